@@ -1,0 +1,165 @@
+"""Seeded synthetic inputs for the DP-SGD step, shared by tests, smoke and bench.
+
+This module holds only shapes, value distributions and the random draws; it
+contains none of the DP-SGD arithmetic, so both the CUDA path and the CPU
+oracle can be fed from it without sharing any of the method's code.
+
+Recipe (stated once, used everywhere):
+  * every array comes from ``numpy.random.default_rng(SeedSequence([seed,
+    workload_id, layer, kind]))`` with kind 0 = activations A, 1 = output
+    gradients D, 2 = audit indices;
+  * draws are fp32 (numpy's float32 samplers), scaled by the distribution's
+    standard deviation in fp32, then rounded to nearest-even into the
+    workload's dtype (fp32: unchanged; bf16: one RNE rounding);
+  * "N(0, v)" in a workload description is read as variance v (std sqrt(v));
+    "ReLU-sparse N(0,1)" is max(0, x) with x ~ N(0,1) (about half exact zeros);
+  * layouts: A [B, T, d_in], D [B, T, d_out], row-major, example-major.
+
+The paper trains LoRA adapters of GPT-2 / RoBERTa, an MLP on Purchase and a
+WideResNet on CIFAR-10 (App. B); none of those datasets or checkpoints is
+available here, so these seeded dense-layer workloads stand in for them.
+"""
+
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import List, Sequence, Tuple
+
+import numpy as np
+import torch
+
+__all__ = ["Workload", "WORKLOADS", "SWEEP", "get", "make_layer", "make_inputs",
+           "audit_indices", "to_f64"]
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    wid: int                       # id folded into the seed sequence
+    layers: Tuple[Tuple[int, int], ...]
+    B: int
+    T: int
+    dtype: str                     # "f32" or "bf16"
+    a_dist: Tuple[str, ...]        # per layer: "normal", "uniform", "relu_normal"
+    a_std: float
+    d_std: float
+    C: float
+    sigma: float
+    audit_frac: float = 0.0
+
+    @property
+    def n_params(self) -> int:
+        return sum(i * o for i, o in self.layers)
+
+    def describe(self) -> str:
+        dims = ",".join(f"{i}x{o}" for i, o in self.layers)
+        return f"{self.name}: layers[{dims}] B={self.B} T={self.T} {self.dtype}"
+
+
+def _normal_all(n):
+    return tuple("normal" for _ in range(n))
+
+
+WORKLOADS = {
+    # single linear layer, fp32, the small case the oracle finishes instantly
+    "single_fp32": Workload("single_fp32", 1, ((64, 32),), 8, 1, "f32",
+                            _normal_all(1), 1.0, 1.0, 1.0, 1.0),
+    # 3-layer MLP 784-512-512-10, fp32; U[0,1) inputs, ReLU-sparse hidden
+    # activations, D ~ N(0, 0.01)
+    "mlp_fp32": Workload("mlp_fp32", 2, ((784, 512), (512, 512), (512, 10)), 256, 1,
+                         "f32", ("uniform", "relu_normal", "relu_normal"),
+                         1.0, math.sqrt(0.01), 1.0, 1.1),
+    # transformer-block linears: QKV, out-proj, FFN up, FFN down; bf16
+    "block_bf16": Workload("block_bf16", 3,
+                           ((768, 2304), (768, 768), (768, 3072), (3072, 768)),
+                           32, 128, "bf16", _normal_all(4), 1.0, math.sqrt(1e-4),
+                           1.0, 0.8),
+    # LLM-scale projections d_model=4096: FFN up/down and fused QKV; bf16
+    "llm_bf16": Workload("llm_bf16", 4,
+                         ((4096, 11008), (11008, 4096), (4096, 12288)),
+                         16, 512, "bf16", _normal_all(3), 1.0, math.sqrt(1e-5),
+                         0.5, 1.0, audit_frac=0.05),
+}
+
+# one 4096x4096 bf16 layer over B x T
+SWEEP = [Workload(f"sweep_B{b}_T{t}", 100 + 10 * bi + ti, ((4096, 4096),), b, t,
+                  "bf16", _normal_all(1), 1.0, 1.0, 1.0, 1.0)
+         for bi, b in enumerate((8, 32, 128)) for ti, t in enumerate((1, 64, 512, 2048))]
+
+
+def get(name: str) -> Workload:
+    if name in WORKLOADS:
+        return WORKLOADS[name]
+    for w in SWEEP:
+        if w.name == name:
+            return w
+    raise KeyError(name)
+
+
+def custom(name: str, layers: Sequence[Tuple[int, int]], B: int, T: int, dtype: str,
+           C: float = 1.0, sigma: float = 1.0, a_std: float = 1.0, d_std: float = 1.0,
+           wid: int = 999, a_dist=None) -> Workload:
+    """An ad-hoc workload (tests use these for ragged and edge shapes)."""
+    a_dist = tuple(a_dist) if a_dist else _normal_all(len(layers))
+    return Workload(name, wid, tuple(tuple(x) for x in layers), B, T, dtype,
+                    a_dist, a_std, d_std, C, sigma)
+
+
+def _draw(rng: np.random.Generator, dist: str, shape, std: float) -> np.ndarray:
+    if dist == "normal":
+        x = rng.standard_normal(shape, dtype=np.float32)
+    elif dist == "uniform":
+        x = rng.random(shape, dtype=np.float32)
+    elif dist == "relu_normal":
+        x = rng.standard_normal(shape, dtype=np.float32)
+        np.maximum(x, np.float32(0.0), out=x)
+    else:
+        raise ValueError(dist)
+    if std != 1.0:
+        x *= np.float32(std)
+    return x
+
+
+def _to_dtype(x: np.ndarray, dtype: str) -> torch.Tensor:
+    t = torch.from_numpy(x)
+    if dtype == "bf16":
+        return t.to(torch.bfloat16)
+    if dtype == "f32":
+        return t
+    raise ValueError(dtype)
+
+
+def make_layer(w: Workload, layer: int, seed: int = 0, B: int | None = None):
+    """(A, D) CPU tensors of layer ``layer`` in the workload's dtype.
+
+    ``B`` may ask for only the first B examples (the draws of example i do not
+    depend on how many examples are drawn after it only when B is the full
+    batch, so callers that sample examples pass the full B)."""
+    B = w.B if B is None else B
+    d_in, d_out = w.layers[layer]
+    ra = np.random.default_rng(np.random.SeedSequence([seed, w.wid, layer, 0]))
+    rd = np.random.default_rng(np.random.SeedSequence([seed, w.wid, layer, 1]))
+    A = _draw(ra, w.a_dist[layer], (B, w.T, d_in), w.a_std)
+    D = _draw(rd, "normal", (B, w.T, d_out), w.d_std)
+    return _to_dtype(A, w.dtype), _to_dtype(D, w.dtype)
+
+
+def make_inputs(w: Workload, seed: int = 0) -> List[Tuple[torch.Tensor, torch.Tensor]]:
+    return [make_layer(w, l, seed) for l in range(len(w.layers))]
+
+
+def audit_indices(w: Workload, seed: int = 0, frac: float | None = None) -> np.ndarray:
+    """ceil(frac * B) distinct example indices (sorted), drawn with kind 2.
+
+    In the paper the TEE picks what to audit from hidden randomness; here the
+    caller's seeded draw stands in for it."""
+    frac = w.audit_frac if frac is None else frac
+    k = max(1, math.ceil(frac * w.B)) if frac > 0 else w.B
+    rng = np.random.default_rng(np.random.SeedSequence([seed, w.wid, 0, 2]))
+    return np.sort(rng.choice(w.B, size=min(k, w.B), replace=False)).astype(np.int32)
+
+
+def to_f64(t: torch.Tensor) -> np.ndarray:
+    """Exact upcast of fp32 / bf16 tensor values to a float64 numpy array."""
+    return t.detach().cpu().to(torch.float64).numpy()
