@@ -1,0 +1,385 @@
+"""Benchmark of the DP-SGD gradient step on GB300.
+
+One step = the whole hot path over one batch: per-example norms of every
+layer, clip factors, clipped sum + fused Philox noise of every layer, and the
+audit emit of the sampled examples (5% of the batch).  Default workload:
+the LLM-scale projections (FFN 4096x11008, 11008x4096, QKV 4096x12288),
+bf16, B=16, T=512.  Prints ONE JSON line on rank 0.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the fp64 CPU oracle (the baseline this build is
+checked against) on a bounded sample of the same workload.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "examples/sec per DP-SGD step (1 GB300) + % BF16 tensor peak / % HBM GB/s"
+UNIT = "examples/s"
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained"), "src": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "src": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        ids = [x.strip() for x in vis.split(",")] if vis else []
+        self.gpu = ids[gpu_index] if gpu_index < len(ids) else str(gpu_index)
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, ValueError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for ln in self.proc.stdout:
+            self.lines.append(ln.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.lines:
+            return None
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax = float(f[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _kernel_sha(path):
+    return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
+
+
+def _traffic(kernel_key, src_file):
+    """DRAM bytes per launch of a kernel from a committed ncu summary, or None
+    when the kernel source changed since the counters were taken."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    d = json.load(open(p)).get(kernel_key)
+    if not d or d.get("src_sha256_16") != _kernel_sha(src_file):
+        return None
+    return d.get("dram_bytes_per_step")
+
+
+def cpu_baseline_sample(w, seed=0):
+    """The fp64 oracle, as it stands, on a bounded sample of the workload:
+    example 0 through every layer (materialised norms, clip factor, its
+    clipped-sum contribution) plus the noise of a 1/B share of the
+    parameters.  Returns (examples/s, seconds, description)."""
+    import numpy as np
+
+    import workloads as W
+    from oracle import dp_oracle as O
+    layers = [W.make_layer(w, l, seed=seed, B=1) for l in range(len(w.layers))]
+    l64 = [(W.to_f64(A), W.to_f64(D)) for A, D in layers]
+    share = w.n_params // w.B
+    t0 = time.perf_counter()
+    n = np.stack([O.layer_sqnorms_materialised(A, D) for A, D in l64])
+    s, c = O.clip_factors(n, float(np.float32(w.C)))
+    S = [O.clipped_sum(A, D, c) for A, D in l64]
+    z = O.gaussian_noise(seed, 0, 0, share)
+    dt = time.perf_counter() - t0
+    del S, z
+    desc = (f"oracle on example 0 of {w.name} (all {len(w.layers)} layers: materialised "
+            f"norms, clip, clipped-sum share) + noise for P/B = {share} parameters")
+    return 1.0 / dt, dt, desc
+
+
+def run_reference(args, rank, world):
+    import numpy as np  # noqa: F401
+    import workloads as W
+    if rank != 0:
+        return
+    w = W.get(args.workload)
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    for _ in range(args.warmup):
+        cpu_baseline_sample(w)
+    times = []
+    desc = ""
+    for _ in range(args.steps):
+        _, dt, desc = cpu_baseline_sample(w)
+        times.append(dt)
+    tot = sum(times)
+    val = args.steps / tot
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": w.describe(), "sample": desc},
+            "cpu_baseline": {"value": val, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": val, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_ours(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+
+    import paper_2609_20532_gb300 as dp
+    import workloads as W
+
+    dev = torch.device(f"cuda:{local_rank}")
+    torch.cuda.set_device(dev)
+    w = W.get(args.workload)
+    L = len(w.layers)
+    layers = W.make_inputs(w, seed=rank)
+    A_d = [A.to(dev) for A, _ in layers]
+    D_d = [D.to(dev) for _, D in layers]
+    outs = [torch.empty(i, o, device=dev, dtype=torch.float32) for i, o in w.layers]
+    idx = W.audit_indices(w, seed=rank)
+    stream = torch.cuda.current_stream()
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
+                         seed=1234 + rank, step=0, audit_capacity=len(idx))
+    ctx = dp.dp_step_init(cfg, stream)
+    in_bytes = sum(A.numel() * A.element_size() + D.numel() * D.element_size()
+                   for A, D in layers)
+    out_bytes = sum(o.numel() * 4 for o in outs)
+    rec_bytes = len(idx) * dp.dp_audit_record_bytes(L)
+
+    ev = {k: [] for k in ("norm", "clip", "gemm")}
+
+    def step(t, timed=False):
+        cfg.step = t
+        dp.dp_step_init(cfg, stream, ctx)
+        for l in range(L):
+            if timed:
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+            dp.dp_layer_norms(ctx, l, A_d[l], D_d[l])
+            if timed:
+                e1.record(stream)
+                ev["norm"].append((l, e0, e1))
+        if timed:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+        dp.dp_clip_factors(ctx)
+        if timed:
+            e1.record(stream)
+            ev["clip"].append((0, e0, e1))
+        for l in range(L):
+            if timed:
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+            dp.dp_clipped_sum_noise(ctx, l, A_d[l], D_d[l], outs[l], 0)
+            if timed:
+                e1.record(stream)
+                ev["gemm"].append((l, e0, e1))
+        return dp.dp_audit_emit(ctx, idx, L)
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for t in range(args.warmup):
+        step(t)
+    torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local_rank) as clk:
+        start.record(stream)
+        for t in range(args.steps):
+            step(args.warmup + t, timed=True)
+        stop.record(stream)
+        torch.cuda.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    ms = start.elapsed_time(stop)
+    if world > 1:
+        import torch.distributed as dist
+        tt = torch.tensor([ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_step = ms / args.steps
+    value = world * w.B / (ms_step * 1e-3)
+
+    def per_step_ms(kind, layer=None):
+        tot = sum(e0.elapsed_time(e1) for l, e0, e1 in ev[kind] if layer is None or l == layer)
+        return tot / args.steps
+
+    peaks = _peaks()
+    gemm_flops = sum(2.0 * w.B * w.T * i * o for i, o in w.layers)
+    gemm_ms = per_step_ms("gemm")
+    gemm_tflops = gemm_flops / (gemm_ms * 1e-3) / 1e12
+    in_total = in_bytes
+    norm_ms = per_step_ms("norm")
+    norm_gbs = in_total / (norm_ms * 1e-3) / 1e9
+    src = os.path.join(ROOT, "paper_2609_20532_gb300", "csrc", "k_tc.cu")
+    traffic = _traffic("clipsum_gemm", src)
+    kernels = {
+        "clipsum_gemm": {"ms_per_step": gemm_ms, "tflops": gemm_tflops,
+                         "frac_bf16_peak": gemm_tflops / peaks["bf16_tflops"],
+                         "per_layer_ms": [per_step_ms("gemm", l) for l in range(L)]},
+        "layer_norms": {"ms_per_step": norm_ms, "gbs_inputs_read_once": norm_gbs,
+                        "frac_hbm": norm_gbs / peaks["hbm_gbs"],
+                        "per_layer_ms": [per_step_ms("norm", l) for l in range(L)]},
+        "clip": {"ms_per_step": per_step_ms("clip")},
+    }
+
+    # ---- end to end through the C ABI with host buffers ----
+    e2e = None
+    if not args.no_e2e:
+        A_h = [A.pin_memory() for A, _ in layers]
+        D_h = [D.pin_memory() for _, D in layers]
+        O_h = [torch.empty(o.shape, dtype=torch.float32).pin_memory() for o in outs]
+
+        def e2e_step(t):
+            for l in range(L):
+                A_d[l].copy_(A_h[l], non_blocking=True)
+                D_d[l].copy_(D_h[l], non_blocking=True)
+            cfg.step = t
+            dp.dp_step_init(cfg, stream, ctx)
+            for l in range(L):
+                dp.dp_layer_norms(ctx, l, A_d[l], D_d[l])
+            dp.dp_clip_factors(ctx)
+            for l in range(L):
+                dp.dp_clipped_sum_noise(ctx, l, A_d[l], D_d[l], outs[l], 0)
+                O_h[l].copy_(outs[l], non_blocking=True)
+            return dp.dp_audit_emit(ctx, idx, L)   # synchronises the stream
+
+        for t in range(max(1, args.warmup)):
+            e2e_step(t)
+        torch.cuda.synchronize()
+        barrier()
+        k = max(1, args.e2e_steps)
+        t0 = time.perf_counter()
+        for t in range(k):
+            e2e_step(t)
+        torch.cuda.synchronize()
+        wall = (time.perf_counter() - t0) / k
+        if world > 1:
+            import torch.distributed as dist
+            tt = torch.tensor([wall], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            wall = float(tt.item())
+        e2e = {"value": world * w.B / wall, "unit": UNIT, "ms_per_step": 1e3 * wall,
+               "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes + rec_bytes,
+               "steps": k}
+
+    dp.dp_step_destroy(ctx)
+    if rank != 0:
+        return
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+        v, dt, desc = cpu_baseline_sample(w)
+        cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
+               "seconds": dt}
+    dominant = "clipsum_gemm"
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
+        "data": "synthetic: seeded N(0,1) activations, N(0,1e-5) output grads, rounded to bf16",
+        "config": {"workload": w.describe(), "layers": [list(x) for x in w.layers], "B": w.B,
+                   "T": w.T, "C": w.C, "sigma": w.sigma, "out_scale": "1/B",
+                   "audit_examples": len(idx),
+                   "l2": f"inputs {in_bytes / 1e6:.0f} MB > 129 MB L2 (no flush needed)",
+                   "parallelism": "replicas" if world > 1 else "single"},
+        "roofline": {"kernel": dominant, "bound": "tensor", "achieved": gemm_tflops,
+                     "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                     "frac": gemm_tflops / peaks["bf16_tflops"], "traffic": traffic,
+                     "peak_src": f"{peaks['src']} bf16 burst"},
+        "kernels": kernels,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": args.steps * (2 * L + 2),
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="llm_bf16")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    try:
+        run_ours(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,210 @@
+/*
+ * dp_step.h -- C ABI of the GB300 (sm_103a) DP-SGD gradient-step library.
+ *
+ * The library runs, on one GPU, the work the untrusted accelerator does in the
+ * paper's verifiable DP-SGD protocol (Algorithm 2): per-example gradients of
+ * dense layers, their L2 norms across all layers, per-example clipping, the
+ * clipped sum, and the seeded Gaussian noise that the trusted side can
+ * regenerate (Sec. 2.2 "DP-SGD"; Algorithms 2 and 3; Sec. 7.2 "Communication-
+ * efficient split execution").  It also emits per-example audit records for
+ * the partial recomputation a CPU-side checker performs (Sec. 7).
+ *
+ * Notation.  A step has B examples of T positions each and L dense layers;
+ * layer l has weight shape d_in x d_out.  For example i the caller supplies
+ *   A_{i,l} in R^{T x d_in}   activations entering layer l,
+ *   D_{i,l} in R^{T x d_out}  gradients of the loss w.r.t. layer l's outputs,
+ * so that the per-example weight gradient is G_{i,l} = A_{i,l}^T D_{i,l}
+ * (laid out [d_in, d_out]).
+ *
+ * Memory layout of every A / D argument: one dense row-major array
+ * [B][T][d] (example-major, then position, then feature), element type from
+ * dp_config.dtype, base address 16-byte aligned, rows d * elemsize bytes
+ * apart.  d * elemsize must be a multiple of 16 bytes for bf16 inputs.
+ * Outputs are fp32 row-major [d_in][d_out], 16-byte aligned.
+ *
+ * Ownership.  The caller owns every A, D and output buffer and the CUDA
+ * stream; buffers are device pointers unless a parameter says "host".  The
+ * context owns its scratch (per-layer norm partials, norms, clip factors,
+ * audit staging, an error flag) and frees it in dp_step_destroy.
+ *
+ * Asynchrony.  Every call except dp_audit_emit only enqueues work on the
+ * context's stream and returns; dp_audit_emit synchronises that stream.
+ *
+ * Errors.  Argument, shape, dtype and call-order errors are detected on the
+ * host before anything is launched, and the call returns without side
+ * effects.  Device-detected conditions (a non-finite squared norm) set a
+ * sticky flag in the context that the next synchronising call
+ * (dp_audit_emit) reports as DP_ERR_NONFINITE.  dp_last_error() returns a
+ * message for the last failing call on the calling thread.
+ *
+ * Call order within one step:
+ *   dp_step_init  ->  dp_layer_norms (every layer, any order)
+ *                 ->  dp_clip_factors
+ *                 ->  dp_clipped_sum_noise (any layers, any order, any number)
+ *                 ->  dp_audit_emit (optional, any number of times)
+ * Anything else returns DP_ERR_ORDER, except dp_clipped_sum_noise with
+ * DP_NOISE_ONLY, which needs only an initialised context.
+ */
+#ifndef DP_STEP_H
+#define DP_STEP_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct dp_ctx dp_ctx; /* opaque, owned by the library */
+
+typedef enum {
+    DP_OK = 0,
+    DP_ERR_ARG = 1,         /* null pointer, misaligned buffer, bad scalar, index out of range */
+    DP_ERR_SHAPE = 2,       /* shape disagrees with the context / limits exceeded */
+    DP_ERR_DTYPE = 3,       /* unknown element type */
+    DP_ERR_ORDER = 4,       /* call made out of the order documented above */
+    DP_ERR_NONFINITE = 5,   /* a per-example squared norm was NaN or infinite */
+    DP_ERR_CUDA = 6,        /* a CUDA runtime / driver call failed */
+    DP_ERR_TIMEOUT = 7,     /* a bounded device wait gave up */
+    DP_ERR_OOM = 8,         /* device or pinned host allocation failed */
+    DP_ERR_UNSUPPORTED = 9  /* the device is not an sm_103 GPU or a path is not built */
+} dp_status;
+
+typedef enum { DP_F32 = 0, DP_BF16 = 1 } dp_dtype;
+
+/* How the per-example squared norm ||A_i^T D_i||_F^2 of a layer is formed.
+ * RANK1: T must be 1, n_i = ||a_i||^2 ||d_i||^2.
+ * GHOST: n_i = sum_{t,s} (a_t . a_s)(d_t . d_s), from the two T x T Gram matrices.
+ * MATERIALISED: the d_in x d_out gradient is formed tile by tile on chip,
+ *   squared and summed; it is never written to memory.
+ * AUTO: RANK1 when T == 1, else whichever of GHOST / MATERIALISED has the
+ *   smaller arithmetic cost (T <= 2 d_in d_out / (d_in + d_out) picks GHOST). */
+typedef enum {
+    DP_NORM_AUTO = 0,
+    DP_NORM_RANK1 = 1,
+    DP_NORM_GHOST = 2,
+    DP_NORM_MATERIALISED = 3
+} dp_norm_mode;
+
+typedef struct {
+    int64_t d_in;
+    int64_t d_out;
+} dp_layer;
+
+/* Parameters of Algorithm 2 for one step: batch B (also the aggregation
+ * denominator when out_scale = 1/B), clip norm C, noise multiplier sigma and
+ * the released per-step noise seed (seed, step). */
+typedef struct {
+    int32_t B;                 /* examples per step, >= 1 */
+    int32_t T;                 /* positions per example, >= 1 */
+    int32_t n_layers;          /* L, 1 .. 64 */
+    const dp_layer* layers;    /* host array of L layer shapes; copied by dp_step_init */
+    dp_dtype dtype;            /* element type of every A and D */
+    float clip_C;              /* C > 0 */
+    float sigma;               /* noise multiplier, >= 0 */
+    float out_scale;           /* 1 (sum) or 1/B (Algorithm 2 average); any finite value */
+    uint64_t seed;             /* Philox key; the trusted side's s_noise,t */
+    uint64_t step;             /* step index t; upper Philox counter words */
+    dp_norm_mode norm_mode;    /* applies to every layer (AUTO picks per layer) */
+    int32_t audit_capacity;    /* max records per dp_audit_emit call, 0 .. B */
+} dp_config;
+
+/* Flags of dp_clipped_sum_noise. */
+#define DP_NO_NOISE   0x1u /* write out_scale * S only: the noiseless commitment of Algorithm 2 */
+#define DP_NOISE_ONLY 0x2u /* out += out_scale * sigma * C * z; A and D are ignored (may be NULL) */
+#define DP_ACCUMULATE 0x4u /* add into out instead of overwriting it (micro-batch accumulation) */
+
+/* Create (*ctx == NULL) or re-key (*ctx != NULL) a step context.
+ * Create: validates cfg, allocates scratch on the current device and binds
+ *   cuda_stream (a cudaStream_t; NULL = the legacy default stream).
+ * Re-key: cfg must have the same B, T, dtype and layer shapes as the context
+ *   (else DP_ERR_SHAPE and the context is unchanged); clip_C, sigma,
+ *   out_scale, seed, step, norm_mode, audit_capacity and the stream are
+ *   replaced and the per-step call-order state is reset.  Used once per
+ *   training step, and again to supply the seed the trusted side releases
+ *   after the commitment (Algorithm 3, Derive/release) before a
+ *   DP_NOISE_ONLY call.
+ * Limits: B * T <= 2^31 - 1; every d_in, d_out in 1 .. 2^20; the device must
+ *   be compute capability 10.3.
+ * Errors: DP_ERR_ARG, DP_ERR_SHAPE, DP_ERR_DTYPE, DP_ERR_UNSUPPORTED,
+ *   DP_ERR_OOM, DP_ERR_CUDA. On failure of a create, *ctx stays NULL. */
+dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream);
+
+/* Per-example squared gradient norms of one layer (Sec. 2.2 clipping
+ * equation: ||g_t(x_i)||_2^2 restricted to layer l):
+ *   n_{l,i} = ||A_{i,l}^T D_{i,l}||_F^2,  i = 0 .. B-1,
+ * kept in the context.  A: [B][T][d_in], D: [B][T][d_out] device arrays.
+ * Errors: DP_ERR_ARG (null / misaligned), DP_ERR_ORDER (after
+ * dp_clip_factors of this step), DP_ERR_CUDA. */
+dp_status dp_layer_norms(dp_ctx* ctx, int32_t layer, const void* A, const void* D);
+
+/* Sum the per-layer norms and form the clip factors (Sec. 2.2; Algorithm 2):
+ *   s_i = sum_l n_{l,i},   c_i = 1 if s_i <= C^2 else C / sqrt(s_i).
+ * d_sqnorm_out [B] and d_clip_out [B] are optional device fp32 arrays that
+ * receive s and c (NULL to skip).  A non-finite s_i sets the sticky flag and
+ * gives c_i = NaN.
+ * Errors: DP_ERR_ORDER (a layer's norms are missing), DP_ERR_ARG, DP_ERR_CUDA. */
+dp_status dp_clip_factors(dp_ctx* ctx, float* d_sqnorm_out, float* d_clip_out);
+
+/* Clipped sum and noise of one layer (Algorithm 2; Sec. 2.2 aggregation):
+ *   S_l = sum_i c_i A_{i,l}^T D_{i,l} = A_l^T diag(c (x) 1_T) D_l   [d_in x d_out]
+ *   out = out_scale * (S_l + sigma * C * z_l)       (flags = 0)
+ *   z_p = Gaussian number of global parameter index p = off_l + j*d_out + k,
+ *         off_l = sum_{l' < l} d_in^{l'} d_out^{l'};
+ *   Philox4x32-10 with key = (lo32 seed, hi32 seed) and counter =
+ *   (lo32 q, hi32 q, lo32 step, hi32 step), q = p >> 2, gives words x0..x3;
+ *   u0 = RN_fp32((x_{2m}+1) / 2^32), u1 = RN_fp32(x_{2m+1} / 2^32);
+ *   slots 2m, 2m+1 of the quad are sqrt(-2 ln u0) * (cos, sin)(2 pi u1).
+ * flags: DP_NO_NOISE, DP_NOISE_ONLY, DP_ACCUMULATE (see above).
+ * d_out: device fp32 [d_in][d_out], 16-byte aligned, owned by the caller.
+ * Errors: DP_ERR_ARG, DP_ERR_ORDER (clip factors not formed yet, unless
+ *   DP_NOISE_ONLY), DP_ERR_CUDA. */
+dp_status dp_clipped_sum_noise(dp_ctx* ctx, int32_t layer, const void* A, const void* D,
+                               float* d_out, uint32_t flags);
+
+/* Audit emit: for the n example indices in h_idx (host array, each in
+ * 0 .. B-1, n <= audit_capacity) copy records into h_records (host memory,
+ * n * dp_audit_record_bytes(L) bytes) with layout per record:
+ *   int32_t example; float total_sqnorm (s_i); float clip_factor (c_i);
+ *   float layer_sqnorm[L] (n_{1..L,i})
+ * -- what a checker needs to recompute the audited examples (Sec. 7, partial
+ * recomputation; Algorithm 1 consumes the recomputed aggregate).
+ * Synchronises the context's stream.  Returns DP_ERR_NONFINITE if the sticky
+ * flag was set during this step (records are still written).
+ * Errors: DP_ERR_ARG, DP_ERR_ORDER (before dp_clip_factors), DP_ERR_NONFINITE,
+ *   DP_ERR_CUDA. */
+dp_status dp_audit_emit(dp_ctx* ctx, const int32_t* h_idx, int32_t n, void* h_records);
+
+/* Bytes of one audit record for L layers: 12 + 4 L. */
+int64_t dp_audit_record_bytes(int32_t n_layers);
+
+/* Norm mode chosen for a layer (resolves DP_NORM_AUTO). */
+dp_status dp_layer_norm_mode(const dp_ctx* ctx, int32_t layer, dp_norm_mode* mode_out);
+
+/* Release the context and all of its scratch; NULL is a no-op.  Waits for
+ * the context's pending work first. */
+void dp_step_destroy(dp_ctx* ctx);
+
+/* Message of the last failing call on this thread ("" if none). */
+const char* dp_last_error(void);
+
+/* Name of a status code. */
+const char* dp_status_string(dp_status s);
+
+/* ---- test exports (not part of the step API) ---------------------------
+ * They expose the generator the noise uses so tests can compare it with the
+ * oracle: raw Philox4x32-10 blocks and the Gaussian numbers z_p.
+ * d_out is a device array; stream is a cudaStream_t (NULL = default).    */
+
+/* d_out[4 r + w] = word w of the block for quad first_quad + r, r < n_quads. */
+dp_status dp_debug_philox(uint64_t seed, uint64_t step, uint64_t first_quad, int64_t n_quads,
+                          uint32_t* d_out, void* stream);
+
+/* d_out[r] = z_{first_index + r} (unit variance, as defined above), r < n. */
+dp_status dp_debug_gaussian(uint64_t seed, uint64_t step, uint64_t first_index, int64_t n,
+                            float* d_out, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DP_STEP_H */

@@ -1,0 +1,225 @@
+"""Python binding of the GB300 DP-SGD step library (``libdpstep.so``).
+
+Argument marshalling only: every function here forwards to the C entry point
+of the same name declared in ``include/dp_step.h`` (device pointers, sizes,
+the CUDA stream handle).  All arithmetic of the step runs in the library's
+CUDA kernels; there is no CPU fallback, and importing a function whose
+library is missing raises :class:`LibraryNotBuilt`.
+
+PyTorch appears here only as the owner of device memory and streams.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Iterable, List, Optional, Sequence
+
+import numpy as np
+
+__all__ = [
+    "DPError", "LibraryNotBuilt", "lib", "lib_path",
+    "DP_OK", "DP_F32", "DP_BF16",
+    "DP_NORM_AUTO", "DP_NORM_RANK1", "DP_NORM_GHOST", "DP_NORM_MATERIALISED",
+    "DP_NO_NOISE", "DP_NOISE_ONLY", "DP_ACCUMULATE",
+    "dp_layer", "dp_config", "make_config",
+    "dp_step_init", "dp_layer_norms", "dp_clip_factors", "dp_clipped_sum_noise",
+    "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_step_destroy",
+    "dp_last_error", "dp_debug_philox", "dp_debug_gaussian", "EXPORTED_SYMBOLS",
+]
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+lib_path = os.path.join(HERE, "libdpstep.so")
+
+DP_OK = 0
+DP_F32, DP_BF16 = 0, 1
+DP_NORM_AUTO, DP_NORM_RANK1, DP_NORM_GHOST, DP_NORM_MATERIALISED = 0, 1, 2, 3
+DP_NO_NOISE, DP_NOISE_ONLY, DP_ACCUMULATE = 0x1, 0x2, 0x4
+
+STATUS_NAMES = {0: "DP_OK", 1: "DP_ERR_ARG", 2: "DP_ERR_SHAPE", 3: "DP_ERR_DTYPE",
+                4: "DP_ERR_ORDER", 5: "DP_ERR_NONFINITE", 6: "DP_ERR_CUDA",
+                7: "DP_ERR_TIMEOUT", 8: "DP_ERR_OOM", 9: "DP_ERR_UNSUPPORTED"}
+
+# every symbol include/dp_step.h declares
+EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_clip_factors", "dp_clipped_sum_noise",
+                    "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode",
+                    "dp_step_destroy", "dp_last_error", "dp_status_string", "dp_debug_philox",
+                    "dp_debug_gaussian"]
+
+
+class DPError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        self.status = status
+        self.name = STATUS_NAMES.get(status, str(status))
+        super().__init__(f"{self.name}: {msg}")
+
+
+class LibraryNotBuilt(ImportError):
+    pass
+
+
+class dp_layer(ctypes.Structure):
+    _fields_ = [("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64)]
+
+
+class dp_config(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int32), ("T", ctypes.c_int32), ("n_layers", ctypes.c_int32),
+                ("layers", ctypes.POINTER(dp_layer)), ("dtype", ctypes.c_int32),
+                ("clip_C", ctypes.c_float), ("sigma", ctypes.c_float),
+                ("out_scale", ctypes.c_float), ("seed", ctypes.c_uint64),
+                ("step", ctypes.c_uint64), ("norm_mode", ctypes.c_int32),
+                ("audit_capacity", ctypes.c_int32)]
+
+
+_LIB = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load ``libdpstep.so`` (once).  Raises LibraryNotBuilt if it is missing."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    if not os.path.exists(lib_path):
+        raise LibraryNotBuilt(
+            f"{lib_path} is missing: build it with `python -c 'import __graft_entry__ as g; "
+            f"g.build()'` (nvcc, sm_103a)")
+    L = ctypes.CDLL(lib_path)
+    vp, i32, i64, u32, u64 = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32,
+                              ctypes.c_uint64)
+    sig = {
+        "dp_step_init": ([ctypes.POINTER(vp), ctypes.POINTER(dp_config), vp], i32),
+        "dp_layer_norms": ([vp, i32, vp, vp], i32),
+        "dp_clip_factors": ([vp, vp, vp], i32),
+        "dp_clipped_sum_noise": ([vp, i32, vp, vp, vp, u32], i32),
+        "dp_audit_emit": ([vp, vp, i32, vp], i32),
+        "dp_audit_record_bytes": ([i32], i64),
+        "dp_layer_norm_mode": ([vp, i32, ctypes.POINTER(i32)], i32),
+        "dp_step_destroy": ([vp], None),
+        "dp_last_error": ([], ctypes.c_char_p),
+        "dp_status_string": ([i32], ctypes.c_char_p),
+        "dp_debug_philox": ([u64, u64, u64, i64, vp, vp], i32),
+        "dp_debug_gaussian": ([u64, u64, u64, i64, vp, vp], i32),
+    }
+    for name, (args, res) in sig.items():
+        f = getattr(L, name)
+        f.argtypes = args
+        f.restype = res
+    _LIB = L
+    return L
+
+
+def _check(st: int):
+    if st != DP_OK:
+        raise DPError(st, lib().dp_last_error().decode())
+
+
+def _ptr(x) -> Optional[int]:
+    """Device pointer of a torch tensor (contiguity checked), an int, or None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        if not x.is_contiguous():
+            raise ValueError("tensor arguments must be contiguous")
+        return x.data_ptr()
+    raise TypeError(f"cannot take a pointer of {type(x)}")
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def make_config(layers: Sequence[Sequence[int]], B: int, T: int, dtype: str, C: float,
+                sigma: float, out_scale: float = 1.0, seed: int = 0, step: int = 0,
+                norm_mode: int = DP_NORM_AUTO, audit_capacity: int = 0) -> dp_config:
+    arr = (dp_layer * len(layers))(*[dp_layer(int(i), int(o)) for i, o in layers])
+    cfg = dp_config(B=B, T=T, n_layers=len(layers), layers=arr,
+                    dtype=DP_BF16 if dtype == "bf16" else DP_F32, clip_C=C, sigma=sigma,
+                    out_scale=out_scale, seed=seed & (2 ** 64 - 1), step=step & (2 ** 64 - 1),
+                    norm_mode=norm_mode, audit_capacity=audit_capacity)
+    cfg._keep = arr  # keep the layer array alive with the struct
+    return cfg
+
+
+def dp_step_init(cfg: dp_config, stream=None, ctx: Optional[int] = None) -> int:
+    """Create a context (ctx None) or re-key an existing one; returns the handle."""
+    h = ctypes.c_void_p(ctx)
+    _check(lib().dp_step_init(ctypes.byref(h), ctypes.byref(cfg), _stream(stream)))
+    return h.value
+
+
+def dp_layer_norms(ctx: int, layer: int, A, D) -> None:
+    _check(lib().dp_layer_norms(ctx, layer, _ptr(A), _ptr(D)))
+
+
+def dp_clip_factors(ctx: int, sqnorm_out=None, clip_out=None) -> None:
+    _check(lib().dp_clip_factors(ctx, _ptr(sqnorm_out), _ptr(clip_out)))
+
+
+def dp_clipped_sum_noise(ctx: int, layer: int, A, D, out, flags: int = 0) -> None:
+    _check(lib().dp_clipped_sum_noise(ctx, layer, _ptr(A), _ptr(D), _ptr(out), flags))
+
+
+def dp_audit_record_bytes(n_layers: int) -> int:
+    return int(lib().dp_audit_record_bytes(n_layers))
+
+
+def dp_audit_emit(ctx: int, idx: Iterable[int], n_layers: int) -> List[dict]:
+    """Records for the listed examples: dicts with example, total_sqnorm,
+    clip_factor and layer_sqnorm (numpy [L])."""
+    idx = np.ascontiguousarray(np.asarray(list(idx), dtype=np.int32))
+    n = int(idx.size)
+    words = 3 + n_layers
+    buf = np.zeros(max(n, 1) * words, dtype=np.float32)
+    st = lib().dp_audit_emit(ctx, idx.ctypes.data if n else None, n, buf.ctypes.data)
+    if st not in (DP_OK, 5):
+        _check(st)
+    recs = []
+    for r in range(n):
+        w = buf[r * words:(r + 1) * words]
+        recs.append({"example": int(w[:1].view(np.int32)[0]), "total_sqnorm": float(w[1]),
+                     "clip_factor": float(w[2]), "layer_sqnorm": w[3:].astype(np.float64)})
+    if st != DP_OK:
+        _check(st)
+    return recs
+
+
+def dp_layer_norm_mode(ctx: int, layer: int) -> int:
+    m = ctypes.c_int32(0)
+    _check(lib().dp_layer_norm_mode(ctx, layer, ctypes.byref(m)))
+    return m.value
+
+
+def dp_step_destroy(ctx: Optional[int]) -> None:
+    if ctx:
+        lib().dp_step_destroy(ctx)
+
+
+def dp_last_error() -> str:
+    return lib().dp_last_error().decode()
+
+
+def dp_debug_philox(seed: int, step: int, first_quad: int, n_quads: int, out, stream=None):
+    _check(lib().dp_debug_philox(seed & (2 ** 64 - 1), step & (2 ** 64 - 1),
+                                 first_quad & (2 ** 64 - 1), n_quads, _ptr(out), _stream(stream)))
+
+
+def dp_debug_gaussian(seed: int, step: int, first_index: int, n: int, out, stream=None):
+    _check(lib().dp_debug_gaussian(seed & (2 ** 64 - 1), step & (2 ** 64 - 1),
+                                   first_index & (2 ** 64 - 1), n, _ptr(out), _stream(stream)))
+
+
+def run_step(ctx: int, A_list, D_list, outs, flags: int = 0) -> None:
+    """The five calls of one step in order (norms of every layer, clip,
+    clipped sum + noise of every layer); audit is left to the caller."""
+    for l, (A, D) in enumerate(zip(A_list, D_list)):
+        dp_layer_norms(ctx, l, A, D)
+    dp_clip_factors(ctx)
+    for l, (A, D) in enumerate(zip(A_list, D_list)):
+        dp_clipped_sum_noise(ctx, l, A, D, outs[l], flags)

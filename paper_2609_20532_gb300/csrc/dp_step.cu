@@ -1,0 +1,479 @@
+// C-ABI layer of the DP-SGD step library: argument checking, the per-step
+// call-order state machine, scratch ownership and kernel dispatch.  See
+// include/dp_step.h for the contract of every entry point.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/dp_step.h"
+#include "internal.h"
+#include "tc.h"
+
+namespace {
+
+thread_local std::string g_err;
+
+dp_status fail(dp_status st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  std::vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return st;
+}
+
+#define DP_CUDA(call)                                                                      \
+  do {                                                                                     \
+    cudaError_t e_ = (call);                                                               \
+    if (e_ != cudaSuccess)                                                                 \
+      return fail(DP_ERR_CUDA, "%s failed: %s", #call, cudaGetErrorString(e_));            \
+  } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+// Per-layer execution plan, fixed at init from the shapes and the norm mode.
+struct LayerPlan {
+  int64_t d_in, d_out;
+  uint64_t p_base;     // global parameter index of element (0, 0)
+  dp_norm_mode mode;   // resolved norm mode
+  int norm_tc;         // 1: tensor-core norm kernel
+  int nparts;          // partial sums per example
+  int gemm_tc;         // 1: tcgen05 clipped sum
+};
+
+struct dp_ctx {
+  int B = 0, T = 0, L = 0;
+  dp_dtype dtype = DP_F32;
+  float C = 1.f, sigma = 0.f, out_scale = 1.f;
+  uint64_t seed = 0, step = 0;
+  dp_norm_mode norm_mode = DP_NORM_AUTO;
+  int audit_capacity = 0;
+  cudaStream_t stream = nullptr;
+  int device = 0;
+  std::vector<LayerPlan> plan;
+  int NP = 1;  // partial-sum stride
+  // scratch
+  float* d_part = nullptr;      // [L][B][NP]
+  int* d_nparts = nullptr;      // [L]
+  float* d_layer_sq = nullptr;  // [L][B]
+  float* d_s = nullptr;         // [B]
+  float* d_c = nullptr;         // [B]
+  int* d_flag = nullptr;        // sticky error bits
+  int* d_idx = nullptr;         // [cap]
+  float* d_rec = nullptr;       // [cap][3 + L]
+  int* h_idx = nullptr;         // pinned [cap]
+  float* h_rec = nullptr;       // pinned [cap][3 + L]
+  int* h_flag = nullptr;        // pinned
+  size_t part_bytes = 0;
+  // per-step state
+  std::vector<char> norm_done;
+  bool clip_done = false;
+};
+
+namespace {
+
+dp_status check_config(const dp_config* cfg) {
+  if (!cfg) return fail(DP_ERR_ARG, "cfg is NULL");
+  if (cfg->B < 1 || cfg->T < 1) return fail(DP_ERR_SHAPE, "B and T must be >= 1");
+  if (static_cast<int64_t>(cfg->B) * cfg->T > 0x7fffffffLL)
+    return fail(DP_ERR_SHAPE, "B*T exceeds 2^31-1");
+  if (cfg->n_layers < 1 || cfg->n_layers > 64)
+    return fail(DP_ERR_SHAPE, "n_layers must be in 1..64");
+  if (!cfg->layers) return fail(DP_ERR_ARG, "layers is NULL");
+  if (cfg->dtype != DP_F32 && cfg->dtype != DP_BF16) return fail(DP_ERR_DTYPE, "unknown dtype");
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    const dp_layer& ly = cfg->layers[l];
+    if (ly.d_in < 1 || ly.d_out < 1 || ly.d_in > (1 << 20) || ly.d_out > (1 << 20))
+      return fail(DP_ERR_SHAPE, "layer %d: d_in, d_out must be in 1..2^20", l);
+    if (cfg->dtype == DP_BF16 && ((ly.d_in * 2) % 16 || (ly.d_out * 2) % 16))
+      return fail(DP_ERR_SHAPE, "layer %d: bf16 rows must be a multiple of 16 bytes", l);
+  }
+  if (!(cfg->clip_C > 0.f) || !std::isfinite(cfg->clip_C))
+    return fail(DP_ERR_ARG, "clip_C must be finite and > 0");
+  if (!(cfg->sigma >= 0.f) || !std::isfinite(cfg->sigma))
+    return fail(DP_ERR_ARG, "sigma must be finite and >= 0");
+  if (!std::isfinite(cfg->out_scale)) return fail(DP_ERR_ARG, "out_scale must be finite");
+  if (cfg->norm_mode < DP_NORM_AUTO || cfg->norm_mode > DP_NORM_MATERIALISED)
+    return fail(DP_ERR_ARG, "unknown norm_mode");
+  if (cfg->norm_mode == DP_NORM_RANK1 && cfg->T != 1)
+    return fail(DP_ERR_SHAPE, "DP_NORM_RANK1 needs T == 1");
+  if (cfg->audit_capacity < 0 || cfg->audit_capacity > cfg->B)
+    return fail(DP_ERR_ARG, "audit_capacity must be in 0..B");
+  return DP_OK;
+}
+
+dp_norm_mode resolve_mode(dp_norm_mode m, int T, int64_t d_in, int64_t d_out) {
+  if (m != DP_NORM_AUTO) return m;
+  if (T == 1) return DP_NORM_RANK1;
+  // Multiply-adds per example: Gram form about T^2 (d_in + d_out) / 2 with
+  // the symmetric half, materialised form T d_in d_out.
+  const double ghost = 0.5 * double(T) * T * double(d_in + d_out);
+  const double mat = double(T) * double(d_in) * double(d_out);
+  return ghost <= mat ? DP_NORM_GHOST : DP_NORM_MATERIALISED;
+}
+
+void build_plan(dp_ctx* c, const dp_config* cfg) {
+  c->plan.resize(cfg->n_layers);
+  uint64_t off = 0;
+  int NP = 1;
+  for (int l = 0; l < cfg->n_layers; ++l) {
+    LayerPlan& p = c->plan[l];
+    p.d_in = cfg->layers[l].d_in;
+    p.d_out = cfg->layers[l].d_out;
+    p.p_base = off;
+    off += static_cast<uint64_t>(p.d_in) * p.d_out;
+    p.mode = resolve_mode(cfg->norm_mode, cfg->T, p.d_in, p.d_out);
+    const bool bf16 = cfg->dtype == DP_BF16;
+    p.norm_tc = 0;
+    if (p.mode == DP_NORM_RANK1) {
+      p.nparts = dpk::rank1_parts();
+    } else if (p.mode == DP_NORM_GHOST) {
+      p.norm_tc = bf16 && dpk::tc_ghost_supported(cfg->T, p.d_in, p.d_out);
+      p.nparts = p.norm_tc ? dpk::tc_ghost_parts(cfg->T) : dpk::ghost_simt_parts(cfg->T);
+    } else {
+      p.norm_tc = bf16 && dpk::tc_gemm_supported(cfg->T, p.d_in, p.d_out);
+      p.nparts = p.norm_tc ? dpk::tc_mat_parts(p.d_in, p.d_out)
+                           : dpk::mat_simt_parts(static_cast<int>(p.d_in), static_cast<int>(p.d_out));
+    }
+    p.gemm_tc = bf16 && dpk::tc_gemm_supported(cfg->T, p.d_in, p.d_out);
+    if (p.nparts > NP) NP = p.nparts;
+  }
+  c->NP = NP;
+}
+
+void free_scratch(dp_ctx* c) {
+  cudaFree(c->d_part);
+  cudaFree(c->d_nparts);
+  cudaFree(c->d_layer_sq);
+  cudaFree(c->d_s);
+  cudaFree(c->d_c);
+  cudaFree(c->d_flag);
+  cudaFree(c->d_idx);
+  cudaFree(c->d_rec);
+  cudaFreeHost(c->h_idx);
+  cudaFreeHost(c->h_rec);
+  cudaFreeHost(c->h_flag);
+  c->d_part = nullptr;
+  c->d_nparts = nullptr;
+  c->d_layer_sq = c->d_s = c->d_c = nullptr;
+  c->d_flag = nullptr;
+  c->d_idx = nullptr;
+  c->d_rec = nullptr;
+  c->h_idx = nullptr;
+  c->h_rec = nullptr;
+  c->h_flag = nullptr;
+}
+
+dp_status alloc_scratch(dp_ctx* c) {
+  const int L = c->L, B = c->B;
+  const int cap = c->B;  // audit staging sized for the whole batch
+  c->part_bytes = sizeof(float) * static_cast<size_t>(L) * B * c->NP;
+#define DP_ALLOC(ptr, bytes)                                                           \
+  do {                                                                                 \
+    if (cudaMalloc(reinterpret_cast<void**>(&(ptr)), (bytes)) != cudaSuccess) {        \
+      cudaGetLastError();                                                              \
+      free_scratch(c);                                                                 \
+      return fail(DP_ERR_OOM, "cudaMalloc of %zu bytes failed", size_t(bytes));        \
+    }                                                                                  \
+  } while (0)
+  DP_ALLOC(c->d_part, c->part_bytes);
+  DP_ALLOC(c->d_nparts, sizeof(int) * L);
+  DP_ALLOC(c->d_layer_sq, sizeof(float) * L * B);
+  DP_ALLOC(c->d_s, sizeof(float) * B);
+  DP_ALLOC(c->d_c, sizeof(float) * B);
+  DP_ALLOC(c->d_flag, sizeof(int));
+  DP_ALLOC(c->d_idx, sizeof(int) * cap);
+  DP_ALLOC(c->d_rec, sizeof(float) * cap * (3 + L));
+#undef DP_ALLOC
+  if (cudaMallocHost(reinterpret_cast<void**>(&c->h_idx), sizeof(int) * cap) != cudaSuccess ||
+      cudaMallocHost(reinterpret_cast<void**>(&c->h_rec), sizeof(float) * cap * (3 + L)) !=
+          cudaSuccess ||
+      cudaMallocHost(reinterpret_cast<void**>(&c->h_flag), sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    free_scratch(c);
+    return fail(DP_ERR_OOM, "pinned host allocation failed");
+  }
+  return DP_OK;
+}
+
+dp_status upload_plan(dp_ctx* c) {
+  // Pageable-source copy: returns once the source has been staged, so the
+  // vector may go out of scope without a stream synchronisation.
+  std::vector<int> np(c->L);
+  for (int l = 0; l < c->L; ++l) np[l] = c->plan[l].nparts;
+  DP_CUDA(cudaMemcpyAsync(c->d_nparts, np.data(), sizeof(int) * c->L, cudaMemcpyHostToDevice,
+                          c->stream));
+  return DP_OK;
+}
+
+bool same_parts(const std::vector<LayerPlan>& a, const std::vector<LayerPlan>& b) {
+  if (a.size() != b.size()) return false;
+  for (size_t l = 0; l < a.size(); ++l)
+    if (a[l].nparts != b[l].nparts) return false;
+  return true;
+}
+
+void reset_step(dp_ctx* c) {
+  c->norm_done.assign(c->L, 0);
+  c->clip_done = false;
+}
+
+void set_scalars(dp_ctx* c, const dp_config* cfg, void* stream) {
+  c->C = cfg->clip_C;
+  c->sigma = cfg->sigma;
+  c->out_scale = cfg->out_scale;
+  c->seed = cfg->seed;
+  c->step = cfg->step;
+  c->norm_mode = cfg->norm_mode;
+  c->audit_capacity = cfg->audit_capacity;
+  c->stream = static_cast<cudaStream_t>(stream);
+}
+
+dp_status check_device() {
+  int dev = 0;
+  DP_CUDA(cudaGetDevice(&dev));
+  int major = 0, minor = 0;
+  DP_CUDA(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev));
+  DP_CUDA(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev));
+  if (major != 10 || minor != 3)
+    return fail(DP_ERR_UNSUPPORTED, "device %d is sm_%d%d; this library is built for sm_103a",
+                dev, major, minor);
+  return DP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
+  if (!ctx) return fail(DP_ERR_ARG, "ctx is NULL");
+  dp_status st = check_config(cfg);
+  if (st != DP_OK) return st;
+  if (*ctx) {
+    dp_ctx* c = *ctx;
+    bool same = c->B == cfg->B && c->T == cfg->T && c->L == cfg->n_layers &&
+                c->dtype == cfg->dtype;
+    for (int l = 0; same && l < c->L; ++l)
+      same = c->plan[l].d_in == cfg->layers[l].d_in && c->plan[l].d_out == cfg->layers[l].d_out;
+    if (!same) return fail(DP_ERR_SHAPE, "re-key with different shapes; destroy and re-create");
+    // The norm mode may change; the partial buffer must still be large enough.
+    std::vector<LayerPlan> old = c->plan;
+    const int oldNP = c->NP;
+    build_plan(c, cfg);
+    if (c->NP > oldNP) {
+      c->plan = old;
+      c->NP = oldNP;
+      return fail(DP_ERR_SHAPE, "norm_mode change needs more scratch; destroy and re-create");
+    }
+    c->NP = oldNP;  // keep the allocated stride
+    set_scalars(c, cfg, cuda_stream);
+    if (!same_parts(old, c->plan)) {
+      st = upload_plan(c);
+      if (st != DP_OK) return st;
+    }
+    // the sticky flag reports conditions of the current step only
+    DP_CUDA(cudaMemsetAsync(c->d_flag, 0, sizeof(int), c->stream));
+    reset_step(c);
+    return DP_OK;
+  }
+  st = check_device();
+  if (st != DP_OK) return st;
+  dp_ctx* c = new dp_ctx();
+  c->B = cfg->B;
+  c->T = cfg->T;
+  c->L = cfg->n_layers;
+  c->dtype = cfg->dtype;
+  cudaGetDevice(&c->device);
+  set_scalars(c, cfg, cuda_stream);
+  build_plan(c, cfg);
+  st = alloc_scratch(c);
+  if (st != DP_OK) {
+    delete c;
+    return st;
+  }
+  st = upload_plan(c);
+  if (st == DP_OK) {
+    cudaError_t e = cudaMemsetAsync(c->d_flag, 0, sizeof(int), c->stream);
+    if (e != cudaSuccess) st = fail(DP_ERR_CUDA, "cudaMemsetAsync: %s", cudaGetErrorString(e));
+  }
+  if (st != DP_OK) {
+    free_scratch(c);
+    delete c;
+    return st;
+  }
+  reset_step(c);
+  *ctx = c;
+  return DP_OK;
+}
+
+dp_status dp_layer_norms(dp_ctx* c, int32_t layer, const void* A, const void* D) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
+  if (!A || !D) return fail(DP_ERR_ARG, "A or D is NULL");
+  if (!aligned16(A) || !aligned16(D)) return fail(DP_ERR_ARG, "A and D must be 16-byte aligned");
+  if (c->clip_done) return fail(DP_ERR_ORDER, "dp_layer_norms after dp_clip_factors");
+  const LayerPlan& p = c->plan[layer];
+  const dpk::InType it = c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32;
+  const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
+  const int row0 = layer * c->B;
+  cudaError_t e = cudaSuccess;
+  if (p.mode == DP_NORM_RANK1) {
+    e = dpk::launch_norm_rank1(it, A, D, c->B, din, dout, c->d_part, c->NP, row0, c->stream);
+  } else if (p.mode == DP_NORM_GHOST) {
+    e = p.norm_tc ? dpk::tc_launch_ghost(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
+                                         c->stream)
+                  : dpk::launch_norm_ghost_simt(it, A, D, c->B, c->T, din, dout, c->d_part,
+                                                c->NP, row0, c->stream);
+  } else {
+    e = p.norm_tc ? dpk::tc_launch_mat_norm(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
+                                            c->stream)
+                  : dpk::launch_norm_mat_simt(it, A, D, c->B, c->T, din, dout, c->d_part, c->NP,
+                                              row0, c->stream);
+  }
+  if (e != cudaSuccess) return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
+  c->norm_done[layer] = 1;
+  return DP_OK;
+}
+
+dp_status dp_clip_factors(dp_ctx* c, float* d_sqnorm_out, float* d_clip_out) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  for (int l = 0; l < c->L; ++l)
+    if (!c->norm_done[l]) return fail(DP_ERR_ORDER, "norms of layer %d not computed", l);
+  if (c->clip_done) return fail(DP_ERR_ORDER, "dp_clip_factors already called this step");
+  cudaError_t e = dpk::launch_clip(c->d_part, c->L, c->B, c->NP, c->d_nparts, c->C,
+                                   c->d_layer_sq, c->d_s, c->d_c, d_sqnorm_out, d_clip_out,
+                                   c->d_flag, c->stream);
+  if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clip kernel launch: %s", cudaGetErrorString(e));
+  c->clip_done = true;
+  return DP_OK;
+}
+
+dp_status dp_clipped_sum_noise(dp_ctx* c, int32_t layer, const void* A, const void* D,
+                               float* d_out, uint32_t flags) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
+  if (flags & ~(DP_NO_NOISE | DP_NOISE_ONLY | DP_ACCUMULATE))
+    return fail(DP_ERR_ARG, "unknown flag bits 0x%x", flags);
+  if ((flags & DP_NO_NOISE) && (flags & DP_NOISE_ONLY))
+    return fail(DP_ERR_ARG, "DP_NO_NOISE and DP_NOISE_ONLY are exclusive");
+  if (!d_out) return fail(DP_ERR_ARG, "d_out is NULL");
+  if (!aligned16(d_out)) return fail(DP_ERR_ARG, "d_out must be 16-byte aligned");
+  const LayerPlan& p = c->plan[layer];
+  const float sigmaC = c->sigma * c->C;
+  if (flags & DP_NOISE_ONLY) {
+    cudaError_t e = dpk::launch_noise_add(d_out, p.d_in * p.d_out, p.p_base, c->seed, c->step,
+                                          c->out_scale * sigmaC, c->stream);
+    if (e != cudaSuccess) return fail(DP_ERR_CUDA, "noise kernel: %s", cudaGetErrorString(e));
+    return DP_OK;
+  }
+  if (!A || !D) return fail(DP_ERR_ARG, "A or D is NULL");
+  if (!aligned16(A) || !aligned16(D)) return fail(DP_ERR_ARG, "A and D must be 16-byte aligned");
+  if (!c->clip_done) return fail(DP_ERR_ORDER, "dp_clipped_sum_noise before dp_clip_factors");
+  dpk::Epilogue ep{};
+  ep.seed = c->seed;
+  ep.step = c->step;
+  ep.p_base = p.p_base;
+  ep.out_scale = c->out_scale;
+  ep.sigmaC = sigmaC;
+  ep.add_noise = (flags & DP_NO_NOISE) ? 0 : 1;
+  ep.accumulate = (flags & DP_ACCUMULATE) ? 1 : 0;
+  const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
+  cudaError_t e;
+  if (p.gemm_tc)
+    e = dpk::tc_launch_clipsum(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep, c->stream);
+  else
+    e = dpk::launch_gemm_simt(c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, A, D, c->d_c,
+                              c->B, c->T, din, dout, d_out, ep, c->stream);
+  if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clipped-sum kernel: %s", cudaGetErrorString(e));
+  return DP_OK;
+}
+
+dp_status dp_audit_emit(dp_ctx* c, const int32_t* h_idx, int32_t n, void* h_records) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (n < 0 || n > c->audit_capacity)
+    return fail(DP_ERR_ARG, "n=%d outside 0..audit_capacity=%d", n, c->audit_capacity);
+  if (n > 0 && (!h_idx || !h_records)) return fail(DP_ERR_ARG, "h_idx or h_records is NULL");
+  if (!c->clip_done) return fail(DP_ERR_ORDER, "dp_audit_emit before dp_clip_factors");
+  for (int r = 0; r < n; ++r)
+    if (h_idx[r] < 0 || h_idx[r] >= c->B)
+      return fail(DP_ERR_ARG, "audit index %d out of range 0..%d", h_idx[r], c->B - 1);
+  // Staging buffers are reused by every call: wait for the previous user.
+  DP_CUDA(cudaStreamSynchronize(c->stream));
+  const size_t rec_words = static_cast<size_t>(3 + c->L);
+  if (n > 0) {
+    std::memcpy(c->h_idx, h_idx, sizeof(int) * n);
+    DP_CUDA(cudaMemcpyAsync(c->d_idx, c->h_idx, sizeof(int) * n, cudaMemcpyHostToDevice,
+                            c->stream));
+    DP_CUDA(dpk::launch_audit(c->d_idx, n, c->L, c->B, c->d_layer_sq, c->d_s, c->d_c, c->d_rec,
+                              c->stream));
+    DP_CUDA(cudaMemcpyAsync(c->h_rec, c->d_rec, sizeof(float) * rec_words * n,
+                            cudaMemcpyDeviceToHost, c->stream));
+  }
+  DP_CUDA(cudaMemcpyAsync(c->h_flag, c->d_flag, sizeof(int), cudaMemcpyDeviceToHost, c->stream));
+  DP_CUDA(cudaStreamSynchronize(c->stream));
+  if (n > 0) std::memcpy(h_records, c->h_rec, sizeof(float) * rec_words * n);
+  if (*c->h_flag) return fail(DP_ERR_NONFINITE, "a per-example squared norm was not finite");
+  return DP_OK;
+}
+
+int64_t dp_audit_record_bytes(int32_t n_layers) { return 12 + 4 * static_cast<int64_t>(n_layers); }
+
+dp_status dp_layer_norm_mode(const dp_ctx* c, int32_t layer, dp_norm_mode* mode_out) {
+  if (!c || !mode_out) return fail(DP_ERR_ARG, "NULL argument");
+  if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
+  *mode_out = c->plan[layer].mode;
+  return DP_OK;
+}
+
+void dp_step_destroy(dp_ctx* c) {
+  if (!c) return;
+  cudaStreamSynchronize(c->stream);
+  free_scratch(c);
+  delete c;
+}
+
+const char* dp_last_error(void) { return g_err.c_str(); }
+
+const char* dp_status_string(dp_status s) {
+  switch (s) {
+    case DP_OK: return "DP_OK";
+    case DP_ERR_ARG: return "DP_ERR_ARG";
+    case DP_ERR_SHAPE: return "DP_ERR_SHAPE";
+    case DP_ERR_DTYPE: return "DP_ERR_DTYPE";
+    case DP_ERR_ORDER: return "DP_ERR_ORDER";
+    case DP_ERR_NONFINITE: return "DP_ERR_NONFINITE";
+    case DP_ERR_CUDA: return "DP_ERR_CUDA";
+    case DP_ERR_TIMEOUT: return "DP_ERR_TIMEOUT";
+    case DP_ERR_OOM: return "DP_ERR_OOM";
+    case DP_ERR_UNSUPPORTED: return "DP_ERR_UNSUPPORTED";
+  }
+  return "DP_ERR_UNKNOWN";
+}
+
+dp_status dp_debug_philox(uint64_t seed, uint64_t step, uint64_t first_quad, int64_t n_quads,
+                          uint32_t* d_out, void* stream) {
+  if (n_quads < 0) return fail(DP_ERR_ARG, "n_quads < 0");
+  if (n_quads > 0 && !d_out) return fail(DP_ERR_ARG, "d_out is NULL");
+  DP_CUDA(dpk::launch_debug_philox(seed, step, first_quad, n_quads, d_out,
+                                   static_cast<cudaStream_t>(stream)));
+  return DP_OK;
+}
+
+dp_status dp_debug_gaussian(uint64_t seed, uint64_t step, uint64_t first_index, int64_t n,
+                            float* d_out, void* stream) {
+  if (n < 0) return fail(DP_ERR_ARG, "n < 0");
+  if (n > 0 && !d_out) return fail(DP_ERR_ARG, "d_out is NULL");
+  DP_CUDA(dpk::launch_debug_gauss(seed, step, first_index, n, d_out,
+                                  static_cast<cudaStream_t>(stream)));
+  return DP_OK;
+}
+
+}  // extern "C"

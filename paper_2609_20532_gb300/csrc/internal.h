@@ -1,0 +1,57 @@
+// Launchers shared between the C-ABI layer (dp_step.cu) and the kernel files.
+#pragma once
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace dpk {
+
+enum InType { IN_F32 = 0, IN_BF16 = 1 };
+
+// How the output tile of a clipped-sum kernel is written.
+struct Epilogue {
+  uint64_t seed;
+  uint64_t step;
+  uint64_t p_base;     // global index of element (0, 0) of this layer
+  float out_scale;     // applied to (S + sigmaC * z)
+  float sigmaC;        // sigma * C
+  int add_noise;       // 0: out_scale * S
+  int accumulate;      // 1: out += value
+};
+
+// ---- per-example squared norms: partial sums into part[(row) * NP + p] ----
+// row = layer * B + example; every kernel writes exactly nparts(...) entries.
+int rank1_parts();
+int ghost_simt_parts(int T);
+int mat_simt_parts(int d_in, int d_out);
+
+cudaError_t launch_norm_rank1(InType t, const void* A, const void* D, int B, int d_in, int d_out,
+                              float* part, int NP, int row0, cudaStream_t s);
+cudaError_t launch_norm_ghost_simt(InType t, const void* A, const void* D, int B, int T, int d_in,
+                                   int d_out, float* part, int NP, int row0, cudaStream_t s);
+cudaError_t launch_norm_mat_simt(InType t, const void* A, const void* D, int B, int T, int d_in,
+                                 int d_out, float* part, int NP, int row0, cudaStream_t s);
+
+// ---- cross-layer sum and clip factors ----
+cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_nparts, float C,
+                        float* layer_sq, float* s_out, float* c_out, float* user_s, float* user_c,
+                        int* flag, cudaStream_t s);
+
+// ---- clipped sum + noise (CUDA-core FFMA path) ----
+cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float* c, int B, int T,
+                             int d_in, int d_out, float* out, const Epilogue& ep, cudaStream_t s);
+
+// ---- standalone noise add: out[e] += scale * z_{p_base + e}, e < n ----
+cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, uint64_t seed, uint64_t step,
+                             float scale, cudaStream_t s);
+
+// ---- audit gather ----
+cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer_sq,
+                         const float* s_vec, const float* c_vec, float* rec, cudaStream_t s);
+
+// ---- generator exports for tests ----
+cudaError_t launch_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
+                                uint32_t* out, cudaStream_t s);
+cudaError_t launch_debug_gauss(uint64_t seed, uint64_t step, uint64_t p0, int64_t n, float* out,
+                               cudaStream_t s);
+
+}  // namespace dpk

@@ -1,0 +1,458 @@
+// CUDA-core kernels of the DP-SGD step: per-example norms (rank-1, Gram and
+// materialised forms), the cross-layer clip-factor kernel, the fp32 clipped
+// sum with its fused noise epilogue, the standalone noise add, the audit
+// gather and the generator exports.
+//
+// The clipped sum here is the fp32 path (an FFMA GEMM, exact in the inputs'
+// precision); bf16 layers whose T is a multiple of the tensor-core K-block
+// go through the tcgen05 kernels instead.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "internal.h"
+#include "philox.cuh"
+
+namespace dpk {
+
+namespace {
+
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+// Sum of v over the block (blockDim.x a multiple of 32, <= 1024); result in
+// every thread.  Fixed reduction order, so results are reproducible.
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  __syncthreads();
+  if (lane == 0) red[w] = v;
+  __syncthreads();
+  const int nw = blockDim.x >> 5;
+  float t = lane < nw ? red[lane] : 0.f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+  return t;
+}
+
+// ---------------------------------------------------------------------------
+// Rank-1 norm (T = 1): n_i = ||a_i||^2 ||d_i||^2
+// ---------------------------------------------------------------------------
+template <typename TIn>
+__global__ void __launch_bounds__(256) k_norm_rank1(const TIn* __restrict__ A,
+                                                    const TIn* __restrict__ D, int d_in, int d_out,
+                                                    float* __restrict__ part, int NP, int row0) {
+  __shared__ float red[32];
+  const int i = blockIdx.x;
+  const TIn* a = A + static_cast<int64_t>(i) * d_in;
+  const TIn* d = D + static_cast<int64_t>(i) * d_out;
+  float sa = 0.f, sd = 0.f;
+  for (int j = threadIdx.x; j < d_in; j += blockDim.x) {
+    const float v = to_f(a[j]);
+    sa = fmaf(v, v, sa);
+  }
+  for (int k = threadIdx.x; k < d_out; k += blockDim.x) {
+    const float v = to_f(d[k]);
+    sd = fmaf(v, v, sd);
+  }
+  sa = block_sum(sa, red);
+  sd = block_sum(sd, red);
+  if (threadIdx.x == 0) part[static_cast<int64_t>(row0 + i) * NP] = sa * sd;
+}
+
+// ---------------------------------------------------------------------------
+// Gram ("ghost") norm: n_i = sum_{t,s} (a_t . a_s)(d_t . d_s).
+// One block per (example, 64x64 tile pair (bt <= bs) of the T x T Grams);
+// off-diagonal tiles count twice, the upper and lower halves being equal.
+// ---------------------------------------------------------------------------
+constexpr int GT = 64;   // Gram tile edge
+constexpr int GF = 32;   // features per staged chunk
+
+__device__ __forceinline__ void pair_of(int pid, int nb, int& bt, int& bs) {
+  // enumerate (bt, bs), bt <= bs, row by row
+  int r = 0, left = pid;
+  while (left >= nb - r) {
+    left -= nb - r;
+    ++r;
+  }
+  bt = r;
+  bs = r + left;
+}
+
+template <typename TIn>
+__device__ __forceinline__ void gram_tile(const TIn* __restrict__ X, int T, int d, int t0, int s0,
+                                          float (&g)[4][4], float (*Xt)[GT + 4],
+                                          float (*Xs)[GT + 4]) {
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  for (int f0 = 0; f0 < d; f0 += GF) {
+#pragma unroll
+    for (int r = 0; r < (GT * GF) / 256; ++r) {
+      const int e = tid + 256 * r;
+      const int row = e / GF, f = e % GF;
+      const int t = t0 + row, s = s0 + row, ff = f0 + f;
+      Xt[f][row] = (t < T && ff < d) ? to_f(X[static_cast<int64_t>(t) * d + ff]) : 0.f;
+      Xs[f][row] = (s < T && ff < d) ? to_f(X[static_cast<int64_t>(s) * d + ff]) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 8
+    for (int f = 0; f < GF; ++f) {
+      const float4 a = *reinterpret_cast<const float4*>(&Xt[f][ty * 4]);
+      const float4 b = *reinterpret_cast<const float4*>(&Xs[f][tx * 4]);
+      const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) g[u][v] = fmaf(av[u], bv[v], g[u][v]);
+    }
+    __syncthreads();
+  }
+}
+
+template <typename TIn>
+__global__ void __launch_bounds__(256) k_norm_ghost_simt(const TIn* __restrict__ A,
+                                                         const TIn* __restrict__ D, int T, int d_in,
+                                                         int d_out, float* __restrict__ part,
+                                                         int NP, int row0) {
+  __shared__ __align__(16) float Xt[GF][GT + 4];
+  __shared__ __align__(16) float Xs[GF][GT + 4];
+  __shared__ float red[32];
+  const int nb = (T + GT - 1) / GT;
+  int bt, bs;
+  pair_of(blockIdx.x, nb, bt, bs);
+  const int i = blockIdx.y;
+  const int t0 = bt * GT, s0 = bs * GT;
+  float ga[4][4] = {}, gd[4][4] = {};
+  gram_tile(A + static_cast<int64_t>(i) * T * d_in, T, d_in, t0, s0, ga, Xt, Xs);
+  gram_tile(D + static_cast<int64_t>(i) * T * d_out, T, d_out, t0, s0, gd, Xt, Xs);
+  float acc = 0.f;
+#pragma unroll
+  for (int u = 0; u < 4; ++u)
+#pragma unroll
+    for (int v = 0; v < 4; ++v) acc = fmaf(ga[u][v], gd[u][v], acc);
+  acc = block_sum(acc, red);
+  if (threadIdx.x == 0)
+    part[static_cast<int64_t>(row0 + i) * NP + blockIdx.x] = (bt == bs ? 1.f : 2.f) * acc;
+}
+
+// ---------------------------------------------------------------------------
+// FFMA GEMM over positions: tile 128 (d_in) x 128 (d_out), K-chunks of 16.
+// CLIPSUM: S = sum_k c[k / T] A[k, :]^T D[k, :] over all B*T rows, + epilogue.
+// NORM:    per example (blockIdx.z), G tile = A_i^T D_i, writes sum of squares.
+// ---------------------------------------------------------------------------
+constexpr int SB = 128, SK = 16;
+
+template <typename TIn, bool NORM>
+__global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
+                                                   const TIn* __restrict__ D,
+                                                   const float* __restrict__ cvec, int T, int B,
+                                                   int d_in, int d_out, float* __restrict__ out,
+                                                   Epilogue ep, float* __restrict__ part, int NP,
+                                                   int row0) {
+  __shared__ __align__(16) float As[SK][SB];
+  __shared__ __align__(16) float Ds[SK][SB];
+  __shared__ float red[32];
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const int j0 = blockIdx.y * SB, k0 = blockIdx.x * SB;
+  int64_t K;
+  if (NORM) {
+    const int64_t i = blockIdx.z;
+    A += i * T * d_in;
+    D += i * T * d_out;
+    K = T;
+  } else {
+    K = static_cast<int64_t>(B) * T;
+  }
+  float acc[8][8] = {};
+  for (int64_t kk = 0; kk < K; kk += SK) {
+#pragma unroll
+    for (int r = 0; r < (SK * SB) / 256; ++r) {
+      const int e = tid + 256 * r;
+      const int row = e / SB, col = e % SB;
+      const int64_t kr = kk + row;
+      const int j = j0 + col, k = k0 + col;
+      float va = 0.f, vd = 0.f;
+      if (kr < K) {
+        if (j < d_in) {
+          va = to_f(A[kr * d_in + j]);
+          if (!NORM) va *= cvec[kr / T];
+        }
+        if (k < d_out) vd = to_f(D[kr * d_out + k]);
+      }
+      As[row][col] = va;
+      Ds[row][col] = vd;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < SK; ++q) {
+      const float4 a0 = *reinterpret_cast<const float4*>(&As[q][ty * 4]);
+      const float4 a1 = *reinterpret_cast<const float4*>(&As[q][64 + ty * 4]);
+      const float4 b0 = *reinterpret_cast<const float4*>(&Ds[q][tx * 4]);
+      const float4 b1 = *reinterpret_cast<const float4*>(&Ds[q][64 + tx * 4]);
+      const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+#pragma unroll
+        for (int v = 0; v < 8; ++v) acc[u][v] = fmaf(av[u], bv[v], acc[u][v]);
+    }
+    __syncthreads();
+  }
+
+  if constexpr (NORM) {
+    float sq = 0.f;
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+#pragma unroll
+      for (int v = 0; v < 8; ++v) sq = fmaf(acc[u][v], acc[u][v], sq);  // padding is zero
+    sq = block_sum(sq, red);
+    if (tid == 0) {
+      const int tile = blockIdx.y * gridDim.x + blockIdx.x;
+      part[static_cast<int64_t>(row0 + blockIdx.z) * NP + tile] = sq;
+    }
+  } else {
+#pragma unroll
+  for (int u = 0; u < 8; ++u) {
+    const int j = j0 + (u < 4 ? ty * 4 + u : 64 + ty * 4 + (u - 4));
+    if (j >= d_in) continue;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int kb = k0 + h * 64 + tx * 4;
+      if (kb >= d_out) continue;
+      float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+      const uint64_t p0 = ep.p_base + static_cast<uint64_t>(j) * d_out + kb;
+      if (ep.add_noise) z = gauss4_at(ep.seed, ep.step, p0);
+      const float zv[4] = {z.x, z.y, z.z, z.w};
+      float* o = out + static_cast<int64_t>(j) * d_out;
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        const int k = kb + v;
+        if (k < d_out) {
+          const float val = ep.out_scale * fmaf(ep.sigmaC, zv[v], acc[u][h * 4 + v]);
+          o[k] = ep.accumulate ? o[k] + val : val;
+        }
+      }
+    }
+  }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Cross-layer sum and clip factors (one thread per example, fixed order)
+// ---------------------------------------------------------------------------
+__global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
+                       const int* __restrict__ nparts, float C, float* __restrict__ layer_sq,
+                       float* __restrict__ s_out, float* __restrict__ c_out,
+                       float* __restrict__ user_s, float* __restrict__ user_c, int* flag) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B) return;
+  float s = 0.f;
+  for (int l = 0; l < L; ++l) {
+    const float* p = part + static_cast<int64_t>(l * B + i) * NP;
+    float n = 0.f;
+    const int np = nparts[l];
+    for (int q = 0; q < np; ++q) n += p[q];
+    layer_sq[l * B + i] = n;
+    s += n;
+  }
+  float c;
+  if (!isfinite(s)) {
+    atomicOr(flag, 1);
+    c = __int_as_float(0x7fc00000);  // NaN
+  } else {
+    c = (s <= C * C) ? 1.f : C / sqrtf(s);
+  }
+  s_out[i] = s;
+  c_out[i] = c;
+  if (user_s) user_s[i] = s;
+  if (user_c) user_c[i] = c;
+}
+
+// ---------------------------------------------------------------------------
+// Standalone noise add: out[e] += scale * z_{p_base + e}
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_noise_add(float* __restrict__ out, int64_t n,
+                                                   uint64_t p_base, uint64_t seed, uint64_t step,
+                                                   float scale) {
+  // quads that overlap [p_base, p_base + n)
+  const uint64_t q_first = p_base >> 2;
+  const uint64_t q_last = (p_base + n - 1) >> 2;
+  const int64_t nq = static_cast<int64_t>(q_last - q_first + 1);
+  const bool vec = ((p_base & 3) == 0) && ((reinterpret_cast<uintptr_t>(out) & 15) == 0);
+  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < nq;
+       g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const uint64_t q = q_first + g;
+    const float4 z = gauss_quad(seed, step, q);
+    const int64_t e0 = static_cast<int64_t>(4 * q) - static_cast<int64_t>(p_base);
+    if (vec && e0 + 3 < n) {
+      float4* o = reinterpret_cast<float4*>(out + e0);
+      float4 v = *o;
+      v.x = fmaf(scale, z.x, v.x);
+      v.y = fmaf(scale, z.y, v.y);
+      v.z = fmaf(scale, z.z, v.z);
+      v.w = fmaf(scale, z.w, v.w);
+      *o = v;
+    } else {
+      const float zv[4] = {z.x, z.y, z.z, z.w};
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const int64_t e = e0 + w;
+        if (e >= 0 && e < n) out[e] = fmaf(scale, zv[w], out[e]);
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Audit gather: rec[r] = {idx, s, c, n_1..n_L}
+// ---------------------------------------------------------------------------
+__global__ void k_audit(const int* __restrict__ idx, int n, int L, int B,
+                        const float* __restrict__ layer_sq, const float* __restrict__ s_vec,
+                        const float* __restrict__ c_vec, float* __restrict__ rec) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= n) return;
+  const int i = idx[r];
+  float* o = rec + static_cast<int64_t>(r) * (3 + L);
+  reinterpret_cast<int*>(o)[0] = i;
+  o[1] = s_vec[i];
+  o[2] = c_vec[i];
+  for (int l = 0; l < L; ++l) o[3 + l] = layer_sq[l * B + i];
+}
+
+__global__ void k_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
+                               uint32_t* __restrict__ out) {
+  for (int64_t r = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; r < nq;
+       r += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const uint64_t q = q0 + r;
+    const uint4 w = philox4x32_10(
+        make_uint4(static_cast<uint32_t>(q), static_cast<uint32_t>(q >> 32),
+                   static_cast<uint32_t>(step), static_cast<uint32_t>(step >> 32)),
+        static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
+    out[4 * r + 0] = w.x;
+    out[4 * r + 1] = w.y;
+    out[4 * r + 2] = w.z;
+    out[4 * r + 3] = w.w;
+  }
+}
+
+__global__ void k_debug_gauss(uint64_t seed, uint64_t step, uint64_t p0, int64_t n,
+                              float* __restrict__ out) {
+  for (int64_t r = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; r < n;
+       r += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const uint64_t p = p0 + r;
+    const float4 z = gauss_quad(seed, step, p >> 2);
+    const float zv[4] = {z.x, z.y, z.z, z.w};
+    out[r] = zv[p & 3];
+  }
+}
+
+int grid_for(int64_t work, int threads) {
+  const int64_t g = (work + threads - 1) / threads;
+  const int64_t cap = 152 * 16;
+  return static_cast<int>(g < 1 ? 1 : (g > cap ? cap : g));
+}
+
+}  // namespace
+
+int rank1_parts() { return 1; }
+int ghost_simt_parts(int T) {
+  const int nb = (T + GT - 1) / GT;
+  return nb * (nb + 1) / 2;
+}
+int mat_simt_parts(int d_in, int d_out) {
+  return ((d_in + SB - 1) / SB) * ((d_out + SB - 1) / SB);
+}
+
+cudaError_t launch_norm_rank1(InType t, const void* A, const void* D, int B, int d_in, int d_out,
+                              float* part, int NP, int row0, cudaStream_t s) {
+  if (t == IN_F32)
+    k_norm_rank1<float><<<B, 256, 0, s>>>(static_cast<const float*>(A),
+                                           static_cast<const float*>(D), d_in, d_out, part, NP,
+                                           row0);
+  else
+    k_norm_rank1<__nv_bfloat16><<<B, 256, 0, s>>>(static_cast<const __nv_bfloat16*>(A),
+                                                   static_cast<const __nv_bfloat16*>(D), d_in,
+                                                   d_out, part, NP, row0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_norm_ghost_simt(InType t, const void* A, const void* D, int B, int T, int d_in,
+                                   int d_out, float* part, int NP, int row0, cudaStream_t s) {
+  const dim3 grid(ghost_simt_parts(T), B);
+  if (t == IN_F32)
+    k_norm_ghost_simt<float><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
+                                                   static_cast<const float*>(D), T, d_in, d_out,
+                                                   part, NP, row0);
+  else
+    k_norm_ghost_simt<__nv_bfloat16><<<grid, 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(A), static_cast<const __nv_bfloat16*>(D), T, d_in,
+        d_out, part, NP, row0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_norm_mat_simt(InType t, const void* A, const void* D, int B, int T, int d_in,
+                                 int d_out, float* part, int NP, int row0, cudaStream_t s) {
+  const dim3 grid((d_out + SB - 1) / SB, (d_in + SB - 1) / SB, B);
+  Epilogue ep{};
+  if (t == IN_F32)
+    k_gemm_simt<float, true><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
+                                                   static_cast<const float*>(D), nullptr, T, B,
+                                                   d_in, d_out, nullptr, ep, part, NP, row0);
+  else
+    k_gemm_simt<__nv_bfloat16, true><<<grid, 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(A), static_cast<const __nv_bfloat16*>(D), nullptr, T,
+        B, d_in, d_out, nullptr, ep, part, NP, row0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_nparts, float C,
+                        float* layer_sq, float* s_out, float* c_out, float* user_s, float* user_c,
+                        int* flag, cudaStream_t s) {
+  k_clip<<<(B + 127) / 128, 128, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out,
+                                         user_s, user_c, flag);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float* c, int B, int T,
+                             int d_in, int d_out, float* out, const Epilogue& ep, cudaStream_t s) {
+  const dim3 grid((d_out + SB - 1) / SB, (d_in + SB - 1) / SB, 1);
+  if (t == IN_F32)
+    k_gemm_simt<float, false><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
+                                                    static_cast<const float*>(D), c, T, B, d_in,
+                                                    d_out, out, ep, nullptr, 0, 0);
+  else
+    k_gemm_simt<__nv_bfloat16, false><<<grid, 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(A), static_cast<const __nv_bfloat16*>(D), c, T, B,
+        d_in, d_out, out, ep, nullptr, 0, 0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, uint64_t seed, uint64_t step,
+                             float scale, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int64_t nq = static_cast<int64_t>(((p_base + n - 1) >> 2) - (p_base >> 2) + 1);
+  k_noise_add<<<grid_for(nq, 256), 256, 0, s>>>(out, n, p_base, seed, step, scale);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer_sq,
+                         const float* s_vec, const float* c_vec, float* rec, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  k_audit<<<(n + 127) / 128, 128, 0, s>>>(idx, n, L, B, layer_sq, s_vec, c_vec, rec);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
+                                uint32_t* out, cudaStream_t s) {
+  if (nq <= 0) return cudaSuccess;
+  k_debug_philox<<<grid_for(nq, 256), 256, 0, s>>>(seed, step, q0, nq, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_debug_gauss(uint64_t seed, uint64_t step, uint64_t p0, int64_t n, float* out,
+                               cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  k_debug_gauss<<<grid_for(n, 256), 256, 0, s>>>(seed, step, p0, n, out);
+  return cudaGetLastError();
+}
+
+}  // namespace dpk

@@ -1,0 +1,89 @@
+"""Helpers shared by the GPU tests: run one step through the C ABI and compare
+it with the fp64 oracle on the same stored input bits."""
+
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+import paper_2609_20532_gb300 as dp
+import workloads as W
+from oracle import dp_oracle as O
+
+TOL = {"f32": 1e-5, "bf16": 2e-3}
+
+
+def f32(x: float) -> float:
+    """The fp32 value the library receives for a config scalar."""
+    return float(np.float32(x))
+
+
+def run_gpu_step(w: W.Workload, layers, seed=0, step=0, out_scale=1.0, flags=0,
+                 norm_mode=dp.DP_NORM_AUTO, audit=True):
+    """Run norms -> clip -> clipped sum (+noise) on cuda:0.
+
+    layers: list of (A, D) CPU tensors.  Returns dict with n [L,B], s, c
+    (from the audit records of every example), out (list of fp32 numpy) and
+    the chosen norm modes."""
+    dev = torch.device("cuda:0")
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    outs = [torch.zeros(i, o, device=dev, dtype=torch.float32) for i, o in w.layers]
+    s_dev = torch.empty(w.B, device=dev)
+    c_dev = torch.empty(w.B, device=dev)
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=out_scale,
+                         seed=seed, step=step, norm_mode=norm_mode, audit_capacity=w.B)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        for l in range(len(layers)):
+            dp.dp_layer_norms(ctx, l, Ad[l], Dd[l])
+        dp.dp_clip_factors(ctx, s_dev, c_dev)
+        for l in range(len(layers)):
+            dp.dp_clipped_sum_noise(ctx, l, Ad[l], Dd[l], outs[l], flags)
+        recs = dp.dp_audit_emit(ctx, range(w.B), len(layers)) if audit else None
+        modes = [dp.dp_layer_norm_mode(ctx, l) for l in range(len(layers))]
+    finally:
+        dp.dp_step_destroy(ctx)
+    torch.cuda.synchronize()
+    res = {"out": [o.cpu().numpy() for o in outs], "s": s_dev.cpu().numpy(),
+           "c": c_dev.cpu().numpy(), "modes": modes}
+    if recs is not None:
+        res["n"] = np.stack([r["layer_sqnorm"] for r in recs], axis=1)
+        res["rec_s"] = np.array([r["total_sqnorm"] for r in recs])
+        res["rec_c"] = np.array([r["clip_factor"] for r in recs])
+        res["rec_i"] = np.array([r["example"] for r in recs])
+    return res
+
+
+def rel_err_elementwise(got, ref):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    return float(np.max(np.abs(got - ref) / np.maximum(np.abs(ref), 1e-30)))
+
+
+def rel_err_normwise(got, ref):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    den = np.linalg.norm(ref)
+    return float(np.linalg.norm(got - ref) / den) if den > 0 else float(np.linalg.norm(got))
+
+
+def assert_step_matches(res, ref, dtype: str, what=("n", "s", "c", "out")):
+    tol = TOL[dtype]
+    if "n" in what:
+        e = rel_err_elementwise(res["n"], ref["n"])
+        assert e <= tol, f"per-layer norms rel err {e:.3e} > {tol}"
+    if "s" in what:
+        e = rel_err_elementwise(res["s"], ref["s"])
+        assert e <= tol, f"s rel err {e:.3e}"
+        assert np.array_equal(res["rec_s"].astype(np.float32), res["s"].astype(np.float32))
+    if "c" in what:
+        e = rel_err_elementwise(res["c"], ref["c"])
+        assert e <= tol, f"clip factor rel err {e:.3e}"
+        assert np.all(res["c"] <= 1.0) and np.all(res["c"] > 0)
+    if "out" in what:
+        for l, (o, r) in enumerate(zip(res["out"], ref["out"])):
+            e = rel_err_normwise(o, r)
+            assert e <= tol, f"layer {l} output normwise rel err {e:.3e} > {tol}"

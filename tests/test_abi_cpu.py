@@ -1,0 +1,97 @@
+"""C-ABI checks that need no GPU: the library loads, exports every symbol the
+header declares, and rejects bad arguments on the host before touching the
+device."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2609_20532_gb300 as dp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "dp_step.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    if not os.path.exists(dp.lib_path):
+        from paper_2609_20532_gb300 import build
+        build.build()
+    return dp.lib()
+
+
+def header_functions():
+    txt = open(HEADER).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"\b(dp_[a-z_0-9]+)\s*\(", txt)))
+
+
+def test_header_and_binding_agree():
+    assert header_functions() == sorted(dp.EXPORTED_SYMBOLS)
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in header_functions():
+        assert hasattr(L, name), name
+
+
+def _cfg(**kw):
+    base = dict(layers=[(64, 32)], B=8, T=1, dtype="f32", C=1.0, sigma=1.0)
+    base.update(kw)
+    return dp.make_config(**base)
+
+
+def _init_status(L, cfg):
+    h = ctypes.c_void_p(None)
+    st = L.dp_step_init(ctypes.byref(h), ctypes.byref(cfg) if cfg is not None else None, None)
+    return st, h.value
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(B=0), 2), (dict(T=0), 2), (dict(layers=[(0, 4)]), 2),
+    (dict(layers=[(1 << 21, 4)]), 2), (dict(dtype="bf16", layers=[(12, 8)]), 2),
+    (dict(C=0.0), 1), (dict(C=float("inf")), 1), (dict(sigma=-1.0), 1),
+    (dict(sigma=float("nan")), 1), (dict(out_scale=float("inf")), 1),
+    (dict(norm_mode=7), 1), (dict(norm_mode=dp.DP_NORM_RANK1, T=4), 2),
+    (dict(audit_capacity=9), 1), (dict(audit_capacity=-1), 1),
+])
+def test_init_rejects_bad_config_on_host(L, kw, status):
+    st, h = _init_status(L, _cfg(**kw))
+    assert st == status, dp.dp_last_error()
+    assert h is None
+    assert dp.dp_last_error()
+
+
+def test_init_rejects_null_and_bad_dtype(L):
+    st, _ = _init_status(L, None)
+    assert st == 1
+    cfg = _cfg()
+    cfg.dtype = 5
+    st, _ = _init_status(L, cfg)
+    assert st == 3
+    cfg = _cfg()
+    cfg.n_layers = 0
+    st, _ = _init_status(L, cfg)
+    assert st == 2
+    assert L.dp_step_init(None, ctypes.byref(_cfg()), None) == 1
+
+
+def test_calls_reject_null_context(L):
+    assert L.dp_layer_norms(None, 0, 16, 16) == 1
+    assert L.dp_clip_factors(None, None, None) == 1
+    assert L.dp_clipped_sum_noise(None, 0, 16, 16, 16, 0) == 1
+    assert L.dp_audit_emit(None, None, 0, None) == 1
+    m = ctypes.c_int32()
+    assert L.dp_layer_norm_mode(None, 0, ctypes.byref(m)) == 1
+    L.dp_step_destroy(None)  # no-op
+
+
+def test_misc_exports(L):
+    assert L.dp_audit_record_bytes(3) == 24
+    assert L.dp_status_string(5) == b"DP_ERR_NONFINITE"
+    assert L.dp_debug_philox(0, 0, 0, -1, None, None) == 1
+    assert L.dp_debug_gaussian(0, 0, 0, -1, None, None) == 1
+    # zero-length requests launch nothing
+    assert L.dp_debug_philox(0, 0, 0, 0, None, None) == 0

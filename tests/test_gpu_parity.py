@@ -1,0 +1,325 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle.
+
+Tolerances: Philox words bit-exact; Gaussian numbers within 1e-6 relative
+elementwise; per-example norms, s_i and c_i within 2e-3 (bf16 inputs) or
+1e-5 (fp32 inputs) relative elementwise; clipped sums and noisy outputs
+within the same bounds normwise per layer.
+"""
+
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_20532_gb300 as dp
+import workloads as W
+from oracle import dp_oracle as O
+
+from gpu_harness import (TOL, assert_step_matches, f32, rel_err_elementwise, rel_err_normwise,
+                         run_gpu_step)
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _gpu():
+    if not torch.cuda.is_available():
+        pytest.fail("CUDA GPU required for -m gpu tests")
+    dp.lib()  # fails loudly if the library was not built
+
+
+def oracle_step(w, layers, seed=0, step=0, out_scale=1.0, noise=True, norm="materialised"):
+    return O.dp_step([(W.to_f64(A), W.to_f64(D)) for A, D in layers], f32(w.C), f32(w.sigma),
+                     seed, step, out_scale=f32(out_scale), noise=noise, norm=norm)
+
+
+# ---------------------------------------------------------------------------
+# generator
+# ---------------------------------------------------------------------------
+
+M64 = (1 << 64) - 1
+
+
+@pytest.mark.parametrize("seed,step,q0,n", [
+    (0, 0, 0, 1 << 22),
+    (0x123456789ABCDEF0, 7, (1 << 32) - 1000, 1 << 16),     # crosses the 32-bit counter carry
+    (M64, M64, M64 - 4095, 4096),                             # wraps the 64-bit quad counter
+    (1, 1 << 32, 35_000_000, 1 << 16),
+])
+def test_philox_words_bit_exact(seed, step, q0, n):
+    out = torch.empty(4 * n, dtype=torch.int32, device=DEV)
+    dp.dp_debug_philox(seed, step, q0, n, out)
+    got = out.cpu().numpy().view(np.uint32).reshape(n, 4)
+    if q0 + n - 1 > M64:  # the oracle's quad range is defined modulo 2^64
+        ref = np.concatenate([O.philox_quads(seed, step, q0, M64 - q0 + 1),
+                              O.philox_quads(seed, step, 0, q0 + n - 1 - M64)])
+    else:
+        ref = O.philox_quads(seed, step, q0, n)
+    assert np.array_equal(got, ref)
+
+
+@pytest.mark.parametrize("seed,step,p0,n", [
+    (0, 0, 0, 1 << 22), (5, 9, 3, 100_003), (M64, 2, (1 << 34) + 1, 1 << 16)])
+def test_gaussian_within_1e6(seed, step, p0, n):
+    out = torch.empty(n, dtype=torch.float32, device=DEV)
+    dp.dp_debug_gaussian(seed, step, p0, n, out)
+    got = out.cpu().numpy().astype(np.float64)
+    ref = O.gaussian_noise(seed, step, p0, n)
+    e = rel_err_elementwise(got, ref)
+    assert e <= 1e-6, e
+
+
+# ---------------------------------------------------------------------------
+# whole-step parity on the workloads
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("name", ["single_fp32", "mlp_fp32", "block_bf16"])
+@pytest.mark.parametrize("out_scale", ["sum", "mean"])
+def test_step_matches_oracle(name, out_scale):
+    w = W.get(name)
+    layers = W.make_inputs(w, seed=0)
+    scale = 1.0 if out_scale == "sum" else 1.0 / w.B
+    res = run_gpu_step(w, layers, seed=0, step=0, out_scale=scale)
+    ref = oracle_step(w, layers, seed=0, step=0, out_scale=scale)
+    assert_step_matches(res, ref, w.dtype)
+    assert np.array_equal(res["rec_i"], np.arange(w.B))
+
+
+@pytest.mark.parametrize("name", ["single_fp32", "mlp_fp32", "block_bf16"])
+def test_commitment_is_noiseless_clipped_sum(name):
+    """DP_NO_NOISE writes the commitment of Algorithm 2: S_l (times out_scale)."""
+    w = W.get(name)
+    layers = W.make_inputs(w, seed=0)
+    res = run_gpu_step(w, layers, flags=dp.DP_NO_NOISE, audit=False)
+    ref = oracle_step(w, layers, noise=False)
+    for l, (o, r) in enumerate(zip(res["out"], ref["out"])):
+        assert rel_err_normwise(o, r) <= TOL[w.dtype], l
+    # the structural check of Sec. 6.2 on the averaged commitment
+    agg = math.sqrt(sum(float(np.sum(o.astype(np.float64) ** 2)) for o in res["out"])) / w.B
+    assert agg <= f32(w.C) * (1 + 1e-4)
+
+
+def _llm_sample_check(w, layers, res, sample_rows=24, seed=0, step=0):
+    """Full-size check at the LLM workload: every per-example norm from the
+    oracle's Gram form (pinned equal to the materialised one), clip factors,
+    and sampled rows of the clipped sum and of the noisy output."""
+    L = len(w.layers)
+    n_ref = np.stack([O.layer_sqnorms_ghost(W.to_f64(A), W.to_f64(D)) for A, D in layers])
+    s_ref, c_ref = O.clip_factors(n_ref, f32(w.C))
+    tol = TOL[w.dtype]
+    assert rel_err_elementwise(res["n"], n_ref) <= tol
+    assert rel_err_elementwise(res["c"], c_ref) <= tol
+    rng = np.random.default_rng(123)
+    off = 0
+    for l, (A, D) in enumerate(layers):
+        d_in, d_out = w.layers[l]
+        rows = np.sort(rng.choice(d_in, size=sample_rows, replace=False))
+        A64 = W.to_f64(A[:, :, rows])
+        S_rows = O.clipped_sum(A64, W.to_f64(D), c_ref)          # = S_l[rows, :]
+        z = np.stack([O.gaussian_noise(seed, step, off + int(j) * d_out, d_out) for j in rows])
+        ref = S_rows + f32(w.sigma) * f32(w.C) * z
+        got = res["out"][l][rows]
+        assert rel_err_normwise(got, ref) <= tol, l
+        off += d_in * d_out
+
+
+def test_llm_workload_sampled():
+    w = W.get("llm_bf16")
+    layers = W.make_inputs(w, seed=0)
+    res = run_gpu_step(w, layers)
+    _llm_sample_check(w, layers, res)
+
+
+# ---------------------------------------------------------------------------
+# norm modes, edge shapes and flags
+# ---------------------------------------------------------------------------
+
+EDGE = [
+    # (layers, B, T, dtype)
+    ([(8, 8)], 1, 1, "bf16"),
+    ([(136, 72), (64, 200)], 3, 80, "bf16"),
+    ([(24, 264)], 2, 129, "bf16"),
+    ([(130, 70), (70, 3)], 5, 3, "f32"),
+    ([(1, 1)], 1, 1, "f32"),
+    ([(5, 7)], 4, 65, "f32"),
+    ([(256, 128)], 2, 256, "bf16"),
+]
+
+
+@pytest.mark.parametrize("case", range(len(EDGE)))
+@pytest.mark.parametrize("mode", [dp.DP_NORM_AUTO, dp.DP_NORM_GHOST, dp.DP_NORM_MATERIALISED])
+def test_edge_shapes_and_norm_modes(case, mode):
+    layers_shape, B, T, dtype = EDGE[case]
+    w = W.custom(f"edge{case}", layers_shape, B, T, dtype, C=0.3, sigma=0.9, d_std=0.5,
+                 wid=500 + case)
+    layers = W.make_inputs(w, seed=1)
+    res = run_gpu_step(w, layers, seed=11, step=3, norm_mode=mode)
+    ref = oracle_step(w, layers, seed=11, step=3)
+    assert_step_matches(res, ref, dtype)
+    if mode != dp.DP_NORM_AUTO:
+        assert all(m == mode for m in res["modes"])
+
+
+def test_zero_example_keeps_clip_factor_one():
+    w = W.custom("zero", [(64, 48)], 4, 16, "bf16", C=1e-3, sigma=0.0, wid=600)
+    layers = W.make_inputs(w)
+    A, D = layers[0]
+    A = A.clone()
+    A[2].zero_()
+    layers = [(A, D)]
+    res = run_gpu_step(w, layers)
+    assert res["c"][2] == 1.0 and res["n"][0, 2] == 0.0
+    ref = oracle_step(w, layers)
+    assert_step_matches(res, ref, "bf16")
+
+
+def test_nonfinite_input_is_reported():
+    w = W.custom("nan", [(32, 16)], 3, 4, "f32", wid=601)
+    layers = W.make_inputs(w)
+    A, D = layers[0]
+    A = A.clone()
+    A[1, 2, 5] = float("nan")
+    dev = torch.device(DEV)
+    Ad, Dd = A.to(dev), D.to(dev)
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, audit_capacity=w.B)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.dp_layer_norms(ctx, 0, Ad, Dd)
+        c = torch.empty(w.B, device=dev)
+        dp.dp_clip_factors(ctx, None, c)
+        with pytest.raises(dp.DPError) as ei:
+            dp.dp_audit_emit(ctx, [0, 1], 1)
+        assert ei.value.status == 5
+        cc = c.cpu().numpy()
+        assert np.isnan(cc[1]) and np.isfinite(cc[0]) and np.isfinite(cc[2])
+        # a re-keyed step with clean inputs clears the flag
+        dp.dp_step_init(cfg, ctx=ctx)
+        A2 = layers[0][0].to(dev)
+        dp.dp_layer_norms(ctx, 0, A2, Dd)
+        dp.dp_clip_factors(ctx)
+        dp.dp_audit_emit(ctx, [1], 1)
+    finally:
+        dp.dp_step_destroy(ctx)
+
+
+def test_call_order_errors():
+    w = W.custom("order", [(32, 16), (16, 8)], 2, 3, "f32", wid=602)
+    layers = W.make_inputs(w)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    out = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, audit_capacity=1)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        def status(fn, *a):
+            with pytest.raises(dp.DPError) as ei:
+                fn(*a)
+            return ei.value.status
+        assert status(dp.dp_clipped_sum_noise, ctx, 0, Ad[0], Dd[0], out[0]) == 4
+        assert status(dp.dp_audit_emit, ctx, [0], 2) == 4
+        dp.dp_layer_norms(ctx, 0, Ad[0], Dd[0])
+        assert status(dp.dp_clip_factors, ctx) == 4          # layer 1 missing
+        dp.dp_layer_norms(ctx, 1, Ad[1], Dd[1])
+        dp.dp_clip_factors(ctx)
+        assert status(dp.dp_layer_norms, ctx, 0, Ad[0], Dd[0]) == 4
+        assert status(dp.dp_clip_factors, ctx) == 4
+        assert status(dp.dp_audit_emit, ctx, [0, 1], 2) == 1  # over capacity
+        assert status(dp.dp_audit_emit, ctx, [5], 2) == 1     # index out of range
+        assert status(dp.dp_layer_norms, ctx, 2, Ad[0], Dd[0]) == 1
+        assert status(dp.dp_clipped_sum_noise, ctx, 0, Ad[0], Dd[0], out[0],
+                      dp.DP_NO_NOISE | dp.DP_NOISE_ONLY) == 1
+        misaligned = out[0].view(-1)[1:]
+        assert status(dp.dp_clipped_sum_noise, ctx, 0, Ad[0], Dd[0], misaligned.data_ptr()) == 1
+        dp.dp_clipped_sum_noise(ctx, 0, Ad[0], Dd[0], out[0])
+        # re-key with other shapes is refused, the context stays usable
+        bad = dp.make_config([(32, 16)], w.B, w.T, w.dtype, w.C, w.sigma)
+        assert status(dp.dp_step_init, bad, None, ctx) == 2
+        dp.dp_audit_emit(ctx, [1], 2)
+    finally:
+        dp.dp_step_destroy(ctx)
+
+
+def test_commit_then_noise_equals_one_shot():
+    """Commit (DP_NO_NOISE), re-key with the released seed, DP_NOISE_ONLY:
+    equals the one-shot noisy output (Algorithm 2 commit-then-release)."""
+    w = W.get("block_bf16")
+    layers = W.make_inputs(w)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    one = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    two = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    scale = 1.0 / w.B
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=scale,
+                         seed=77, step=4)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.run_step(ctx, Ad, Dd, one)
+        cfg0 = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=scale,
+                              seed=0, step=4)   # seed not released yet
+        dp.dp_step_init(cfg0, ctx=ctx)
+        dp.run_step(ctx, Ad, Dd, two, flags=dp.DP_NO_NOISE)
+        dp.dp_step_init(cfg, ctx=ctx)           # released seed
+        for l in range(len(layers)):
+            dp.dp_clipped_sum_noise(ctx, l, None, None, two[l], dp.DP_NOISE_ONLY)
+    finally:
+        dp.dp_step_destroy(ctx)
+    for a, b in zip(one, two):
+        assert rel_err_normwise(b.cpu().numpy(), a.cpu().numpy()) <= 1e-6
+
+
+def test_accumulate_over_microbatches():
+    """Two micro-batches with DP_ACCUMULATE | DP_NO_NOISE sum their clipped sums."""
+    w = W.custom("micro", [(96, 40)], 6, 32, "bf16", C=0.05, sigma=1.0, d_std=0.2, wid=603)
+    layers = W.make_inputs(w)
+    A, D = layers[0]
+    dev = torch.device(DEV)
+    out = torch.zeros(96, 40, device=dev)
+    halves = [(A[:3], D[:3]), (A[3:], D[3:])]
+    ref = np.zeros((96, 40))
+    for Ah, Dh in halves:
+        wh = W.custom("micro_h", [(96, 40)], 3, 32, "bf16", C=0.05, sigma=1.0, wid=603)
+        cfg = dp.make_config(wh.layers, 3, 32, "bf16", wh.C, wh.sigma)
+        ctx = dp.dp_step_init(cfg)
+        try:
+            dp.run_step(ctx, [Ah.contiguous().to(dev)], [Dh.contiguous().to(dev)], [out],
+                        flags=dp.DP_NO_NOISE | dp.DP_ACCUMULATE)
+        finally:
+            dp.dp_step_destroy(ctx)
+        r = oracle_step(wh, [(Ah, Dh)], noise=False)
+        ref += r["out"][0]
+    assert rel_err_normwise(out.cpu().numpy(), ref) <= 2e-3
+
+
+def test_deterministic_and_step_keyed():
+    w = W.get("block_bf16")
+    layers = W.make_inputs(w)
+    r1 = run_gpu_step(w, layers, seed=3, step=10)
+    r2 = run_gpu_step(w, layers, seed=3, step=10)
+    r3 = run_gpu_step(w, layers, seed=3, step=11)
+    for a, b, c in zip(r1["out"], r2["out"], r3["out"]):
+        assert np.array_equal(a, b)
+        assert not np.array_equal(a, c)
+    assert np.array_equal(r1["n"], r2["n"]) and np.array_equal(r1["c"], r2["c"])
+
+
+def test_noise_statistics_on_device():
+    """Noise-only output over a large layer: mean ~ 0, variance ~ (out_scale sigma C)^2."""
+    w = W.custom("stat", [(4096, 4096)], 2, 1, "bf16", C=0.5, sigma=1.3, wid=604)
+    dev = torch.device(DEV)
+    out = torch.zeros(4096, 4096, device=dev)
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=0.5, seed=9)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.dp_clipped_sum_noise(ctx, 0, None, None, out, dp.DP_NOISE_ONLY)
+    finally:
+        dp.dp_step_destroy(ctx)
+    x = out.double().cpu().numpy().ravel()
+    sd = 0.5 * f32(1.3) * f32(0.5)
+    n = x.size
+    assert abs(x.mean()) <= 5 * sd / math.sqrt(n)
+    assert abs(x.var() / sd ** 2 - 1) <= 5 * math.sqrt(2 / n)
