@@ -180,6 +180,12 @@ int64_t dp_audit_record_bytes(int32_t n_layers);
 /* Norm mode chosen for a layer (resolves DP_NORM_AUTO). */
 dp_status dp_layer_norm_mode(const dp_ctx* ctx, int32_t layer, dp_norm_mode* mode_out);
 
+/* Which kernels serve a layer: *norm_tc = 1 if its per-example norms run on
+ * the tcgen05 tensor cores (0: CUDA cores), *sum_tc = 1 if its clipped sum
+ * does.  bf16 layers use tensor cores when T is a multiple of 64 (clipped
+ * sum, materialised norm) or always (Gram norm); fp32 layers never do. */
+dp_status dp_layer_path(const dp_ctx* ctx, int32_t layer, int32_t* norm_tc, int32_t* sum_tc);
+
 /* Release the context and all of its scratch; NULL is a no-op.  Waits for
  * the context's pending work first. */
 void dp_step_destroy(dp_ctx* ctx);

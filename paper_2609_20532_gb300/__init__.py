@@ -24,7 +24,8 @@ __all__ = [
     "DP_NO_NOISE", "DP_NOISE_ONLY", "DP_ACCUMULATE",
     "dp_layer", "dp_config", "make_config",
     "dp_step_init", "dp_layer_norms", "dp_clip_factors", "dp_clipped_sum_noise",
-    "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_step_destroy",
+    "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_layer_path",
+    "dp_step_destroy",
     "dp_last_error", "dp_debug_philox", "dp_debug_gaussian", "EXPORTED_SYMBOLS",
 ]
 
@@ -43,8 +44,8 @@ STATUS_NAMES = {0: "DP_OK", 1: "DP_ERR_ARG", 2: "DP_ERR_SHAPE", 3: "DP_ERR_DTYPE
 # every symbol include/dp_step.h declares
 EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_clip_factors", "dp_clipped_sum_noise",
                     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode",
-                    "dp_step_destroy", "dp_last_error", "dp_status_string", "dp_debug_philox",
-                    "dp_debug_gaussian"]
+                    "dp_layer_path", "dp_step_destroy", "dp_last_error", "dp_status_string",
+                    "dp_debug_philox", "dp_debug_gaussian"]
 
 
 class DPError(RuntimeError):
@@ -94,6 +95,7 @@ def lib() -> ctypes.CDLL:
         "dp_audit_emit": ([vp, vp, i32, vp], i32),
         "dp_audit_record_bytes": ([i32], i64),
         "dp_layer_norm_mode": ([vp, i32, ctypes.POINTER(i32)], i32),
+        "dp_layer_path": ([vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], i32),
         "dp_step_destroy": ([vp], None),
         "dp_last_error": ([], ctypes.c_char_p),
         "dp_status_string": ([i32], ctypes.c_char_p),
@@ -194,6 +196,13 @@ def dp_layer_norm_mode(ctx: int, layer: int) -> int:
     m = ctypes.c_int32(0)
     _check(lib().dp_layer_norm_mode(ctx, layer, ctypes.byref(m)))
     return m.value
+
+
+def dp_layer_path(ctx: int, layer: int):
+    """(norm_on_tensor_cores, sum_on_tensor_cores) for a layer."""
+    a, b = ctypes.c_int32(0), ctypes.c_int32(0)
+    _check(lib().dp_layer_path(ctx, layer, ctypes.byref(a), ctypes.byref(b)))
+    return bool(a.value), bool(b.value)
 
 
 def dp_step_destroy(ctx: Optional[int]) -> None:

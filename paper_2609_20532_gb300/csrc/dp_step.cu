@@ -329,12 +329,12 @@ dp_status dp_layer_norms(dp_ctx* c, int32_t layer, const void* A, const void* D)
     e = dpk::launch_norm_rank1(it, A, D, c->B, din, dout, c->d_part, c->NP, row0, c->stream);
   } else if (p.mode == DP_NORM_GHOST) {
     e = p.norm_tc ? dpk::tc_launch_ghost(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
-                                         c->stream)
+                                         c->d_flag, c->stream)
                   : dpk::launch_norm_ghost_simt(it, A, D, c->B, c->T, din, dout, c->d_part,
                                                 c->NP, row0, c->stream);
   } else {
     e = p.norm_tc ? dpk::tc_launch_mat_norm(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
-                                            c->stream)
+                                            c->d_flag, c->stream)
                   : dpk::launch_norm_mat_simt(it, A, D, c->B, c->T, din, dout, c->d_part, c->NP,
                                               row0, c->stream);
   }
@@ -388,7 +388,8 @@ dp_status dp_clipped_sum_noise(dp_ctx* c, int32_t layer, const void* A, const vo
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
   cudaError_t e;
   if (p.gemm_tc)
-    e = dpk::tc_launch_clipsum(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep, c->stream);
+    e = dpk::tc_launch_clipsum(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep, c->d_flag,
+                               c->stream);
   else
     e = dpk::launch_gemm_simt(c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, A, D, c->d_c,
                               c->B, c->T, din, dout, d_out, ep, c->stream);
@@ -420,7 +421,9 @@ dp_status dp_audit_emit(dp_ctx* c, const int32_t* h_idx, int32_t n, void* h_reco
   DP_CUDA(cudaMemcpyAsync(c->h_flag, c->d_flag, sizeof(int), cudaMemcpyDeviceToHost, c->stream));
   DP_CUDA(cudaStreamSynchronize(c->stream));
   if (n > 0) std::memcpy(h_records, c->h_rec, sizeof(float) * rec_words * n);
-  if (*c->h_flag) return fail(DP_ERR_NONFINITE, "a per-example squared norm was not finite");
+  if (*c->h_flag & 2)
+    return fail(DP_ERR_TIMEOUT, "a tensor-core kernel gave up waiting on a pipeline barrier");
+  if (*c->h_flag & 1) return fail(DP_ERR_NONFINITE, "a per-example squared norm was not finite");
   return DP_OK;
 }
 
@@ -430,6 +433,14 @@ dp_status dp_layer_norm_mode(const dp_ctx* c, int32_t layer, dp_norm_mode* mode_
   if (!c || !mode_out) return fail(DP_ERR_ARG, "NULL argument");
   if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
   *mode_out = c->plan[layer].mode;
+  return DP_OK;
+}
+
+dp_status dp_layer_path(const dp_ctx* c, int32_t layer, int32_t* norm_tc, int32_t* sum_tc) {
+  if (!c || !norm_tc || !sum_tc) return fail(DP_ERR_ARG, "NULL argument");
+  if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
+  *norm_tc = c->plan[layer].norm_tc;
+  *sum_tc = c->plan[layer].gemm_tc;
   return DP_OK;
 }
 

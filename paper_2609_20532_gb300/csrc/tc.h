@@ -1,7 +1,9 @@
 // Tensor-core (tcgen05 / TMEM / TMA) kernels of the DP-SGD step, bf16 inputs.
 #pragma once
-#include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
+
+#include <cstdint>
 
 #include "internal.h"
 
@@ -11,16 +13,24 @@ namespace dpk {
 bool tc_ghost_supported(int T, int64_t d_in, int64_t d_out);
 int tc_ghost_parts(int T);
 cudaError_t tc_launch_ghost(const void* A, const void* D, int B, int T, int d_in, int d_out,
-                            float* part, int NP, int row0, cudaStream_t s);
+                            float* part, int NP, int row0, int* err, cudaStream_t s);
 
 // Clipped sum S = A^T diag(c) D with the noise epilogue, and the materialised
 // per-example norm that shares its main loop.
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out);
 int tc_mat_parts(int64_t d_in, int64_t d_out);
 cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d_in, int d_out,
-                               float* part, int NP, int row0, cudaStream_t s);
+                               float* part, int NP, int row0, int* err, cudaStream_t s);
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
-                              int d_in, int d_out, float* out, const Epilogue& ep,
+                              int d_in, int d_out, float* out, const Epilogue& ep, int* err,
                               cudaStream_t s);
+
+// Host helpers shared by the tensor-core launchers (tc_host.cu).
+bool tma_encode_available();
+// bf16 tensor map, 128-byte swizzle, zero fill out of bounds; dims[0] innermost,
+// strides_bytes[r] is the byte stride of dimension r+1.
+bool make_tma_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
+                   const uint64_t* strides_bytes, const uint32_t* box);
+int device_sm_count();
 
 }  // namespace dpk

@@ -44,11 +44,12 @@ def run_gpu_step(w: W.Workload, layers, seed=0, step=0, out_scale=1.0, flags=0,
             dp.dp_clipped_sum_noise(ctx, l, Ad[l], Dd[l], outs[l], flags)
         recs = dp.dp_audit_emit(ctx, range(w.B), len(layers)) if audit else None
         modes = [dp.dp_layer_norm_mode(ctx, l) for l in range(len(layers))]
+        paths = [dp.dp_layer_path(ctx, l) for l in range(len(layers))]
     finally:
         dp.dp_step_destroy(ctx)
     torch.cuda.synchronize()
     res = {"out": [o.cpu().numpy() for o in outs], "s": s_dev.cpu().numpy(),
-           "c": c_dev.cpu().numpy(), "modes": modes}
+           "c": c_dev.cpu().numpy(), "modes": modes, "paths": paths}
     if recs is not None:
         res["n"] = np.stack([r["layer_sqnorm"] for r in recs], axis=1)
         res["rec_s"] = np.array([r["total_sqnorm"] for r in recs])

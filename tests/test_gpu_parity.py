@@ -323,3 +323,51 @@ def test_noise_statistics_on_device():
     n = x.size
     assert abs(x.mean()) <= 5 * sd / math.sqrt(n)
     assert abs(x.var() / sd ** 2 - 1) <= 5 * math.sqrt(2 / n)
+
+
+# ---------------------------------------------------------------------------
+# tensor-core paths: ragged tiles, persistence across many tiles, both norms
+# ---------------------------------------------------------------------------
+
+TC_CASES = [
+    # (layers, B, T): every layer bf16 with T % 64 == 0, so both the clipped
+    # sum and the norms run on tcgen05
+    ([(200, 264)], 3, 64),               # ragged M and N tiles
+    ([(8, 8), (16, 24)], 2, 64),         # tiles far smaller than one MMA
+    ([(520, 1000), (1000, 136)], 2, 128),
+    ([(4096, 4096)], 2, 64),             # 512 tiles > SM count: persistent loop
+    ([(384, 512)], 5, 192),              # 3 K-blocks per example, T not a power of 2
+]
+
+
+@pytest.mark.parametrize("case", range(len(TC_CASES)))
+@pytest.mark.parametrize("mode", [dp.DP_NORM_GHOST, dp.DP_NORM_MATERIALISED])
+def test_tensor_core_paths(case, mode):
+    shapes, B, T = TC_CASES[case]
+    w = W.custom(f"tc{case}", shapes, B, T, "bf16", C=0.2, sigma=0.5, d_std=0.05,
+                 wid=700 + case)
+    layers = W.make_inputs(w, seed=2)
+    res = run_gpu_step(w, layers, seed=5, step=1, norm_mode=mode)
+    assert all(n and s for n, s in res["paths"]), res["paths"]
+    ref = oracle_step(w, layers, seed=5, step=1)
+    assert_step_matches(res, ref, "bf16")
+
+
+def test_workload_paths_use_tensor_cores():
+    for name, expect in [("block_bf16", True), ("llm_bf16", True), ("mlp_fp32", False)]:
+        w = W.get(name)
+        cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma)
+        ctx = dp.dp_step_init(cfg)
+        try:
+            paths = [dp.dp_layer_path(ctx, l) for l in range(len(w.layers))]
+        finally:
+            dp.dp_step_destroy(ctx)
+        assert all(p == (expect, expect) for p in paths), (name, paths)
+
+
+def test_ghost_and_materialised_agree_on_block_workload():
+    w = W.get("block_bf16")
+    layers = W.make_inputs(w)
+    g = run_gpu_step(w, layers, norm_mode=dp.DP_NORM_GHOST, flags=dp.DP_NO_NOISE)
+    m = run_gpu_step(w, layers, norm_mode=dp.DP_NORM_MATERIALISED, flags=dp.DP_NO_NOISE)
+    assert rel_err_elementwise(g["n"], m["n"]) <= 1e-4
