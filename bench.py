@@ -108,16 +108,17 @@ def _kernel_sha(path):
     return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
 
 
-def _traffic(kernel_key, src_file):
-    """DRAM bytes per launch of a kernel from a committed ncu summary, or None
+def _traffic(kernel_key, flops_per_launch):
+    """DRAM bytes per launch of the GEMM from the committed ncu capture
+    (profiles/traffic.json), scaled from the captured shape by FLOPs, or None
     when the kernel source changed since the counters were taken."""
     p = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
     d = json.load(open(p)).get(kernel_key)
-    if not d or d.get("src_sha256_16") != _kernel_sha(src_file):
+    if not d or d.get("src_sha256_16") != _kernel_sha(os.path.join(ROOT, d["src"])):
         return None
-    return d.get("dram_bytes_per_step")
+    return d["captured_dram_bytes"] * flops_per_launch / d["captured_flops"]
 
 
 def cpu_baseline_sample(w, seed=0):
@@ -265,8 +266,8 @@ def run_ours(args, rank, world, local_rank):
     in_total = in_bytes
     norm_ms = per_step_ms("norm")
     norm_gbs = in_total / (norm_ms * 1e-3) / 1e9
-    src = os.path.join(ROOT, "paper_2609_20532_gb300", "csrc", "k_tc.cu")
-    traffic = _traffic("clipsum_gemm", src)
+    # roofline of the dominant kernel, per launch (average over the L launches)
+    traffic = _traffic("clipsum_gemm", gemm_flops / L)
     kernels = {
         "clipsum_gemm": {"ms_per_step": gemm_ms, "tflops": gemm_tflops,
                          "frac_bf16_peak": gemm_tflops / peaks["bf16_tflops"],

@@ -82,6 +82,12 @@ WORKLOADS = {
                          0.5, 1.0, audit_frac=0.05),
 }
 
+# the FFN-up layer of the LLM workload alone (profiling case: 247 MB of
+# inputs, larger than L2, a few hundred MB on the device)
+WORKLOADS["llm_ffn_up_bf16"] = Workload("llm_ffn_up_bf16", 5, ((4096, 11008),), 16, 512, "bf16",
+                                        _normal_all(1), 1.0, math.sqrt(1e-5), 0.5, 1.0,
+                                        audit_frac=0.05)
+
 # one 4096x4096 bf16 layer over B x T
 SWEEP = [Workload(f"sweep_B{b}_T{t}", 100 + 10 * bi + ti, ((4096, 4096),), b, t,
                   "bf16", _normal_all(1), 1.0, 1.0, 1.0, 1.0)
