@@ -190,6 +190,29 @@ dp_status dp_layer_path(const dp_ctx* ctx, int32_t layer, int32_t* norm_tc, int3
  * the context's pending work first. */
 void dp_step_destroy(dp_ctx* ctx);
 
+/* Per-example squared norms of one layer without allocating any memory.
+ * The paper has no counterpart: this exists for callers that cannot call
+ * cudaMalloc at the point of use (inside a CUDA stream capture in global
+ * capture mode, a process whose device-memory budget is fixed at start-up,
+ * or a caller that must avoid the device synchronisation allocation can
+ * cause) and so cannot create a step context.
+ *   d_sqnorm_out[i] = ||A_i^T D_i||_F^2, i < B, by the Gram form (the same
+ *   kernels as dp_layer_norms with DP_NORM_GHOST).
+ * A: [B][T][d_in], D: [B][T][d_out] device arrays of dtype, 16-byte aligned;
+ * d_sqnorm_out: device fp32 [B]; cuda_stream: cudaStream_t (NULL = default).
+ * Asynchronous.  Scratch is a library-owned static device array of 2^20 fp32
+ * partial sums (4 MiB, held by every GPU that loads the library until exit):
+ * B * ceil(T/128) * (ceil(T/128) + 1) * 2 (bf16) or
+ * B * ceil(T/64) * (ceil(T/64) + 1) / 2 (fp32) must not exceed 2^20, else
+ * DP_ERR_SHAPE.  The first call on a device looks up the array's address
+ * and should come before any stream capture.  Calls share the array: calls
+ * that overlap on the GPU race and must be ordered by the caller.  If a
+ * tensor-core pipeline wait gives up, the outputs are NaN.
+ * Errors: DP_ERR_ARG, DP_ERR_DTYPE, DP_ERR_SHAPE, DP_ERR_CUDA. */
+dp_status dp_layer_sqnorms_noalloc(const void* A, const void* D, int32_t B, int32_t T,
+                                   int64_t d_in, int64_t d_out, dp_dtype dtype,
+                                   float* d_sqnorm_out, void* cuda_stream);
+
 /* Message of the last failing call on this thread ("" if none). */
 const char* dp_last_error(void);
 

@@ -26,7 +26,8 @@ __all__ = [
     "dp_step_init", "dp_layer_norms", "dp_clip_factors", "dp_clipped_sum_noise",
     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_layer_path",
     "dp_step_destroy",
-    "dp_last_error", "dp_debug_philox", "dp_debug_gaussian", "EXPORTED_SYMBOLS",
+    "dp_last_error", "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
+    "EXPORTED_SYMBOLS",
 ]
 
 HERE = os.path.dirname(os.path.abspath(__file__))
@@ -45,7 +46,7 @@ STATUS_NAMES = {0: "DP_OK", 1: "DP_ERR_ARG", 2: "DP_ERR_SHAPE", 3: "DP_ERR_DTYPE
 EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_clip_factors", "dp_clipped_sum_noise",
                     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode",
                     "dp_layer_path", "dp_step_destroy", "dp_last_error", "dp_status_string",
-                    "dp_debug_philox", "dp_debug_gaussian"]
+                    "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc"]
 
 
 class DPError(RuntimeError):
@@ -101,6 +102,7 @@ def lib() -> ctypes.CDLL:
         "dp_status_string": ([i32], ctypes.c_char_p),
         "dp_debug_philox": ([u64, u64, u64, i64, vp, vp], i32),
         "dp_debug_gaussian": ([u64, u64, u64, i64, vp, vp], i32),
+        "dp_layer_sqnorms_noalloc": ([vp, vp, i32, i32, i64, i64, i32, vp, vp], i32),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)
@@ -222,6 +224,16 @@ def dp_debug_philox(seed: int, step: int, first_quad: int, n_quads: int, out, st
 def dp_debug_gaussian(seed: int, step: int, first_index: int, n: int, out, stream=None):
     _check(lib().dp_debug_gaussian(seed & (2 ** 64 - 1), step & (2 ** 64 - 1),
                                    first_index & (2 ** 64 - 1), n, _ptr(out), _stream(stream)))
+
+
+def dp_layer_sqnorms_noalloc(A, D, B: int, T: int, d_in: int, d_out: int, dtype: str, out,
+                             stream=None) -> None:
+    """Per-example squared norms of one layer into ``out`` [B] without any
+    allocation by the library (for callers that cannot allocate at the point
+    of use; see include/dp_step.h)."""
+    _check(lib().dp_layer_sqnorms_noalloc(_ptr(A), _ptr(D), B, T, d_in, d_out,
+                                          DP_BF16 if dtype == "bf16" else DP_F32, _ptr(out),
+                                          _stream(stream)))
 
 
 def run_step(ctx: int, A_list, D_list, outs, flags: int = 0) -> None:

@@ -39,6 +39,10 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 }  // namespace
 
+namespace dpk {
+void set_last_error(const char* msg) { g_err = msg; }
+}  // namespace dpk
+
 // Per-layer execution plan, fixed at init from the shapes and the norm mode.
 struct LayerPlan {
   int64_t d_in, d_out;

@@ -48,6 +48,9 @@ cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, uint64_t se
 cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer_sq,
                          const float* s_vec, const float* c_vec, float* rec, cudaStream_t s);
 
+// ---- error message of the calling thread, read back by dp_last_error() ----
+void set_last_error(const char* msg);
+
 // ---- generator exports for tests ----
 cudaError_t launch_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
                                 uint32_t* out, cudaStream_t s);
