@@ -8,8 +8,8 @@ bf16, B=16, T=512.  Prints ONE JSON line on rank 0.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 
---impl reference times the fp64 CPU oracle (the baseline this build is
-checked against) on a bounded sample of the same workload.
+--impl reference times the fp64 CPU oracle (the plain implementation the
+kernels are checked against) on a bounded sample of the same workload.
 """
 
 from __future__ import annotations

@@ -193,7 +193,7 @@ def clipped_sum(A, D, c) -> np.ndarray:
 
 # ---------------------------------------------------------------------------
 # Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) -- the counter-based
-# generator this build uses for Noise(s; sigma C); the paper names none.
+# generator used for Noise(s; sigma C); the paper names none.
 # ---------------------------------------------------------------------------
 
 PHILOX_M0 = 0xD2511F53  # round multiplier for counter word 0
