@@ -6,7 +6,8 @@
 // Operands: A is [B*T, d_in] and D is [B*T, d_out], both row-major, so as
 // GEMM operands (M = d_in, N = d_out, K = B*T) both are MN-major; TMA loads
 // 64-column x 64-row boxes with 128-byte swizzle straight into the canonical
-// MN-major layout the tensor core reads.
+// MN-major layout the tensor core reads (LBO = 8 KB between 64-element MN
+// chunks, SBO = 1 KB between 8-row K groups).
 //
 // The clip factor varies along K (one value per example).  Instead of
 // rescaling operand tiles in shared memory, the kernel folds it exactly:
@@ -16,9 +17,19 @@
 // fp32 register accumulator while the tensor core already works on the
 // next example.  No extra rounding, no operand rewrite.
 //
+// Two variants of the same kernel:
+//   single CTA (PAIR = false): tile 128 x 256, 4 stages of 48 KB;
+//   CTA pair (PAIR = true, cluster of 2, tcgen05 cta_group::2): tile
+//     256 x 256; each CTA stages its 128 rows of A and its 128 columns of D
+//     (6 stages of 32 KB), the leader CTA issues the pair MMA and its
+//     commits arrive on the barriers of both CTAs; each CTA's TMEM holds its
+//     128 rows.  Half the shared-memory bytes per MMA, so the same stage
+//     memory covers 1.5x more load latency.
+//
 // Warp roles (3 warpgroups = 384 threads, one CTA per SM, persistent):
 //   warpgroup 0: warp 0 TMA producer (one lane), warp 1 TMEM allocator +
-//                MMA issuer (one lane), warps 2-3 idle; drops to 48 regs.
+//                MMA issuer (one lane; leader CTA only in a pair), warps 2-3
+//                idle; drops to 48 regs.
 //   warpgroups 1-2 (warps 4-11): fold / epilogue, raised to 224 regs; warp w
 //                reads TMEM lanes 32*(w%4)..+31, column half (w-4)/4.
 // Register budget: launched at 168 x 384 = 64512; after the split
@@ -39,21 +50,26 @@ namespace {
 
 using namespace tc;
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
-constexpr int A_STAGE = BM * BK * 2;           // 16 KB: two 64-col chunks of 64 rows x 128 B
-constexpr int B_STAGE = BN * BK * 2;           // 32 KB: four chunks
-constexpr int CHUNK = 64 * BK * 2;             // 8 KB: one 64-column chunk
-constexpr int STAGE_BYTES = A_STAGE + B_STAGE;
+constexpr int BM = 128, BN = 256, BK = 64;
+constexpr int CHUNK = 64 * BK * 2;  // 8 KB: one 64-column chunk of 64 rows
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int FIRST_EPI_WARP = 4;
 constexpr int GEMM_THREADS = 128 + 32 * NUM_EPI_WARPS;
 constexpr int REGS_CTRL = 48, REGS_EPI = 224;
 constexpr uint32_t TMEM_COLS = 512;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;
-// MN-major, 128-byte swizzle: LBO = distance between 64-element MN chunks,
-// SBO = distance between 8-row K groups.
 constexpr uint32_t LBO = CHUNK, SBO = 1024;
-constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN, /*a_mn=*/1, /*b_mn=*/1);
+
+template <bool PAIR>
+struct Cfg {
+  static constexpr int STAGES = PAIR ? 6 : 4;
+  static constexpr int B_COLS = PAIR ? BN / 2 : BN;         // D columns staged per CTA
+  static constexpr int A_STAGE = BM * BK * 2;               // 16 KB
+  static constexpr int B_STAGE = B_COLS * BK * 2;           // 16 / 32 KB
+  static constexpr int STAGE_BYTES = A_STAGE + B_STAGE;     // 32 / 48 KB
+  static constexpr int TILE_M = PAIR ? 2 * BM : BM;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;
+  static constexpr uint32_t IDESC = idesc_bf16_f32(TILE_M, BN, /*a_mn=*/1, /*b_mn=*/1);
+};
 
 struct GemmArgs {
   const float* c;
@@ -66,10 +82,23 @@ struct GemmArgs {
   Epilogue ep;
 };
 
-template <bool NORM>
+// Bounded wait used only at teardown (ignores the abort flag).
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* err) {
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      atomicOr(err, kErrTimeout);
+      return;
+    }
+  }
+}
+
+template <bool NORM, bool PAIR>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapD,
               const GemmArgs g) {
+  using C = Cfg<PAIR>;
+  constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -78,6 +107,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   __shared__ int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0;
+  const bool leader = rank == 0;
+  const int unit = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int n_units = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
   const int kpe = g.T / BK;
   const int n_tiles = g.n_m * g.n_n;
   volatile int* abrt = &abort_flag;
@@ -89,7 +122,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull_bar[b], 1);
-      mbar_init(&tempty_bar[b], NUM_EPI_WARPS);
+      mbar_init(&tempty_bar[b], PAIR ? 2 * NUM_EPI_WARPS : NUM_EPI_WARPS);
     }
     mbar_init(&done_bar, 1);
     abort_flag = 0;
@@ -99,34 +132,51 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     tma_prefetch_desc(&mapA);
     tma_prefetch_desc(&mapD);
   }
-  if (warp == 1) tmem_alloc(&tmem_slot, TMEM_COLS);
+  if (warp == 1) {
+    if constexpr (PAIR)
+      tmem_alloc_pair(&tmem_slot, TMEM_COLS);
+    else
+      tmem_alloc(&tmem_slot, TMEM_COLS);
+  }
   tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) cluster_sync();  // the peer's barriers exist before any remote arrive
   tc_fence_after();
   const uint32_t tmem_base = tmem_slot;
 
   if (warp < FIRST_EPI_WARP) {
     asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(REGS_CTRL));
-  if (warp == 0) {
-    if (lane == 0) {
-      // ---------------- TMA producer ----------------
+    if (warp == 0 && lane == 0) {
+      // ---------------- TMA producer (both CTAs of a pair) ----------------
       int stage = 0;
       uint32_t phase = 0;
       uint32_t uses[STAGES] = {};
-      for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-        const int m0 = (tile % g.n_m) * BM, n0 = (tile / g.n_m) * BN;
+      for (int tile = unit; tile < n_tiles; tile += n_units) {
+        const int m0 = (tile % g.n_m) * C::TILE_M + static_cast<int>(rank) * BM;
+        const int n0 = (tile / g.n_m) * BN + (PAIR ? static_cast<int>(rank) * (BN / 2) : 0);
         for (int ex = 0; ex < g.B; ++ex) {
           for (int kb = 0; kb < kpe; ++kb) {
             if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
-            uint8_t* sa = smem + stage * STAGE_BYTES;
-            uint8_t* sb = sa + A_STAGE;
-            mbar_arrive_expect_tx(&full_bar[stage], STAGE_BYTES);
+            uint8_t* sa = smem + stage * C::STAGE_BYTES;
+            uint8_t* sb = sa + C::A_STAGE;
             const int krow = ex * g.T + kb * BK;
-            tma_load_2d(&mapA, &full_bar[stage], sa, m0, krow);
-            tma_load_2d(&mapA, &full_bar[stage], sa + CHUNK, m0 + 64, krow);
+            if constexpr (PAIR) {
+              // both CTAs' loads complete on the leader's full barrier
+              const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
+              if (leader) mbar_arrive_expect_tx(&full_bar[stage], 2 * C::STAGE_BYTES);
+              tma_load_2d_pair(&mapA, fb, sa, m0, krow);
+              tma_load_2d_pair(&mapA, fb, sa + CHUNK, m0 + 64, krow);
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
-              tma_load_2d(&mapD, &full_bar[stage], sb + q * CHUNK, n0 + 64 * q, krow);
+              for (int q = 0; q < C::B_COLS / 64; ++q)
+                tma_load_2d_pair(&mapD, fb, sb + q * CHUNK, n0 + 64 * q, krow);
+            } else {
+              mbar_arrive_expect_tx(&full_bar[stage], C::STAGE_BYTES);
+              tma_load_2d(&mapA, &full_bar[stage], sa, m0, krow);
+              tma_load_2d(&mapA, &full_bar[stage], sa + CHUNK, m0 + 64, krow);
+#pragma unroll
+              for (int q = 0; q < C::B_COLS / 64; ++q)
+                tma_load_2d(&mapD, &full_bar[stage], sb + q * CHUNK, n0 + 64 * q, krow);
+            }
             ++uses[stage];
             if (++stage == STAGES) {
               stage = 0;
@@ -137,24 +187,21 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       }
     producer_done:
       // No TMA write may still be landing in shared memory when the CTA exits.
+      // Completion of a stage is recorded on the leader's full barrier; a
+      // peer waits instead for the leader's release of each stage it loaded.
       for (int s = 0; s < STAGES; ++s) {
         if (uses[s] == 0) continue;
-        const uint64_t t0 = globaltimer_ns();
-        while (!mbar_try_wait(&full_bar[s], (uses[s] - 1) & 1)) {
-          if (globaltimer_ns() - t0 > kWaitLimitNs) {
-            atomicOr(g.err, kErrTimeout);
-            break;
-          }
-        }
+        if (leader)
+          drain_wait(&full_bar[s], (uses[s] - 1) & 1, g.err);
+        else
+          drain_wait(&empty_bar[s], (uses[s] - 1) & 1, g.err);
       }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
+    } else if (warp == 1 && lane == 0 && leader) {
       // ---------------- MMA issuer ----------------
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
-      for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+      for (int tile = unit; tile < n_tiles; tile += n_units) {
         for (int ex = 0; ex < g.B; ++ex, ++it) {
           const int buf = it & 1;
           const uint32_t tph = (it >> 1) & 1;
@@ -164,35 +211,39 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           for (int kb = 0; kb < kpe; ++kb) {
             if (!mbar_wait(&full_bar[stage], phase, abrt, g.err)) goto mma_done;
             tc_fence_after();
-            const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
-            const uint32_t sb = sa + A_STAGE;
+            const uint32_t sa = smem_u32(smem + stage * C::STAGE_BYTES);
+            const uint32_t sb = sa + C::A_STAGE;
 #pragma unroll
             for (int kk = 0; kk < BK / 16; ++kk) {
               const uint64_t ad = smem_desc_sw128(sa + kk * 16 * 128, LBO, SBO);
               const uint64_t bd = smem_desc_sw128(sb + kk * 16 * 128, LBO, SBO);
-              mma_bf16(d_tmem, ad, bd, IDESC, (kb | kk) != 0);
+              if constexpr (PAIR)
+                mma_bf16_pair(d_tmem, ad, bd, C::IDESC, (kb | kk) != 0);
+              else
+                mma_bf16(d_tmem, ad, bd, C::IDESC, (kb | kk) != 0);
             }
-            mma_commit(&empty_bar[stage]);
+            if constexpr (PAIR)
+              mma_commit_pair(&empty_bar[stage]);
+            else
+              mma_commit(&empty_bar[stage]);
             if (++stage == STAGES) {
               stage = 0;
               phase ^= 1;
             }
           }
-          mma_commit(&tfull_bar[buf]);
+          if constexpr (PAIR)
+            mma_commit_pair(&tfull_bar[buf]);
+          else
+            mma_commit(&tfull_bar[buf]);
         }
       }
     mma_done:
-      // all issued MMAs must complete before TMEM is released
-      mma_commit(&done_bar);
-      const uint64_t t0 = globaltimer_ns();
-      while (!mbar_try_wait(&done_bar, 0)) {
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
-          atomicOr(g.err, kErrTimeout);
-          break;
-        }
-      }
+      // all issued MMAs must complete before TMEM is released (both CTAs wait)
+      if constexpr (PAIR)
+        mma_commit_pair(&done_bar);
+      else
+        mma_commit(&done_bar);
     }
-  }
   } else {
     asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REGS_EPI));
     // ---------------- fold / epilogue warps ----------------
@@ -202,14 +253,47 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int row = quad * 32 + lane;  // tile row held by this thread
     const uint32_t t_lane = static_cast<uint32_t>(quad * 32) << 16;
     int it = 0;
-    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-      const int m0 = (tile % g.n_m) * BM, n0 = (tile / g.n_m) * BN;
+    // The tile's noise (32 Philox quads per thread) is generated in slices
+    // of qpe quads while the tensor core works on each example and added
+    // into the register accumulator (sum and noise commute), so the tile end
+    // only scales and stores.
+    const int qpe = (32 + g.B - 1) / g.B;
+    const Epilogue& ep = g.ep;
+    for (int tile = unit; tile < n_tiles; tile += n_units) {
+      const int m0 = (tile % g.n_m) * C::TILE_M + static_cast<int>(rank) * BM;
+      const int n0 = (tile / g.n_m) * BN;
+      const int j = m0 + row;
+      const int k0 = n0 + half * 128;
+      const uint64_t prow = ep.p_base + static_cast<uint64_t>(j) * g.d_out;
       float S[128];
       if constexpr (!NORM) {
 #pragma unroll
         for (int i = 0; i < 128; ++i) S[i] = 0.f;
       }
       for (int ex = 0; ex < g.B; ++ex, ++it) {
+        if constexpr (!NORM) {
+          if (ep.add_noise && j < g.d_in) {
+            const int q_lo = ex * qpe;
+            const int q_hi = q_lo + qpe < 32 ? q_lo + qpe : 32;
+#pragma unroll 1
+            for (int q = q_lo; q < q_hi; ++q) {
+              // p_base and d_out are multiples of 8 on this path, so the four
+              // parameters prow+k .. +3 form exactly one Philox quad
+              if (k0 + 4 * q >= g.d_out) break;
+              const float4 z = gauss_quad(ep.seed, ep.step, (prow + k0 + 4 * q) >> 2);
+              // static register indices: select the slot with a predicate
+#pragma unroll
+              for (int t = 0; t < 32; ++t) {
+                if (t == q) {
+                  S[4 * t + 0] = fmaf(ep.sigmaC, z.x, S[4 * t + 0]);
+                  S[4 * t + 1] = fmaf(ep.sigmaC, z.y, S[4 * t + 1]);
+                  S[4 * t + 2] = fmaf(ep.sigmaC, z.z, S[4 * t + 2]);
+                  S[4 * t + 3] = fmaf(ep.sigmaC, z.w, S[4 * t + 3]);
+                }
+              }
+            }
+          }
+        }
         const int buf = it & 1;
         const uint32_t tph = (it >> 1) & 1;
         if (!mbar_wait(&tfull_bar[buf], tph, abrt, g.err)) goto epi_done;
@@ -231,34 +315,33 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty_bar[buf]);
+        if (lane == 0) {
+          if constexpr (PAIR)
+            mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[buf]), 0));
+          else
+            mbar_arrive(&tempty_bar[buf]);
+        }
         if constexpr (NORM) {
           // one partial per epilogue warp; the clip kernel sums them in order
 #pragma unroll
           for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
           if (lane == 0)
-            g.part[static_cast<int64_t>(g.row0 + ex) * g.NP + tile * NUM_EPI_WARPS + ew] = sq;
+            g.part[static_cast<int64_t>(g.row0 + ex) * g.NP +
+                   (tile * (PAIR ? 2 : 1) + static_cast<int>(rank)) * NUM_EPI_WARPS + ew] = sq;
         }
       }
       if constexpr (!NORM) {
-        const int j = m0 + row;
         if (j < g.d_in) {
           float* orow = g.out + static_cast<int64_t>(j) * g.d_out;
-          const Epilogue& ep = g.ep;
-          const uint64_t prow = ep.p_base + static_cast<uint64_t>(j) * g.d_out;
 #pragma unroll
           for (int q = 0; q < 32; ++q) {
-            const int k = n0 + half * 128 + 4 * q;
+            const int k = k0 + 4 * q;
             if (k < g.d_out) {
-              float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-              // p_base and d_out are multiples of 8 on this path, so the four
-              // parameters prow+k .. +3 form exactly one Philox quad
-              if (ep.add_noise) z = gauss_quad(ep.seed, ep.step, (prow + k) >> 2);
               float4 v;
-              v.x = ep.out_scale * fmaf(ep.sigmaC, z.x, S[4 * q + 0]);
-              v.y = ep.out_scale * fmaf(ep.sigmaC, z.y, S[4 * q + 1]);
-              v.z = ep.out_scale * fmaf(ep.sigmaC, z.z, S[4 * q + 2]);
-              v.w = ep.out_scale * fmaf(ep.sigmaC, z.w, S[4 * q + 3]);
+              v.x = ep.out_scale * S[4 * q + 0];
+              v.y = ep.out_scale * S[4 * q + 1];
+              v.z = ep.out_scale * S[4 * q + 2];
+              v.w = ep.out_scale * S[4 * q + 3];
               float4* o = reinterpret_cast<float4*>(orow + k);  // d_out % 8 == 0: aligned
               if (ep.accumulate) {
                 const float4 p = *o;
@@ -278,9 +361,16 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 
   tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    // the leader's last commit tells both CTAs that no MMA still writes TMEM
+    if (lane == 0) drain_wait(&done_bar, 0, g.err);
+    __syncwarp();
+    if constexpr (PAIR)
+      tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    else
+      tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -296,26 +386,65 @@ bool make_map_2d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows,
   return make_tma_bf16(m, base, 2, dims, strides, box);
 }
 
-template <bool NORM>
+// CTA pairs for every layer wider than one 128-row tile.
+bool use_pair(int64_t d_in) { return d_in > BM; }
+
+template <bool NORM, bool PAIR>
 cudaError_t launch_gemm(const void* A, const void* D, GemmArgs& g, cudaStream_t s) {
+  using C = Cfg<PAIR>;
   CUtensorMap mA, mD;
   const uint64_t rows = static_cast<uint64_t>(g.B) * g.T;
   if (!make_map_2d(&mA, A, g.d_in, rows, BK) || !make_map_2d(&mD, D, g.d_out, rows, BK))
     return cudaErrorInvalidValue;
-  static bool attr_set[2] = {false, false};
-  if (!attr_set[NORM]) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<NORM>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<NORM, PAIR>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
-    attr_set[NORM] = true;
+    attr_set = true;
   }
-  g.n_m = (g.d_in + BM - 1) / BM;
+  g.n_m = (g.d_in + C::TILE_M - 1) / C::TILE_M;
   g.n_n = (g.d_out + BN - 1) / BN;
   const int tiles = g.n_m * g.n_n;
   const int sms = device_sm_count();
-  const int grid = tiles < sms ? tiles : sms;
-  k_gemm_tc<NORM><<<grid, GEMM_THREADS, SMEM_BYTES, s>>>(mA, mD, g);
-  return cudaGetLastError();
+  if constexpr (PAIR) {
+    // persistent grid: as many pairs as can be resident at once
+    static int max_pairs = 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.blockDim = dim3(GEMM_THREADS);
+    cfg.dynamicSmemBytes = C::SMEM_BYTES;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (max_pairs == 0) {
+      cfg.gridDim = dim3(sms);
+      int n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<NORM, PAIR>, &cfg) != cudaSuccess || n < 1) {
+        cudaGetLastError();
+        n = sms / 2;
+      }
+      max_pairs = n < sms / 2 ? n : sms / 2;
+    }
+    const int pairs = tiles < max_pairs ? tiles : max_pairs;
+    cfg.gridDim = dim3(2 * pairs);
+    return cudaLaunchKernelEx(&cfg, k_gemm_tc<NORM, PAIR>, mA, mD, g);
+  } else {
+    const int grid = tiles < sms ? tiles : sms;
+    k_gemm_tc<NORM, PAIR><<<grid, GEMM_THREADS, C::SMEM_BYTES, s>>>(mA, mD, g);
+    return cudaGetLastError();
+  }
+}
+
+template <bool NORM>
+cudaError_t launch_any(const void* A, const void* D, GemmArgs& g, cudaStream_t s) {
+  return use_pair(g.d_in) ? launch_gemm<NORM, true>(A, D, g, s)
+                          : launch_gemm<NORM, false>(A, D, g, s);
 }
 
 }  // namespace
@@ -325,7 +454,10 @@ bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out) {
 }
 
 int tc_mat_parts(int64_t d_in, int64_t d_out) {
-  return static_cast<int>(((d_in + BM - 1) / BM) * ((d_out + BN - 1) / BN)) * NUM_EPI_WARPS;
+  const int64_t tile_m = use_pair(d_in) ? 2 * BM : BM;
+  const int64_t ctas_per_tile = use_pair(d_in) ? 2 : 1;
+  return static_cast<int>(((d_in + tile_m - 1) / tile_m) * ((d_out + BN - 1) / BN) *
+                          ctas_per_tile * NUM_EPI_WARPS);
 }
 
 cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d_in, int d_out,
@@ -339,7 +471,7 @@ cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d
   g.d_out = d_out;
   g.NP = NP;
   g.row0 = row0;
-  return launch_gemm<true>(A, D, g, s);
+  return launch_any<true>(A, D, g, s);
 }
 
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
@@ -354,7 +486,7 @@ cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int 
   g.d_in = d_in;
   g.d_out = d_out;
   g.ep = ep;
-  return launch_gemm<false>(A, D, g, s);
+  return launch_any<false>(A, D, g, s);
 }
 
 }  // namespace dpk
