@@ -351,6 +351,100 @@ def run_ours(args, rank, world, local_rank):
     print(json.dumps(line), flush=True)
 
 
+def run_sweep(args):
+    """One JSON line with a record per point of the 4096x4096 sweep: step
+    time, per-kernel times, the norm kernel the cost model picked, both norm
+    kernels timed (the measured crossover) and roofline fractions.  Inputs are
+    drawn on the device (torch's seeded CUDA generator, N(0,1) rounded to
+    bf16) so the whole sweep stays under a minute."""
+    import torch
+
+    import paper_2609_20532_gb300 as dp
+    import workloads as W
+
+    dev = torch.device("cuda:0")
+    torch.cuda.set_device(dev)
+    peaks = _peaks()
+    stream = torch.cuda.current_stream()
+    points = []
+    for w in W.SWEEP:
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(w.wid)
+        d = 4096
+        A = torch.randn(w.B, w.T, d, generator=gen, device=dev).to(torch.bfloat16)
+        D = torch.randn(w.B, w.T, d, generator=gen, device=dev).to(torch.bfloat16)
+        out = torch.empty(d, d, device=dev)
+
+        def timed(fn, reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            ts = []
+            for _ in range(reps):
+                e0.record(stream)
+                fn()
+                e1.record(stream)
+                torch.cuda.synchronize()
+                ts.append(e0.elapsed_time(e1))
+            return statistics.median(ts)
+
+        rec = {"B": w.B, "T": w.T}
+        for mode_name, mode in (("auto", dp.DP_NORM_AUTO), ("ghost", dp.DP_NORM_GHOST),
+                                ("materialised", dp.DP_NORM_MATERIALISED)):
+            if mode_name != "auto" and w.T == 1:
+                continue  # both reduce to the rank-1 form
+            cfg = dp.make_config(w.layers, w.B, w.T, "bf16", w.C, w.sigma, out_scale=1.0 / w.B,
+                                 seed=7, norm_mode=mode)
+            ctx = dp.dp_step_init(cfg, stream)
+
+            def norms():
+                dp.dp_step_init(cfg, stream, ctx)
+                dp.dp_layer_norms(ctx, 0, A, D)
+
+            def gemm():
+                dp.dp_clipped_sum_noise(ctx, 0, A, D, out, 0)
+
+            def step():
+                norms()
+                dp.dp_clip_factors(ctx)
+                gemm()
+
+            for _ in range(args.warmup):
+                step()
+            torch.cuda.synchronize()
+            rec[f"norm_{mode_name}_ms"] = timed(norms, args.steps)
+            if mode_name == "auto":
+                rec["auto_picked"] = {1: "rank1", 2: "ghost", 3: "materialised"}[
+                    dp.dp_layer_norm_mode(ctx, 0)]
+                norms()
+                dp.dp_clip_factors(ctx)
+                rec["gemm_ms"] = timed(gemm, args.steps)
+                rec["step_ms"] = timed(step, args.steps)
+            dp.dp_step_destroy(ctx)
+        flops = 2.0 * w.B * w.T * d * d
+        tf = flops / (rec["gemm_ms"] * 1e-3) / 1e12
+        in_bytes = 2.0 * w.B * w.T * 2 * d
+        rec["examples_per_s"] = w.B / (rec["step_ms"] * 1e-3)
+        rec["gemm_tflops"] = tf
+        rec["gemm_frac_bf16_peak"] = tf / peaks["bf16_tflops"]
+        # the output write (+ read of A, D) bounds the clipped sum at short T
+        gemm_bytes = in_bytes + 4.0 * d * d
+        rec["gemm_gbs"] = gemm_bytes / (rec["gemm_ms"] * 1e-3) / 1e9
+        rec["gemm_frac_hbm"] = rec["gemm_gbs"] / peaks["hbm_gbs"]
+        rec["norm_gbs_inputs"] = in_bytes / (rec["norm_auto_ms"] * 1e-3) / 1e9
+        rec["norm_frac_hbm"] = rec["norm_gbs_inputs"] / peaks["hbm_gbs"]
+        if w.T > 1:
+            rec["faster_norm"] = ("ghost" if rec["norm_ghost_ms"] <= rec["norm_materialised_ms"]
+                                  else "materialised")
+        points.append(rec)
+        del A, D, out
+        torch.cuda.empty_cache()
+    line = {"metric": METRIC, "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "dtype": "bf16", "data": "synthetic (device RNG, N(0,1) bf16)",
+            "config": {"workload": "sweep: one 4096x4096 layer, B in {8,32,128}, "
+                                   "T in {1,64,512,2048}, C=1, sigma=1"},
+            "peaks": peaks, "sweep": points}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -361,6 +455,8 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="time every point of the 4096x4096 sweep instead of one workload")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -368,6 +464,9 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.sweep:
+        run_sweep(args)
         return
     if world > 1:
         import torch

@@ -182,8 +182,11 @@ dp_status dp_layer_norm_mode(const dp_ctx* ctx, int32_t layer, dp_norm_mode* mod
 
 /* Which kernels serve a layer: *norm_tc = 1 if its per-example norms run on
  * the tcgen05 tensor cores (0: CUDA cores), *sum_tc = 1 if its clipped sum
- * does.  bf16 layers use tensor cores when T is a multiple of 64 (clipped
- * sum, materialised norm) or always (Gram norm); fp32 layers never do. */
+ * does.  For bf16 layers the Gram norm always does; the clipped sum and the
+ * materialised norm do when T is a multiple of 64 or T >= 32 (each example
+ * padded to 64 positions), and for T < 32 the clipped sum runs on a
+ * pre-scaled copy of A (c_i folded into a bf16 hi + lo pair held in context
+ * scratch).  fp32 layers never use tensor cores. */
 dp_status dp_layer_path(const dp_ctx* ctx, int32_t layer, int32_t* norm_tc, int32_t* sum_tc);
 
 /* Release the context and all of its scratch; NULL is a no-op.  Waits for

@@ -50,7 +50,7 @@ struct LayerPlan {
   dp_norm_mode mode;   // resolved norm mode
   int norm_tc;         // 1: tensor-core norm kernel
   int nparts;          // partial sums per example
-  int gemm_tc;         // 1: tcgen05 clipped sum
+  int gemm_tc;         // 0: CUDA-core clipped sum, 1: tcgen05, 2: tcgen05 on a pre-scaled operand
 };
 
 struct dp_ctx {
@@ -76,6 +76,8 @@ struct dp_ctx {
   int* h_idx = nullptr;         // pinned [cap]
   float* h_rec = nullptr;       // pinned [cap][3 + L]
   int* h_flag = nullptr;        // pinned
+  void* d_prescaled = nullptr;  // pre-scaled operand of short-example layers
+  int64_t prescaled_bytes = 0;
   size_t part_bytes = 0;
   // per-step state
   std::vector<char> norm_done;
@@ -147,7 +149,14 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
       p.nparts = p.norm_tc ? dpk::tc_mat_parts(p.d_in, p.d_out)
                            : dpk::mat_simt_parts(static_cast<int>(p.d_in), static_cast<int>(p.d_out));
     }
-    p.gemm_tc = bf16 && dpk::tc_gemm_supported(cfg->T, p.d_in, p.d_out);
+    p.gemm_tc = 0;
+    if (bf16 && dpk::tc_gemm_supported(cfg->T, p.d_in, p.d_out)) {
+      p.gemm_tc = 1;
+    } else if (bf16 && dpk::tc_prescaled_supported(cfg->T, p.d_in, p.d_out)) {
+      p.gemm_tc = 2;
+      const int64_t need = dpk::tc_prescaled_scratch_bytes(cfg->B, cfg->T, p.d_in);
+      if (need > c->prescaled_bytes) c->prescaled_bytes = need;
+    }
     if (p.nparts > NP) NP = p.nparts;
   }
   c->NP = NP;
@@ -165,6 +174,8 @@ void free_scratch(dp_ctx* c) {
   cudaFreeHost(c->h_idx);
   cudaFreeHost(c->h_rec);
   cudaFreeHost(c->h_flag);
+  cudaFree(c->d_prescaled);
+  c->d_prescaled = nullptr;
   c->d_part = nullptr;
   c->d_nparts = nullptr;
   c->d_layer_sq = c->d_s = c->d_c = nullptr;
@@ -196,6 +207,7 @@ dp_status alloc_scratch(dp_ctx* c) {
   DP_ALLOC(c->d_flag, sizeof(int));
   DP_ALLOC(c->d_idx, sizeof(int) * cap);
   DP_ALLOC(c->d_rec, sizeof(float) * cap * (3 + L));
+  if (c->prescaled_bytes > 0) DP_ALLOC(c->d_prescaled, static_cast<size_t>(c->prescaled_bytes));
 #undef DP_ALLOC
   if (cudaMallocHost(reinterpret_cast<void**>(&c->h_idx), sizeof(int) * cap) != cudaSuccess ||
       cudaMallocHost(reinterpret_cast<void**>(&c->h_rec), sizeof(float) * cap * (3 + L)) !=
@@ -271,7 +283,9 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     // The norm mode may change; the partial buffer must still be large enough.
     std::vector<LayerPlan> old = c->plan;
     const int oldNP = c->NP;
+    const int64_t old_pre = c->prescaled_bytes;
     build_plan(c, cfg);
+    c->prescaled_bytes = old_pre;  // shapes are unchanged, so is the pre-scale need
     if (c->NP > oldNP) {
       c->plan = old;
       c->NP = oldNP;
@@ -391,9 +405,12 @@ dp_status dp_clipped_sum_noise(dp_ctx* c, int32_t layer, const void* A, const vo
   ep.accumulate = (flags & DP_ACCUMULATE) ? 1 : 0;
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
   cudaError_t e;
-  if (p.gemm_tc)
+  if (p.gemm_tc == 1)
     e = dpk::tc_launch_clipsum(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep, c->d_flag,
                                c->stream);
+  else if (p.gemm_tc == 2)
+    e = dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep,
+                                         c->d_flag, c->d_prescaled, c->stream);
   else
     e = dpk::launch_gemm_simt(c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, A, D, c->d_c,
                               c->B, c->T, din, dout, d_out, ep, c->stream);
@@ -444,7 +461,7 @@ dp_status dp_layer_path(const dp_ctx* c, int32_t layer, int32_t* norm_tc, int32_
   if (!c || !norm_tc || !sum_tc) return fail(DP_ERR_ARG, "NULL argument");
   if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
   *norm_tc = c->plan[layer].norm_tc;
-  *sum_tc = c->plan[layer].gemm_tc;
+  *sum_tc = c->plan[layer].gemm_tc != 0;
   return DP_OK;
 }
 

@@ -79,6 +79,8 @@ struct GemmArgs {
   int B, T, d_in, d_out;
   int n_m, n_n;
   int NP, row0;
+  int pad3d;   // 1: maps are [B][T][d] and each example's K range is padded to 64 rows
+  int d_rows;  // > 0: pre-scaled mode, D row of K row k is k % d_rows (A holds [hi; lo])
   Epilogue ep;
 };
 
@@ -89,6 +91,52 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* 
     if (globaltimer_ns() - t0 > kWaitLimitNs) {
       atomicOr(err, kErrTimeout);
       return;
+    }
+  }
+}
+
+// TMA loads of one stage: A rows m0.. (two 64-column chunks) and the D
+// columns this CTA stages, for K block kb of example ex.
+template <bool PAIR>
+__device__ __forceinline__ void issue_stage_loads(const CUtensorMap* mapA, const CUtensorMap* mapD,
+                                                  const GemmArgs& g, uint64_t* full, bool leader,
+                                                  uint8_t* sa, uint8_t* sb, int m0, int n0, int ex,
+                                                  int kb) {
+  using C = Cfg<PAIR>;
+  const int arow = ex * g.T + kb * BK;                       // row of [B*T, d]
+  const int drow = g.d_rows > 0 ? arow % g.d_rows : arow;    // pre-scaled: hi and lo share D
+  const int trow = kb * BK;                                  // 3-D maps: position in example
+  if constexpr (PAIR) {
+    // both CTAs' loads complete on the leader's full barrier
+    const uint32_t fb = mapa_shared(smem_u32(full), 0);
+    if (leader) mbar_arrive_expect_tx(full, 2 * C::STAGE_BYTES);
+    if (g.pad3d) {
+      tma_load_3d_pair(mapA, fb, sa, m0, trow, ex);
+      tma_load_3d_pair(mapA, fb, sa + CHUNK, m0 + 64, trow, ex);
+#pragma unroll
+      for (int q = 0; q < C::B_COLS / 64; ++q)
+        tma_load_3d_pair(mapD, fb, sb + q * CHUNK, n0 + 64 * q, trow, ex);
+    } else {
+      tma_load_2d_pair(mapA, fb, sa, m0, arow);
+      tma_load_2d_pair(mapA, fb, sa + CHUNK, m0 + 64, arow);
+#pragma unroll
+      for (int q = 0; q < C::B_COLS / 64; ++q)
+        tma_load_2d_pair(mapD, fb, sb + q * CHUNK, n0 + 64 * q, drow);
+    }
+  } else {
+    mbar_arrive_expect_tx(full, C::STAGE_BYTES);
+    if (g.pad3d) {
+      tma_load_3d(mapA, full, sa, m0, trow, ex);
+      tma_load_3d(mapA, full, sa + CHUNK, m0 + 64, trow, ex);
+#pragma unroll
+      for (int q = 0; q < C::B_COLS / 64; ++q)
+        tma_load_3d(mapD, full, sb + q * CHUNK, n0 + 64 * q, trow, ex);
+    } else {
+      tma_load_2d(mapA, full, sa, m0, arow);
+      tma_load_2d(mapA, full, sa + CHUNK, m0 + 64, arow);
+#pragma unroll
+      for (int q = 0; q < C::B_COLS / 64; ++q)
+        tma_load_2d(mapD, full, sb + q * CHUNK, n0 + 64 * q, drow);
     }
   }
 }
@@ -111,7 +159,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   const bool leader = rank == 0;
   const int unit = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
   const int n_units = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
-  const int kpe = g.T / BK;
+  const int kpe = (g.T + BK - 1) / BK;  // K-blocks per example
   const int n_tiles = g.n_m * g.n_n;
   volatile int* abrt = &abort_flag;
 
@@ -159,24 +207,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
             if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
             uint8_t* sa = smem + stage * C::STAGE_BYTES;
             uint8_t* sb = sa + C::A_STAGE;
-            const int krow = ex * g.T + kb * BK;
-            if constexpr (PAIR) {
-              // both CTAs' loads complete on the leader's full barrier
-              const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
-              if (leader) mbar_arrive_expect_tx(&full_bar[stage], 2 * C::STAGE_BYTES);
-              tma_load_2d_pair(&mapA, fb, sa, m0, krow);
-              tma_load_2d_pair(&mapA, fb, sa + CHUNK, m0 + 64, krow);
-#pragma unroll
-              for (int q = 0; q < C::B_COLS / 64; ++q)
-                tma_load_2d_pair(&mapD, fb, sb + q * CHUNK, n0 + 64 * q, krow);
-            } else {
-              mbar_arrive_expect_tx(&full_bar[stage], C::STAGE_BYTES);
-              tma_load_2d(&mapA, &full_bar[stage], sa, m0, krow);
-              tma_load_2d(&mapA, &full_bar[stage], sa + CHUNK, m0 + 64, krow);
-#pragma unroll
-              for (int q = 0; q < C::B_COLS / 64; ++q)
-                tma_load_2d(&mapD, &full_bar[stage], sb + q * CHUNK, n0 + 64 * q, krow);
-            }
+            issue_stage_loads<PAIR>(&mapA, &mapD, g, &full_bar[stage], leader, sa, sb, m0, n0,
+                                    ex, kb);
             ++uses[stage];
             if (++stage == STAGES) {
               stage = 0;
@@ -300,7 +332,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         tc_fence_after();
         const uint32_t tcol = t_lane + buf * BN + half * 128;
         float sq = 0.f;
-        const float ci = NORM ? 0.f : g.c[ex];
+        const float ci = NORM ? 0.f : (g.c ? g.c[ex] : 1.f);
 #pragma unroll
         for (int ch = 0; ch < 4; ++ch) {
           float v[32];
@@ -386,16 +418,23 @@ bool make_map_2d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows,
   return make_tma_bf16(m, base, 2, dims, strides, box);
 }
 
+// 3D bf16 map over [B][T][cols], box {64 cols, box_rows positions, 1 example}:
+// positions t >= T of an example read as zeros.
+bool make_map_3d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t T, uint64_t B,
+                 uint32_t box_rows) {
+  const uint64_t dims[3] = {cols, T, B};
+  const uint64_t strides[2] = {cols * 2, T * cols * 2};
+  const uint32_t box[3] = {64, box_rows, 1};
+  return make_tma_bf16(m, base, 3, dims, strides, box);
+}
+
 // CTA pairs for every layer wider than one 128-row tile.
 bool use_pair(int64_t d_in) { return d_in > BM; }
 
 template <bool NORM, bool PAIR>
-cudaError_t launch_gemm(const void* A, const void* D, GemmArgs& g, cudaStream_t s) {
+cudaError_t launch_gemm(const CUtensorMap& mA, const CUtensorMap& mD, GemmArgs& g,
+                        cudaStream_t s) {
   using C = Cfg<PAIR>;
-  CUtensorMap mA, mD;
-  const uint64_t rows = static_cast<uint64_t>(g.B) * g.T;
-  if (!make_map_2d(&mA, A, g.d_in, rows, BK) || !make_map_2d(&mD, D, g.d_out, rows, BK))
-    return cudaErrorInvalidValue;
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<NORM, PAIR>,
@@ -441,16 +480,106 @@ cudaError_t launch_gemm(const void* A, const void* D, GemmArgs& g, cudaStream_t 
   }
 }
 
+// Maps over the caller's [B][T][d] arrays: 2-D [B*T, d] when T is a multiple
+// of the K block, else 3-D with each example's positions padded to it.
+bool make_input_maps(const void* A, const void* D, GemmArgs& g, CUtensorMap* mA,
+                     CUtensorMap* mD) {
+  g.pad3d = (g.T % BK) != 0;
+  if (g.pad3d)
+    return make_map_3d(mA, A, g.d_in, g.T, g.B, BK) && make_map_3d(mD, D, g.d_out, g.T, g.B, BK);
+  const uint64_t rows = static_cast<uint64_t>(g.B) * g.T;
+  return make_map_2d(mA, A, g.d_in, rows, BK) && make_map_2d(mD, D, g.d_out, rows, BK);
+}
+
 template <bool NORM>
 cudaError_t launch_any(const void* A, const void* D, GemmArgs& g, cudaStream_t s) {
-  return use_pair(g.d_in) ? launch_gemm<NORM, true>(A, D, g, s)
-                          : launch_gemm<NORM, false>(A, D, g, s);
+  CUtensorMap mA, mD;
+  if (!make_input_maps(A, D, g, &mA, &mD)) return cudaErrorInvalidValue;
+  return use_pair(g.d_in) ? launch_gemm<NORM, true>(mA, mD, g, s)
+                          : launch_gemm<NORM, false>(mA, mD, g, s);
 }
+
+// Pre-scaled operand for short examples: rows [0, R) of A2 hold
+// hi = RN_bf16(c_i a) and rows [R, 2R) hold lo = RN_bf16(c_i a - hi) for the
+// B*T input rows (zeros in the padding rows), so hi + lo carries c_i a to
+// about 2^-16 relative and S = A2^T [D; D] needs no per-example fold.
+__global__ void k_prescale_hilo(const __nv_bfloat16* __restrict__ A, const float* __restrict__ c,
+                                int T, int64_t BT, int64_t R, int d_in,
+                                __nv_bfloat16* __restrict__ A2) {
+  const int vpr = d_in / 8;  // 16-byte vectors per row
+  const int64_t nvec = 2 * R * vpr;
+  for (int64_t v = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; v < nvec;
+       v += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t row = v / vpr;
+    const int col = static_cast<int>(v % vpr) * 8;
+    const bool lo = row >= R;
+    const int64_t k = lo ? row - R : row;
+    uint4 outv = make_uint4(0u, 0u, 0u, 0u);
+    if (k < BT) {
+      const float ci = c[k / T];
+      const uint4 in = *reinterpret_cast<const uint4*>(A + k * d_in + col);
+      const __nv_bfloat16* x = reinterpret_cast<const __nv_bfloat16*>(&in);
+      __nv_bfloat16 y[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float p = ci * __bfloat162float(x[u]);
+        const __nv_bfloat16 h = __float2bfloat16_rn(p);
+        y[u] = lo ? __float2bfloat16_rn(p - __bfloat162float(h)) : h;
+      }
+      outv = *reinterpret_cast<const uint4*>(y);
+    }
+    *reinterpret_cast<uint4*>(A2 + row * d_in + col) = outv;
+  }
+}
+
+int64_t prescale_rows(int B, int T) { return ((static_cast<int64_t>(B) * T + BK - 1) / BK) * BK; }
 
 }  // namespace
 
+// Direct path: T a multiple of 64, or T >= 32 (3-D padding wastes at most half).
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out) {
-  return T % BK == 0 && d_in % 8 == 0 && d_out % 8 == 0 && tma_encode_available();
+  return (T % BK == 0 || T >= 32) && d_in % 8 == 0 && d_out % 8 == 0 && tma_encode_available();
+}
+
+bool tc_prescaled_supported(int T, int64_t d_in, int64_t d_out) {
+  return T < 32 && d_in % 8 == 0 && d_out % 8 == 0 && tma_encode_available();
+}
+
+int64_t tc_prescaled_scratch_bytes(int B, int T, int64_t d_in) {
+  return 2 * prescale_rows(B, T) * d_in * 2;
+}
+
+cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const float* c, int B,
+                                        int T, int d_in, int d_out, float* out,
+                                        const Epilogue& ep, int* err, void* scratch,
+                                        cudaStream_t s) {
+  const int64_t BT = static_cast<int64_t>(B) * T;
+  const int64_t R = prescale_rows(B, T);
+  auto* A2 = static_cast<__nv_bfloat16*>(scratch);
+  const int64_t nvec = 2 * R * (d_in / 8);
+  int64_t blocks = (nvec + 255) / 256;
+  const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
+  if (blocks > cap) blocks = cap;
+  k_prescale_hilo<<<static_cast<int>(blocks), 256, 0, s>>>(
+      static_cast<const __nv_bfloat16*>(A), c, T, BT, R, d_in, A2);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  GemmArgs g{};
+  g.c = nullptr;  // clip factors already applied
+  g.out = out;
+  g.err = err;
+  g.B = 1;
+  g.T = static_cast<int>(2 * R);
+  g.d_in = d_in;
+  g.d_out = d_out;
+  g.d_rows = static_cast<int>(R);
+  g.ep = ep;
+  CUtensorMap mA, mD;
+  if (!make_map_2d(&mA, A2, d_in, 2 * R, BK) || !make_map_2d(&mD, D, d_out, BT, BK))
+    return cudaErrorInvalidValue;
+  g.pad3d = 0;
+  return use_pair(d_in) ? launch_gemm<false, true>(mA, mD, g, s)
+                        : launch_gemm<false, false>(mA, mD, g, s);
 }
 
 int tc_mat_parts(int64_t d_in, int64_t d_out) {

@@ -25,6 +25,15 @@ cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int 
                               int d_in, int d_out, float* out, const Epilogue& ep, int* err,
                               cudaStream_t s);
 
+// Clipped sum for short examples (T < 32): c_i folded into a bf16 hi+lo
+// split of A in scratch (tc_prescaled_scratch_bytes), then one plain GEMM.
+bool tc_prescaled_supported(int T, int64_t d_in, int64_t d_out);
+int64_t tc_prescaled_scratch_bytes(int B, int T, int64_t d_in);
+cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const float* c, int B,
+                                        int T, int d_in, int d_out, float* out,
+                                        const Epilogue& ep, int* err, void* scratch,
+                                        cudaStream_t s);
+
 // Host helpers shared by the tensor-core launchers (tc_host.cu).
 bool tma_encode_available();
 // bf16 tensor map, 128-byte swizzle, zero fill out of bounds; dims[0] innermost,

@@ -330,13 +330,21 @@ def test_noise_statistics_on_device():
 # ---------------------------------------------------------------------------
 
 TC_CASES = [
-    # (layers, B, T): every layer bf16 with T % 64 == 0, so both the clipped
-    # sum and the norms run on tcgen05
+    # (layers, B, T): bf16 layers whose clipped sum and norms run on tcgen05
     ([(200, 264)], 3, 64),               # ragged M and N tiles
     ([(8, 8), (16, 24)], 2, 64),         # tiles far smaller than one MMA
     ([(520, 1000), (1000, 136)], 2, 128),
     ([(4096, 4096)], 2, 64),             # 512 tiles > SM count: persistent loop
     ([(384, 512)], 5, 192),              # 3 K-blocks per example, T not a power of 2
+    ([(200, 520)], 3, 45),               # T padded to 64 per example (3-D maps)
+    ([(264, 136), (64, 8)], 4, 97),      # padded, ragged
+]
+
+SMALL_T_CASES = [
+    # T < 32: the clipped sum runs on the pre-scaled hi+lo operand
+    ([(264, 136)], 7, 3),
+    ([(4096, 1024)], 16, 1),
+    ([(136, 72), (72, 8)], 33, 31),
 ]
 
 
@@ -351,6 +359,22 @@ def test_tensor_core_paths(case, mode):
     assert all(n and s for n, s in res["paths"]), res["paths"]
     ref = oracle_step(w, layers, seed=5, step=1)
     assert_step_matches(res, ref, "bf16")
+
+
+@pytest.mark.parametrize("case", range(len(SMALL_T_CASES)))
+def test_small_T_prescaled_clipped_sum(case):
+    shapes, B, T = SMALL_T_CASES[case]
+    w = W.custom(f"smallT{case}", shapes, B, T, "bf16", C=0.2, sigma=0.5, d_std=0.05,
+                 wid=750 + case)
+    layers = W.make_inputs(w, seed=3)
+    res = run_gpu_step(w, layers, seed=8, step=2)
+    assert all(s for _, s in res["paths"]), res["paths"]
+    ref = oracle_step(w, layers, seed=8, step=2)
+    assert_step_matches(res, ref, "bf16")
+    nz = run_gpu_step(w, layers, flags=dp.DP_NO_NOISE, audit=False)
+    r0 = oracle_step(w, layers, noise=False)
+    for o, r in zip(nz["out"], r0["out"]):
+        assert rel_err_normwise(o, r) <= 1e-4   # hi+lo split keeps c_i a to ~2^-16
 
 
 def test_workload_paths_use_tensor_cores():
@@ -371,3 +395,31 @@ def test_ghost_and_materialised_agree_on_block_workload():
     g = run_gpu_step(w, layers, norm_mode=dp.DP_NORM_GHOST, flags=dp.DP_NO_NOISE)
     m = run_gpu_step(w, layers, norm_mode=dp.DP_NORM_MATERIALISED, flags=dp.DP_NO_NOISE)
     assert rel_err_elementwise(g["n"], m["n"]) <= 1e-4
+
+
+# ---------------------------------------------------------------------------
+# the 4096 x 4096 sweep at full size (sampled against the oracle)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("name", [w.name for w in W.SWEEP])
+def test_sweep_point_full_size(name):
+    w = W.get(name)
+    A, D = W.make_layer(w, 0, seed=0)
+    res = run_gpu_step(w, [(A, D)], seed=4, step=9)
+    rng = np.random.default_rng(w.wid)
+    ex = np.sort(rng.choice(w.B, size=min(3, w.B), replace=False))
+    n_ref = O.layer_sqnorms_ghost(W.to_f64(A[ex]), W.to_f64(D[ex]))
+    assert rel_err_elementwise(res["n"][0, ex], n_ref) <= TOL["bf16"]
+    # c_i of the sampled examples (one layer: s_i = n_i)
+    _, c_ref = O.clip_factors(n_ref[None, :], f32(w.C))
+    assert rel_err_elementwise(res["c"][ex], c_ref) <= TOL["bf16"]
+    # unclipped, noiseless sum on sampled rows: S[rows] = sum_i A_i[:, rows]^T D_i
+    wu = W.custom(name + "_unclipped", w.layers, w.B, w.T, "bf16", C=1e30, sigma=0.0,
+                  wid=w.wid)
+    resu = run_gpu_step(wu, [(A, D)], flags=dp.DP_NO_NOISE, audit=False)
+    rows = np.sort(rng.choice(4096, size=16, replace=False))
+    ones = np.ones(1)
+    S = np.zeros((rows.size, 4096))
+    for i in range(w.B):                     # the oracle's sum, one example at a time
+        S += O.clipped_sum(W.to_f64(A[i:i + 1, :, rows]), W.to_f64(D[i:i + 1]), ones)
+    assert rel_err_normwise(resu["out"][0][rows], S) <= TOL["bf16"]
