@@ -199,17 +199,18 @@ def run_ours(args, rank, world, local_rank):
 
     ev = {k: [] for k in ("norm", "clip", "gemm")}
 
+    layer_ids = list(range(L))
+
     def step(t, timed=False):
         cfg.step = t
         dp.dp_step_init(cfg, stream, ctx)
-        for l in range(L):
-            if timed:
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record(stream)
-            dp.dp_layer_norms(ctx, l, A_d[l], D_d[l])
-            if timed:
-                e1.record(stream)
-                ev["norm"].append((l, e0, e1))
+        if timed:
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+        dp.dp_layer_norms_batch(ctx, layer_ids, A_d, D_d)   # every layer, one launch
+        if timed:
+            e1.record(stream)
+            ev["norm"].append((None, e0, e1))
         if timed:
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
@@ -274,9 +275,27 @@ def run_ours(args, rank, world, local_rank):
                          "per_layer_ms": [per_step_ms("gemm", l) for l in range(L)]},
         "layer_norms": {"ms_per_step": norm_ms, "gbs_inputs_read_once": norm_gbs,
                         "frac_hbm": norm_gbs / peaks["hbm_gbs"],
-                        "per_layer_ms": [per_step_ms("norm", l) for l in range(L)]},
+                        "launches_per_step": 1},
         "clip": {"ms_per_step": per_step_ms("clip")},
     }
+
+    # standalone noise add over every layer (the DP_NOISE_ONLY call that adds
+    # the released seed's noise to a committed sum): 8 bytes per parameter
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    nts = []
+    for r in range(args.warmup + args.steps):
+        e0.record(stream)
+        for l in range(L):
+            dp.dp_clipped_sum_noise(ctx, l, None, None, outs[l], dp.DP_NOISE_ONLY)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if r >= args.warmup:
+            nts.append(e0.elapsed_time(e1))
+    noise_ms = statistics.median(nts)
+    noise_gbs = 8.0 * w.n_params / (noise_ms * 1e-3) / 1e9
+    kernels["noise_add"] = {"ms_per_step": noise_ms, "gbs": noise_gbs,
+                            "frac_hbm": noise_gbs / peaks["hbm_gbs"], "launches": L,
+                            "bytes": 8 * w.n_params}
 
     # ---- end to end through the C ABI with host buffers ----
     e2e = None
@@ -291,8 +310,7 @@ def run_ours(args, rank, world, local_rank):
                 D_d[l].copy_(D_h[l], non_blocking=True)
             cfg.step = t
             dp.dp_step_init(cfg, stream, ctx)
-            for l in range(L):
-                dp.dp_layer_norms(ctx, l, A_d[l], D_d[l])
+            dp.dp_layer_norms_batch(ctx, layer_ids, A_d, D_d)
             dp.dp_clip_factors(ctx)
             for l in range(L):
                 dp.dp_clipped_sum_noise(ctx, l, A_d[l], D_d[l], outs[l], 0)
@@ -345,7 +363,7 @@ def run_ours(args, rank, world, local_rank):
         "kernels": kernels,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": args.steps * (2 * L + 2),
+        "gpu_launches": args.steps * (L + 3),
         "clocks": clk.summary(),
     }
     print(json.dumps(line), flush=True)

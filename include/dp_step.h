@@ -137,6 +137,16 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream);
  * dp_clip_factors of this step), DP_ERR_CUDA. */
 dp_status dp_layer_norms(dp_ctx* ctx, int32_t layer, const void* A, const void* D);
 
+/* The same per-example squared norms for n listed layers at once (one call
+ * per step for the whole trainable set of Algorithm 2): layers[r] is a layer
+ * index (each at most once), A[r] and D[r] its device arrays (host arrays of
+ * n pointers).  Equivalent to dp_layer_norms on each; Gram-form tensor-core
+ * layers share kernel launches, so the work of several layers balances
+ * across the SMs.  Errors: as dp_layer_norms; nothing is launched if any
+ * argument is invalid. */
+dp_status dp_layer_norms_batch(dp_ctx* ctx, int32_t n, const int32_t* layers,
+                               const void* const* A, const void* const* D);
+
 /* Sum the per-layer norms and form the clip factors (Sec. 2.2; Algorithm 2):
  *   s_i = sum_l n_{l,i},   c_i = 1 if s_i <= C^2 else C / sqrt(s_i).
  * d_sqnorm_out [B] and d_clip_out [B] are optional device fp32 arrays that

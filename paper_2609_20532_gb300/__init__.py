@@ -23,7 +23,8 @@ __all__ = [
     "DP_NORM_AUTO", "DP_NORM_RANK1", "DP_NORM_GHOST", "DP_NORM_MATERIALISED",
     "DP_NO_NOISE", "DP_NOISE_ONLY", "DP_ACCUMULATE",
     "dp_layer", "dp_config", "make_config",
-    "dp_step_init", "dp_layer_norms", "dp_clip_factors", "dp_clipped_sum_noise",
+    "dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "dp_clip_factors",
+    "dp_clipped_sum_noise",
     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_layer_path",
     "dp_step_destroy",
     "dp_last_error", "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
@@ -43,7 +44,8 @@ STATUS_NAMES = {0: "DP_OK", 1: "DP_ERR_ARG", 2: "DP_ERR_SHAPE", 3: "DP_ERR_DTYPE
                 7: "DP_ERR_TIMEOUT", 8: "DP_ERR_OOM", 9: "DP_ERR_UNSUPPORTED"}
 
 # every symbol include/dp_step.h declares
-EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_clip_factors", "dp_clipped_sum_noise",
+EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "dp_clip_factors",
+                    "dp_clipped_sum_noise",
                     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode",
                     "dp_layer_path", "dp_step_destroy", "dp_last_error", "dp_status_string",
                     "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc"]
@@ -91,6 +93,7 @@ def lib() -> ctypes.CDLL:
     sig = {
         "dp_step_init": ([ctypes.POINTER(vp), ctypes.POINTER(dp_config), vp], i32),
         "dp_layer_norms": ([vp, i32, vp, vp], i32),
+        "dp_layer_norms_batch": ([vp, i32, vp, vp, vp], i32),
         "dp_clip_factors": ([vp, vp, vp], i32),
         "dp_clipped_sum_noise": ([vp, i32, vp, vp, vp, u32], i32),
         "dp_audit_emit": ([vp, vp, i32, vp], i32),
@@ -160,6 +163,14 @@ def dp_step_init(cfg: dp_config, stream=None, ctx: Optional[int] = None) -> int:
 
 def dp_layer_norms(ctx: int, layer: int, A, D) -> None:
     _check(lib().dp_layer_norms(ctx, layer, _ptr(A), _ptr(D)))
+
+
+def dp_layer_norms_batch(ctx: int, layers: Sequence[int], A_list, D_list) -> None:
+    n = len(layers)
+    ids = (ctypes.c_int32 * n)(*layers)
+    a = (ctypes.c_void_p * n)(*[_ptr(x) for x in A_list])
+    d = (ctypes.c_void_p * n)(*[_ptr(x) for x in D_list])
+    _check(lib().dp_layer_norms_batch(ctx, n, ids, a, d))
 
 
 def dp_clip_factors(ctx: int, sqnorm_out=None, clip_out=None) -> None:
@@ -237,10 +248,10 @@ def dp_layer_sqnorms_noalloc(A, D, B: int, T: int, d_in: int, d_out: int, dtype:
 
 
 def run_step(ctx: int, A_list, D_list, outs, flags: int = 0) -> None:
-    """The five calls of one step in order (norms of every layer, clip,
-    clipped sum + noise of every layer); audit is left to the caller."""
-    for l, (A, D) in enumerate(zip(A_list, D_list)):
-        dp_layer_norms(ctx, l, A, D)
+    """The calls of one step in order (norms of every layer in one batched
+    call, clip, clipped sum + noise of every layer); audit is left to the
+    caller."""
+    dp_layer_norms_batch(ctx, list(range(len(A_list))), A_list, D_list)
     dp_clip_factors(ctx)
     for l, (A, D) in enumerate(zip(A_list, D_list)):
         dp_clipped_sum_noise(ctx, l, A, D, outs[l], flags)

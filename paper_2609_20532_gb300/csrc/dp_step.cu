@@ -265,6 +265,32 @@ dp_status check_device() {
   return DP_OK;
 }
 
+dp_status check_norm_args(dp_ctx* c, int32_t layer, const void* A, const void* D) {
+  if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
+  if (!A || !D) return fail(DP_ERR_ARG, "A or D is NULL");
+  if (!aligned16(A) || !aligned16(D)) return fail(DP_ERR_ARG, "A and D must be 16-byte aligned");
+  if (c->clip_done) return fail(DP_ERR_ORDER, "dp_layer_norms after dp_clip_factors");
+  return DP_OK;
+}
+
+cudaError_t launch_layer_norms(dp_ctx* c, int32_t layer, const void* A, const void* D) {
+  const LayerPlan& p = c->plan[layer];
+  const dpk::InType it = c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32;
+  const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
+  const int row0 = layer * c->B;
+  if (p.mode == DP_NORM_RANK1)
+    return dpk::launch_norm_rank1(it, A, D, c->B, din, dout, c->d_part, c->NP, row0, c->stream);
+  if (p.mode == DP_NORM_GHOST)
+    return p.norm_tc ? dpk::tc_launch_ghost(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
+                                            c->d_flag, c->stream)
+                     : dpk::launch_norm_ghost_simt(it, A, D, c->B, c->T, din, dout, c->d_part,
+                                                   c->NP, row0, c->stream);
+  return p.norm_tc ? dpk::tc_launch_mat_norm(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
+                                             c->d_flag, c->stream)
+                   : dpk::launch_norm_mat_simt(it, A, D, c->B, c->T, din, dout, c->d_part, c->NP,
+                                               row0, c->stream);
+}
+
 }  // namespace
 
 extern "C" {
@@ -334,30 +360,63 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
 
 dp_status dp_layer_norms(dp_ctx* c, int32_t layer, const void* A, const void* D) {
   if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
-  if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
-  if (!A || !D) return fail(DP_ERR_ARG, "A or D is NULL");
-  if (!aligned16(A) || !aligned16(D)) return fail(DP_ERR_ARG, "A and D must be 16-byte aligned");
-  if (c->clip_done) return fail(DP_ERR_ORDER, "dp_layer_norms after dp_clip_factors");
-  const LayerPlan& p = c->plan[layer];
-  const dpk::InType it = c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32;
-  const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
-  const int row0 = layer * c->B;
-  cudaError_t e = cudaSuccess;
-  if (p.mode == DP_NORM_RANK1) {
-    e = dpk::launch_norm_rank1(it, A, D, c->B, din, dout, c->d_part, c->NP, row0, c->stream);
-  } else if (p.mode == DP_NORM_GHOST) {
-    e = p.norm_tc ? dpk::tc_launch_ghost(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
-                                         c->d_flag, c->stream)
-                  : dpk::launch_norm_ghost_simt(it, A, D, c->B, c->T, din, dout, c->d_part,
-                                                c->NP, row0, c->stream);
-  } else {
-    e = p.norm_tc ? dpk::tc_launch_mat_norm(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
-                                            c->d_flag, c->stream)
-                  : dpk::launch_norm_mat_simt(it, A, D, c->B, c->T, din, dout, c->d_part, c->NP,
-                                              row0, c->stream);
-  }
+  dp_status st = check_norm_args(c, layer, A, D);
+  if (st != DP_OK) return st;
+  cudaError_t e = launch_layer_norms(c, layer, A, D);
   if (e != cudaSuccess) return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
   c->norm_done[layer] = 1;
+  return DP_OK;
+}
+
+dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, const void* const* A,
+                               const void* const* D) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (n < 1 || n > c->L) return fail(DP_ERR_ARG, "n=%d outside 1..L", n);
+  if (!layers || !A || !D) return fail(DP_ERR_ARG, "NULL array argument");
+  std::vector<char> seen(c->L, 0);
+  for (int r = 0; r < n; ++r) {
+    dp_status st = check_norm_args(c, layers[r], A[r], D[r]);
+    if (st != DP_OK) return st;
+    if (seen[layers[r]]) return fail(DP_ERR_ARG, "layer %d listed twice", layers[r]);
+    seen[layers[r]] = 1;
+  }
+  // Gram-form tensor-core layers share launches (up to kGhostMaxLayers each);
+  // every other layer gets its own kernel.
+  std::vector<int> grp;
+  auto flush = [&]() -> cudaError_t {
+    if (grp.empty()) return cudaSuccess;
+    const void* a[dpk::kGhostMaxLayers];
+    const void* d[dpk::kGhostMaxLayers];
+    int din[dpk::kGhostMaxLayers], dout[dpk::kGhostMaxLayers], row0[dpk::kGhostMaxLayers];
+    for (size_t q = 0; q < grp.size(); ++q) {
+      const int r = grp[q], l = layers[r];
+      a[q] = A[r];
+      d[q] = D[r];
+      din[q] = static_cast<int>(c->plan[l].d_in);
+      dout[q] = static_cast<int>(c->plan[l].d_out);
+      row0[q] = l * c->B;
+    }
+    cudaError_t e = dpk::tc_launch_ghost_batch(static_cast<int>(grp.size()), a, d, din, dout, row0,
+                                               c->B, c->T, c->d_part, c->NP, c->d_flag,
+                                               c->stream);
+    grp.clear();
+    return e;
+  };
+  for (int r = 0; r < n; ++r) {
+    const LayerPlan& p = c->plan[layers[r]];
+    cudaError_t e = cudaSuccess;
+    if (p.mode == DP_NORM_GHOST && p.norm_tc) {
+      grp.push_back(r);
+      if (static_cast<int>(grp.size()) == dpk::kGhostMaxLayers) e = flush();
+    } else {
+      e = launch_layer_norms(c, layers[r], A[r], D[r]);
+    }
+    if (e != cudaSuccess)
+      return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
+  }
+  cudaError_t e = flush();
+  if (e != cudaSuccess) return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
+  for (int r = 0; r < n; ++r) c->norm_done[layers[r]] = 1;
   return DP_OK;
 }
 

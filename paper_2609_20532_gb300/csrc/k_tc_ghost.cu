@@ -1,20 +1,28 @@
-// tcgen05 Gram-form ("ghost") per-example squared norm of a dense layer:
+// tcgen05 Gram-form ("ghost") per-example squared norm of dense layers:
 //   n_i = ||A_i^T D_i||_F^2 = sum_{t,s} (A_i A_i^T)_{ts} (D_i D_i^T)_{ts}
 // (the expansion of the Frobenius norm of a sum of outer products), which
 // never forms the d_in x d_out gradient.
 //
-// Work item = (example i, 128x128 tile pair (tb <= sb) of the T x T Grams).
-// For an item the tensor core accumulates the A-Gram tile (K = d_in) and the
-// D-Gram tile (K = d_out) into two TMEM accumulators; the epilogue multiplies
-// them elementwise and reduces.  Off-diagonal tile pairs count twice, the
-// Grams being symmetric, so only the upper triangle of tile pairs is
-// computed.  Both operands are rows of A_i (or D_i): K-major, loaded by TMA
-// through a 3-D tensor map [B][T][d] so positions t >= T of an example read
-// as zeros.  Diagonal pairs load one tile and use it for both operands.
+// The T x T Grams are cut into 128-position blocks; only the upper triangle
+// of block pairs is computed (off-diagonal pairs count twice, the Grams
+// being symmetric).  A work item is a strip: one 128-row t-block against up
+// to two consecutive s-blocks (N = 256 MMAs), for one example of one layer.
+// For the strip the tensor core accumulates the A-Gram (K = d_in) and the
+// D-Gram (K = d_out) into two 256-column TMEM accumulators; the epilogue
+// multiplies them elementwise and reduces.  Strips that start on the
+// diagonal load each 128-row tile once and use it for both operands.
+// Operands are K-major rows of A_i / D_i read through 3-D tensor maps
+// [B][T][d], so positions t >= T of an example read as zeros.
 //
-// Warp roles (192 threads, persistent, TMEM double-buffered across items):
-//   warp 0 TMA producer, warp 1 TMEM allocator + MMA issuer,
-//   warps 2-5 epilogue (warp w reads TMEM lanes 32*(w%4)..+31).
+// One launch can serve up to kMaxLayers layers of a step (they share B and
+// T): the persistent grid walks a work list ordered full strips first, half
+// strips last, which keeps the SMs evenly loaded when there are only a few
+// items per SM.
+//
+// Warp roles (384 threads, one CTA per SM):
+//   warp 0 TMA producer, warp 1 TMEM allocator + MMA issuer, warps 2-3
+//   idle, warps 4-11 epilogue (warp w reads TMEM lanes 32*(w%4)..+31,
+//   column half (w-4)/4 of each 256-column accumulator).
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -29,50 +37,106 @@ namespace {
 
 using namespace tc;
 
-constexpr int GT = 128;                 // Gram tile edge (positions)
-constexpr int FK = 64;                  // features per stage (128 bytes of bf16)
-constexpr int STAGES = 6;
-constexpr int TILE_BYTES = GT * FK * 2;  // 16 KB
-constexpr int STAGE_BYTES = 2 * TILE_BYTES;
-constexpr int NUM_EPI_WARPS = 4;
-constexpr int GHOST_THREADS = 64 + 32 * NUM_EPI_WARPS;
-constexpr uint32_t TMEM_COLS = 512;     // 2 buffers x (A-Gram 128 + D-Gram 128)
+constexpr int GT = 128;                  // Gram block edge (positions)
+constexpr int FK = 64;                   // features per stage (128 bytes of bf16)
+constexpr int STAGES = 4;
+constexpr int TILE_BYTES = GT * FK * 2;  // 16 KB: one 128-position tile
+constexpr int A_OFF = 0;                 // t-tile (off-diagonal strips only)
+constexpr int B_OFF = TILE_BYTES;        // two s-tiles, 256 rows
+constexpr int STAGE_BYTES = 3 * TILE_BYTES;
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int FIRST_EPI_WARP = 4;
+constexpr int GHOST_THREADS = 128 + 32 * NUM_EPI_WARPS;
+constexpr uint32_t TMEM_COLS = 512;      // A-Gram strip 256 + D-Gram strip 256
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;
 // K-major, 128-byte swizzle: rows 128 B apart, 8-row groups 1024 B apart.
 constexpr uint32_t LBO = 16, SBO = 1024;
-constexpr uint32_t IDESC = idesc_bf16_f32(GT, GT, /*a_mn=*/0, /*b_mn=*/0);
+constexpr uint32_t IDESC_N256 = idesc_bf16_f32(GT, 2 * GT, 0, 0);
+constexpr uint32_t IDESC_N128 = idesc_bf16_f32(GT, GT, 0, 0);
 
-struct GhostArgs {
+struct GhostBatch {
+  CUtensorMap mapA[kGhostMaxLayers];
+  CUtensorMap mapD[kGhostMaxLayers];
+  int d_in[kGhostMaxLayers];
+  int d_out[kGhostMaxLayers];
+  int row0[kGhostMaxLayers];   // partial-sum row of example 0 of the layer
+  int L, B, T, nb;             // layers in this launch, examples, positions, blocks
+  int n_full, n_half;          // strips per example
   float* part;
   int* err;
-  int B, T, d_in, d_out;
-  int nb, npairs;
-  int NP, row0;
+  int NP;
 };
 
-__device__ __forceinline__ void pair_of(int pid, int nb, int& tb, int& sb) {
-  int r = 0, left = pid;
-  while (left >= nb - r) {
-    left -= nb - r;
-    ++r;
+struct Strip {
+  int layer, ex, tb, sb, ns, slot;
+};
+
+// Full strips of row tb: floor((nb - tb) / 2); a half strip ends every row
+// with an odd number of blocks left.
+__device__ __forceinline__ void full_strip(int k, int nb, int& tb, int& sb) {
+  for (int t = 0; t < nb; ++t) {
+    const int f = (nb - t) / 2;
+    if (k < f) {
+      tb = t;
+      sb = t + 2 * k;
+      return;
+    }
+    k -= f;
   }
-  tb = r;
-  sb = r + left;
+  tb = sb = 0;
+}
+__device__ __forceinline__ void half_strip(int k, int nb, int& tb, int& sb) {
+  for (int t = 0; t < nb; ++t) {
+    if ((nb - t) & 1) {
+      if (k == 0) {
+        tb = t;
+        sb = nb - 1;
+        return;
+      }
+      --k;
+    }
+  }
+  tb = sb = 0;
+}
+
+// Work list: all full strips (layer-major, then example), then all half strips.
+__device__ __forceinline__ Strip decode(int item, const GhostBatch& g) {
+  Strip s;
+  const int per_full = g.B * g.n_full;
+  const int all_full = g.L * per_full;
+  if (item < all_full) {
+    s.layer = item / per_full;
+    const int r = item % per_full;
+    s.ex = r / g.n_full;
+    const int k = r % g.n_full;
+    full_strip(k, g.nb, s.tb, s.sb);
+    s.ns = 2;
+    s.slot = k;
+  } else {
+    const int i2 = item - all_full;
+    const int per_half = g.B * g.n_half;
+    s.layer = i2 / per_half;
+    const int r = i2 % per_half;
+    s.ex = r / g.n_half;
+    const int k = r % g.n_half;
+    half_strip(k, g.nb, s.tb, s.sb);
+    s.ns = 1;
+    s.slot = g.n_full + k;
+  }
+  return s;
 }
 
 __global__ void __launch_bounds__(GHOST_THREADS, 1)
-    k_ghost_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapD,
-               const GhostArgs g) {
+    k_ghost_tc(const __grid_constant__ GhostBatch g) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  __shared__ uint64_t full_bar[STAGES], empty_bar[STAGES], tfull_bar[2], tempty_bar[2], done_bar;
+  __shared__ uint64_t full_bar[STAGES], empty_bar[STAGES], tfull_bar, tempty_bar, done_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ int abort_flag;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_items = g.B * g.npairs;
-  const int ka = (g.d_in + FK - 1) / FK, kd = (g.d_out + FK - 1) / FK;
+  const int n_items = g.L * g.B * (g.n_full + g.n_half);
   volatile int* abrt = &abort_flag;
 
   if (threadIdx.x == 0) {
@@ -80,17 +144,11 @@ __global__ void __launch_bounds__(GHOST_THREADS, 1)
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&tfull_bar[b], 1);
-      mbar_init(&tempty_bar[b], NUM_EPI_WARPS);
-    }
+    mbar_init(&tfull_bar, 1);
+    mbar_init(&tempty_bar, NUM_EPI_WARPS);
     mbar_init(&done_bar, 1);
     abort_flag = 0;
     fence_mbar_init();
-  }
-  if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&mapA);
-    tma_prefetch_desc(&mapD);
   }
   if (warp == 1) tmem_alloc(&tmem_slot, TMEM_COLS);
   tc_fence_before();
@@ -105,18 +163,23 @@ __global__ void __launch_bounds__(GHOST_THREADS, 1)
       uint32_t phase = 0;
       uint32_t uses[STAGES] = {};
       for (int item = blockIdx.x; item < n_items; item += gridDim.x) {
-        const int ex = item / g.npairs;
-        int tb, sb;
-        pair_of(item % g.npairs, g.nb, tb, sb);
-        const bool diag = tb == sb;
+        const Strip st = decode(item, g);
+        const bool diag = st.tb == st.sb;
+        const CUtensorMap* mA = &g.mapA[st.layer];
+        const CUtensorMap* mD = &g.mapD[st.layer];
+        const int ka = (g.d_in[st.layer] + FK - 1) / FK, kd = (g.d_out[st.layer] + FK - 1) / FK;
+        const uint32_t bytes = (diag ? 0 : TILE_BYTES) + st.ns * TILE_BYTES;
         for (int k = 0; k < ka + kd; ++k) {
-          const CUtensorMap* map = k < ka ? &mapA : &mapD;
+          const CUtensorMap* map = k < ka ? mA : mD;
           const int f0 = (k < ka ? k : k - ka) * FK;
           if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
-          uint8_t* st = smem + stage * STAGE_BYTES;
-          mbar_arrive_expect_tx(&full_bar[stage], diag ? TILE_BYTES : 2 * TILE_BYTES);
-          tma_load_3d(map, &full_bar[stage], st, f0, tb * GT, ex);
-          if (!diag) tma_load_3d(map, &full_bar[stage], st + TILE_BYTES, f0, sb * GT, ex);
+          uint8_t* sp = smem + stage * STAGE_BYTES;
+          mbar_arrive_expect_tx(&full_bar[stage], bytes);
+          if (!diag) tma_load_3d(map, &full_bar[stage], sp + A_OFF, f0, st.tb * GT, st.ex);
+          tma_load_3d(map, &full_bar[stage], sp + B_OFF, f0, st.sb * GT, st.ex);
+          if (st.ns == 2)
+            tma_load_3d(map, &full_bar[stage], sp + B_OFF + TILE_BYTES, f0, (st.sb + 1) * GT,
+                        st.ex);
           ++uses[stage];
           if (++stage == STAGES) {
             stage = 0;
@@ -143,26 +206,26 @@ __global__ void __launch_bounds__(GHOST_THREADS, 1)
       uint32_t phase = 0;
       int it = 0;
       for (int item = blockIdx.x; item < n_items; item += gridDim.x, ++it) {
-        int tb, sb;
-        pair_of(item % g.npairs, g.nb, tb, sb);
-        const bool diag = tb == sb;
-        const int buf = it & 1;
-        const uint32_t tph = (it >> 1) & 1;
-        if (!mbar_wait(&tempty_bar[buf], tph ^ 1, abrt, g.err)) goto mma_done;
+        const Strip st = decode(item, g);
+        const bool diag = st.tb == st.sb;
+        const uint32_t idesc = st.ns == 2 ? IDESC_N256 : IDESC_N128;
+        const int ka = (g.d_in[st.layer] + FK - 1) / FK, kd = (g.d_out[st.layer] + FK - 1) / FK;
+        if (!mbar_wait(&tempty_bar, (it & 1) ^ 1, abrt, g.err)) goto mma_done;
         tc_fence_after();
         for (int k = 0; k < ka + kd; ++k) {
           const bool is_a = k < ka;
           const int kl = is_a ? k : k - ka;
-          const uint32_t d_tmem = tmem_base + buf * 2 * GT + (is_a ? 0 : GT);
+          const uint32_t d_tmem = tmem_base + (is_a ? 0 : 2 * GT);
           if (!mbar_wait(&full_bar[stage], phase, abrt, g.err)) goto mma_done;
           tc_fence_after();
-          const uint32_t st = smem_u32(smem + stage * STAGE_BYTES);
-          const uint32_t ss = diag ? st : st + TILE_BYTES;
+          const uint32_t sp = smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sb = sp + B_OFF;
+          const uint32_t sa = diag ? sb : sp + A_OFF;
 #pragma unroll
           for (int kk = 0; kk < FK / 16; ++kk) {
-            const uint64_t ad = smem_desc_sw128(st + kk * 32, LBO, SBO);
-            const uint64_t bd = smem_desc_sw128(ss + kk * 32, LBO, SBO);
-            mma_bf16(d_tmem, ad, bd, IDESC, (kl | kk) != 0);
+            const uint64_t ad = smem_desc_sw128(sa + kk * 32, LBO, SBO);
+            const uint64_t bd = smem_desc_sw128(sb + kk * 32, LBO, SBO);
+            mma_bf16(d_tmem, ad, bd, idesc, (kl | kk) != 0);
           }
           mma_commit(&empty_bar[stage]);
           if (++stage == STAGES) {
@@ -170,10 +233,53 @@ __global__ void __launch_bounds__(GHOST_THREADS, 1)
             phase ^= 1;
           }
         }
-        mma_commit(&tfull_bar[buf]);
+        mma_commit(&tfull_bar);
       }
     mma_done:
       mma_commit(&done_bar);
+    }
+  } else if (warp >= FIRST_EPI_WARP) {
+    // ---------------- epilogue: weighted sum of GA * GD ----------------
+    const int ew = warp - FIRST_EPI_WARP;
+    const int quad = warp & 3;
+    const int half = ew >> 2;  // which 128-column half of the strip
+    const uint32_t t_lane = static_cast<uint32_t>(quad * 32) << 16;
+    int it = 0;
+    for (int item = blockIdx.x; item < n_items; item += gridDim.x, ++it) {
+      const Strip st = decode(item, g);
+      if (!mbar_wait(&tfull_bar, it & 1, abrt, g.err)) break;
+      tc_fence_after();
+      float acc = 0.f;
+      if (half < st.ns) {
+        const uint32_t ta = tmem_base + t_lane + half * GT;
+#pragma unroll
+        for (int ch = 0; ch < GT / 32; ++ch) {
+          float va[32], vd[32];
+          tmem_ld32(ta + ch * 32, va);
+          tmem_ld32(ta + 2 * GT + ch * 32, vd);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) acc = fmaf(va[i], vd[i], acc);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty_bar);
+      // the diagonal block (first half of a diagonal strip) counts once,
+      // every off-diagonal block twice
+      const float wgt = (st.tb == st.sb && half == 0) ? 1.f : 2.f;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+      if (lane == 0)
+        g.part[static_cast<int64_t>(g.row0[st.layer] + st.ex) * g.NP +
+               st.slot * NUM_EPI_WARPS + ew] = wgt * acc;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    if (lane == 0) {
       const uint64_t t0 = globaltimer_ns();
       while (!mbar_try_wait(&done_bar, 0)) {
         if (globaltimer_ns() - t0 > kWaitLimitNs) {
@@ -182,46 +288,7 @@ __global__ void __launch_bounds__(GHOST_THREADS, 1)
         }
       }
     }
-  } else {
-    // ---------------- epilogue: sum_{s} GA[t][s] * GD[t][s] ----------------
-    const int ew = warp - 2;
-    const int quad = warp & 3;
-    const uint32_t t_lane = static_cast<uint32_t>(quad * 32) << 16;
-    int it = 0;
-    for (int item = blockIdx.x; item < n_items; item += gridDim.x, ++it) {
-      const int ex = item / g.npairs;
-      const int pid = item % g.npairs;
-      int tb, sb;
-      pair_of(pid, g.nb, tb, sb);
-      const int buf = it & 1;
-      const uint32_t tph = (it >> 1) & 1;
-      if (!mbar_wait(&tfull_bar[buf], tph, abrt, g.err)) break;
-      tc_fence_after();
-      const uint32_t ta = tmem_base + t_lane + buf * 2 * GT;
-      float acc = 0.f;
-#pragma unroll
-      for (int ch = 0; ch < GT / 32; ++ch) {
-        float va[32], vd[32];
-        tmem_ld32(ta + ch * 32, va);
-        tmem_ld32(ta + GT + ch * 32, vd);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) acc = fmaf(va[i], vd[i], acc);
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty_bar[buf]);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-      if (lane == 0)
-        g.part[static_cast<int64_t>(g.row0 + ex) * g.NP + pid * NUM_EPI_WARPS + ew] =
-            (tb == sb ? 1.f : 2.f) * acc;
-    }
-  }
-
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
+    __syncwarp();
     tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
@@ -234,6 +301,14 @@ bool make_map_3d(CUtensorMap* m, const void* base, int B, int T, int d) {
   return make_tma_bf16(m, base, 3, dims, strides, box);
 }
 
+int blocks_of(int T) { return (T + GT - 1) / GT; }
+int full_strips(int nb) {
+  int f = 0;
+  for (int t = 0; t < nb; ++t) f += (nb - t) / 2;
+  return f;
+}
+int half_strips(int nb) { return (nb + 1) / 2; }
+
 }  // namespace
 
 bool tc_ghost_supported(int T, int64_t d_in, int64_t d_out) {
@@ -242,15 +317,23 @@ bool tc_ghost_supported(int T, int64_t d_in, int64_t d_out) {
 }
 
 int tc_ghost_parts(int T) {
-  const int nb = (T + GT - 1) / GT;
-  return nb * (nb + 1) / 2 * NUM_EPI_WARPS;
+  const int nb = blocks_of(T);
+  return (full_strips(nb) + half_strips(nb)) * NUM_EPI_WARPS;
 }
 
-cudaError_t tc_launch_ghost(const void* A, const void* D, int B, int T, int d_in, int d_out,
-                            float* part, int NP, int row0, int* err, cudaStream_t s) {
-  CUtensorMap mA, mD;
-  if (!make_map_3d(&mA, A, B, T, d_in) || !make_map_3d(&mD, D, B, T, d_out))
-    return cudaErrorInvalidValue;
+cudaError_t tc_launch_ghost_batch(int L, const void* const* A, const void* const* D,
+                                  const int* d_in, const int* d_out, const int* row0, int B,
+                                  int T, float* part, int NP, int* err, cudaStream_t s) {
+  if (L < 1 || L > kGhostMaxLayers) return cudaErrorInvalidValue;
+  GhostBatch g{};
+  for (int l = 0; l < L; ++l) {
+    if (!make_map_3d(&g.mapA[l], A[l], B, T, d_in[l]) ||
+        !make_map_3d(&g.mapD[l], D[l], B, T, d_out[l]))
+      return cudaErrorInvalidValue;
+    g.d_in[l] = d_in[l];
+    g.d_out[l] = d_out[l];
+    g.row0[l] = row0[l];
+  }
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e =
@@ -258,22 +341,25 @@ cudaError_t tc_launch_ghost(const void* A, const void* D, int B, int T, int d_in
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  GhostArgs g{};
-  g.part = part;
-  g.err = err;
+  g.L = L;
   g.B = B;
   g.T = T;
-  g.d_in = d_in;
-  g.d_out = d_out;
-  g.nb = (T + GT - 1) / GT;
-  g.npairs = g.nb * (g.nb + 1) / 2;
+  g.nb = blocks_of(T);
+  g.n_full = full_strips(g.nb);
+  g.n_half = half_strips(g.nb);
+  g.part = part;
+  g.err = err;
   g.NP = NP;
-  g.row0 = row0;
-  const int items = B * g.npairs;
+  const int items = L * B * (g.n_full + g.n_half);
   const int sms = device_sm_count();
   const int grid = items < sms ? items : sms;
-  k_ghost_tc<<<grid, GHOST_THREADS, SMEM_BYTES, s>>>(mA, mD, g);
+  k_ghost_tc<<<grid, GHOST_THREADS, SMEM_BYTES, s>>>(g);
   return cudaGetLastError();
+}
+
+cudaError_t tc_launch_ghost(const void* A, const void* D, int B, int T, int d_in, int d_out,
+                            float* part, int NP, int row0, int* err, cudaStream_t s) {
+  return tc_launch_ghost_batch(1, &A, &D, &d_in, &d_out, &row0, B, T, part, NP, err, s);
 }
 
 }  // namespace dpk

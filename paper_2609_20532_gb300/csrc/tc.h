@@ -9,11 +9,16 @@
 
 namespace dpk {
 
-// Gram-form per-example norms on tensor cores.
+// Gram-form per-example norms on tensor cores; one launch can serve up to
+// kGhostMaxLayers layers of a step.
+constexpr int kGhostMaxLayers = 8;
 bool tc_ghost_supported(int T, int64_t d_in, int64_t d_out);
 int tc_ghost_parts(int T);
 cudaError_t tc_launch_ghost(const void* A, const void* D, int B, int T, int d_in, int d_out,
                             float* part, int NP, int row0, int* err, cudaStream_t s);
+cudaError_t tc_launch_ghost_batch(int L, const void* const* A, const void* const* D,
+                                  const int* d_in, const int* d_out, const int* row0, int B,
+                                  int T, float* part, int NP, int* err, cudaStream_t s);
 
 // Clipped sum S = A^T diag(c) D with the noise epilogue, and the materialised
 // per-example norm that shares its main loop.

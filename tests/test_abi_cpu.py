@@ -80,6 +80,7 @@ def test_init_rejects_null_and_bad_dtype(L):
 
 def test_calls_reject_null_context(L):
     assert L.dp_layer_norms(None, 0, 16, 16) == 1
+    assert L.dp_layer_norms_batch(None, 1, None, None, None) == 1
     assert L.dp_clip_factors(None, None, None) == 1
     assert L.dp_clipped_sum_noise(None, 0, 16, 16, 16, 0) == 1
     assert L.dp_audit_emit(None, None, 0, None) == 1

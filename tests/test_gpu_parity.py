@@ -423,3 +423,42 @@ def test_sweep_point_full_size(name):
     for i in range(w.B):                     # the oracle's sum, one example at a time
         S += O.clipped_sum(W.to_f64(A[i:i + 1, :, rows]), W.to_f64(D[i:i + 1]), ones)
     assert rel_err_normwise(resu["out"][0][rows], S) <= TOL["bf16"]
+
+
+def test_batched_norms_equal_per_layer_calls():
+    """dp_layer_norms_batch gives the same norms as one dp_layer_norms per layer."""
+    w = W.get("block_bf16")
+    layers = W.make_inputs(w)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    outs = []
+    for batched in (False, True):
+        cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, audit_capacity=w.B)
+        ctx = dp.dp_step_init(cfg)
+        try:
+            if batched:
+                order = [2, 0, 3, 1]
+                dp.dp_layer_norms_batch(ctx, order, [Ad[l] for l in order], [Dd[l] for l in order])
+            else:
+                for l in range(len(layers)):
+                    dp.dp_layer_norms(ctx, l, Ad[l], Dd[l])
+            dp.dp_clip_factors(ctx)
+            recs = dp.dp_audit_emit(ctx, range(w.B), len(layers))
+        finally:
+            dp.dp_step_destroy(ctx)
+        outs.append(np.stack([r["layer_sqnorm"] for r in recs]))
+    assert np.array_equal(outs[0], outs[1])
+    ref = oracle_step(w, layers, noise=False)
+    assert rel_err_elementwise(outs[1].T, ref["n"]) <= 2e-3
+    # invalid batch: duplicate layer, nothing launched, context still usable
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        with pytest.raises(dp.DPError) as ei:
+            dp.dp_layer_norms_batch(ctx, [0, 0], [Ad[0], Ad[0]], [Dd[0], Dd[0]])
+        assert ei.value.status == 1
+        dp.dp_layer_norms_batch(ctx, [0, 1, 2, 3], Ad, Dd)
+        dp.dp_clip_factors(ctx)
+    finally:
+        dp.dp_step_destroy(ctx)
