@@ -171,6 +171,16 @@ dp_status dp_clip_factors(dp_ctx* ctx, float* d_sqnorm_out, float* d_clip_out);
 dp_status dp_clipped_sum_noise(dp_ctx* ctx, int32_t layer, const void* A, const void* D,
                                float* d_out, uint32_t flags);
 
+/* Clipped sum and noise of n listed layers (host arrays of n entries:
+ * layer indices, each at most once, and their A, D and d_out pointers; A
+ * and D may be NULL with DP_NOISE_ONLY).  Equivalent to dp_clipped_sum_noise
+ * on each; tensor-core layers share kernel launches, so the last round of
+ * output tiles of one layer overlaps the next layer's.  Errors: as
+ * dp_clipped_sum_noise; nothing is launched if any argument is invalid. */
+dp_status dp_clipped_sum_noise_batch(dp_ctx* ctx, int32_t n, const int32_t* layers,
+                                     const void* const* A, const void* const* D,
+                                     float* const* d_out, uint32_t flags);
+
 /* Audit emit: for the n example indices in h_idx (host array, each in
  * 0 .. B-1, n <= audit_capacity) copy records into h_records (host memory,
  * n * dp_audit_record_bytes(L) bytes) with layout per record:

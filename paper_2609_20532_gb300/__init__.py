@@ -24,7 +24,7 @@ __all__ = [
     "DP_NO_NOISE", "DP_NOISE_ONLY", "DP_ACCUMULATE",
     "dp_layer", "dp_config", "make_config",
     "dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "dp_clip_factors",
-    "dp_clipped_sum_noise",
+    "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_layer_path",
     "dp_step_destroy",
     "dp_last_error", "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
@@ -45,7 +45,7 @@ STATUS_NAMES = {0: "DP_OK", 1: "DP_ERR_ARG", 2: "DP_ERR_SHAPE", 3: "DP_ERR_DTYPE
 
 # every symbol include/dp_step.h declares
 EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "dp_clip_factors",
-                    "dp_clipped_sum_noise",
+                    "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
                     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode",
                     "dp_layer_path", "dp_step_destroy", "dp_last_error", "dp_status_string",
                     "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc"]
@@ -96,6 +96,7 @@ def lib() -> ctypes.CDLL:
         "dp_layer_norms_batch": ([vp, i32, vp, vp, vp], i32),
         "dp_clip_factors": ([vp, vp, vp], i32),
         "dp_clipped_sum_noise": ([vp, i32, vp, vp, vp, u32], i32),
+        "dp_clipped_sum_noise_batch": ([vp, i32, vp, vp, vp, vp, u32], i32),
         "dp_audit_emit": ([vp, vp, i32, vp], i32),
         "dp_audit_record_bytes": ([i32], i64),
         "dp_layer_norm_mode": ([vp, i32, ctypes.POINTER(i32)], i32),
@@ -181,6 +182,16 @@ def dp_clipped_sum_noise(ctx: int, layer: int, A, D, out, flags: int = 0) -> Non
     _check(lib().dp_clipped_sum_noise(ctx, layer, _ptr(A), _ptr(D), _ptr(out), flags))
 
 
+def dp_clipped_sum_noise_batch(ctx: int, layers: Sequence[int], A_list, D_list, outs,
+                               flags: int = 0) -> None:
+    n = len(layers)
+    ids = (ctypes.c_int32 * n)(*layers)
+    a = (ctypes.c_void_p * n)(*[_ptr(x) for x in A_list]) if A_list is not None else None
+    d = (ctypes.c_void_p * n)(*[_ptr(x) for x in D_list]) if D_list is not None else None
+    o = (ctypes.c_void_p * n)(*[_ptr(x) for x in outs])
+    _check(lib().dp_clipped_sum_noise_batch(ctx, n, ids, a, d, o, flags))
+
+
 def dp_audit_record_bytes(n_layers: int) -> int:
     return int(lib().dp_audit_record_bytes(n_layers))
 
@@ -251,7 +262,7 @@ def run_step(ctx: int, A_list, D_list, outs, flags: int = 0) -> None:
     """The calls of one step in order (norms of every layer in one batched
     call, clip, clipped sum + noise of every layer); audit is left to the
     caller."""
-    dp_layer_norms_batch(ctx, list(range(len(A_list))), A_list, D_list)
+    ids = list(range(len(A_list)))
+    dp_layer_norms_batch(ctx, ids, A_list, D_list)
     dp_clip_factors(ctx)
-    for l, (A, D) in enumerate(zip(A_list, D_list)):
-        dp_clipped_sum_noise(ctx, l, A, D, outs[l], flags)
+    dp_clipped_sum_noise_batch(ctx, ids, A_list, D_list, outs, flags)

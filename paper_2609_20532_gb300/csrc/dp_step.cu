@@ -291,6 +291,52 @@ cudaError_t launch_layer_norms(dp_ctx* c, int32_t layer, const void* A, const vo
                                                row0, c->stream);
 }
 
+dp_status check_sum_args(dp_ctx* c, int32_t layer, const void* A, const void* D,
+                         const float* d_out, uint32_t flags) {
+  if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
+  if (flags & ~(DP_NO_NOISE | DP_NOISE_ONLY | DP_ACCUMULATE))
+    return fail(DP_ERR_ARG, "unknown flag bits 0x%x", flags);
+  if ((flags & DP_NO_NOISE) && (flags & DP_NOISE_ONLY))
+    return fail(DP_ERR_ARG, "DP_NO_NOISE and DP_NOISE_ONLY are exclusive");
+  if (!d_out) return fail(DP_ERR_ARG, "d_out is NULL");
+  if (!aligned16(d_out)) return fail(DP_ERR_ARG, "d_out must be 16-byte aligned");
+  if (flags & DP_NOISE_ONLY) return DP_OK;
+  if (!A || !D) return fail(DP_ERR_ARG, "A or D is NULL");
+  if (!aligned16(A) || !aligned16(D)) return fail(DP_ERR_ARG, "A and D must be 16-byte aligned");
+  if (!c->clip_done) return fail(DP_ERR_ORDER, "dp_clipped_sum_noise before dp_clip_factors");
+  return DP_OK;
+}
+
+dpk::Epilogue make_epilogue(const dp_ctx* c, uint32_t flags, uint64_t p_base) {
+  dpk::Epilogue ep{};
+  ep.seed = c->seed;
+  ep.step = c->step;
+  ep.p_base = p_base;
+  ep.out_scale = c->out_scale;
+  ep.sigmaC = c->sigma * c->C;
+  ep.add_noise = (flags & DP_NO_NOISE) ? 0 : 1;
+  ep.accumulate = (flags & DP_ACCUMULATE) ? 1 : 0;
+  return ep;
+}
+
+cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const void* D,
+                               float* d_out, uint32_t flags) {
+  const LayerPlan& p = c->plan[layer];
+  const dpk::Epilogue ep = make_epilogue(c, flags, p.p_base);
+  if (flags & DP_NOISE_ONLY)
+    return dpk::launch_noise_add(d_out, p.d_in * p.d_out, p.p_base, c->seed, c->step,
+                                 c->out_scale * ep.sigmaC, c->stream);
+  const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
+  if (p.gemm_tc == 1)
+    return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep, c->d_flag,
+                                  c->stream);
+  if (p.gemm_tc == 2)
+    return dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep,
+                                            c->d_flag, c->d_prescaled, c->stream);
+  return dpk::launch_gemm_simt(c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, A, D, c->d_c,
+                               c->B, c->T, din, dout, d_out, ep, c->stream);
+}
+
 }  // namespace
 
 extern "C" {
@@ -436,43 +482,71 @@ dp_status dp_clip_factors(dp_ctx* c, float* d_sqnorm_out, float* d_clip_out) {
 dp_status dp_clipped_sum_noise(dp_ctx* c, int32_t layer, const void* A, const void* D,
                                float* d_out, uint32_t flags) {
   if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
-  if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
-  if (flags & ~(DP_NO_NOISE | DP_NOISE_ONLY | DP_ACCUMULATE))
-    return fail(DP_ERR_ARG, "unknown flag bits 0x%x", flags);
-  if ((flags & DP_NO_NOISE) && (flags & DP_NOISE_ONLY))
-    return fail(DP_ERR_ARG, "DP_NO_NOISE and DP_NOISE_ONLY are exclusive");
-  if (!d_out) return fail(DP_ERR_ARG, "d_out is NULL");
-  if (!aligned16(d_out)) return fail(DP_ERR_ARG, "d_out must be 16-byte aligned");
-  const LayerPlan& p = c->plan[layer];
-  const float sigmaC = c->sigma * c->C;
-  if (flags & DP_NOISE_ONLY) {
-    cudaError_t e = dpk::launch_noise_add(d_out, p.d_in * p.d_out, p.p_base, c->seed, c->step,
-                                          c->out_scale * sigmaC, c->stream);
-    if (e != cudaSuccess) return fail(DP_ERR_CUDA, "noise kernel: %s", cudaGetErrorString(e));
-    return DP_OK;
+  dp_status st = check_sum_args(c, layer, A, D, d_out, flags);
+  if (st != DP_OK) return st;
+  cudaError_t e = launch_clipped_sum(c, layer, A, D, d_out, flags);
+  if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clipped-sum kernel: %s", cudaGetErrorString(e));
+  return DP_OK;
+}
+
+dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers,
+                                     const void* const* A, const void* const* D,
+                                     float* const* d_out, uint32_t flags) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (n < 1 || n > c->L) return fail(DP_ERR_ARG, "n=%d outside 1..L", n);
+  if (!layers || !d_out || (!(flags & DP_NOISE_ONLY) && (!A || !D)))
+    return fail(DP_ERR_ARG, "NULL array argument");
+  std::vector<char> seen(c->L, 0);
+  for (int r = 0; r < n; ++r) {
+    const int32_t l = layers[r];
+    dp_status st = check_sum_args(c, l, (flags & DP_NOISE_ONLY) ? nullptr : A[r],
+                                  (flags & DP_NOISE_ONLY) ? nullptr : D[r], d_out[r], flags);
+    if (st != DP_OK) return st;
+    if (seen[l]) return fail(DP_ERR_ARG, "layer %d listed twice", l);
+    seen[l] = 1;
   }
-  if (!A || !D) return fail(DP_ERR_ARG, "A or D is NULL");
-  if (!aligned16(A) || !aligned16(D)) return fail(DP_ERR_ARG, "A and D must be 16-byte aligned");
-  if (!c->clip_done) return fail(DP_ERR_ORDER, "dp_clipped_sum_noise before dp_clip_factors");
-  dpk::Epilogue ep{};
-  ep.seed = c->seed;
-  ep.step = c->step;
-  ep.p_base = p.p_base;
-  ep.out_scale = c->out_scale;
-  ep.sigmaC = sigmaC;
-  ep.add_noise = (flags & DP_NO_NOISE) ? 0 : 1;
-  ep.accumulate = (flags & DP_ACCUMULATE) ? 1 : 0;
-  const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
-  cudaError_t e;
-  if (p.gemm_tc == 1)
-    e = dpk::tc_launch_clipsum(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep, c->d_flag,
-                               c->stream);
-  else if (p.gemm_tc == 2)
-    e = dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep,
-                                         c->d_flag, c->d_prescaled, c->stream);
-  else
-    e = dpk::launch_gemm_simt(c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, A, D, c->d_c,
-                              c->B, c->T, din, dout, d_out, ep, c->stream);
+  // Direct tensor-core layers with the same tile shape share launches (up to
+  // kGemmMaxLayers each); every other layer gets its own kernel.
+  std::vector<int> grp;
+  dpk::Epilogue ep = make_epilogue(c, flags, 0);
+  auto flush = [&]() -> cudaError_t {
+    if (grp.empty()) return cudaSuccess;
+    const void* a[dpk::kGemmMaxLayers];
+    const void* d[dpk::kGemmMaxLayers];
+    float* o[dpk::kGemmMaxLayers];
+    int din[dpk::kGemmMaxLayers], dout[dpk::kGemmMaxLayers];
+    uint64_t pb[dpk::kGemmMaxLayers];
+    for (size_t q = 0; q < grp.size(); ++q) {
+      const int r = grp[q];
+      const LayerPlan& p = c->plan[layers[r]];
+      a[q] = A[r];
+      d[q] = D[r];
+      o[q] = d_out[r];
+      din[q] = static_cast<int>(p.d_in);
+      dout[q] = static_cast<int>(p.d_out);
+      pb[q] = p.p_base;
+    }
+    cudaError_t e = dpk::tc_launch_clipsum_batch(static_cast<int>(grp.size()), a, d, o, din, dout,
+                                                 pb, c->d_c, c->B, c->T, ep, c->d_flag, c->stream);
+    grp.clear();
+    return e;
+  };
+  for (int r = 0; r < n; ++r) {
+    const int32_t l = layers[r];
+    const LayerPlan& p = c->plan[l];
+    cudaError_t e = cudaSuccess;
+    if (!(flags & DP_NOISE_ONLY) && p.gemm_tc == 1) {
+      if (!grp.empty() && !dpk::tc_clipsum_same_launch(c->plan[layers[grp[0]]].d_in, p.d_in))
+        e = flush();
+      grp.push_back(r);
+      if (e == cudaSuccess && static_cast<int>(grp.size()) == dpk::kGemmMaxLayers) e = flush();
+    } else {
+      e = launch_clipped_sum(c, l, (flags & DP_NOISE_ONLY) ? nullptr : A[r],
+                             (flags & DP_NOISE_ONLY) ? nullptr : D[r], d_out[r], flags);
+    }
+    if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clipped-sum kernel: %s", cudaGetErrorString(e));
+  }
+  cudaError_t e = flush();
   if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clipped-sum kernel: %s", cudaGetErrorString(e));
   return DP_OK;
 }

@@ -71,17 +71,28 @@ struct Cfg {
   static constexpr uint32_t IDESC = idesc_bf16_f32(TILE_M, BN, /*a_mn=*/1, /*b_mn=*/1);
 };
 
+// One launch serves up to kGemmMaxLayers layers of a step (same B and T):
+// their tiles form one persistent work list, so the last round of tiles is
+// shared by all layers instead of idling most of the GPU once per layer.
 struct GemmArgs {
-  const float* c;
-  float* out;
-  float* part;
+  CUtensorMap mapA[kGemmMaxLayers];
+  CUtensorMap mapD[kGemmMaxLayers];
+  float* out[kGemmMaxLayers];
+  uint64_t p_base[kGemmMaxLayers];  // global parameter index of element (0, 0)
+  int d_in[kGemmMaxLayers], d_out[kGemmMaxLayers];
+  int n_m[kGemmMaxLayers], n_n[kGemmMaxLayers];
+  int tile_start[kGemmMaxLayers + 1];
+  int L;
+  const float* c;  // clip factors [B]; nullptr: all ones (pre-scaled operand)
+  float* part;     // materialised-norm partials (L == 1)
   int* err;
-  int B, T, d_in, d_out;
-  int n_m, n_n;
+  int B, T;
   int NP, row0;
   int pad3d;   // 1: maps are [B][T][d] and each example's K range is padded to 64 rows
   int d_rows;  // > 0: pre-scaled mode, D row of K row k is k % d_rows (A holds [hi; lo])
-  Epilogue ep;
+  uint64_t seed, step;
+  float out_scale, sigmaC;
+  int add_noise, accumulate;
 };
 
 // Bounded wait used only at teardown (ignores the abort flag).
@@ -98,11 +109,12 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* 
 // TMA loads of one stage: A rows m0.. (two 64-column chunks) and the D
 // columns this CTA stages, for K block kb of example ex.
 template <bool PAIR>
-__device__ __forceinline__ void issue_stage_loads(const CUtensorMap* mapA, const CUtensorMap* mapD,
-                                                  const GemmArgs& g, uint64_t* full, bool leader,
-                                                  uint8_t* sa, uint8_t* sb, int m0, int n0, int ex,
-                                                  int kb) {
+__device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, uint64_t* full,
+                                                  bool leader, uint8_t* sa, uint8_t* sb, int m0,
+                                                  int n0, int ex, int kb) {
   using C = Cfg<PAIR>;
+  const CUtensorMap* mapA = &g.mapA[layer];
+  const CUtensorMap* mapD = &g.mapD[layer];
   const int arow = ex * g.T + kb * BK;                       // row of [B*T, d]
   const int drow = g.d_rows > 0 ? arow % g.d_rows : arow;    // pre-scaled: hi and lo share D
   const int trow = kb * BK;                                  // 3-D maps: position in example
@@ -143,8 +155,7 @@ __device__ __forceinline__ void issue_stage_loads(const CUtensorMap* mapA, const
 
 template <bool NORM, bool PAIR>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
-    k_gemm_tc(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapD,
-              const GemmArgs g) {
+    k_gemm_tc(const __grid_constant__ GemmArgs g) {
   using C = Cfg<PAIR>;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
@@ -160,7 +171,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   const int unit = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
   const int n_units = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
   const int kpe = (g.T + BK - 1) / BK;  // K-blocks per example
-  const int n_tiles = g.n_m * g.n_n;
+  const int n_tiles = g.tile_start[g.L];
   volatile int* abrt = &abort_flag;
 
   if (threadIdx.x == 0) {
@@ -177,8 +188,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&mapA);
-    tma_prefetch_desc(&mapD);
+    for (int l = 0; l < g.L; ++l) {
+      tma_prefetch_desc(&g.mapA[l]);
+      tma_prefetch_desc(&g.mapD[l]);
+    }
   }
   if (warp == 1) {
     if constexpr (PAIR)
@@ -200,15 +213,17 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       uint32_t phase = 0;
       uint32_t uses[STAGES] = {};
       for (int tile = unit; tile < n_tiles; tile += n_units) {
-        const int m0 = (tile % g.n_m) * C::TILE_M + static_cast<int>(rank) * BM;
-        const int n0 = (tile / g.n_m) * BN + (PAIR ? static_cast<int>(rank) * (BN / 2) : 0);
+        int l = 0;
+        while (tile >= g.tile_start[l + 1]) ++l;
+        const int lt = tile - g.tile_start[l];
+        const int m0 = (lt % g.n_m[l]) * C::TILE_M + static_cast<int>(rank) * BM;
+        const int n0 = (lt / g.n_m[l]) * BN + (PAIR ? static_cast<int>(rank) * (BN / 2) : 0);
         for (int ex = 0; ex < g.B; ++ex) {
           for (int kb = 0; kb < kpe; ++kb) {
             if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
             uint8_t* sa = smem + stage * C::STAGE_BYTES;
             uint8_t* sb = sa + C::A_STAGE;
-            issue_stage_loads<PAIR>(&mapA, &mapD, g, &full_bar[stage], leader, sa, sb, m0, n0,
-                                    ex, kb);
+            issue_stage_loads<PAIR>(g, l, &full_bar[stage], leader, sa, sb, m0, n0, ex, kb);
             ++uses[stage];
             if (++stage == STAGES) {
               stage = 0;
@@ -290,13 +305,16 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     // into the register accumulator (sum and noise commute), so the tile end
     // only scales and stores.
     const int qpe = (32 + g.B - 1) / g.B;
-    const Epilogue& ep = g.ep;
     for (int tile = unit; tile < n_tiles; tile += n_units) {
-      const int m0 = (tile % g.n_m) * C::TILE_M + static_cast<int>(rank) * BM;
-      const int n0 = (tile / g.n_m) * BN;
+      int l = 0;
+      while (tile >= g.tile_start[l + 1]) ++l;
+      const int lt = tile - g.tile_start[l];
+      const int d_in = g.d_in[l], d_out = g.d_out[l];
+      const int m0 = (lt % g.n_m[l]) * C::TILE_M + static_cast<int>(rank) * BM;
+      const int n0 = (lt / g.n_m[l]) * BN;
       const int j = m0 + row;
       const int k0 = n0 + half * 128;
-      const uint64_t prow = ep.p_base + static_cast<uint64_t>(j) * g.d_out;
+      const uint64_t prow = g.p_base[l] + static_cast<uint64_t>(j) * d_out;
       float S[128];
       if constexpr (!NORM) {
 #pragma unroll
@@ -304,23 +322,23 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       }
       for (int ex = 0; ex < g.B; ++ex, ++it) {
         if constexpr (!NORM) {
-          if (ep.add_noise && j < g.d_in) {
+          if (g.add_noise && j < d_in) {
             const int q_lo = ex * qpe;
             const int q_hi = q_lo + qpe < 32 ? q_lo + qpe : 32;
 #pragma unroll 1
             for (int q = q_lo; q < q_hi; ++q) {
               // p_base and d_out are multiples of 8 on this path, so the four
               // parameters prow+k .. +3 form exactly one Philox quad
-              if (k0 + 4 * q >= g.d_out) break;
-              const float4 z = gauss_quad(ep.seed, ep.step, (prow + k0 + 4 * q) >> 2);
+              if (k0 + 4 * q >= d_out) break;
+              const float4 z = gauss_quad(g.seed, g.step, (prow + k0 + 4 * q) >> 2);
               // static register indices: select the slot with a predicate
 #pragma unroll
               for (int t = 0; t < 32; ++t) {
                 if (t == q) {
-                  S[4 * t + 0] = fmaf(ep.sigmaC, z.x, S[4 * t + 0]);
-                  S[4 * t + 1] = fmaf(ep.sigmaC, z.y, S[4 * t + 1]);
-                  S[4 * t + 2] = fmaf(ep.sigmaC, z.z, S[4 * t + 2]);
-                  S[4 * t + 3] = fmaf(ep.sigmaC, z.w, S[4 * t + 3]);
+                  S[4 * t + 0] = fmaf(g.sigmaC, z.x, S[4 * t + 0]);
+                  S[4 * t + 1] = fmaf(g.sigmaC, z.y, S[4 * t + 1]);
+                  S[4 * t + 2] = fmaf(g.sigmaC, z.z, S[4 * t + 2]);
+                  S[4 * t + 3] = fmaf(g.sigmaC, z.w, S[4 * t + 3]);
                 }
               }
             }
@@ -359,23 +377,23 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
           if (lane == 0)
             g.part[static_cast<int64_t>(g.row0 + ex) * g.NP +
-                   (tile * (PAIR ? 2 : 1) + static_cast<int>(rank)) * NUM_EPI_WARPS + ew] = sq;
+                   (lt * (PAIR ? 2 : 1) + static_cast<int>(rank)) * NUM_EPI_WARPS + ew] = sq;
         }
       }
       if constexpr (!NORM) {
-        if (j < g.d_in) {
-          float* orow = g.out + static_cast<int64_t>(j) * g.d_out;
+        if (j < d_in) {
+          float* orow = g.out[l] + static_cast<int64_t>(j) * d_out;
 #pragma unroll
           for (int q = 0; q < 32; ++q) {
             const int k = k0 + 4 * q;
-            if (k < g.d_out) {
+            if (k < d_out) {
               float4 v;
-              v.x = ep.out_scale * S[4 * q + 0];
-              v.y = ep.out_scale * S[4 * q + 1];
-              v.z = ep.out_scale * S[4 * q + 2];
-              v.w = ep.out_scale * S[4 * q + 3];
+              v.x = g.out_scale * S[4 * q + 0];
+              v.y = g.out_scale * S[4 * q + 1];
+              v.z = g.out_scale * S[4 * q + 2];
+              v.w = g.out_scale * S[4 * q + 3];
               float4* o = reinterpret_cast<float4*>(orow + k);  // d_out % 8 == 0: aligned
-              if (ep.accumulate) {
+              if (g.accumulate) {
                 const float4 p = *o;
                 v.x += p.x;
                 v.y += p.y;
@@ -432,8 +450,7 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t T, ui
 bool use_pair(int64_t d_in) { return d_in > BM; }
 
 template <bool NORM, bool PAIR>
-cudaError_t launch_gemm(const CUtensorMap& mA, const CUtensorMap& mD, GemmArgs& g,
-                        cudaStream_t s) {
+cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
   using C = Cfg<PAIR>;
   static bool attr_set = false;
   if (!attr_set) {
@@ -443,9 +460,13 @@ cudaError_t launch_gemm(const CUtensorMap& mA, const CUtensorMap& mD, GemmArgs& 
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  g.n_m = (g.d_in + C::TILE_M - 1) / C::TILE_M;
-  g.n_n = (g.d_out + BN - 1) / BN;
-  const int tiles = g.n_m * g.n_n;
+  g.tile_start[0] = 0;
+  for (int l = 0; l < g.L; ++l) {
+    g.n_m[l] = (g.d_in[l] + C::TILE_M - 1) / C::TILE_M;
+    g.n_n[l] = (g.d_out[l] + BN - 1) / BN;
+    g.tile_start[l + 1] = g.tile_start[l] + g.n_m[l] * g.n_n[l];
+  }
+  const int tiles = g.tile_start[g.L];
   const int sms = device_sm_count();
   if constexpr (PAIR) {
     // persistent grid: as many pairs as can be resident at once
@@ -472,31 +493,39 @@ cudaError_t launch_gemm(const CUtensorMap& mA, const CUtensorMap& mD, GemmArgs& 
     }
     const int pairs = tiles < max_pairs ? tiles : max_pairs;
     cfg.gridDim = dim3(2 * pairs);
-    return cudaLaunchKernelEx(&cfg, k_gemm_tc<NORM, PAIR>, mA, mD, g);
+    return cudaLaunchKernelEx(&cfg, k_gemm_tc<NORM, PAIR>, g);
   } else {
     const int grid = tiles < sms ? tiles : sms;
-    k_gemm_tc<NORM, PAIR><<<grid, GEMM_THREADS, C::SMEM_BYTES, s>>>(mA, mD, g);
+    k_gemm_tc<NORM, PAIR><<<grid, GEMM_THREADS, C::SMEM_BYTES, s>>>(g);
     return cudaGetLastError();
   }
 }
 
-// Maps over the caller's [B][T][d] arrays: 2-D [B*T, d] when T is a multiple
-// of the K block, else 3-D with each example's positions padded to it.
-bool make_input_maps(const void* A, const void* D, GemmArgs& g, CUtensorMap* mA,
-                     CUtensorMap* mD) {
+// Maps over the caller's [B][T][d] arrays of layer slot l: 2-D [B*T, d] when
+// T is a multiple of the K block, else 3-D with each example's positions
+// padded to it.
+bool make_input_maps(const void* A, const void* D, GemmArgs& g, int l) {
   g.pad3d = (g.T % BK) != 0;
   if (g.pad3d)
-    return make_map_3d(mA, A, g.d_in, g.T, g.B, BK) && make_map_3d(mD, D, g.d_out, g.T, g.B, BK);
+    return make_map_3d(&g.mapA[l], A, g.d_in[l], g.T, g.B, BK) &&
+           make_map_3d(&g.mapD[l], D, g.d_out[l], g.T, g.B, BK);
   const uint64_t rows = static_cast<uint64_t>(g.B) * g.T;
-  return make_map_2d(mA, A, g.d_in, rows, BK) && make_map_2d(mD, D, g.d_out, rows, BK);
+  return make_map_2d(&g.mapA[l], A, g.d_in[l], rows, BK) &&
+         make_map_2d(&g.mapD[l], D, g.d_out[l], rows, BK);
 }
 
 template <bool NORM>
-cudaError_t launch_any(const void* A, const void* D, GemmArgs& g, cudaStream_t s) {
-  CUtensorMap mA, mD;
-  if (!make_input_maps(A, D, g, &mA, &mD)) return cudaErrorInvalidValue;
-  return use_pair(g.d_in) ? launch_gemm<NORM, true>(mA, mD, g, s)
-                          : launch_gemm<NORM, false>(mA, mD, g, s);
+cudaError_t launch_any(GemmArgs& g, cudaStream_t s) {
+  return use_pair(g.d_in[0]) ? launch_gemm<NORM, true>(g, s) : launch_gemm<NORM, false>(g, s);
+}
+
+void set_epilogue(GemmArgs& g, const Epilogue& ep) {
+  g.seed = ep.seed;
+  g.step = ep.step;
+  g.out_scale = ep.out_scale;
+  g.sigmaC = ep.sigmaC;
+  g.add_noise = ep.add_noise;
+  g.accumulate = ep.accumulate;
 }
 
 // Pre-scaled operand for short examples: rows [0, R) of A2 hold
@@ -565,21 +594,21 @@ cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const floa
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   GemmArgs g{};
+  g.L = 1;
   g.c = nullptr;  // clip factors already applied
-  g.out = out;
+  g.out[0] = out;
+  g.p_base[0] = ep.p_base;
   g.err = err;
   g.B = 1;
   g.T = static_cast<int>(2 * R);
-  g.d_in = d_in;
-  g.d_out = d_out;
+  g.d_in[0] = d_in;
+  g.d_out[0] = d_out;
   g.d_rows = static_cast<int>(R);
-  g.ep = ep;
-  CUtensorMap mA, mD;
-  if (!make_map_2d(&mA, A2, d_in, 2 * R, BK) || !make_map_2d(&mD, D, d_out, BT, BK))
+  set_epilogue(g, ep);
+  if (!make_map_2d(&g.mapA[0], A2, d_in, 2 * R, BK) || !make_map_2d(&g.mapD[0], D, d_out, BT, BK))
     return cudaErrorInvalidValue;
   g.pad3d = 0;
-  return use_pair(d_in) ? launch_gemm<false, true>(mA, mD, g, s)
-                        : launch_gemm<false, false>(mA, mD, g, s);
+  return launch_any<false>(g, s);
 }
 
 int tc_mat_parts(int64_t d_in, int64_t d_out) {
@@ -592,30 +621,51 @@ int tc_mat_parts(int64_t d_in, int64_t d_out) {
 cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d_in, int d_out,
                                float* part, int NP, int row0, int* err, cudaStream_t s) {
   GemmArgs g{};
+  g.L = 1;
   g.part = part;
   g.err = err;
   g.B = B;
   g.T = T;
-  g.d_in = d_in;
-  g.d_out = d_out;
+  g.d_in[0] = d_in;
+  g.d_out[0] = d_out;
   g.NP = NP;
   g.row0 = row0;
-  return launch_any<true>(A, D, g, s);
+  if (!make_input_maps(A, D, g, 0)) return cudaErrorInvalidValue;
+  return launch_any<true>(g, s);
+}
+
+cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
+                                    float* const* out, const int* d_in, const int* d_out,
+                                    const uint64_t* p_base, const float* c, int B, int T,
+                                    const Epilogue& ep, int* err, cudaStream_t s) {
+  if (L < 1 || L > kGemmMaxLayers) return cudaErrorInvalidValue;
+  const bool pair = use_pair(d_in[0]);
+  GemmArgs g{};
+  g.L = L;
+  g.c = c;
+  g.err = err;
+  g.B = B;
+  g.T = T;
+  set_epilogue(g, ep);
+  for (int l = 0; l < L; ++l) {
+    if (use_pair(d_in[l]) != pair) return cudaErrorInvalidValue;  // caller groups by tile shape
+    g.d_in[l] = d_in[l];
+    g.d_out[l] = d_out[l];
+    g.out[l] = out[l];
+    g.p_base[l] = p_base[l];
+    if (!make_input_maps(A[l], D[l], g, l)) return cudaErrorInvalidValue;
+  }
+  return launch_any<false>(g, s);
 }
 
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
                               int d_in, int d_out, float* out, const Epilogue& ep, int* err,
                               cudaStream_t s) {
-  GemmArgs g{};
-  g.c = c;
-  g.out = out;
-  g.err = err;
-  g.B = B;
-  g.T = T;
-  g.d_in = d_in;
-  g.d_out = d_out;
-  g.ep = ep;
-  return launch_any<false>(A, D, g, s);
+  return tc_launch_clipsum_batch(1, &A, &D, &out, &d_in, &d_out, &ep.p_base, c, B, T, ep, err, s);
+}
+
+bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_in_b) {
+  return use_pair(d_in_a) == use_pair(d_in_b);
 }
 
 }  // namespace dpk

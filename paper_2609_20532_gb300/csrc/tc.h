@@ -21,7 +21,15 @@ cudaError_t tc_launch_ghost_batch(int L, const void* const* A, const void* const
                                   int T, float* part, int NP, int* err, cudaStream_t s);
 
 // Clipped sum S = A^T diag(c) D with the noise epilogue, and the materialised
-// per-example norm that shares its main loop.
+// per-example norm that shares its main loop.  One clipped-sum launch can
+// serve up to kGemmMaxLayers layers whose tiles have the same shape
+// (tc_clipsum_same_launch).
+constexpr int kGemmMaxLayers = 8;
+bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_in_b);
+cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
+                                    float* const* out, const int* d_in, const int* d_out,
+                                    const uint64_t* p_base, const float* c, int B, int T,
+                                    const Epilogue& ep, int* err, cudaStream_t s);
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out);
 int tc_mat_parts(int64_t d_in, int64_t d_out);
 cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d_in, int d_out,

@@ -462,3 +462,35 @@ def test_batched_norms_equal_per_layer_calls():
         dp.dp_clip_factors(ctx)
     finally:
         dp.dp_step_destroy(ctx)
+
+
+def test_batched_clipped_sum_equals_per_layer_calls():
+    """dp_clipped_sum_noise_batch writes the same outputs as per-layer calls."""
+    w = W.get("block_bf16")
+    layers = W.make_inputs(w)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    res = []
+    for batched in (False, True):
+        outs = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+        cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, seed=3, step=1)
+        ctx = dp.dp_step_init(cfg)
+        try:
+            dp.dp_layer_norms_batch(ctx, [0, 1, 2, 3], Ad, Dd)
+            dp.dp_clip_factors(ctx)
+            if batched:
+                order = [3, 1, 0, 2]
+                dp.dp_clipped_sum_noise_batch(ctx, order, [Ad[l] for l in order],
+                                              [Dd[l] for l in order], [outs[l] for l in order])
+            else:
+                for l in range(4):
+                    dp.dp_clipped_sum_noise(ctx, l, Ad[l], Dd[l], outs[l])
+        finally:
+            dp.dp_step_destroy(ctx)
+        res.append([o.cpu().numpy() for o in outs])
+    for a, b in zip(*res):
+        assert np.array_equal(a, b)
+    ref = oracle_step(w, layers, seed=3, step=1)
+    for o, r in zip(res[1], ref["out"]):
+        assert rel_err_normwise(o, r) <= 2e-3
