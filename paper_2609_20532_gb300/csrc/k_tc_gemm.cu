@@ -67,7 +67,9 @@ struct Cfg {
   static constexpr int B_STAGE = B_COLS * BK * 2;           // 16 / 32 KB
   static constexpr int STAGE_BYTES = A_STAGE + B_STAGE;     // 32 / 48 KB
   static constexpr int TILE_M = PAIR ? 2 * BM : BM;
-  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;
+  // pipeline stages, then one 4 KB store-staging block per epilogue warp
+  static constexpr int STAGING = STAGES * STAGE_BYTES;
+  static constexpr int SMEM_BYTES = STAGING + NUM_EPI_WARPS * 4096 + 1024;
   static constexpr uint32_t IDESC = idesc_bf16_f32(TILE_M, BN, /*a_mn=*/1, /*b_mn=*/1);
 };
 
@@ -77,6 +79,7 @@ struct Cfg {
 struct GemmArgs {
   CUtensorMap mapA[kGemmMaxLayers];
   CUtensorMap mapD[kGemmMaxLayers];
+  CUtensorMap mapO[kGemmMaxLayers];  // fp32 outputs, 32 x 32 boxes
   float* out[kGemmMaxLayers];
   uint64_t p_base[kGemmMaxLayers];  // global parameter index of element (0, 0)
   int d_in[kGemmMaxLayers], d_out[kGemmMaxLayers];
@@ -381,32 +384,41 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
       }
       if constexpr (!NORM) {
-        if (j < d_in) {
-          float* orow = g.out[l] + static_cast<int64_t>(j) * d_out;
+        // Store through shared memory: 4 rounds of a 32 x 32 block per warp
+        // (rows of this warp's lane quadrant, 32 columns), written with the
+        // 128-byte swizzle the output tensor map uses, then sent by one TMA
+        // store (or reduce-add) that clips at the tensor bounds.
+        uint8_t* stg = smem + C::STAGING + ew * 4096;
+        const int y = m0 + quad * 32;
 #pragma unroll
-          for (int q = 0; q < 32; ++q) {
-            const int k = k0 + 4 * q;
-            if (k < d_out) {
-              float4 v;
-              v.x = g.out_scale * S[4 * q + 0];
-              v.y = g.out_scale * S[4 * q + 1];
-              v.z = g.out_scale * S[4 * q + 2];
-              v.w = g.out_scale * S[4 * q + 3];
-              float4* o = reinterpret_cast<float4*>(orow + k);  // d_out % 8 == 0: aligned
-              if (g.accumulate) {
-                const float4 p = *o;
-                v.x += p.x;
-                v.y += p.y;
-                v.z += p.z;
-                v.w += p.w;
-              }
-              *o = v;
-            }
+        for (int c4 = 0; c4 < 4; ++c4) {
+          if (lane == 0) bulk_wait_read_all();  // previous block has been read
+          __syncwarp();
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            float4 v;
+            v.x = g.out_scale * S[32 * c4 + 4 * k + 0];
+            v.y = g.out_scale * S[32 * c4 + 4 * k + 1];
+            v.z = g.out_scale * S[32 * c4 + 4 * k + 2];
+            v.w = g.out_scale * S[32 * c4 + 4 * k + 3];
+            *reinterpret_cast<float4*>(stg + lane * 128 + ((k ^ (lane & 7)) << 4)) = v;
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            if (g.accumulate)
+              tma_reduce_add_2d(&g.mapO[l], stg, k0 + 32 * c4, y);
+            else
+              tma_store_2d(&g.mapO[l], stg, k0 + 32 * c4, y);
+            bulk_commit_group();
           }
         }
       }
     }
-  epi_done:;
+  epi_done:
+    if constexpr (!NORM) {
+      if (lane == 0) bulk_wait_all();  // every output write performed before exit
+    }
   }
 
   tc_fence_before();
@@ -605,7 +617,8 @@ cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const floa
   g.d_out[0] = d_out;
   g.d_rows = static_cast<int>(R);
   set_epilogue(g, ep);
-  if (!make_map_2d(&g.mapA[0], A2, d_in, 2 * R, BK) || !make_map_2d(&g.mapD[0], D, d_out, BT, BK))
+  if (!make_map_2d(&g.mapA[0], A2, d_in, 2 * R, BK) || !make_map_2d(&g.mapD[0], D, d_out, BT, BK) ||
+      !make_tma_f32_out(&g.mapO[0], out, d_in, d_out))
     return cudaErrorInvalidValue;
   g.pad3d = 0;
   return launch_any<false>(g, s);
@@ -653,7 +666,8 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
     g.d_out[l] = d_out[l];
     g.out[l] = out[l];
     g.p_base[l] = p_base[l];
-    if (!make_input_maps(A[l], D[l], g, l)) return cudaErrorInvalidValue;
+    if (!make_input_maps(A[l], D[l], g, l) || !make_tma_f32_out(&g.mapO[l], out[l], d_in[l], d_out[l]))
+      return cudaErrorInvalidValue;
   }
   return launch_any<false>(g, s);
 }

@@ -53,6 +53,8 @@ bool tma_encode_available();
 // strides_bytes[r] is the byte stride of dimension r+1.
 bool make_tma_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
                    const uint64_t* strides_bytes, const uint32_t* box);
+// fp32 output map over [rows][cols], box 32 x 32 (128-byte rows), 128-byte swizzle.
+bool make_tma_f32_out(CUtensorMap* m, void* base, uint64_t rows, uint64_t cols);
 int device_sm_count();
 
 }  // namespace dpk

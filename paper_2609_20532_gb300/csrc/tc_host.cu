@@ -47,6 +47,18 @@ bool make_tma_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* d
          CUDA_SUCCESS;
 }
 
+bool make_tma_f32_out(CUtensorMap* m, void* base, uint64_t rows, uint64_t cols) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t d[2] = {cols, rows};
+  cuuint64_t st[1] = {cols * 4};
+  cuuint32_t b[2] = {32, 32};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, base, d, st, b, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int device_sm_count() {
   int dev = 0, n = 0;
   cudaGetDevice(&dev);
