@@ -156,6 +156,20 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
   }
 }
 
+// Tile t of a layer -> (m tile, n tile).  Grouped raster: groups of
+// kRasterM consecutive m tiles, n runs over the whole layer inside a group
+// with m fastest, so the tiles in flight at one time share an A panel of
+// kRasterM tiles that stays in L2 while the D panels stream past it.
+constexpr int kRasterM = 8;
+__device__ __forceinline__ void tile_mn(int t, int n_m, int n_n, int& mt, int& nt) {
+  const int per_group = kRasterM * n_n;
+  const int grp = t / per_group;
+  const int r = t - grp * per_group;
+  const int gm = (n_m - grp * kRasterM) < kRasterM ? (n_m - grp * kRasterM) : kRasterM;
+  mt = grp * kRasterM + r % gm;
+  nt = r / gm;
+}
+
 template <bool NORM, bool PAIR>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_gemm_tc(const __grid_constant__ GemmArgs g) {
@@ -219,8 +233,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         int l = 0;
         while (tile >= g.tile_start[l + 1]) ++l;
         const int lt = tile - g.tile_start[l];
-        const int m0 = (lt % g.n_m[l]) * C::TILE_M + static_cast<int>(rank) * BM;
-        const int n0 = (lt / g.n_m[l]) * BN + (PAIR ? static_cast<int>(rank) * (BN / 2) : 0);
+        int mt, nt;
+        tile_mn(lt, g.n_m[l], g.n_n[l], mt, nt);
+        const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
+        const int n0 = nt * BN + (PAIR ? static_cast<int>(rank) * (BN / 2) : 0);
         for (int ex = 0; ex < g.B; ++ex) {
           for (int kb = 0; kb < kpe; ++kb) {
             if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
@@ -313,8 +329,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       while (tile >= g.tile_start[l + 1]) ++l;
       const int lt = tile - g.tile_start[l];
       const int d_in = g.d_in[l], d_out = g.d_out[l];
-      const int m0 = (lt % g.n_m[l]) * C::TILE_M + static_cast<int>(rank) * BM;
-      const int n0 = (lt / g.n_m[l]) * BN;
+      int mt, nt;
+      tile_mn(lt, g.n_m[l], g.n_n[l], mt, nt);
+      const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
+      const int n0 = nt * BN;
       const int j = m0 + row;
       const int k0 = n0 + half * 128;
       const uint64_t prow = g.p_base[l] + static_cast<uint64_t>(j) * d_out;

@@ -14,10 +14,8 @@
 // Operands are K-major rows of A_i / D_i read through 3-D tensor maps
 // [B][T][d], so positions t >= T of an example read as zeros.
 //
-// One launch can serve up to kMaxLayers layers of a step (they share B and
-// T): the persistent grid walks a work list ordered full strips first, half
-// strips last, which keeps the SMs evenly loaded when there are only a few
-// items per SM.
+// One launch can serve up to kGhostMaxLayers layers of a step (they share B
+// and T), so the few items of each layer balance across all SMs.
 //
 // Warp roles (384 threads, one CTA per SM):
 //   warp 0 TMA producer, warp 1 TMEM allocator + MMA issuer, warps 2-3
@@ -99,30 +97,26 @@ __device__ __forceinline__ void half_strip(int k, int nb, int& tb, int& sb) {
   tb = sb = 0;
 }
 
-// Work list: all full strips (layer-major, then example), then all half strips.
+// Work list: layer-major, then example, then that example's strips (full
+// strips first).  The strips of one example run at about the same time and
+// share its rows in L2; with a few items per SM the largest makespan is the
+// same as for a full-strips-first order.
 __device__ __forceinline__ Strip decode(int item, const GhostBatch& g) {
   Strip s;
-  const int per_full = g.B * g.n_full;
-  const int all_full = g.L * per_full;
-  if (item < all_full) {
-    s.layer = item / per_full;
-    const int r = item % per_full;
-    s.ex = r / g.n_full;
-    const int k = r % g.n_full;
+  const int per_ex = g.n_full + g.n_half;
+  const int per_layer = g.B * per_ex;
+  s.layer = item / per_layer;
+  const int r = item - s.layer * per_layer;
+  s.ex = r / per_ex;
+  const int k = r - s.ex * per_ex;
+  if (k < g.n_full) {
     full_strip(k, g.nb, s.tb, s.sb);
     s.ns = 2;
-    s.slot = k;
   } else {
-    const int i2 = item - all_full;
-    const int per_half = g.B * g.n_half;
-    s.layer = i2 / per_half;
-    const int r = i2 % per_half;
-    s.ex = r / g.n_half;
-    const int k = r % g.n_half;
-    half_strip(k, g.nb, s.tb, s.sb);
+    half_strip(k - g.n_full, g.nb, s.tb, s.sb);
     s.ns = 1;
-    s.slot = g.n_full + k;
   }
+  s.slot = k;
   return s;
 }
 
