@@ -278,25 +278,35 @@ __global__ void __launch_bounds__(256) k_noise_add(float* __restrict__ out, int6
   const uint64_t q_last = (p_base + n - 1) >> 2;
   const int64_t nq = static_cast<int64_t>(q_last - q_first + 1);
   const bool vec = ((p_base & 3) == 0) && ((reinterpret_cast<uintptr_t>(out) & 15) == 0);
+  // Two quads per iteration, a grid-stride apart: two independent Philox /
+  // Box-Muller chains give the scheduler instruction-level parallelism.
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < nq;
-       g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const uint64_t q = q_first + g;
-    const float4 z = gauss_quad(seed, step, q);
-    const int64_t e0 = static_cast<int64_t>(4 * q) - static_cast<int64_t>(p_base);
-    if (vec && e0 + 3 < n) {
-      float4* o = reinterpret_cast<float4*>(out + e0);
-      float4 v = *o;
-      v.x = fmaf(scale, z.x, v.x);
-      v.y = fmaf(scale, z.y, v.y);
-      v.z = fmaf(scale, z.z, v.z);
-      v.w = fmaf(scale, z.w, v.w);
-      *o = v;
-    } else {
-      const float zv[4] = {z.x, z.y, z.z, z.w};
+       g += 2 * stride) {
+    const bool has_b = g + stride < nq;
+    const float4 za = gauss_quad(seed, step, q_first + g);
+    const float4 zb = gauss_quad(seed, step, q_first + (has_b ? g + stride : g));
 #pragma unroll
-      for (int w = 0; w < 4; ++w) {
-        const int64_t e = e0 + w;
-        if (e >= 0 && e < n) out[e] = fmaf(scale, zv[w], out[e]);
+    for (int h = 0; h < 2; ++h) {
+      if (h == 1 && !has_b) break;
+      const uint64_t q = q_first + g + h * stride;
+      const float4 z = h == 0 ? za : zb;
+      const int64_t e0 = static_cast<int64_t>(4 * q) - static_cast<int64_t>(p_base);
+      if (vec && e0 + 3 < n) {
+        float4* o = reinterpret_cast<float4*>(out + e0);
+        float4 v = *o;
+        v.x = fmaf(scale, z.x, v.x);
+        v.y = fmaf(scale, z.y, v.y);
+        v.z = fmaf(scale, z.z, v.z);
+        v.w = fmaf(scale, z.w, v.w);
+        *o = v;
+      } else {
+        const float zv[4] = {z.x, z.y, z.z, z.w};
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          const int64_t e = e0 + w;
+          if (e >= 0 && e < n) out[e] = fmaf(scale, zv[w], out[e]);
+        }
       }
     }
   }
