@@ -104,6 +104,24 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """Largest value of x over all ranks (one all-reduce), x itself at world 1."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64,
+                     device=device if device is not None else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(examples_per_rank: int, world: int, seconds_per_step: float) -> float:
+    """Whole-job examples/s: every rank runs its own replica of the step, so the
+    job processes world * B examples per (slowest-rank) step time."""
+    return world * examples_per_rank / seconds_per_step
+
+
 def _kernel_sha(path):
     return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
 
@@ -246,14 +264,9 @@ def run_ours(args, rank, world, local_rank):
         torch.cuda.synchronize()
     barrier()
     torch.cuda.synchronize()
-    ms = start.elapsed_time(stop)
-    if world > 1:
-        import torch.distributed as dist
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(start.elapsed_time(stop), world, dev)
     ms_step = ms / args.steps
-    value = world * w.B / (ms_step * 1e-3)
+    value = replica_throughput(w.B, world, ms_step * 1e-3)
 
     def per_step_ms(kind, layer=None):
         tot = sum(e0.elapsed_time(e1) for l, e0, e1 in ev[kind] if layer is None or l == layer)
@@ -358,13 +371,8 @@ def run_ours(args, rank, world, local_rank):
         t0 = time.perf_counter()
         run(k, 1000)
         torch.cuda.synchronize()                   # last outputs are in host memory
-        wall = (time.perf_counter() - t0) / k
-        if world > 1:
-            import torch.distributed as dist
-            tt = torch.tensor([wall], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            wall = float(tt.item())
-        e2e = {"value": world * w.B / wall, "unit": UNIT, "ms_per_step": 1e3 * wall,
+        wall = max_over_ranks((time.perf_counter() - t0) / k, world, dev)
+        e2e = {"value": replica_throughput(w.B, world, wall), "unit": UNIT, "ms_per_step": 1e3 * wall,
                "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes + rec_bytes,
                "steps": k, "overlap": "double-buffered copies on separate streams"}
 

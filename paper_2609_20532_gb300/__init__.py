@@ -13,7 +13,7 @@ from __future__ import annotations
 
 import ctypes
 import os
-from typing import Iterable, List, Optional, Sequence
+from typing import Iterable, Optional, Sequence
 
 import numpy as np
 
@@ -25,7 +25,7 @@ __all__ = [
     "dp_layer", "dp_config", "make_config",
     "dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "dp_clip_factors",
     "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
-    "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_layer_path",
+    "dp_audit_emit", "audit_dtype", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_layer_path",
     "dp_step_destroy",
     "dp_last_error", "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
     "EXPORTED_SYMBOLS",
@@ -196,24 +196,21 @@ def dp_audit_record_bytes(n_layers: int) -> int:
     return int(lib().dp_audit_record_bytes(n_layers))
 
 
-def dp_audit_emit(ctx: int, idx: Iterable[int], n_layers: int) -> List[dict]:
-    """Records for the listed examples: dicts with example, total_sqnorm,
-    clip_factor and layer_sqnorm (numpy [L])."""
+def audit_dtype(n_layers: int) -> np.dtype:
+    """numpy layout of one audit record (12 + 4 L bytes, see dp_step.h)."""
+    return np.dtype([("example", "<i4"), ("total_sqnorm", "<f4"), ("clip_factor", "<f4"),
+                     ("layer_sqnorm", "<f4", (n_layers,))])
+
+
+def dp_audit_emit(ctx: int, idx: Iterable[int], n_layers: int) -> np.ndarray:
+    """Records for the listed examples as a numpy structured array with fields
+    example, total_sqnorm, clip_factor and layer_sqnorm [L]."""
     idx = np.ascontiguousarray(np.asarray(list(idx), dtype=np.int32))
     n = int(idx.size)
-    words = 3 + n_layers
-    buf = np.zeros(max(n, 1) * words, dtype=np.float32)
-    st = lib().dp_audit_emit(ctx, idx.ctypes.data if n else None, n, buf.ctypes.data)
-    if st not in (DP_OK, 5):
-        _check(st)
-    recs = []
-    for r in range(n):
-        w = buf[r * words:(r + 1) * words]
-        recs.append({"example": int(w[:1].view(np.int32)[0]), "total_sqnorm": float(w[1]),
-                     "clip_factor": float(w[2]), "layer_sqnorm": w[3:].astype(np.float64)})
-    if st != DP_OK:
-        _check(st)
-    return recs
+    recs = np.zeros(max(n, 1), dtype=audit_dtype(n_layers))
+    st = lib().dp_audit_emit(ctx, idx.ctypes.data if n else None, n, recs.ctypes.data)
+    _check(st)
+    return recs[:n]
 
 
 def dp_layer_norm_mode(ctx: int, layer: int) -> int:

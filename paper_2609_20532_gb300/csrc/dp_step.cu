@@ -560,8 +560,8 @@ dp_status dp_audit_emit(dp_ctx* c, const int32_t* h_idx, int32_t n, void* h_reco
   for (int r = 0; r < n; ++r)
     if (h_idx[r] < 0 || h_idx[r] >= c->B)
       return fail(DP_ERR_ARG, "audit index %d out of range 0..%d", h_idx[r], c->B - 1);
-  // Staging buffers are reused by every call: wait for the previous user.
-  DP_CUDA(cudaStreamSynchronize(c->stream));
+  // The staging buffers are free here: every call synchronises before it
+  // returns, so no earlier copy can still be using them.
   const size_t rec_words = static_cast<size_t>(3 + c->L);
   if (n > 0) {
     std::memcpy(c->h_idx, h_idx, sizeof(int) * n);

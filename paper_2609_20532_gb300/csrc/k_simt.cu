@@ -135,24 +135,27 @@ __global__ void __launch_bounds__(256) k_norm_ghost_simt(const TIn* __restrict__
 }
 
 // ---------------------------------------------------------------------------
-// FFMA GEMM over positions: tile 128 (d_in) x 128 (d_out), K-chunks of 16.
+// FFMA GEMM over positions: tile TB (d_in) x TB (d_out), K-chunks of 16,
+// 256 threads with (TB/16) x (TB/16) outputs each.
 // CLIPSUM: S = sum_k c[k / T] A[k, :]^T D[k, :] over all B*T rows, + epilogue.
 // NORM:    per example (blockIdx.z), G tile = A_i^T D_i, writes sum of squares.
 // ---------------------------------------------------------------------------
 constexpr int SB = 128, SK = 16;
 
-template <typename TIn, bool NORM>
+template <typename TIn, bool NORM, int TB>
 __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
                                                    const TIn* __restrict__ D,
                                                    const float* __restrict__ cvec, int T, int B,
                                                    int d_in, int d_out, float* __restrict__ out,
                                                    Epilogue ep, float* __restrict__ part, int NP,
                                                    int row0) {
-  __shared__ __align__(16) float As[SK][SB];
-  __shared__ __align__(16) float Ds[SK][SB];
+  constexpr int MT = TB / 16;  // outputs per thread along each axis
+  constexpr int NH = MT / 4;   // 4-wide groups per thread along each axis
+  __shared__ __align__(16) float As[SK][TB];
+  __shared__ __align__(16) float Ds[SK][TB];
   __shared__ float red[32];
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
-  const int j0 = blockIdx.y * SB, k0 = blockIdx.x * SB;
+  const int j0 = blockIdx.y * TB, k0 = blockIdx.x * TB;
   int64_t K;
   if (NORM) {
     const int64_t i = blockIdx.z;
@@ -162,12 +165,12 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
   } else {
     K = static_cast<int64_t>(B) * T;
   }
-  float acc[8][8] = {};
+  float acc[MT][MT] = {};
   for (int64_t kk = 0; kk < K; kk += SK) {
 #pragma unroll
-    for (int r = 0; r < (SK * SB) / 256; ++r) {
+    for (int r = 0; r < (SK * TB) / 256; ++r) {
       const int e = tid + 256 * r;
-      const int row = e / SB, col = e % SB;
+      const int row = e / TB, col = e % TB;
       const int64_t kr = kk + row;
       const int j = j0 + col, k = k0 + col;
       float va = 0.f, vd = 0.f;
@@ -184,16 +187,18 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
     __syncthreads();
 #pragma unroll
     for (int q = 0; q < SK; ++q) {
-      const float4 a0 = *reinterpret_cast<const float4*>(&As[q][ty * 4]);
-      const float4 a1 = *reinterpret_cast<const float4*>(&As[q][64 + ty * 4]);
-      const float4 b0 = *reinterpret_cast<const float4*>(&Ds[q][tx * 4]);
-      const float4 b1 = *reinterpret_cast<const float4*>(&Ds[q][64 + tx * 4]);
-      const float av[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-      const float bv[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+      float av[MT], bv[MT];
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
+      for (int h = 0; h < NH; ++h) {
+        const float4 a = *reinterpret_cast<const float4*>(&As[q][h * 64 + ty * 4]);
+        const float4 b = *reinterpret_cast<const float4*>(&Ds[q][h * 64 + tx * 4]);
+        av[4 * h + 0] = a.x; av[4 * h + 1] = a.y; av[4 * h + 2] = a.z; av[4 * h + 3] = a.w;
+        bv[4 * h + 0] = b.x; bv[4 * h + 1] = b.y; bv[4 * h + 2] = b.z; bv[4 * h + 3] = b.w;
+      }
 #pragma unroll
-        for (int v = 0; v < 8; ++v) acc[u][v] = fmaf(av[u], bv[v], acc[u][v]);
+      for (int u = 0; u < MT; ++u)
+#pragma unroll
+        for (int v = 0; v < MT; ++v) acc[u][v] = fmaf(av[u], bv[v], acc[u][v]);
     }
     __syncthreads();
   }
@@ -201,9 +206,9 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
   if constexpr (NORM) {
     float sq = 0.f;
 #pragma unroll
-    for (int u = 0; u < 8; ++u)
+    for (int u = 0; u < MT; ++u)
 #pragma unroll
-      for (int v = 0; v < 8; ++v) sq = fmaf(acc[u][v], acc[u][v], sq);  // padding is zero
+      for (int v = 0; v < MT; ++v) sq = fmaf(acc[u][v], acc[u][v], sq);  // padding is zero
     sq = block_sum(sq, red);
     if (tid == 0) {
       const int tile = blockIdx.y * gridDim.x + blockIdx.x;
@@ -211,28 +216,28 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
     }
   } else {
 #pragma unroll
-  for (int u = 0; u < 8; ++u) {
-    const int j = j0 + (u < 4 ? ty * 4 + u : 64 + ty * 4 + (u - 4));
-    if (j >= d_in) continue;
+    for (int u = 0; u < MT; ++u) {
+      const int j = j0 + (u / 4) * 64 + ty * 4 + (u % 4);
+      if (j >= d_in) continue;
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int kb = k0 + h * 64 + tx * 4;
-      if (kb >= d_out) continue;
-      float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-      const uint64_t p0 = ep.p_base + static_cast<uint64_t>(j) * d_out + kb;
-      if (ep.add_noise) z = gauss4_at(ep.seed, ep.step, p0);
-      const float zv[4] = {z.x, z.y, z.z, z.w};
-      float* o = out + static_cast<int64_t>(j) * d_out;
+      for (int h = 0; h < NH; ++h) {
+        const int kb = k0 + h * 64 + tx * 4;
+        if (kb >= d_out) continue;
+        float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+        const uint64_t p0 = ep.p_base + static_cast<uint64_t>(j) * d_out + kb;
+        if (ep.add_noise) z = gauss4_at(ep.seed, ep.step, p0);
+        const float zv[4] = {z.x, z.y, z.z, z.w};
+        float* o = out + static_cast<int64_t>(j) * d_out;
 #pragma unroll
-      for (int v = 0; v < 4; ++v) {
-        const int k = kb + v;
-        if (k < d_out) {
-          const float val = ep.out_scale * fmaf(ep.sigmaC, zv[v], acc[u][h * 4 + v]);
-          o[k] = ep.accumulate ? o[k] + val : val;
+        for (int v = 0; v < 4; ++v) {
+          const int k = kb + v;
+          if (k < d_out) {
+            const float val = ep.out_scale * fmaf(ep.sigmaC, zv[v], acc[u][h * 4 + v]);
+            o[k] = ep.accumulate ? o[k] + val : val;
+          }
         }
       }
     }
-  }
   }
 }
 
@@ -404,11 +409,11 @@ cudaError_t launch_norm_mat_simt(InType t, const void* A, const void* D, int B, 
   const dim3 grid((d_out + SB - 1) / SB, (d_in + SB - 1) / SB, B);
   Epilogue ep{};
   if (t == IN_F32)
-    k_gemm_simt<float, true><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
-                                                   static_cast<const float*>(D), nullptr, T, B,
-                                                   d_in, d_out, nullptr, ep, part, NP, row0);
+    k_gemm_simt<float, true, SB><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
+                                                       static_cast<const float*>(D), nullptr, T,
+                                                       B, d_in, d_out, nullptr, ep, part, NP, row0);
   else
-    k_gemm_simt<__nv_bfloat16, true><<<grid, 256, 0, s>>>(
+    k_gemm_simt<__nv_bfloat16, true, SB><<<grid, 256, 0, s>>>(
         static_cast<const __nv_bfloat16*>(A), static_cast<const __nv_bfloat16*>(D), nullptr, T,
         B, d_in, d_out, nullptr, ep, part, NP, row0);
   return cudaGetLastError();
@@ -422,17 +427,28 @@ cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_np
   return cudaGetLastError();
 }
 
-cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float* c, int B, int T,
-                             int d_in, int d_out, float* out, const Epilogue& ep, cudaStream_t s) {
-  const dim3 grid((d_out + SB - 1) / SB, (d_in + SB - 1) / SB, 1);
+template <int TB>
+void launch_gemm_simt_tb(InType t, const void* A, const void* D, const float* c, int B, int T,
+                         int d_in, int d_out, float* out, const Epilogue& ep, cudaStream_t s) {
+  const dim3 grid((d_out + TB - 1) / TB, (d_in + TB - 1) / TB, 1);
   if (t == IN_F32)
-    k_gemm_simt<float, false><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
-                                                    static_cast<const float*>(D), c, T, B, d_in,
-                                                    d_out, out, ep, nullptr, 0, 0);
+    k_gemm_simt<float, false, TB><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
+                                                        static_cast<const float*>(D), c, T, B,
+                                                        d_in, d_out, out, ep, nullptr, 0, 0);
   else
-    k_gemm_simt<__nv_bfloat16, false><<<grid, 256, 0, s>>>(
+    k_gemm_simt<__nv_bfloat16, false, TB><<<grid, 256, 0, s>>>(
         static_cast<const __nv_bfloat16*>(A), static_cast<const __nv_bfloat16*>(D), c, T, B,
         d_in, d_out, out, ep, nullptr, 0, 0);
+}
+
+cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float* c, int B, int T,
+                             int d_in, int d_out, float* out, const Epilogue& ep, cudaStream_t s) {
+  // 128 x 128 tiles when they alone fill the GPU twice, else 64 x 64 tiles
+  const int64_t big = static_cast<int64_t>((d_out + SB - 1) / SB) * ((d_in + SB - 1) / SB);
+  if (big >= 2 * 152)
+    launch_gemm_simt_tb<SB>(t, A, D, c, B, T, d_in, d_out, out, ep, s);
+  else
+    launch_gemm_simt_tb<64>(t, A, D, c, B, T, d_in, d_out, out, ep, s);
   return cudaGetLastError();
 }
 

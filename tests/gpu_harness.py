@@ -51,10 +51,10 @@ def run_gpu_step(w: W.Workload, layers, seed=0, step=0, out_scale=1.0, flags=0,
     res = {"out": [o.cpu().numpy() for o in outs], "s": s_dev.cpu().numpy(),
            "c": c_dev.cpu().numpy(), "modes": modes, "paths": paths}
     if recs is not None:
-        res["n"] = np.stack([r["layer_sqnorm"] for r in recs], axis=1)
-        res["rec_s"] = np.array([r["total_sqnorm"] for r in recs])
-        res["rec_c"] = np.array([r["clip_factor"] for r in recs])
-        res["rec_i"] = np.array([r["example"] for r in recs])
+        res["n"] = recs["layer_sqnorm"].astype(np.float64).T
+        res["rec_s"] = recs["total_sqnorm"].astype(np.float64)
+        res["rec_c"] = recs["clip_factor"].astype(np.float64)
+        res["rec_i"] = recs["example"].astype(np.int64)
     return res
 
 

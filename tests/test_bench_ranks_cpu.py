@@ -1,0 +1,60 @@
+"""Multi-rank bookkeeping of bench.py on CPU (gloo, world size 2).
+
+The step has no data-path collective: every rank runs its own replica, the
+job's time is the slowest rank's and its throughput counts every rank's
+examples.  This checks that host logic with two gloo processes."""
+
+import os
+import socket
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, out):
+    sys.path.insert(0, ROOT)
+    import torch.distributed as dist
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    import bench
+    local = [2.5, 4.0][rank]                      # per-rank step time (ms)
+    m = bench.max_over_ranks(local, world)
+    v = bench.replica_throughput(16, world, m * 1e-3)
+    out[rank] = (m, v)
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_take_the_slowest_step_and_count_all_examples():
+    world = 2
+    port = _free_port()
+    ctx = mp.get_context("spawn")
+    mgr = ctx.Manager()
+    out = mgr.dict()
+    procs = [ctx.Process(target=_worker, args=(r, world, port, out)) for r in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=120)
+        assert p.exitcode == 0
+    for r in range(world):
+        m, v = out[r]
+        assert m == 4.0                          # slowest rank
+        assert v == pytest.approx(2 * 16 / 4.0e-3)
+
+
+def test_single_rank_is_identity():
+    sys.path.insert(0, ROOT)
+    import bench
+    assert bench.max_over_ranks(3.0, 1) == 3.0
+    assert bench.replica_throughput(16, 1, 2e-3) == pytest.approx(8000.0)

@@ -447,7 +447,7 @@ def test_batched_norms_equal_per_layer_calls():
             recs = dp.dp_audit_emit(ctx, range(w.B), len(layers))
         finally:
             dp.dp_step_destroy(ctx)
-        outs.append(np.stack([r["layer_sqnorm"] for r in recs]))
+        outs.append(recs["layer_sqnorm"].astype(np.float64))
     assert np.array_equal(outs[0], outs[1])
     ref = oracle_step(w, layers, noise=False)
     assert rel_err_elementwise(outs[1].T, ref["n"]) <= 2e-3
@@ -494,3 +494,27 @@ def test_batched_clipped_sum_equals_per_layer_calls():
     ref = oracle_step(w, layers, seed=3, step=1)
     for o, r in zip(res[1], ref["out"]):
         assert rel_err_normwise(o, r) <= 2e-3
+
+
+# ---------------------------------------------------------------------------
+# the paper's own acceptance test on the commitment (Sec. 6.2, Algorithm 1)
+# ---------------------------------------------------------------------------
+
+TAU_ABS = 1.60e-3   # tightest LLM routing threshold of the verifier table (App. E), units of C
+
+
+@pytest.mark.parametrize("name", ["single_fp32", "mlp_fp32", "block_bf16"])
+def test_commitment_passes_the_verifier_body_path(name):
+    """The averaged commitment g = S/B passes the always-on structural check
+    ||g|| <= C(1 + 1e-4) and lands in the FP32 body path of Algorithm 1:
+    z = ||g_GPU - g_ref||_2 / C <= tau_abs against the fp64 recomputation."""
+    w = W.get(name)
+    layers = W.make_inputs(w, seed=0)
+    res = run_gpu_step(w, layers, out_scale=1.0 / w.B, flags=dp.DP_NO_NOISE, audit=False)
+    ref = oracle_step(w, layers, out_scale=1.0 / w.B, noise=False)
+    g_gpu = np.concatenate([o.astype(np.float64).ravel() for o in res["out"]])
+    g_ref = np.concatenate([r.ravel() for r in ref["out"]])
+    C = f32(w.C)
+    assert np.linalg.norm(g_gpu) <= C * (1 + 1e-4)
+    z = np.linalg.norm(g_gpu - g_ref) / C
+    assert z <= TAU_ABS, z

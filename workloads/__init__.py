@@ -156,11 +156,13 @@ def make_inputs(w: Workload, seed: int = 0) -> List[Tuple[torch.Tensor, torch.Te
 
 
 def audit_indices(w: Workload, seed: int = 0, frac: float | None = None) -> np.ndarray:
-    """ceil(frac * B) distinct example indices (sorted), drawn with kind 2.
+    """ceil(frac * B) distinct example indices (sorted), drawn with kind 2;
+    frac defaults to the workload's audit fraction, else 5%.
 
     In the paper the TEE picks what to audit from hidden randomness; here the
     caller's seeded draw stands in for it."""
-    frac = w.audit_frac if frac is None else frac
+    if frac is None:
+        frac = w.audit_frac if w.audit_frac > 0 else 0.05
     k = max(1, math.ceil(frac * w.B)) if frac > 0 else w.B
     rng = np.random.default_rng(np.random.SeedSequence([seed, w.wid, 0, 2]))
     return np.sort(rng.choice(w.B, size=min(k, w.B), replace=False)).astype(np.int32)
