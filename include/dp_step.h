@@ -200,6 +200,15 @@ int64_t dp_audit_record_bytes(int32_t n_layers);
 /* Norm mode chosen for a layer (resolves DP_NORM_AUTO). */
 dp_status dp_layer_norm_mode(const dp_ctx* ctx, int32_t layer, dp_norm_mode* mode_out);
 
+/* Replace the noise key (seed, step) without enqueuing any work, for CUDA
+ * graphs: a step captured from dp_step_init on loads the key from mapped
+ * pinned host memory when the graph runs, so calling this between replays
+ * keys each replay (Algorithm 3's released seed s_noise,t).  The caller must not
+ * call it while a previous replay that copies the key may still be pending
+ * (dp_audit_emit, or any synchronisation of the stream, ensures that).
+ * Host-only; the call-order state is unchanged.  Errors: DP_ERR_ARG. */
+dp_status dp_set_noise_key(dp_ctx* ctx, uint64_t seed, uint64_t step);
+
 /* Which kernels serve a layer: *norm_tc = 1 if its per-example norms run on
  * the tcgen05 tensor cores (0: CUDA cores), *sum_tc = 1 if its clipped sum
  * does.  For bf16 layers the Gram norm always does; the clipped sum and the

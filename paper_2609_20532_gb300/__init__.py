@@ -26,7 +26,7 @@ __all__ = [
     "dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "dp_clip_factors",
     "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
     "dp_audit_emit", "audit_dtype", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_layer_path",
-    "dp_step_destroy",
+    "dp_set_noise_key", "dp_step_destroy",
     "dp_last_error", "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
     "EXPORTED_SYMBOLS",
 ]
@@ -47,7 +47,8 @@ STATUS_NAMES = {0: "DP_OK", 1: "DP_ERR_ARG", 2: "DP_ERR_SHAPE", 3: "DP_ERR_DTYPE
 EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "dp_clip_factors",
                     "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
                     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode",
-                    "dp_layer_path", "dp_step_destroy", "dp_last_error", "dp_status_string",
+                    "dp_layer_path", "dp_set_noise_key", "dp_step_destroy", "dp_last_error",
+                    "dp_status_string",
                     "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc"]
 
 
@@ -101,6 +102,7 @@ def lib() -> ctypes.CDLL:
         "dp_audit_record_bytes": ([i32], i64),
         "dp_layer_norm_mode": ([vp, i32, ctypes.POINTER(i32)], i32),
         "dp_layer_path": ([vp, i32, ctypes.POINTER(i32), ctypes.POINTER(i32)], i32),
+        "dp_set_noise_key": ([vp, u64, u64], i32),
         "dp_step_destroy": ([vp], None),
         "dp_last_error": ([], ctypes.c_char_p),
         "dp_status_string": ([i32], ctypes.c_char_p),
@@ -224,6 +226,10 @@ def dp_layer_path(ctx: int, layer: int):
     a, b = ctypes.c_int32(0), ctypes.c_int32(0)
     _check(lib().dp_layer_path(ctx, layer, ctypes.byref(a), ctypes.byref(b)))
     return bool(a.value), bool(b.value)
+
+
+def dp_set_noise_key(ctx: int, seed: int, step: int) -> None:
+    _check(lib().dp_set_noise_key(ctx, seed & (2 ** 64 - 1), step & (2 ** 64 - 1)))
 
 
 def dp_step_destroy(ctx: Optional[int]) -> None:

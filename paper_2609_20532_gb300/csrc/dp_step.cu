@@ -76,6 +76,9 @@ struct dp_ctx {
   int* h_idx = nullptr;         // pinned [cap]
   float* h_rec = nullptr;       // pinned [cap][3 + L]
   int* h_flag = nullptr;        // pinned
+  uint64_t* d_key = nullptr;    // {seed, step} read by the noise kernels
+  uint64_t* h_key = nullptr;    // mapped pinned source of d_key (host address)
+  uint64_t* h_key_dev = nullptr;  // the same words, device address
   void* d_prescaled = nullptr;  // pre-scaled operand of short-example layers
   int64_t prescaled_bytes = 0;
   size_t part_bytes = 0;
@@ -176,6 +179,11 @@ void free_scratch(dp_ctx* c) {
   cudaFreeHost(c->h_flag);
   cudaFree(c->d_prescaled);
   c->d_prescaled = nullptr;
+  cudaFree(c->d_key);
+  cudaFreeHost(c->h_key);
+  c->d_key = nullptr;
+  c->h_key = nullptr;
+  c->h_key_dev = nullptr;
   c->d_part = nullptr;
   c->d_nparts = nullptr;
   c->d_layer_sq = c->d_s = c->d_c = nullptr;
@@ -208,11 +216,16 @@ dp_status alloc_scratch(dp_ctx* c) {
   DP_ALLOC(c->d_idx, sizeof(int) * cap);
   DP_ALLOC(c->d_rec, sizeof(float) * cap * (3 + L));
   if (c->prescaled_bytes > 0) DP_ALLOC(c->d_prescaled, static_cast<size_t>(c->prescaled_bytes));
+  DP_ALLOC(c->d_key, 2 * sizeof(uint64_t));
 #undef DP_ALLOC
   if (cudaMallocHost(reinterpret_cast<void**>(&c->h_idx), sizeof(int) * cap) != cudaSuccess ||
       cudaMallocHost(reinterpret_cast<void**>(&c->h_rec), sizeof(float) * cap * (3 + L)) !=
           cudaSuccess ||
-      cudaMallocHost(reinterpret_cast<void**>(&c->h_flag), sizeof(int)) != cudaSuccess) {
+      cudaMallocHost(reinterpret_cast<void**>(&c->h_flag), sizeof(int)) != cudaSuccess ||
+      cudaHostAlloc(reinterpret_cast<void**>(&c->h_key), 2 * sizeof(uint64_t),
+                    cudaHostAllocMapped) != cudaSuccess ||
+      cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->h_key_dev), c->h_key, 0) !=
+          cudaSuccess) {
     cudaGetLastError();
     free_scratch(c);
     return fail(DP_ERR_OOM, "pinned host allocation failed");
@@ -235,6 +248,17 @@ bool same_parts(const std::vector<LayerPlan>& a, const std::vector<LayerPlan>& b
   for (size_t l = 0; l < a.size(); ++l)
     if (a[l].nparts != b[l].nparts) return false;
   return true;
+}
+
+// Load the key words into device memory on the context's stream.  A
+// one-thread kernel reads the mapped pinned words when it runs (no copy-engine
+// queueing behind bulk host copies), so a CUDA graph that captured it loads
+// the key current at replay time (set with dp_set_noise_key).
+dp_status upload_key(dp_ctx* c) {
+  c->h_key[0] = c->seed;
+  c->h_key[1] = c->step;
+  DP_CUDA(dpk::launch_load_key(c->h_key_dev, c->d_key, c->stream));
+  return DP_OK;
 }
 
 void reset_step(dp_ctx* c) {
@@ -309,8 +333,7 @@ dp_status check_sum_args(dp_ctx* c, int32_t layer, const void* A, const void* D,
 
 dpk::Epilogue make_epilogue(const dp_ctx* c, uint32_t flags, uint64_t p_base) {
   dpk::Epilogue ep{};
-  ep.seed = c->seed;
-  ep.step = c->step;
+  ep.key = c->d_key;
   ep.p_base = p_base;
   ep.out_scale = c->out_scale;
   ep.sigmaC = c->sigma * c->C;
@@ -324,7 +347,7 @@ cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const vo
   const LayerPlan& p = c->plan[layer];
   const dpk::Epilogue ep = make_epilogue(c, flags, p.p_base);
   if (flags & DP_NOISE_ONLY)
-    return dpk::launch_noise_add(d_out, p.d_in * p.d_out, p.p_base, c->seed, c->step,
+    return dpk::launch_noise_add(d_out, p.d_in * p.d_out, p.p_base, c->d_key,
                                  c->out_scale * ep.sigmaC, c->stream);
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
   if (p.gemm_tc == 1)
@@ -371,6 +394,8 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     }
     // the sticky flag reports conditions of the current step only
     DP_CUDA(cudaMemsetAsync(c->d_flag, 0, sizeof(int), c->stream));
+    st = upload_key(c);
+    if (st != DP_OK) return st;
     reset_step(c);
     return DP_OK;
   }
@@ -394,6 +419,7 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     cudaError_t e = cudaMemsetAsync(c->d_flag, 0, sizeof(int), c->stream);
     if (e != cudaSuccess) st = fail(DP_ERR_CUDA, "cudaMemsetAsync: %s", cudaGetErrorString(e));
   }
+  if (st == DP_OK) st = upload_key(c);
   if (st != DP_OK) {
     free_scratch(c);
     delete c;
@@ -587,6 +613,15 @@ dp_status dp_layer_norm_mode(const dp_ctx* c, int32_t layer, dp_norm_mode* mode_
   if (!c || !mode_out) return fail(DP_ERR_ARG, "NULL argument");
   if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
   *mode_out = c->plan[layer].mode;
+  return DP_OK;
+}
+
+dp_status dp_set_noise_key(dp_ctx* c, uint64_t seed, uint64_t step) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  c->seed = seed;
+  c->step = step;
+  c->h_key[0] = seed;
+  c->h_key[1] = step;
   return DP_OK;
 }
 

@@ -9,8 +9,8 @@ enum InType { IN_F32 = 0, IN_BF16 = 1 };
 
 // How the output tile of a clipped-sum kernel is written.
 struct Epilogue {
-  uint64_t seed;
-  uint64_t step;
+  const uint64_t* key;  // device words {seed, step}: read by the kernel, so a
+                        // captured CUDA graph picks up each step's key
   uint64_t p_base;     // global index of element (0, 0) of this layer
   float out_scale;     // applied to (S + sigmaC * z)
   float sigmaC;        // sigma * C
@@ -41,12 +41,15 @@ cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float
                              int d_in, int d_out, float* out, const Epilogue& ep, cudaStream_t s);
 
 // ---- standalone noise add: out[e] += scale * z_{p_base + e}, e < n ----
-cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, uint64_t seed, uint64_t step,
+cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, const uint64_t* key,
                              float scale, cudaStream_t s);
 
 // ---- audit gather ----
 cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer_sq,
                          const float* s_vec, const float* c_vec, float* rec, cudaStream_t s);
+
+// ---- noise key: device copy of two mapped pinned host words ----
+cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, cudaStream_t s);
 
 // ---- error message of the calling thread, read back by dp_last_error() ----
 void set_last_error(const char* msg);

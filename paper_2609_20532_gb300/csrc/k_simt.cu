@@ -225,7 +225,7 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
         if (kb >= d_out) continue;
         float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
         const uint64_t p0 = ep.p_base + static_cast<uint64_t>(j) * d_out + kb;
-        if (ep.add_noise) z = gauss4_at(ep.seed, ep.step, p0);
+        if (ep.add_noise) z = gauss4_at(ep.key[0], ep.key[1], p0);
         const float zv[4] = {z.x, z.y, z.z, z.w};
         float* o = out + static_cast<int64_t>(j) * d_out;
 #pragma unroll
@@ -276,8 +276,9 @@ __global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
 // Standalone noise add: out[e] += scale * z_{p_base + e}
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_noise_add(float* __restrict__ out, int64_t n,
-                                                   uint64_t p_base, uint64_t seed, uint64_t step,
-                                                   float scale) {
+                                                   uint64_t p_base,
+                                                   const uint64_t* __restrict__ key, float scale) {
+  const uint64_t seed = key[0], step = key[1];
   // quads that overlap [p_base, p_base + n)
   const uint64_t q_first = p_base >> 2;
   const uint64_t q_last = (p_base + n - 1) >> 2;
@@ -331,6 +332,15 @@ __global__ void k_audit(const int* __restrict__ idx, int n, int L, int B,
   o[1] = s_vec[i];
   o[2] = c_vec[i];
   for (int l = 0; l < L; ++l) o[3 + l] = layer_sq[l * B + i];
+}
+
+// Copy the noise key from mapped pinned host memory to device memory.  A
+// kernel instead of a DMA copy: it runs on the SMs, so it never queues behind
+// large host<->device copies on the copy engines, and inside a CUDA graph it
+// reads the host words current at replay time.
+__global__ void k_load_key(const volatile uint64_t* host_key, uint64_t* __restrict__ key) {
+  key[0] = host_key[0];
+  key[1] = host_key[1];
 }
 
 __global__ void k_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
@@ -452,11 +462,11 @@ cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float
   return cudaGetLastError();
 }
 
-cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, uint64_t seed, uint64_t step,
+cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, const uint64_t* key,
                              float scale, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int64_t nq = static_cast<int64_t>(((p_base + n - 1) >> 2) - (p_base >> 2) + 1);
-  k_noise_add<<<grid_for(nq, 256), 256, 0, s>>>(out, n, p_base, seed, step, scale);
+  k_noise_add<<<grid_for(nq, 256), 256, 0, s>>>(out, n, p_base, key, scale);
   return cudaGetLastError();
 }
 
@@ -464,6 +474,11 @@ cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer
                          const float* s_vec, const float* c_vec, float* rec, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   k_audit<<<(n + 127) / 128, 128, 0, s>>>(idx, n, L, B, layer_sq, s_vec, c_vec, rec);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, cudaStream_t s) {
+  k_load_key<<<1, 1, 0, s>>>(host_key_dev, key);
   return cudaGetLastError();
 }
 

@@ -93,7 +93,7 @@ struct GemmArgs {
   int NP, row0;
   int pad3d;   // 1: maps are [B][T][d] and each example's K range is padded to 64 rows
   int d_rows;  // > 0: pre-scaled mode, D row of K row k is k % d_rows (A holds [hi; lo])
-  uint64_t seed, step;
+  const uint64_t* key;  // device {seed, step}
   float out_scale, sigmaC;
   int add_noise, accumulate;
 };
@@ -324,6 +324,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     // into the register accumulator (sum and noise commute), so the tile end
     // only scales and stores.
     const int qpe = (32 + g.B - 1) / g.B;
+    const uint64_t seed = g.add_noise ? g.key[0] : 0, step = g.add_noise ? g.key[1] : 0;
     for (int tile = unit; tile < n_tiles; tile += n_units) {
       int l = 0;
       while (tile >= g.tile_start[l + 1]) ++l;
@@ -351,7 +352,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
               // p_base and d_out are multiples of 8 on this path, so the four
               // parameters prow+k .. +3 form exactly one Philox quad
               if (k0 + 4 * q >= d_out) break;
-              const float4 z = gauss_quad(g.seed, g.step, (prow + k0 + 4 * q) >> 2);
+              const float4 z = gauss_quad(seed, step, (prow + k0 + 4 * q) >> 2);
               // static register indices: select the slot with a predicate
 #pragma unroll
               for (int t = 0; t < 32; ++t) {
@@ -550,8 +551,7 @@ cudaError_t launch_any(GemmArgs& g, cudaStream_t s) {
 }
 
 void set_epilogue(GemmArgs& g, const Epilogue& ep) {
-  g.seed = ep.seed;
-  g.step = ep.step;
+  g.key = ep.key;
   g.out_scale = ep.out_scale;
   g.sigmaC = ep.sigmaC;
   g.add_noise = ep.add_noise;

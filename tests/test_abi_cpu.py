@@ -86,6 +86,7 @@ def test_calls_reject_null_context(L):
     assert L.dp_audit_emit(None, None, 0, None) == 1
     m = ctypes.c_int32()
     assert L.dp_layer_norm_mode(None, 0, ctypes.byref(m)) == 1
+    assert L.dp_set_noise_key(None, 0, 0) == 1
     L.dp_step_destroy(None)  # no-op
 
 

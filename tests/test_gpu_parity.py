@@ -518,3 +518,38 @@ def test_commitment_passes_the_verifier_body_path(name):
     assert np.linalg.norm(g_gpu) <= C * (1 + 1e-4)
     z = np.linalg.norm(g_gpu - g_ref) / C
     assert z <= TAU_ABS, z
+
+
+def test_cuda_graph_replay_matches_eager_steps():
+    """A step captured once in a CUDA graph and replayed under new keys
+    (dp_set_noise_key between replays) writes exactly the eager outputs."""
+    w = W.custom("graph", [(264, 520), (520, 136)], 6, 64, "bf16", C=0.1, sigma=0.7, d_std=0.2,
+                 wid=900)
+    layers = W.make_inputs(w)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    s = torch.cuda.Stream()
+    outs_g = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, seed=5, step=0,
+                         audit_capacity=w.B)
+    ctx = dp.dp_step_init(cfg, s)
+    try:
+        with torch.cuda.stream(s):
+            dp.run_step(ctx, Ad, Dd, outs_g)            # eager warm-up (one-time set-up)
+            dp.dp_audit_emit(ctx, [0], len(layers))
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=s):
+                dp.dp_step_init(cfg, s, ctx)
+                dp.run_step(ctx, Ad, Dd, outs_g)
+            for step in (3, 4):
+                dp.dp_set_noise_key(ctx, 5, step)
+                graph.replay()
+                recs = dp.dp_audit_emit(ctx, range(w.B), len(layers))
+                got = [o.cpu().numpy().copy() for o in outs_g]
+                eager = run_gpu_step(w, layers, seed=5, step=step)
+                for a, b in zip(got, eager["out"]):
+                    assert np.array_equal(a, b)
+                assert np.array_equal(recs["layer_sqnorm"].astype(np.float64).T, eager["n"])
+    finally:
+        dp.dp_step_destroy(ctx)
