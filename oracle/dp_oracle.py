@@ -27,7 +27,12 @@ What is computed (paper: Sec. 2.2 "DP-SGD", and the GPU loop of Algorithm 2):
 * audit records (example, per-layer squared norms, total, clip factor) for a
   caller-chosen subset of examples, the material a CPU checker recomputes when
   it partially re-executes a step (Sec. 7, "recomputes, or partially
-  recomputes").
+  recomputes");
+* the update that follows the seed release in Algorithm 2,
+  g~ = committed average + (1/B) Noise(s; sigma C), then OptStep = AdamW as the
+  paper writes its one-step map (App. A): m = b1 m + (1-b1) g,
+  v = b2 v + (1-b2) g*g, bias corrections 1 - b^t, and
+  theta <- theta - lr (m^/(sqrt(v^) + eps) + wd theta).
 
 Readings where the paper is silent (each also listed with its reason in the
 design notes): c_i = 1 when s_i <= C^2, including s_i = 0; no stabiliser
@@ -48,6 +53,10 @@ Pins (tests/test_oracle_pins.py, all ``-m "not gpu"``):
   (``at::philox_engine``) compiled from its header; counter/key sensitivity.
 * uniforms_from_words: hand-derived edge values (tests/golden/uniform_edges.json).
 * box_muller: the identities z0^2 + z1^2 = -2 ln u0, atan2(z1, z0) = 2 pi u1.
+* adamw_step: pure-Python scalar loop of the App. A equations; the t = 1 and
+  b1 = b2 = 0 special cases where the step is lr (g/(|g| + eps) + wd theta)
+  (tests/golden/adamw_hand.json, worked by hand); g = 0 leaves theta
+  changed by weight decay only.
 * gaussian_noise: sample mean / variance / Kolmogorov-Smirnov against
   N(0, 1); per-coordinate std of the averaged noise against the sigma*C/B
   column printed in the paper's attack-parameter table (App. B.1).
@@ -75,6 +84,8 @@ __all__ = [
     "gaussian_noise",
     "dp_step",
     "audit_records",
+    "adamw_step",
+    "noise_adamw",
     "PHILOX_M0",
     "PHILOX_M1",
     "PHILOX_W0",
@@ -356,3 +367,44 @@ def audit_records(n, s, c, idx):
         recs.append({"example": i, "layer_sqnorm": n[:, i].copy(),
                      "total_sqnorm": float(s[i]), "clip_factor": float(c[i])})
     return recs
+
+
+# ---------------------------------------------------------------------------
+# After the seed release: noisy gradient and OptStep = AdamW (Algorithm 2;
+# the one-step AdamW map of App. A)
+# ---------------------------------------------------------------------------
+
+def adamw_step(theta, m, v, g, lr: float, beta1: float, beta2: float, eps: float,
+               weight_decay: float, t: int):
+    """One AdamW step at step count t >= 1 (bias corrections 1 - beta^t).
+
+    m' = b1 m + (1 - b1) g;  v' = b2 v + (1 - b2) g*g;
+    m^ = m' / (1 - b1^t);    v^ = v' / (1 - b2^t);
+    theta' = theta - lr (m^ / (sqrt(v^) + eps) + wd theta).
+    Returns (theta', m', v') in fp64."""
+    if t < 1:
+        raise ValueError("step count t must be >= 1")
+    theta = _as_f64(theta)
+    m = _as_f64(m)
+    v = _as_f64(v)
+    g = _as_f64(g)
+    m2 = beta1 * m + (1.0 - beta1) * g
+    v2 = beta2 * v + (1.0 - beta2) * g * g
+    mh = m2 / (1.0 - beta1 ** t)
+    vh = v2 / (1.0 - beta2 ** t)
+    theta2 = theta - lr * (mh / (np.sqrt(vh) + eps) + weight_decay * theta)
+    return theta2, m2, v2
+
+
+def noise_adamw(committed, theta, m, v, seed: int, step: int, first_index: int,
+                sigma: float, C: float, out_scale: float, lr: float, beta1: float,
+                beta2: float, eps: float, weight_decay: float, t: int):
+    """The GPU's update after the seed is released (Algorithm 2):
+    g~ = committed + out_scale * sigma * C * z  (committed = out_scale * S, the
+    noiseless commitment), then AdamW.  z uses the parameters' global indices
+    first_index .. first_index + size - 1.  Returns (g~, theta', m', v')."""
+    committed = _as_f64(committed)
+    z = gaussian_noise(seed, step, first_index, committed.size).reshape(committed.shape)
+    g = committed + out_scale * sigma * C * z
+    th, m2, v2 = adamw_step(theta, m, v, g, lr, beta1, beta2, eps, weight_decay, t)
+    return g, th, m2, v2

@@ -456,3 +456,84 @@ def test_planted_mistakes_are_caught(tmp_path_factory):
     assert not check_philox_vs_torch(make_quads(philox_variant(m0=0xD2511F55)), binpath)
     assert not check_philox_vs_torch(make_quads(philox_variant(rounds=7)), binpath)
     assert not check_philox_vs_torch(make_quads(philox_variant(bump_first=True)), binpath)
+
+
+# ---------------------------------------------------------------------------
+# AdamW after the seed release (App. A one-step map; Algorithm 2 OptStep)
+# ---------------------------------------------------------------------------
+
+def adamw_scalar_loop(theta, m, v, g, lr, b1, b2, eps, wd, t):
+    out = []
+    for th, mm, vv, gg in zip(theta.tolist(), m.tolist(), v.tolist(), g.tolist()):
+        m2 = b1 * mm + (1 - b1) * gg
+        v2 = b2 * vv + (1 - b2) * gg * gg
+        mh = m2 / (1 - b1 ** t)
+        vh = v2 / (1 - b2 ** t)
+        out.append((th - lr * (mh / (math.sqrt(vh) + eps) + wd * th), m2, v2))
+    return [np.array(x) for x in zip(*out)]
+
+
+def check_adamw_golden(step_fn) -> bool:
+    g = json.load(open(os.path.join(GOLDEN, "adamw_hand.json")))
+    for c in g["cases"]:
+        th, m, v = step_fn(np.array([c["theta"]]), np.array([c["m"]]), np.array([c["v"]]),
+                           np.array([c["g"]]), c["lr"], c["beta1"], c["beta2"], c["eps"],
+                           c["wd"], c["t"])
+        if not (np.isclose(th[0], c["theta_new"], rtol=1e-14, atol=1e-15)
+                and np.isclose(m[0], c["m_new"], rtol=1e-14, atol=1e-15)
+                and np.isclose(v[0], c["v_new"], rtol=1e-14, atol=1e-15)):
+            return False
+    return True
+
+
+def test_adamw_golden_cases():
+    assert check_adamw_golden(O.adamw_step)
+
+
+def test_adamw_matches_scalar_loop():
+    rng = np.random.default_rng(17)
+    n = 257
+    theta, m, g = rng.standard_normal((3, n))
+    v = rng.random(n)
+    for t in (1, 2, 10, 1000):
+        got = O.adamw_step(theta, m, v, g, 3e-4, 0.9, 0.999, 1e-8, 0.01, t)
+        ref = adamw_scalar_loop(theta, m, v, g, 3e-4, 0.9, 0.999, 1e-8, 0.01, t)
+        for a, b in zip(got, ref):
+            np.testing.assert_allclose(a, b, rtol=1e-14, atol=1e-16)
+    with pytest.raises(ValueError):
+        O.adamw_step(theta, m, v, g, 1e-3, 0.9, 0.999, 1e-8, 0.0, 0)
+
+
+def test_noise_adamw_composes_noise_and_step():
+    rng = np.random.default_rng(3)
+    shape = (7, 9)
+    committed, theta, m = rng.standard_normal((3,) + shape)
+    v = rng.random(shape)
+    g, th, m2, v2 = O.noise_adamw(committed, theta, m, v, 4, 6, 100, 1.1, 0.5, 0.25,
+                                  1e-3, 0.9, 0.99, 1e-8, 0.02, 5)
+    z = O.gaussian_noise(4, 6, 100, 63).reshape(shape)
+    np.testing.assert_allclose(g, committed + 0.25 * 1.1 * 0.5 * z, rtol=1e-15)
+    ref = O.adamw_step(theta, m, v, g, 1e-3, 0.9, 0.99, 1e-8, 0.02, 5)
+    for a, b in zip((th, m2, v2), ref):
+        np.testing.assert_array_equal(a, b)
+
+
+def test_planted_adamw_mistakes_are_caught():
+    def no_bias_correction(theta, m, v, g, lr, b1, b2, eps, wd, t):
+        m2 = b1 * m + (1 - b1) * g
+        v2 = b2 * v + (1 - b2) * g * g
+        return theta - lr * (m2 / (np.sqrt(v2) + eps) + wd * theta), m2, v2
+
+    def coupled_decay(theta, m, v, g, lr, b1, b2, eps, wd, t):
+        return O.adamw_step(theta, m, v, g + wd * theta, lr, b1, b2, eps, 0.0, t)
+
+    def eps_inside_sqrt(theta, m, v, g, lr, b1, b2, eps, wd, t):
+        m2 = b1 * m + (1 - b1) * g
+        v2 = b2 * v + (1 - b2) * g * g
+        mh, vh = m2 / (1 - b1 ** t), v2 / (1 - b2 ** t)
+        return theta - lr * (mh / np.sqrt(vh + eps) + wd * theta), m2, v2
+
+    assert check_adamw_golden(O.adamw_step)
+    assert not check_adamw_golden(no_bias_correction)
+    assert not check_adamw_golden(coupled_decay)
+    assert not check_adamw_golden(eps_inside_sqrt)
