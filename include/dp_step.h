@@ -112,6 +112,16 @@ typedef struct {
 #define DP_NO_NOISE   0x1u /* write out_scale * S only: the noiseless commitment of Algorithm 2 */
 #define DP_NOISE_ONLY 0x2u /* out += out_scale * sigma * C * z; A and D are ignored (may be NULL) */
 #define DP_ACCUMULATE 0x4u /* add into out instead of overwriting it (micro-batch accumulation) */
+#define DP_WRITE_GRAD 0x8u /* dp_noise_adamw: also write the noisy gradient back into d_grad */
+
+/* AdamW hyperparameters of one OptStep (App. A one-step map). */
+typedef struct {
+    float lr;            /* learning rate eta_t, finite */
+    float beta1, beta2;  /* in [0, 1) */
+    float eps;           /* >= 0, added outside the square root */
+    float weight_decay;  /* decoupled weight decay lambda */
+    int64_t t;           /* step count for the bias corrections, >= 1 */
+} dp_adamw;
 
 /* Create (*ctx == NULL) or re-key (*ctx != NULL) a step context.
  * Create: validates cfg, allocates scratch on the current device and binds
@@ -180,6 +190,22 @@ dp_status dp_clipped_sum_noise(dp_ctx* ctx, int32_t layer, const void* A, const 
 dp_status dp_clipped_sum_noise_batch(dp_ctx* ctx, int32_t n, const int32_t* layers,
                                      const void* const* A, const void* const* D,
                                      float* const* d_out, uint32_t flags);
+
+/* The GPU's update after the seed release (Algorithm 2; OptStep = AdamW as
+ * in App. A), one layer, in one pass over its parameters:
+ *   g~    = d_grad + out_scale * sigma * C * z          (z as above, same keys)
+ *   m     = b1 m + (1 - b1) g~,   v = b2 v + (1 - b2) g~^2
+ *   theta = theta - lr (m / (1 - b1^t) / (sqrt(v / (1 - b2^t)) + eps)
+ *                       + weight_decay * theta)
+ * d_grad holds the committed average on entry (dp_clipped_sum_noise with
+ * DP_NO_NOISE); d_theta, d_m, d_v are updated in place.  All are device fp32
+ * [d_in][d_out], 16-byte aligned.  flags: DP_NO_NOISE (g~ = d_grad),
+ * DP_WRITE_GRAD (store g~ into d_grad).  Needs only an initialised context
+ * (the key set by dp_step_init / dp_set_noise_key).
+ * Errors: DP_ERR_ARG (NULL / misaligned pointers, bad hyperparameters or
+ * flags), DP_ERR_CUDA. */
+dp_status dp_noise_adamw(dp_ctx* ctx, int32_t layer, float* d_grad, float* d_theta, float* d_m,
+                         float* d_v, const dp_adamw* hp, uint32_t flags);
 
 /* Audit emit: for the n example indices in h_idx (host array, each in
  * 0 .. B-1, n <= audit_capacity) copy records into h_records (host memory,

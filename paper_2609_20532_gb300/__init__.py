@@ -21,7 +21,7 @@ __all__ = [
     "DPError", "LibraryNotBuilt", "lib", "lib_path",
     "DP_OK", "DP_F32", "DP_BF16",
     "DP_NORM_AUTO", "DP_NORM_RANK1", "DP_NORM_GHOST", "DP_NORM_MATERIALISED",
-    "DP_NO_NOISE", "DP_NOISE_ONLY", "DP_ACCUMULATE",
+    "DP_NO_NOISE", "DP_NOISE_ONLY", "DP_ACCUMULATE", "DP_WRITE_GRAD", "dp_adamw", "dp_noise_adamw",
     "dp_layer", "dp_config", "make_config",
     "dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "dp_clip_factors",
     "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
@@ -37,7 +37,7 @@ lib_path = os.path.join(HERE, "libdpstep.so")
 DP_OK = 0
 DP_F32, DP_BF16 = 0, 1
 DP_NORM_AUTO, DP_NORM_RANK1, DP_NORM_GHOST, DP_NORM_MATERIALISED = 0, 1, 2, 3
-DP_NO_NOISE, DP_NOISE_ONLY, DP_ACCUMULATE = 0x1, 0x2, 0x4
+DP_NO_NOISE, DP_NOISE_ONLY, DP_ACCUMULATE, DP_WRITE_GRAD = 0x1, 0x2, 0x4, 0x8
 
 STATUS_NAMES = {0: "DP_OK", 1: "DP_ERR_ARG", 2: "DP_ERR_SHAPE", 3: "DP_ERR_DTYPE",
                 4: "DP_ERR_ORDER", 5: "DP_ERR_NONFINITE", 6: "DP_ERR_CUDA",
@@ -49,7 +49,8 @@ EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "d
                     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode",
                     "dp_layer_path", "dp_set_noise_key", "dp_step_destroy", "dp_last_error",
                     "dp_status_string",
-                    "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc"]
+                    "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
+                    "dp_noise_adamw"]
 
 
 class DPError(RuntimeError):
@@ -65,6 +66,11 @@ class LibraryNotBuilt(ImportError):
 
 class dp_layer(ctypes.Structure):
     _fields_ = [("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64)]
+
+
+class dp_adamw(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float), ("t", ctypes.c_int64)]
 
 
 class dp_config(ctypes.Structure):
@@ -109,6 +115,7 @@ def lib() -> ctypes.CDLL:
         "dp_debug_philox": ([u64, u64, u64, i64, vp, vp], i32),
         "dp_debug_gaussian": ([u64, u64, u64, i64, vp, vp], i32),
         "dp_layer_sqnorms_noalloc": ([vp, vp, i32, i32, i64, i64, i32, vp, vp], i32),
+        "dp_noise_adamw": ([vp, i32, vp, vp, vp, vp, ctypes.POINTER(dp_adamw), u32], i32),
     }
     for name, (args, res) in sig.items():
         f = getattr(L, name)
@@ -259,6 +266,15 @@ def dp_layer_sqnorms_noalloc(A, D, B: int, T: int, d_in: int, d_out: int, dtype:
     _check(lib().dp_layer_sqnorms_noalloc(_ptr(A), _ptr(D), B, T, d_in, d_out,
                                           DP_BF16 if dtype == "bf16" else DP_F32, _ptr(out),
                                           _stream(stream)))
+
+
+def dp_noise_adamw(ctx: int, layer: int, grad, theta, m, v, lr: float, beta1: float,
+                   beta2: float, eps: float, weight_decay: float, t: int, flags: int = 0) -> None:
+    """Noisy gradient from the committed average, then AdamW on theta, m, v
+    in place (see include/dp_step.h)."""
+    hp = dp_adamw(lr=lr, beta1=beta1, beta2=beta2, eps=eps, weight_decay=weight_decay, t=t)
+    _check(lib().dp_noise_adamw(ctx, layer, _ptr(grad), _ptr(theta), _ptr(m), _ptr(v),
+                                ctypes.byref(hp), flags))
 
 
 def run_step(ctx: int, A_list, D_list, outs, flags: int = 0) -> None:

@@ -577,6 +577,36 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
   return DP_OK;
 }
 
+dp_status dp_noise_adamw(dp_ctx* c, int32_t layer, float* d_grad, float* d_theta, float* d_m,
+                         float* d_v, const dp_adamw* hp, uint32_t flags) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
+  if (flags & ~(DP_NO_NOISE | DP_WRITE_GRAD)) return fail(DP_ERR_ARG, "unknown flag bits 0x%x", flags);
+  if (!d_grad || !d_theta || !d_m || !d_v || !hp) return fail(DP_ERR_ARG, "NULL argument");
+  if (!aligned16(d_grad) || !aligned16(d_theta) || !aligned16(d_m) || !aligned16(d_v))
+    return fail(DP_ERR_ARG, "gradient and optimizer arrays must be 16-byte aligned");
+  if (!(hp->beta1 >= 0.f && hp->beta1 < 1.f) || !(hp->beta2 >= 0.f && hp->beta2 < 1.f) ||
+      !(hp->eps >= 0.f) || !std::isfinite(hp->eps) || !std::isfinite(hp->lr) ||
+      !std::isfinite(hp->weight_decay) || hp->t < 1)
+    return fail(DP_ERR_ARG, "AdamW hyperparameters out of range");
+  const LayerPlan& p = c->plan[layer];
+  dpk::AdamWArgs h{};
+  h.lr = hp->lr;
+  h.beta1 = hp->beta1;
+  h.beta2 = hp->beta2;
+  h.eps = hp->eps;
+  h.weight_decay = hp->weight_decay;
+  h.bc1 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(hp->beta1),
+                                                  static_cast<double>(hp->t))));
+  h.bc2 = static_cast<float>(1.0 / (1.0 - std::pow(static_cast<double>(hp->beta2),
+                                                  static_cast<double>(hp->t))));
+  DP_CUDA(dpk::launch_noise_adamw(d_grad, d_theta, d_m, d_v, p.d_in * p.d_out, p.p_base,
+                                  c->d_key, c->out_scale * (c->sigma * c->C),
+                                  (flags & DP_NO_NOISE) ? 0 : 1, (flags & DP_WRITE_GRAD) ? 1 : 0,
+                                  h, c->stream));
+  return DP_OK;
+}
+
 dp_status dp_audit_emit(dp_ctx* c, const int32_t* h_idx, int32_t n, void* h_records) {
   if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
   if (n < 0 || n > c->audit_capacity)

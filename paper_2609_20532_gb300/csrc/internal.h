@@ -44,6 +44,15 @@ cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float
 cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, const uint64_t* key,
                              float scale, cudaStream_t s);
 
+// ---- noisy gradient + AdamW after the seed release ----
+struct AdamWArgs {
+  float lr, beta1, beta2, eps, weight_decay;
+  float bc1, bc2;  // 1 / (1 - beta1^t), 1 / (1 - beta2^t)
+};
+cudaError_t launch_noise_adamw(float* grad, float* theta, float* m, float* v, int64_t n,
+                               uint64_t p_base, const uint64_t* key, float noise_scale,
+                               int add_noise, int write_grad, const AdamWArgs& h, cudaStream_t s);
+
 // ---- audit gather ----
 cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer_sq,
                          const float* s_vec, const float* c_vec, float* rec, cudaStream_t s);

@@ -87,6 +87,7 @@ def test_calls_reject_null_context(L):
     m = ctypes.c_int32()
     assert L.dp_layer_norm_mode(None, 0, ctypes.byref(m)) == 1
     assert L.dp_set_noise_key(None, 0, 0) == 1
+    assert L.dp_noise_adamw(None, 0, 16, 16, 16, 16, None, 0) == 1
     L.dp_step_destroy(None)  # no-op
 
 

@@ -553,3 +553,156 @@ def test_cuda_graph_replay_matches_eager_steps():
                 assert np.array_equal(recs["layer_sqnorm"].astype(np.float64).T, eager["n"])
     finally:
         dp.dp_step_destroy(ctx)
+
+
+# ---------------------------------------------------------------------------
+# the GPU's update after the seed release (Algorithm 2, OptStep = AdamW, App. A)
+# ---------------------------------------------------------------------------
+
+U32 = 2.0 ** -24          # fp32 unit roundoff
+Z_REL = 1e-6              # elementwise relative error of the device Gaussian (test above)
+
+
+def adamw_error_bound(committed, theta, m, v, z, s, hp):
+    """First-order forward error of the fp32 kernel, per element, from the
+    fp64 values: every fp32 operation rounds once (relative U32), z carries
+    Z_REL, and the errors propagate through m', v', the bias corrections,
+    sqrt, the division and the final update.  Returned with a 4x margin."""
+    b1, b2, lr, eps, wd, t = hp["beta1"], hp["beta2"], hp["lr"], hp["eps"], hp["wd"], hp["t"]
+    g = committed + s * z
+    e_g = s * np.abs(z) * (Z_REL + 3 * U32) + np.abs(g) * U32
+    m2 = b1 * m + (1 - b1) * g
+    e_m = (1 - b1) * (e_g + np.abs(g) * U32) + np.abs(m2) * U32
+    v2 = b2 * v + (1 - b2) * g * g
+    e_v = (1 - b2) * (2 * np.abs(g) * e_g + 2 * g * g * U32) + np.abs(v2) * U32
+    bc1 = 1.0 / (1.0 - b1 ** t)
+    bc2 = 1.0 / (1.0 - b2 ** t)
+    mh, vh = m2 * bc1, v2 * bc2
+    e_mh = bc1 * e_m + np.abs(mh) * 2 * U32
+    e_vh = bc2 * e_v + vh * 2 * U32
+    sq = np.sqrt(vh)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        e_sq = np.minimum(np.where(sq > 0, e_vh / (2 * sq), np.inf), np.sqrt(e_vh)) + sq * U32
+    den = sq + eps
+    e_den = e_sq + den * U32
+    with np.errstate(divide="ignore", invalid="ignore"):
+        r = np.where(den > 0, mh / den, 0.0)
+        e_r = np.where(den > 0, e_mh / den + np.abs(r) * (e_den / den + U32), 0.0)
+    upd = r + wd * theta
+    e_upd = e_r + (np.abs(upd) + np.abs(wd * theta)) * U32
+    th2 = theta - lr * upd
+    e_th = abs(lr) * (e_upd + np.abs(upd) * U32) + np.abs(th2) * U32
+    return {"g": 4 * e_g, "m": 4 * e_m, "v": 4 * e_v, "theta": 4 * e_th}
+
+
+ADAMW_LAYERS = [(4, 5), (264, 520), (3, 7), (128, 1001)]   # aligned, vector+tail, unaligned
+
+
+def _adamw_inputs(layers, seed, zero_state):
+    rng = np.random.default_rng(seed)
+    out = []
+    for i, o in layers:
+        c = rng.normal(0.0, 1e-3, (i, o)).astype(np.float32)
+        th = rng.normal(0.0, 0.05, (i, o)).astype(np.float32)
+        if zero_state:
+            m = np.zeros((i, o), np.float32)
+            v = np.zeros((i, o), np.float32)
+        else:
+            m = rng.normal(0.0, 1e-3, (i, o)).astype(np.float32)
+            v = (rng.normal(0.0, 1e-3, (i, o)) ** 2).astype(np.float32)
+        out.append((c, th, m, v))
+    return out
+
+
+@pytest.mark.parametrize("flags", [0, dp.DP_WRITE_GRAD, dp.DP_NO_NOISE | dp.DP_WRITE_GRAD])
+@pytest.mark.parametrize("hpi", [0, 1, 2])
+def test_noise_adamw_matches_oracle(flags, hpi):
+    """theta', m', v' (and g~ when written back) against oracle.noise_adamw,
+    elementwise within the propagated fp32 error bound, on layers whose
+    parameter ranges start aligned, with a ragged tail, and unaligned."""
+    hps = [dict(lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, wd=0.0, t=1, zero=True),
+           dict(lr=3e-4, beta1=0.9, beta2=0.95, eps=1e-6, wd=0.1, t=1000, zero=False),
+           dict(lr=-2e-2, beta1=0.0, beta2=0.5, eps=0.0, wd=0.01, t=3, zero=False)]
+    hp = {k: (f32(x) if isinstance(x, float) else x) for k, x in hps[hpi].items()}
+    B, C, sigma, seed, step = 64, 0.25, 1.1, 123, 9
+    scale = 1.0 / B
+    data = _adamw_inputs(ADAMW_LAYERS, 40 + hpi, hp["zero"])
+    dev = torch.device(DEV)
+    cfg = dp.make_config(ADAMW_LAYERS, B, 16, "f32", C, sigma, out_scale=scale, seed=seed,
+                         step=step)
+    ctx = dp.dp_step_init(cfg)
+    got = []
+    try:
+        for l, (c, th, m, v) in enumerate(data):
+            t_c, t_th, t_m, t_v = (torch.from_numpy(x.copy()).to(dev) for x in (c, th, m, v))
+            dp.dp_noise_adamw(ctx, l, t_c, t_th, t_m, t_v, hp["lr"], hp["beta1"], hp["beta2"],
+                              hp["eps"], hp["wd"], hp["t"], flags)
+            got.append([x.cpu().numpy().astype(np.float64) for x in (t_c, t_th, t_m, t_v)])
+    finally:
+        dp.dp_step_destroy(ctx)
+    s = 0.0 if flags & dp.DP_NO_NOISE else f32(scale) * f32(sigma) * f32(C)
+    p0 = 0
+    for (c, th, m, v), (g_g, th_g, m_g, v_g), (i, o) in zip(data, got, ADAMW_LAYERS):
+        g_r, th_r, m_r, v_r = O.noise_adamw(c, th, m, v, seed, step, p0, s, 1.0, 1.0,
+                                            hp["lr"], hp["beta1"], hp["beta2"], hp["eps"],
+                                            hp["wd"], hp["t"])
+        z = O.gaussian_noise(seed, step, p0, i * o).reshape(i, o)
+        bound = adamw_error_bound(c.astype(np.float64), th.astype(np.float64),
+                                  m.astype(np.float64), v.astype(np.float64), z, s, hp)
+        for name, a, r in (("theta", th_g, th_r), ("m", m_g, m_r), ("v", v_g, v_r)):
+            bad = np.abs(a - r) > bound[name] + 1e-37
+            assert not bad.any(), (name, np.argwhere(bad)[:5], a[bad][:5], r[bad][:5])
+        if flags & dp.DP_WRITE_GRAD:
+            assert not (np.abs(g_g - g_r) > bound["g"] + 1e-37).any()
+        else:
+            assert np.array_equal(g_g, c.astype(np.float64))     # input left untouched
+        p0 += i * o
+
+
+def test_noise_adamw_gradient_equals_noise_only_path():
+    """The noisy gradient written back by dp_noise_adamw is bit-identical to
+    DP_NOISE_ONLY on the same committed buffer: the released update and the
+    commit-then-noise path draw the same z with the same scale."""
+    layers = [(136, 72), (64, 203)]
+    B = 8
+    rng = np.random.default_rng(5)
+    dev = torch.device(DEV)
+    cfg = dp.make_config(layers, B, 16, "f32", 0.3, 0.8, out_scale=1.0 / B, seed=99, step=17)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        for l, (i, o) in enumerate(layers):
+            c = torch.from_numpy(rng.normal(0, 1e-2, (i, o)).astype(np.float32)).to(dev)
+            a = c.clone()
+            dp.dp_clipped_sum_noise(ctx, l, None, None, a, dp.DP_NOISE_ONLY)
+            th = torch.zeros(i, o, device=dev)
+            m = torch.zeros(i, o, device=dev)
+            v = torch.zeros(i, o, device=dev)
+            dp.dp_noise_adamw(ctx, l, c, th, m, v, 1e-3, 0.9, 0.999, 1e-8, 0.0, 1,
+                              dp.DP_WRITE_GRAD)
+            assert torch.equal(a, c)
+    finally:
+        dp.dp_step_destroy(ctx)
+
+
+def test_noise_adamw_argument_errors():
+    cfg = dp.make_config([(8, 8)], 2, 4, "f32", 1.0, 1.0)
+    ctx = dp.dp_step_init(cfg)
+    dev = torch.device(DEV)
+    x = [torch.zeros(8, 8, device=dev) for _ in range(4)]
+    try:
+        hp = dict(lr=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0, t=1)
+        for bad in (dict(beta1=1.0), dict(beta2=-0.1), dict(eps=-1.0), dict(t=0),
+                    dict(lr=float("nan"))):
+            h = dict(hp, **bad)
+            with pytest.raises(dp.DPError):
+                dp.dp_noise_adamw(ctx, 0, *x, h["lr"], h["beta1"], h["beta2"], h["eps"],
+                                  h["weight_decay"], h["t"])
+        with pytest.raises(dp.DPError):
+            dp.dp_noise_adamw(ctx, 1, *x, **hp)
+        with pytest.raises(dp.DPError):
+            dp.dp_noise_adamw(ctx, 0, *x, **hp, flags=dp.DP_NOISE_ONLY)
+        flat = torch.zeros(8 * 8 + 1, device=dev)
+        with pytest.raises(dp.DPError):
+            dp.dp_noise_adamw(ctx, 0, flat[1:], *x[1:], **hp)
+    finally:
+        dp.dp_step_destroy(ctx)
