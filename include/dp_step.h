@@ -214,9 +214,13 @@ dp_status dp_noise_adamw(dp_ctx* ctx, int32_t layer, float* d_grad, float* d_the
  *   float layer_sqnorm[L] (n_{1..L,i})
  * -- what a checker needs to recompute the audited examples (Sec. 7, partial
  * recomputation; Algorithm 1 consumes the recomputed aggregate).
- * Synchronises the context's stream.  Returns DP_ERR_NONFINITE if the sticky
- * flag was set during this step (records are still written).
+ * Synchronises the context's stream.  The gather kernel reads the indices
+ * and writes the records through mapped pinned staging, so the call uses no
+ * copy engine and never waits behind bulk copies queued on other streams.
+ * Returns DP_ERR_NONFINITE if the sticky flag was set during this step
+ * (records are still written).
  * Errors: DP_ERR_ARG, DP_ERR_ORDER (before dp_clip_factors), DP_ERR_NONFINITE,
+ *   DP_ERR_TIMEOUT (a tensor-core kernel gave up on a bounded wait),
  *   DP_ERR_CUDA. */
 dp_status dp_audit_emit(dp_ctx* ctx, const int32_t* h_idx, int32_t n, void* h_records);
 

@@ -71,11 +71,15 @@ struct dp_ctx {
   float* d_s = nullptr;         // [B]
   float* d_c = nullptr;         // [B]
   int* d_flag = nullptr;        // sticky error bits
-  int* d_idx = nullptr;         // [cap]
-  float* d_rec = nullptr;       // [cap][3 + L]
-  int* h_idx = nullptr;         // pinned [cap]
-  float* h_rec = nullptr;       // pinned [cap][3 + L]
-  int* h_flag = nullptr;        // pinned
+  // audit staging in mapped pinned memory: the gather kernel reads the
+  // indices and writes the records and the flag word over the host link
+  // itself, so an audit never queues behind bulk copies on the copy engines
+  int* h_idx = nullptr;         // mapped [cap]
+  float* h_rec = nullptr;       // mapped [cap][3 + L]
+  int* h_flag = nullptr;        // mapped
+  int* h_idx_dev = nullptr;     // device views of the three
+  float* h_rec_dev = nullptr;
+  int* h_flag_dev = nullptr;
   uint64_t* d_key = nullptr;    // {seed, step} read by the noise kernels
   uint64_t* h_key = nullptr;    // mapped pinned source of d_key (host address)
   uint64_t* h_key_dev = nullptr;  // the same words, device address
@@ -172,8 +176,6 @@ void free_scratch(dp_ctx* c) {
   cudaFree(c->d_s);
   cudaFree(c->d_c);
   cudaFree(c->d_flag);
-  cudaFree(c->d_idx);
-  cudaFree(c->d_rec);
   cudaFreeHost(c->h_idx);
   cudaFreeHost(c->h_rec);
   cudaFreeHost(c->h_flag);
@@ -188,8 +190,6 @@ void free_scratch(dp_ctx* c) {
   c->d_nparts = nullptr;
   c->d_layer_sq = c->d_s = c->d_c = nullptr;
   c->d_flag = nullptr;
-  c->d_idx = nullptr;
-  c->d_rec = nullptr;
   c->h_idx = nullptr;
   c->h_rec = nullptr;
   c->h_flag = nullptr;
@@ -213,15 +213,22 @@ dp_status alloc_scratch(dp_ctx* c) {
   DP_ALLOC(c->d_s, sizeof(float) * B);
   DP_ALLOC(c->d_c, sizeof(float) * B);
   DP_ALLOC(c->d_flag, sizeof(int));
-  DP_ALLOC(c->d_idx, sizeof(int) * cap);
-  DP_ALLOC(c->d_rec, sizeof(float) * cap * (3 + L));
   if (c->prescaled_bytes > 0) DP_ALLOC(c->d_prescaled, static_cast<size_t>(c->prescaled_bytes));
   DP_ALLOC(c->d_key, 2 * sizeof(uint64_t));
 #undef DP_ALLOC
-  if (cudaMallocHost(reinterpret_cast<void**>(&c->h_idx), sizeof(int) * cap) != cudaSuccess ||
-      cudaMallocHost(reinterpret_cast<void**>(&c->h_rec), sizeof(float) * cap * (3 + L)) !=
+  if (cudaHostAlloc(reinterpret_cast<void**>(&c->h_idx), sizeof(int) * (cap > 0 ? cap : 1),
+                    cudaHostAllocMapped) != cudaSuccess ||
+      cudaHostAlloc(reinterpret_cast<void**>(&c->h_rec),
+                    sizeof(float) * (cap > 0 ? cap : 1) * (3 + L), cudaHostAllocMapped) !=
           cudaSuccess ||
-      cudaMallocHost(reinterpret_cast<void**>(&c->h_flag), sizeof(int)) != cudaSuccess ||
+      cudaHostAlloc(reinterpret_cast<void**>(&c->h_flag), sizeof(int), cudaHostAllocMapped) !=
+          cudaSuccess ||
+      cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->h_idx_dev), c->h_idx, 0) !=
+          cudaSuccess ||
+      cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->h_rec_dev), c->h_rec, 0) !=
+          cudaSuccess ||
+      cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->h_flag_dev), c->h_flag, 0) !=
+          cudaSuccess ||
       cudaHostAlloc(reinterpret_cast<void**>(&c->h_key), 2 * sizeof(uint64_t),
                     cudaHostAllocMapped) != cudaSuccess ||
       cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->h_key_dev), c->h_key, 0) !=
@@ -617,18 +624,11 @@ dp_status dp_audit_emit(dp_ctx* c, const int32_t* h_idx, int32_t n, void* h_reco
     if (h_idx[r] < 0 || h_idx[r] >= c->B)
       return fail(DP_ERR_ARG, "audit index %d out of range 0..%d", h_idx[r], c->B - 1);
   // The staging buffers are free here: every call synchronises before it
-  // returns, so no earlier copy can still be using them.
+  // returns, so no earlier gather can still be using them.
   const size_t rec_words = static_cast<size_t>(3 + c->L);
-  if (n > 0) {
-    std::memcpy(c->h_idx, h_idx, sizeof(int) * n);
-    DP_CUDA(cudaMemcpyAsync(c->d_idx, c->h_idx, sizeof(int) * n, cudaMemcpyHostToDevice,
-                            c->stream));
-    DP_CUDA(dpk::launch_audit(c->d_idx, n, c->L, c->B, c->d_layer_sq, c->d_s, c->d_c, c->d_rec,
-                              c->stream));
-    DP_CUDA(cudaMemcpyAsync(c->h_rec, c->d_rec, sizeof(float) * rec_words * n,
-                            cudaMemcpyDeviceToHost, c->stream));
-  }
-  DP_CUDA(cudaMemcpyAsync(c->h_flag, c->d_flag, sizeof(int), cudaMemcpyDeviceToHost, c->stream));
+  if (n > 0) std::memcpy(c->h_idx, h_idx, sizeof(int) * n);
+  DP_CUDA(dpk::launch_audit(c->h_idx_dev, n, c->L, c->B, c->d_layer_sq, c->d_s, c->d_c,
+                            c->d_flag, c->h_rec_dev, c->h_flag_dev, c->stream));
   DP_CUDA(cudaStreamSynchronize(c->stream));
   if (n > 0) std::memcpy(h_records, c->h_rec, sizeof(float) * rec_words * n);
   if (*c->h_flag & 2)

@@ -55,7 +55,8 @@ cudaError_t launch_noise_adamw(float* grad, float* theta, float* m, float* v, in
 
 // ---- audit gather ----
 cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer_sq,
-                         const float* s_vec, const float* c_vec, float* rec, cudaStream_t s);
+                         const float* s_vec, const float* c_vec, const int* flag, float* rec,
+                         int* flag_out, cudaStream_t s);
 
 // ---- noise key: device copy of two mapped pinned host words ----
 cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, cudaStream_t s);

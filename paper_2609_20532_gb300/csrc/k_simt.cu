@@ -321,14 +321,20 @@ __global__ void __launch_bounds__(256) k_noise_add(float* __restrict__ out, int6
 // ---------------------------------------------------------------------------
 // Audit gather: rec[r] = {idx, s, c, n_1..n_L}
 // ---------------------------------------------------------------------------
-__global__ void k_audit(const int* __restrict__ idx, int n, int L, int B,
+// Gather the audit records of the n requested examples.  idx, rec and
+// flag_out are device views of mapped pinned host memory: the indices are
+// read and the records written over the host link by this kernel, so an
+// audit uses no copy engine.  Thread 0 also reports the step's sticky flag.
+__global__ void k_audit(const volatile int* idx, int n, int L, int B,
                         const float* __restrict__ layer_sq, const float* __restrict__ s_vec,
-                        const float* __restrict__ c_vec, float* __restrict__ rec) {
+                        const float* __restrict__ c_vec, const int* __restrict__ flag,
+                        volatile float* rec, volatile int* flag_out) {
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r == 0) *flag_out = *flag;
   if (r >= n) return;
   const int i = idx[r];
-  float* o = rec + static_cast<int64_t>(r) * (3 + L);
-  reinterpret_cast<int*>(o)[0] = i;
+  volatile float* o = rec + static_cast<int64_t>(r) * (3 + L);
+  reinterpret_cast<volatile int*>(o)[0] = i;
   o[1] = s_vec[i];
   o[2] = c_vec[i];
   for (int l = 0; l < L; ++l) o[3 + l] = layer_sq[l * B + i];
@@ -471,9 +477,10 @@ cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, const uint6
 }
 
 cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer_sq,
-                         const float* s_vec, const float* c_vec, float* rec, cudaStream_t s) {
-  if (n <= 0) return cudaSuccess;
-  k_audit<<<(n + 127) / 128, 128, 0, s>>>(idx, n, L, B, layer_sq, s_vec, c_vec, rec);
+                         const float* s_vec, const float* c_vec, const int* flag, float* rec,
+                         int* flag_out, cudaStream_t s) {
+  const int blocks = n > 0 ? (n + 127) / 128 : 1;
+  k_audit<<<blocks, 128, 0, s>>>(idx, n, L, B, layer_sq, s_vec, c_vec, flag, rec, flag_out);
   return cudaGetLastError();
 }
 
