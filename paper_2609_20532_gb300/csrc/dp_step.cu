@@ -257,14 +257,15 @@ bool same_parts(const std::vector<LayerPlan>& a, const std::vector<LayerPlan>& b
   return true;
 }
 
-// Load the key words into device memory on the context's stream.  A
-// one-thread kernel reads the mapped pinned words when it runs (no copy-engine
-// queueing behind bulk host copies), so a CUDA graph that captured it loads
-// the key current at replay time (set with dp_set_noise_key).
+// Load the key words into device memory on the context's stream and clear
+// the sticky flag.  A one-thread kernel reads the mapped pinned words when it
+// runs (no copy-engine queueing behind bulk host copies: a step issues no
+// copy or memset of its own), so a CUDA graph that captured it loads the key
+// current at replay time (set with dp_set_noise_key).
 dp_status upload_key(dp_ctx* c) {
   c->h_key[0] = c->seed;
   c->h_key[1] = c->step;
-  DP_CUDA(dpk::launch_load_key(c->h_key_dev, c->d_key, c->stream));
+  DP_CUDA(dpk::launch_load_key(c->h_key_dev, c->d_key, c->d_flag, c->stream));
   return DP_OK;
 }
 
@@ -399,8 +400,7 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
       st = upload_plan(c);
       if (st != DP_OK) return st;
     }
-    // the sticky flag reports conditions of the current step only
-    DP_CUDA(cudaMemsetAsync(c->d_flag, 0, sizeof(int), c->stream));
+    // the key kernel also clears the sticky flag: it reports this step only
     st = upload_key(c);
     if (st != DP_OK) return st;
     reset_step(c);
@@ -422,10 +422,6 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     return st;
   }
   st = upload_plan(c);
-  if (st == DP_OK) {
-    cudaError_t e = cudaMemsetAsync(c->d_flag, 0, sizeof(int), c->stream);
-    if (e != cudaSuccess) st = fail(DP_ERR_CUDA, "cudaMemsetAsync: %s", cudaGetErrorString(e));
-  }
   if (st == DP_OK) st = upload_key(c);
   if (st != DP_OK) {
     free_scratch(c);

@@ -58,8 +58,10 @@ cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer
                          const float* s_vec, const float* c_vec, const int* flag, float* rec,
                          int* flag_out, cudaStream_t s);
 
-// ---- noise key: device copy of two mapped pinned host words ----
-cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, cudaStream_t s);
+// ---- start of a step: device copy of the two mapped pinned key words, and
+// the sticky flag cleared ----
+cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, int* flag,
+                            cudaStream_t s);
 
 // ---- error message of the calling thread, read back by dp_last_error() ----
 void set_last_error(const char* msg);

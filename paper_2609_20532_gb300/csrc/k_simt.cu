@@ -340,13 +340,16 @@ __global__ void k_audit(const volatile int* idx, int n, int L, int B,
   for (int l = 0; l < L; ++l) o[3 + l] = layer_sq[l * B + i];
 }
 
-// Copy the noise key from mapped pinned host memory to device memory.  A
-// kernel instead of a DMA copy: it runs on the SMs, so it never queues behind
+// Start of a step: copy the noise key from mapped pinned host memory to
+// device memory and clear the step's sticky flag word.  A kernel instead of
+// a DMA copy and a memset: it runs on the SMs, so it never queues behind
 // large host<->device copies on the copy engines, and inside a CUDA graph it
 // reads the host words current at replay time.
-__global__ void k_load_key(const volatile uint64_t* host_key, uint64_t* __restrict__ key) {
+__global__ void k_load_key(const volatile uint64_t* host_key, uint64_t* __restrict__ key,
+                           int* __restrict__ flag) {
   key[0] = host_key[0];
   key[1] = host_key[1];
+  *flag = 0;
 }
 
 __global__ void k_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
@@ -484,8 +487,9 @@ cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer
   return cudaGetLastError();
 }
 
-cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, cudaStream_t s) {
-  k_load_key<<<1, 1, 0, s>>>(host_key_dev, key);
+cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, int* flag,
+                            cudaStream_t s) {
+  k_load_key<<<1, 1, 0, s>>>(host_key_dev, key, flag);
   return cudaGetLastError();
 }
 

@@ -156,6 +156,24 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
   }
 }
 
+// S[4t .. 4t+3] += s * z for the warp-uniform quad slot q in [T0, T0 + N):
+// a binary tree of uniform branches down to static register indices, so the
+// accumulator stays in registers and each quad costs a few branches.
+template <int T0, int N>
+__device__ __forceinline__ void add_noise_slot(float (&S)[128], int q, float4 z, float s) {
+  if constexpr (N == 1) {
+    S[4 * T0 + 0] = fmaf(s, z.x, S[4 * T0 + 0]);
+    S[4 * T0 + 1] = fmaf(s, z.y, S[4 * T0 + 1]);
+    S[4 * T0 + 2] = fmaf(s, z.z, S[4 * T0 + 2]);
+    S[4 * T0 + 3] = fmaf(s, z.w, S[4 * T0 + 3]);
+  } else {
+    if (q < T0 + N / 2)
+      add_noise_slot<T0, N / 2>(S, q, z, s);
+    else
+      add_noise_slot<T0 + N / 2, N / 2>(S, q, z, s);
+  }
+}
+
 // Tile t of a layer -> (m tile, n tile).  Grouped raster: groups of
 // kRasterM consecutive m tiles, n runs over the whole layer inside a group
 // with m fastest, so the tiles in flight at one time share an A panel of
@@ -353,16 +371,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
               // parameters prow+k .. +3 form exactly one Philox quad
               if (k0 + 4 * q >= d_out) break;
               const float4 z = gauss_quad(seed, step, (prow + k0 + 4 * q) >> 2);
-              // static register indices: select the slot with a predicate
-#pragma unroll
-              for (int t = 0; t < 32; ++t) {
-                if (t == q) {
-                  S[4 * t + 0] = fmaf(g.sigmaC, z.x, S[4 * t + 0]);
-                  S[4 * t + 1] = fmaf(g.sigmaC, z.y, S[4 * t + 1]);
-                  S[4 * t + 2] = fmaf(g.sigmaC, z.z, S[4 * t + 2]);
-                  S[4 * t + 3] = fmaf(g.sigmaC, z.w, S[4 * t + 3]);
-                }
-              }
+              add_noise_slot<0, 32>(S, q, z, g.sigmaC);
             }
           }
         }
@@ -374,15 +383,16 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         float sq = 0.f;
         const float ci = NORM ? 0.f : (g.c ? g.c[ex] : 1.f);
 #pragma unroll
-        for (int ch = 0; ch < 4; ++ch) {
-          float v[32];
-          tmem_ld32(tmem_base + tcol + ch * 32, v);
+        for (int ch = 0; ch < 2; ++ch) {
+          uint32_t v[64];
+          tmem_ld64(tmem_base + tcol + ch * 64, v);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
+          for (int i = 0; i < 64; ++i) {
+            const float x = __uint_as_float(v[i]);
             if constexpr (NORM)
-              sq = fmaf(v[i], v[i], sq);
+              sq = fmaf(x, x, sq);
             else
-              S[ch * 32 + i] = fmaf(ci, v[i], S[ch * 32 + i]);
+              S[ch * 64 + i] = fmaf(ci, x, S[ch * 64 + i]);
           }
         }
         tc_fence_before();

@@ -295,6 +295,29 @@ def test_accumulate_over_microbatches():
     assert rel_err_normwise(out.cpu().numpy(), ref) <= 2e-3
 
 
+def test_accumulate_large_layer():
+    """DP_ACCUMULATE on a layer of 13 x 16 pair tiles (reduce-add stores)."""
+    w = W.custom("micro_cl4", [(4096, 3320)], 4, 64, "bf16", C=0.05, sigma=1.0, d_std=0.2,
+                 wid=604)
+    layers = W.make_inputs(w)
+    A, D = layers[0]
+    dev = torch.device(DEV)
+    out = torch.zeros(4096, 3320, device=dev)
+    ref = np.zeros((4096, 3320))
+    for h in range(2):
+        Ah, Dh = A[2 * h:2 * h + 2].contiguous(), D[2 * h:2 * h + 2].contiguous()
+        wh = W.custom("micro_cl4_h", [(4096, 3320)], 2, 64, "bf16", C=0.05, sigma=1.0, wid=604)
+        cfg = dp.make_config(wh.layers, 2, 64, "bf16", wh.C, wh.sigma)
+        ctx = dp.dp_step_init(cfg)
+        try:
+            dp.run_step(ctx, [Ah.to(dev)], [Dh.to(dev)], [out],
+                        flags=dp.DP_NO_NOISE | dp.DP_ACCUMULATE)
+        finally:
+            dp.dp_step_destroy(ctx)
+        ref += oracle_step(wh, [(Ah, Dh)], noise=False)["out"][0]
+    assert rel_err_normwise(out.cpu().numpy(), ref) <= 2e-3
+
+
 def test_deterministic_and_step_keyed():
     w = W.get("block_bf16")
     layers = W.make_inputs(w)
@@ -338,6 +361,8 @@ TC_CASES = [
     ([(384, 512)], 5, 192),              # 3 K-blocks per example, T not a power of 2
     ([(200, 520)], 3, 45),               # T padded to 64 per example (3-D maps)
     ([(264, 136), (64, 8)], 4, 97),      # padded, ragged
+    ([(3320, 3320)], 2, 64),             # 13 x 13 pair tiles, ragged in M and N
+    ([(3320, 4096)], 2, 96),             # 13 x 16 pair tiles, 3-D maps
 ]
 
 SMALL_T_CASES = [
