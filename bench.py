@@ -122,21 +122,32 @@ def replica_throughput(examples_per_rank: int, world: int, seconds_per_step: flo
     return world * examples_per_rank / seconds_per_step
 
 
-def _kernel_sha(path):
-    return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
+def _src_sha(paths):
+    """Hash of a kernel's source and the local headers it includes."""
+    h = hashlib.sha256()
+    for p in paths:
+        h.update(open(os.path.join(ROOT, p), "rb").read())
+    return h.hexdigest()[:16]
 
 
-def _traffic(kernel_key, flops_per_launch):
-    """DRAM bytes per launch of the GEMM from the committed ncu capture
-    (profiles/traffic.json), scaled from the captured shape by FLOPs, or None
-    when the kernel source changed since the counters were taken."""
-    p = os.path.join(ROOT, "profiles", "traffic.json")
+def _traffic(kernel_key, units, path=None):
+    """DRAM bytes per launch of a kernel from the committed ncu capture
+    (profiles/traffic.json), scaled from the captured case by the units of
+    work (FLOPs or input bytes), or None when the kernel's sources changed
+    since the counters were taken (or the entry is incomplete)."""
+    p = path or os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(p):
         return None
     d = json.load(open(p)).get(kernel_key)
-    if not d or d.get("src_sha256_16") != _kernel_sha(os.path.join(ROOT, d["src"])):
+    if not d or not d.get("captured_units") or "captured_dram_bytes" not in d:
         return None
-    return d["captured_dram_bytes"] * flops_per_launch / d["captured_flops"]
+    src = d.get("src")
+    src = [src] if isinstance(src, str) else list(src or [])
+    if not src or not all(os.path.exists(os.path.join(ROOT, f)) for f in src):
+        return None
+    if d.get("src_sha256_16") != _src_sha(src):
+        return None
+    return d["captured_dram_bytes"] * units / d["captured_units"]
 
 
 def cpu_baseline_sample(w, seed=0):
@@ -283,15 +294,18 @@ def run_ours(args, rank, world, local_rank):
     barrier()
     torch.cuda.synchronize()
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    marks = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
     with ClockSampler(local_rank) as clk:
         start.record(stream)
         for t in range(args.steps):
+            marks[t].record(stream)
             if graph is not None:
                 dp.dp_set_noise_key(ctx, cfg.seed, args.warmup + t)
                 graph.replay()
                 dp.dp_audit_emit(ctx, idx, L)
             else:
                 step(args.warmup + t, timed=True)
+        marks[args.steps].record(stream)
         stop.record(stream)
         torch.cuda.synchronize()
     barrier()
@@ -299,6 +313,19 @@ def run_ours(args, rank, world, local_rank):
     ms = max_over_ranks(start.elapsed_time(stop), world, dev)
     ms_step = ms / args.steps
     value = replica_throughput(w.B, world, ms_step * 1e-3)
+    ms_median = statistics.median(marks[t].elapsed_time(marks[t + 1]) for t in range(args.steps))
+
+    # the step without the audit emit: replays back to back under one key
+    # (the emit's synchronisation is what lets each replay take a new key)
+    ms_no_audit = None
+    if graph is not None:
+        e_a, e_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e_a.record(stream)
+        for t in range(args.steps):
+            graph.replay()
+        e_b.record(stream)
+        torch.cuda.synchronize()
+        ms_no_audit = e_a.elapsed_time(e_b) / args.steps
 
     if graph is not None:  # per-kernel split from one eager timed step
         step(args.warmup + args.steps, timed=True)
@@ -317,12 +344,15 @@ def run_ours(args, rank, world, local_rank):
     norm_gbs = in_total / (norm_ms * 1e-3) / 1e9
     # roofline of the dominant kernel (one launch per step covers every layer)
     traffic = _traffic("clipsum_gemm", gemm_flops)
+    norm_traffic = _traffic("ghost_norm", in_total)
     kernels = {
         "clipsum_gemm": {"ms_per_step": gemm_ms, "tflops": gemm_tflops,
                          "frac_bf16_peak": gemm_tflops / peaks["bf16_tflops"],
+                         "frac_bf16_sustained": (gemm_tflops / peaks["bf16_tflops_sustained"]
+                                                 if peaks.get("bf16_tflops_sustained") else None),
                          "launches_per_step": 1},
         "layer_norms": {"ms_per_step": norm_ms, "gbs_inputs_read_once": norm_gbs,
-                        "frac_hbm": norm_gbs / peaks["hbm_gbs"],
+                        "frac_hbm": norm_gbs / peaks["hbm_gbs"], "traffic": norm_traffic,
                         "launches_per_step": 1},
         "clip": {"ms_per_step": per_step_ms("clip")},
     }
@@ -444,7 +474,8 @@ def run_ours(args, rank, world, local_rank):
     dominant = "clipsum_gemm"
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "warmup": args.warmup, "ms_per_step": ms_step, "ms_per_step_median": ms_median,
+        "ms_per_step_no_audit": ms_no_audit, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
         "data": "synthetic: seeded N(0,1) activations, N(0,1e-5) output grads, rounded to bf16",
         "config": {"workload": w.describe(), "layers": [list(x) for x in w.layers], "B": w.B,
@@ -460,7 +491,9 @@ def run_ours(args, rank, world, local_rank):
         "kernels": kernels,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": args.steps * 4,
+        # per step: key + flag reset, norms (all layers), clip, clipped sums
+        # (all layers), audit gather
+        "gpu_launches": args.steps * 5,
         "clocks": clk.summary(),
     }
     print(json.dumps(line), flush=True)

@@ -230,12 +230,14 @@ int64_t dp_audit_record_bytes(int32_t n_layers);
 /* Norm mode chosen for a layer (resolves DP_NORM_AUTO). */
 dp_status dp_layer_norm_mode(const dp_ctx* ctx, int32_t layer, dp_norm_mode* mode_out);
 
-/* Replace the noise key (seed, step) without enqueuing any work, for CUDA
- * graphs: a step captured from dp_step_init on loads the key from mapped
- * pinned host memory when the graph runs, so calling this between replays
- * keys each replay (Algorithm 3's released seed s_noise,t).  The caller must not
- * call it while a previous replay that copies the key may still be pending
- * (dp_audit_emit, or any synchronisation of the stream, ensures that).
+/* Replace the noise key (seed, step) of CUDA graph replays without enqueuing
+ * any work.  A step captured from dp_step_init on loads the key from mapped
+ * pinned host memory when the graph runs (the capture's key until this call
+ * replaces it), so calling this between replays keys each replay (Algorithm
+ * 3's released seed s_noise,t).  The caller must not call it while a
+ * previous replay that copies the key may still be pending (dp_audit_emit,
+ * or any synchronisation of the stream, ensures that).  Eager steps are not
+ * affected: dp_step_init fixes their key when it enqueues them.
  * Host-only; the call-order state is unchanged.  Errors: DP_ERR_ARG. */
 dp_status dp_set_noise_key(dp_ctx* ctx, uint64_t seed, uint64_t step);
 

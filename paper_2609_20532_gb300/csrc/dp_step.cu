@@ -258,14 +258,22 @@ bool same_parts(const std::vector<LayerPlan>& a, const std::vector<LayerPlan>& b
 }
 
 // Load the key words into device memory on the context's stream and clear
-// the sticky flag.  A one-thread kernel reads the mapped pinned words when it
-// runs (no copy-engine queueing behind bulk host copies: a step issues no
-// copy or memset of its own), so a CUDA graph that captured it loads the key
-// current at replay time (set with dp_set_noise_key).
+// the sticky flag, with a one-thread kernel (a step issues no copy or memset
+// of its own, so nothing of it queues behind bulk host copies on the copy
+// engines).  Eager: the key is a kernel argument.  Under stream capture the
+// kernel reads the mapped pinned words when it runs instead, so a replay of
+// the captured step uses the key current at replay time (the capture's key
+// until dp_set_noise_key replaces it); an eager step leaves those words alone.
 dp_status upload_key(dp_ctx* c) {
-  c->h_key[0] = c->seed;
-  c->h_key[1] = c->step;
-  DP_CUDA(dpk::launch_load_key(c->h_key_dev, c->d_key, c->d_flag, c->stream));
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  DP_CUDA(cudaStreamIsCapturing(c->stream, &cs));
+  if (cs == cudaStreamCaptureStatusActive) {
+    c->h_key[0] = c->seed;
+    c->h_key[1] = c->step;
+    DP_CUDA(dpk::launch_load_key(c->h_key_dev, c->d_key, c->d_flag, c->stream));
+  } else {
+    DP_CUDA(dpk::launch_set_key(c->seed, c->step, c->d_key, c->d_flag, c->stream));
+  }
   return DP_OK;
 }
 

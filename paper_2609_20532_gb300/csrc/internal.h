@@ -62,6 +62,8 @@ cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer
 // the sticky flag cleared ----
 cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, int* flag,
                             cudaStream_t s);
+cudaError_t launch_set_key(uint64_t seed, uint64_t step, uint64_t* key, int* flag,
+                           cudaStream_t s);
 
 // ---- error message of the calling thread, read back by dp_last_error() ----
 void set_last_error(const char* msg);

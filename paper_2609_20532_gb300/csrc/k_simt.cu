@@ -352,6 +352,16 @@ __global__ void k_load_key(const volatile uint64_t* host_key, uint64_t* __restri
   *flag = 0;
 }
 
+// The same for eager launches: the key travels as a kernel argument, fixed
+// when the launch is enqueued, so a later re-key cannot reach a step that
+// is still queued.
+__global__ void k_set_key(uint64_t seed, uint64_t step, uint64_t* __restrict__ key,
+                          int* __restrict__ flag) {
+  key[0] = seed;
+  key[1] = step;
+  *flag = 0;
+}
+
 __global__ void k_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
                                uint32_t* __restrict__ out) {
   for (int64_t r = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; r < nq;
@@ -484,6 +494,12 @@ cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer
                          int* flag_out, cudaStream_t s) {
   const int blocks = n > 0 ? (n + 127) / 128 : 1;
   k_audit<<<blocks, 128, 0, s>>>(idx, n, L, B, layer_sq, s_vec, c_vec, flag, rec, flag_out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_set_key(uint64_t seed, uint64_t step, uint64_t* key, int* flag,
+                           cudaStream_t s) {
+  k_set_key<<<1, 1, 0, s>>>(seed, step, key, flag);
   return cudaGetLastError();
 }
 

@@ -58,3 +58,24 @@ def test_single_rank_is_identity():
     import bench
     assert bench.max_over_ranks(3.0, 1) == 3.0
     assert bench.replica_throughput(16, 1, 2e-3) == pytest.approx(8000.0)
+
+
+def test_traffic_lookup(tmp_path):
+    """profiles/traffic.json entries: scaled by units of work while the
+    kernel's sources hash to the recorded value, None once they change, for
+    an old single-file entry, or for an incomplete one."""
+    import json
+    sys.path.insert(0, ROOT)
+    import bench
+    src = ["paper_2609_20532_gb300/csrc/k_tc_gemm.cu", "paper_2609_20532_gb300/csrc/tc_util.cuh"]
+    good = {"src": src, "src_sha256_16": bench._src_sha(src), "captured_units": 100.0,
+            "captured_dram_bytes": 5000.0}
+    data = {"k": good, "stale": dict(good, src_sha256_16="0" * 16),
+            "old": {"src": src[0], "src_sha256_16": "x", "captured_flops": 1.0,
+                    "captured_dram_bytes": 1.0},
+            "partial": {"src": src}}
+    p = tmp_path / "traffic.json"
+    p.write_text(json.dumps(data))
+    assert bench._traffic("k", 250.0, str(p)) == 12500.0
+    for key in ("stale", "old", "partial", "missing"):
+        assert bench._traffic(key, 1.0, str(p)) is None

@@ -318,6 +318,38 @@ def test_accumulate_large_layer():
     assert rel_err_normwise(out.cpu().numpy(), ref) <= 2e-3
 
 
+def test_eager_rekey_does_not_reach_a_queued_step():
+    """Two steps enqueued back to back behind a long queue, re-keyed in
+    between with no synchronisation: each uses its own key (the eager key
+    is fixed when its launch is enqueued)."""
+    w = W.get("block_bf16")
+    layers = W.make_inputs(w)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    s = torch.cuda.Stream()
+    outs = [[torch.zeros(i, o, device=dev) for i, o in w.layers] for _ in range(2)]
+    x = torch.randn(8192, 8192, device=dev, dtype=torch.bfloat16)
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, seed=7, step=1)
+    ctx = dp.dp_step_init(cfg, s)
+    try:
+        torch.cuda.synchronize()
+        with torch.cuda.stream(s):
+            for _ in range(8):
+                x = (x @ x) * 1e-4          # milliseconds of queued work
+            for k, t in enumerate((1, 2)):
+                cfg.step = t
+                dp.dp_step_init(cfg, s, ctx)
+                dp.run_step(ctx, Ad, Dd, outs[k])
+        torch.cuda.synchronize()
+    finally:
+        dp.dp_step_destroy(ctx)
+    for k, t in enumerate((1, 2)):
+        ref = run_gpu_step(w, layers, seed=7, step=t)
+        for a, b in zip(outs[k], ref["out"]):
+            assert np.array_equal(a.cpu().numpy(), b)
+
+
 def test_deterministic_and_step_keyed():
     w = W.get("block_bf16")
     layers = W.make_inputs(w)
