@@ -593,6 +593,81 @@ def run_sweep(args):
     print(json.dumps(line), flush=True)
 
 
+def run_verifier(args):
+    """One JSON line timing the trusted side of Algorithm 1 on the host cores:
+    the structural check of the llm_bf16 commitment (every step), the fp32
+    and fp64 recomputations of a checked step (block_bf16 in full; llm_bf16
+    from one example through every layer, scaled by B), the audit-record
+    check of the audited examples, and what that costs per step at the
+    paper's audit rate.  The GPU commits the average that is checked."""
+    import numpy as np
+    import torch
+
+    import paper_2609_20532_gb300 as dp
+    from paper_2609_20532_gb300 import verifier as V
+    import workloads as W
+
+    def timed(fn, reps=1):
+        best = None
+        for _ in range(reps):
+            t0 = time.perf_counter()
+            out = fn()
+            dt = time.perf_counter() - t0
+            best = dt if best is None else min(best, dt)
+        return out, best
+
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    dev = torch.device("cuda:0")
+    res = {}
+    # block_bf16: a whole checked step against the GPU's commitment
+    w = W.get("block_bf16")
+    layers = W.make_inputs(w, seed=0)
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
+                         audit_capacity=w.B)
+    ctx = dp.dp_step_init(cfg)
+    outs = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    idx = W.audit_indices(w)
+    try:
+        dp.run_step(ctx, [A.to(dev) for A, _ in layers], [D.to(dev) for _, D in layers], outs,
+                    flags=dp.DP_NO_NOISE)
+        recs = dp.dp_audit_emit(ctx, idx, len(layers))
+    finally:
+        dp.dp_step_destroy(ctx)
+    g = [o.cpu().numpy() for o in outs]
+    (g32, _, _), t32 = timed(lambda: V.recompute_average(layers, w.C, np.float32))
+    (g64, _, _), t64 = timed(lambda: V.recompute_average(layers, w.C, np.float64))
+    prm = V.FAMILIES["roberta"]
+    ver = V.Verifier(prm, w.C, w.B, coin_seed=1)
+    r, tstep = timed(lambda: ver.step(g, lambda: g32, lambda: g64, checked=True))
+    rep, taudit = timed(lambda: V.check_audit_records(recs, layers, w.C, rtol=2e-3))
+    res["block_bf16"] = {"fp32_recompute_s": t32, "fp64_recompute_s": t64,
+                         "algorithm1_step_s_given_recomputes": tstep, "verdict": r.verdict,
+                         "path": r.path, "z32": r.z32, "audit_examples": len(idx),
+                         "audit_check_s": taudit, "audit_ok": rep.ok}
+    # llm_bf16: structural check on the real commitment size, recompute from
+    # one example through every layer scaled by B
+    w = W.get("llm_bf16")
+    P = w.n_params
+    flat = np.random.default_rng(0).standard_normal(P).astype(np.float32)
+    flat *= 0.5 * w.C / np.linalg.norm(flat.astype(np.float64))
+    _, tstruct = timed(lambda: bool(np.linalg.norm(flat.astype(np.float64)) <= w.C * 1.0001), 3)
+    one = [W.make_layer(w, l, seed=0, B=1) for l in range(len(w.layers))]
+    _, t1_32 = timed(lambda: V.recompute_average(one, w.C, np.float32))
+    _, t1_64 = timed(lambda: V.recompute_average(one, w.C, np.float64))
+    checked32 = t1_32 * w.B
+    res["llm_bf16"] = {"structural_check_s": tstruct, "fp32_recompute_s_est": checked32,
+                       "fp64_recompute_s_est": t1_64 * w.B,
+                       "estimate": "one example through all 3 layers, times B = 16",
+                       "per_step_s_at_p": tstruct + FAMILY_P * checked32,
+                       "p": FAMILY_P}
+    line = {"impl": "verifier", "metric": "trusted-side verification cost (Algorithm 1)",
+            "unit": "s", "cores": cores, "family": "roberta", "results": res}
+    print(json.dumps(line), flush=True)
+
+
+FAMILY_P = 0.1  # audit rate of every family in the paper's verifier table
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -605,6 +680,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--eager", action="store_true",
                     help="launch every call of a step instead of replaying a captured CUDA graph")
+    ap.add_argument("--verifier", action="store_true",
+                    help="time the trusted-side checker of Algorithm 1 on the host cores")
     ap.add_argument("--sweep", action="store_true",
                     help="time every point of the 4096x4096 sweep instead of one workload")
     args = ap.parse_args()
@@ -617,6 +694,10 @@ def main():
         return
     if args.sweep:
         run_sweep(args)
+        return
+    if args.verifier:
+        if rank == 0:
+            run_verifier(args)
         return
     if world > 1:
         import torch

@@ -763,3 +763,39 @@ def test_noise_adamw_argument_errors():
             dp.dp_noise_adamw(ctx, 0, flat[1:], *x[1:], **hp)
     finally:
         dp.dp_step_destroy(ctx)
+
+
+# ---------------------------------------------------------------------------
+# the trusted side consumes the GPU's commitment and audit records (Algorithm 1)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("name,fam", [("mlp_fp32", "roberta"), ("block_bf16", "gpt2"),
+                                      ("mlp_fp32", "cifar10")])
+def test_verifier_accepts_gpu_commitment_and_rejects_tampering(name, fam):
+    from paper_2609_20532_gb300 import verifier as V
+    w = W.get(name)
+    layers = W.make_inputs(w, seed=0)
+    res = run_gpu_step(w, layers, out_scale=1.0 / w.B, flags=dp.DP_NO_NOISE, audit=True)
+    C = f32(w.C)
+    prm = V.FAMILIES[fam]
+    g32 = V.recompute_average(layers, C, np.float32)[0]
+    g64 = V.recompute_average(layers, C, np.float64)[0]
+    ver = V.Verifier(prm, C, w.B, coin_seed=9)
+    r = ver.step(res["out"], lambda: g32, lambda: g64, checked=True)
+    assert r.verdict == V.ACCEPT and r.path == "body", r
+    assert r.z32 <= prm.tau_abs / 4
+    # the audit records of every example check against the fp64 recomputation
+    recs = np.zeros(w.B, dtype=dp.audit_dtype(len(layers)))
+    recs["example"] = res["rec_i"]
+    recs["total_sqnorm"] = res["rec_s"]
+    recs["clip_factor"] = res["rec_c"]
+    recs["layer_sqnorm"] = res["n"].T
+    rep = V.check_audit_records(recs, layers, C, rtol=TOL[w.dtype])
+    assert rep.ok, rep
+    # one layer's commitment nudged by 3 tau_abs C: the body path cannot hold it
+    bad = [o.copy() for o in res["out"]]
+    bad[0].reshape(-1)[0] += 3 * prm.tau_abs * C
+    r = V.Verifier(prm, C, w.B, coin_seed=9).step(bad, lambda: g32, lambda: g64, checked=True)
+    assert r.path in ("hard_reject", "ambiguity") and r.z32 > prm.tau_abs
+    if fam == "cifar10":
+        assert r.verdict == V.ABORT      # 3 tau_abs > rho_ill = 2 tau_abs
