@@ -19,13 +19,15 @@
  * Memory layout of every A / D argument: one dense row-major array
  * [B][T][d] (example-major, then position, then feature), element type from
  * dp_config.dtype, base address 16-byte aligned, rows d * elemsize bytes
- * apart.  d * elemsize must be a multiple of 16 bytes for bf16 inputs.
+ * apart.  bf16 layers whose d_in and d_out are multiples of 8 can run on
+ * tensor cores; other widths run on CUDA cores.
  * Outputs are fp32 row-major [d_in][d_out], 16-byte aligned.
  *
  * Ownership.  The caller owns every A, D and output buffer and the CUDA
  * stream; buffers are device pointers unless a parameter says "host".  The
  * context owns its scratch (per-layer norm partials, norms, clip factors,
- * audit staging, an error flag) and frees it in dp_step_destroy.
+ * audit staging, an error flag, the per-example gradients of thin layers)
+ * and frees it in dp_step_destroy.
  *
  * Asynchrony.  Every call except dp_audit_emit only enqueues work on the
  * context's stream and returns; dp_audit_emit synchronises that stream.
@@ -96,7 +98,7 @@ typedef struct {
 typedef struct {
     int32_t B;                 /* examples per step, >= 1 */
     int32_t T;                 /* positions per example, >= 1 */
-    int32_t n_layers;          /* L, 1 .. 64 */
+    int32_t n_layers;          /* L, 1 .. 1024 */
     const dp_layer* layers;    /* host array of L layer shapes; copied by dp_step_init */
     dp_dtype dtype;            /* element type of every A and D */
     float clip_C;              /* C > 0 */
@@ -176,6 +178,12 @@ dp_status dp_clip_factors(dp_ctx* ctx, float* d_sqnorm_out, float* d_clip_out);
  *   slots 2m, 2m+1 of the quad are sqrt(-2 ln u0) * (cos, sin)(2 pi u1).
  * flags: DP_NO_NOISE, DP_NOISE_ONLY, DP_ACCUMULATE (see above).
  * d_out: device fp32 [d_in][d_out], 16-byte aligned, owned by the caller.
+ * Thin layers.  When one side of a layer is at most 32 wide (LoRA factors,
+ *   small heads, bias rows) and 8 d_in d_out < T (d_in + d_out) elemsize,
+ *   dp_layer_norms stores the layer's per-example gradients G_{i,l} in the
+ *   context (B d_in d_out floats), and this call sums those in example order
+ *   instead of reading A and D again.  Its A and D must be the arrays given
+ *   to dp_layer_norms in this step; they are checked but not read.
  * Errors: DP_ERR_ARG, DP_ERR_ORDER (clip factors not formed yet, unless
  *   DP_NOISE_ONLY), DP_ERR_CUDA. */
 dp_status dp_clipped_sum_noise(dp_ctx* ctx, int32_t layer, const void* A, const void* D,
@@ -247,7 +255,10 @@ dp_status dp_set_noise_key(dp_ctx* ctx, uint64_t seed, uint64_t step);
  * materialised norm do when T is a multiple of 64 or T >= 32 (each example
  * padded to 64 positions), and for T < 32 the clipped sum runs on a
  * pre-scaled copy of A (c_i folded into a bf16 hi + lo pair held in context
- * scratch).  fp32 layers never use tensor cores. */
+ * scratch).  fp32 layers never use tensor cores.  Thin layers whose
+ * per-example gradients are stored by the norm pass (see
+ * dp_clipped_sum_noise) report *norm_tc = 2 and *sum_tc = 0: both passes run
+ * on CUDA cores. */
 dp_status dp_layer_path(const dp_ctx* ctx, int32_t layer, int32_t* norm_tc, int32_t* sum_tc);
 
 /* Release the context and all of its scratch; NULL is a no-op.  Waits for

@@ -229,10 +229,11 @@ def dp_layer_norm_mode(ctx: int, layer: int) -> int:
 
 
 def dp_layer_path(ctx: int, layer: int):
-    """(norm_on_tensor_cores, sum_on_tensor_cores) for a layer."""
+    """(norm path, sum path) of a layer: 1 = tensor cores, 0 = CUDA cores,
+    norm path 2 = thin layer with stored per-example gradients."""
     a, b = ctypes.c_int32(0), ctypes.c_int32(0)
     _check(lib().dp_layer_path(ctx, layer, ctypes.byref(a), ctypes.byref(b)))
-    return bool(a.value), bool(b.value)
+    return a.value, b.value
 
 
 def dp_set_noise_key(ctx: int, seed: int, step: int) -> None:

@@ -51,6 +51,8 @@ struct LayerPlan {
   int norm_tc;         // 1: tensor-core norm kernel
   int nparts;          // partial sums per example
   int gemm_tc;         // 0: CUDA-core clipped sum, 1: tcgen05, 2: tcgen05 on a pre-scaled operand
+  int pergrad;         // 1: thin layer, per-example gradients stored by the norm pass
+  int64_t g_off;       // offset (floats) of its [B][d_in][d_out] gradients in d_grads
 };
 
 struct dp_ctx {
@@ -85,6 +87,8 @@ struct dp_ctx {
   uint64_t* h_key_dev = nullptr;  // the same words, device address
   void* d_prescaled = nullptr;  // pre-scaled operand of short-example layers
   int64_t prescaled_bytes = 0;
+  float* d_grads = nullptr;     // per-example gradients of thin layers
+  int64_t grads_floats = 0;
   size_t part_bytes = 0;
   // per-step state
   std::vector<char> norm_done;
@@ -98,16 +102,14 @@ dp_status check_config(const dp_config* cfg) {
   if (cfg->B < 1 || cfg->T < 1) return fail(DP_ERR_SHAPE, "B and T must be >= 1");
   if (static_cast<int64_t>(cfg->B) * cfg->T > 0x7fffffffLL)
     return fail(DP_ERR_SHAPE, "B*T exceeds 2^31-1");
-  if (cfg->n_layers < 1 || cfg->n_layers > 64)
-    return fail(DP_ERR_SHAPE, "n_layers must be in 1..64");
+  if (cfg->n_layers < 1 || cfg->n_layers > 1024)
+    return fail(DP_ERR_SHAPE, "n_layers must be in 1..1024");
   if (!cfg->layers) return fail(DP_ERR_ARG, "layers is NULL");
   if (cfg->dtype != DP_F32 && cfg->dtype != DP_BF16) return fail(DP_ERR_DTYPE, "unknown dtype");
   for (int l = 0; l < cfg->n_layers; ++l) {
     const dp_layer& ly = cfg->layers[l];
     if (ly.d_in < 1 || ly.d_out < 1 || ly.d_in > (1 << 20) || ly.d_out > (1 << 20))
       return fail(DP_ERR_SHAPE, "layer %d: d_in, d_out must be in 1..2^20", l);
-    if (cfg->dtype == DP_BF16 && ((ly.d_in * 2) % 16 || (ly.d_out * 2) % 16))
-      return fail(DP_ERR_SHAPE, "layer %d: bf16 rows must be a multiple of 16 bytes", l);
   }
   if (!(cfg->clip_C > 0.f) || !std::isfinite(cfg->clip_C))
     return fail(DP_ERR_ARG, "clip_C must be finite and > 0");
@@ -133,9 +135,23 @@ dp_norm_mode resolve_mode(dp_norm_mode m, int T, int64_t d_in, int64_t d_out) {
   return ghost <= mat ? DP_NORM_GHOST : DP_NORM_MATERIALISED;
 }
 
+// A thin layer (narrow side <= kThinMax) stores its per-example gradients
+// when writing and reading them back moves fewer bytes than reading A and D
+// a second time: 8 d_in d_out < T (d_in + d_out) elem.  That also makes the
+// materialised norm the cheaper one (T > 4 r), so a forced Gram or rank-1
+// mode keeps the other paths.
+bool use_pergrad(const dp_config* cfg, int64_t d_in, int64_t d_out) {
+  if (cfg->norm_mode == DP_NORM_GHOST || cfg->norm_mode == DP_NORM_RANK1) return false;
+  const int64_t r = d_in < d_out ? d_in : d_out;
+  if (r > dpk::kThinMax) return false;
+  const double elem = cfg->dtype == DP_BF16 ? 2.0 : 4.0;
+  return 8.0 * double(d_in) * double(d_out) < double(cfg->T) * double(d_in + d_out) * elem;
+}
+
 void build_plan(dp_ctx* c, const dp_config* cfg) {
   c->plan.resize(cfg->n_layers);
   uint64_t off = 0;
+  int64_t grads = 0;
   int NP = 1;
   for (int l = 0; l < cfg->n_layers; ++l) {
     LayerPlan& p = c->plan[l];
@@ -143,6 +159,18 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
     p.d_out = cfg->layers[l].d_out;
     p.p_base = off;
     off += static_cast<uint64_t>(p.d_in) * p.d_out;
+    p.pergrad = use_pergrad(cfg, p.d_in, p.d_out) ? 1 : 0;
+    p.g_off = 0;
+    if (p.pergrad) {
+      p.mode = DP_NORM_MATERIALISED;
+      p.norm_tc = 0;
+      p.gemm_tc = 0;
+      p.nparts = dpk::pergrad_parts(p.d_in, p.d_out);
+      p.g_off = grads;
+      grads += static_cast<int64_t>(cfg->B) * p.d_in * p.d_out;
+      if (p.nparts > NP) NP = p.nparts;
+      continue;
+    }
     p.mode = resolve_mode(cfg->norm_mode, cfg->T, p.d_in, p.d_out);
     const bool bf16 = cfg->dtype == DP_BF16;
     p.norm_tc = 0;
@@ -167,6 +195,7 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
     if (p.nparts > NP) NP = p.nparts;
   }
   c->NP = NP;
+  c->grads_floats = grads;
 }
 
 void free_scratch(dp_ctx* c) {
@@ -180,7 +209,9 @@ void free_scratch(dp_ctx* c) {
   cudaFreeHost(c->h_rec);
   cudaFreeHost(c->h_flag);
   cudaFree(c->d_prescaled);
+  cudaFree(c->d_grads);
   c->d_prescaled = nullptr;
+  c->d_grads = nullptr;
   cudaFree(c->d_key);
   cudaFreeHost(c->h_key);
   c->d_key = nullptr;
@@ -214,6 +245,7 @@ dp_status alloc_scratch(dp_ctx* c) {
   DP_ALLOC(c->d_c, sizeof(float) * B);
   DP_ALLOC(c->d_flag, sizeof(int));
   if (c->prescaled_bytes > 0) DP_ALLOC(c->d_prescaled, static_cast<size_t>(c->prescaled_bytes));
+  if (c->grads_floats > 0) DP_ALLOC(c->d_grads, sizeof(float) * static_cast<size_t>(c->grads_floats));
   DP_ALLOC(c->d_key, 2 * sizeof(uint64_t));
 #undef DP_ALLOC
   if (cudaHostAlloc(reinterpret_cast<void**>(&c->h_idx), sizeof(int) * (cap > 0 ? cap : 1),
@@ -313,9 +345,51 @@ dp_status check_norm_args(dp_ctx* c, int32_t layer, const void* A, const void* D
   return DP_OK;
 }
 
+void fill_pergrad(const dp_ctx* c, int32_t layer, const void* A, const void* D,
+                  dpk::PerGradLayer& P) {
+  const LayerPlan& p = c->plan[layer];
+  P.wide_is_in = p.d_in >= p.d_out ? 1 : 0;
+  P.X = P.wide_is_in ? A : D;
+  P.Y = P.wide_is_in ? D : A;
+  P.n = static_cast<int>(P.wide_is_in ? p.d_in : p.d_out);
+  P.r = static_cast<int>(P.wide_is_in ? p.d_out : p.d_in);
+  P.G = c->d_grads + p.g_off;
+  P.row0 = layer * c->B;
+}
+
+void fill_pergrad_sum(const dp_ctx* c, int32_t layer, float* d_out, dpk::PerGradSumLayer& P) {
+  const LayerPlan& p = c->plan[layer];
+  P.G = c->d_grads + p.g_off;
+  P.out = d_out;
+  P.count = p.d_in * p.d_out;
+  P.p_base = p.p_base;
+}
+
+dpk::PerGradSumBatch pergrad_sum_batch(const dp_ctx* c, uint32_t flags) {
+  dpk::PerGradSumBatch g{};
+  g.c = c->d_c;
+  g.key = c->d_key;
+  g.out_scale = c->out_scale;
+  g.sigmaC = c->sigma * c->C;
+  g.add_noise = (flags & DP_NO_NOISE) ? 0 : 1;
+  g.accumulate = (flags & DP_ACCUMULATE) ? 1 : 0;
+  g.B = c->B;
+  return g;
+}
+
 cudaError_t launch_layer_norms(dp_ctx* c, int32_t layer, const void* A, const void* D) {
   const LayerPlan& p = c->plan[layer];
   const dpk::InType it = c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32;
+  if (p.pergrad) {
+    dpk::PerGradBatch g{};
+    fill_pergrad(c, layer, A, D, g.l[0]);
+    g.L = 1;
+    g.part = c->d_part;
+    g.B = c->B;
+    g.T = c->T;
+    g.NP = c->NP;
+    return dpk::launch_pergrad_norm(it, g, c->stream);
+  }
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
   const int row0 = layer * c->B;
   if (p.mode == DP_NORM_RANK1)
@@ -365,6 +439,12 @@ cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const vo
   if (flags & DP_NOISE_ONLY)
     return dpk::launch_noise_add(d_out, p.d_in * p.d_out, p.p_base, c->d_key,
                                  c->out_scale * ep.sigmaC, c->stream);
+  if (p.pergrad) {
+    dpk::PerGradSumBatch g = pergrad_sum_batch(c, flags);
+    fill_pergrad_sum(c, layer, d_out, g.l[0]);
+    g.L = 1;
+    return dpk::launch_pergrad_sum(g, c->stream);
+  }
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
   if (p.gemm_tc == 1)
     return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep, c->d_flag,
@@ -395,14 +475,17 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     std::vector<LayerPlan> old = c->plan;
     const int oldNP = c->NP;
     const int64_t old_pre = c->prescaled_bytes;
+    const int64_t old_grads = c->grads_floats;
     build_plan(c, cfg);
     c->prescaled_bytes = old_pre;  // shapes are unchanged, so is the pre-scale need
-    if (c->NP > oldNP) {
+    if (c->NP > oldNP || c->grads_floats > old_grads) {
       c->plan = old;
       c->NP = oldNP;
+      c->grads_floats = old_grads;
       return fail(DP_ERR_SHAPE, "norm_mode change needs more scratch; destroy and re-create");
     }
     c->NP = oldNP;  // keep the allocated stride
+    c->grads_floats = old_grads;
     set_scalars(c, cfg, cuda_stream);
     if (!same_parts(old, c->plan)) {
       st = upload_plan(c);
@@ -485,10 +568,32 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
     grp.clear();
     return e;
   };
+  // Thin layers share launches too, one list per narrow-width bucket.
+  const dpk::InType it = c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32;
+  std::vector<int> thin[6];
+  auto flush_thin = [&](std::vector<int>& v) -> cudaError_t {
+    if (v.empty()) return cudaSuccess;
+    dpk::PerGradBatch g{};
+    for (size_t q = 0; q < v.size(); ++q) fill_pergrad(c, layers[v[q]], A[v[q]], D[v[q]], g.l[q]);
+    g.L = static_cast<int>(v.size());
+    g.part = c->d_part;
+    g.B = c->B;
+    g.T = c->T;
+    g.NP = c->NP;
+    v.clear();
+    return dpk::launch_pergrad_norm(it, g, c->stream);
+  };
   for (int r = 0; r < n; ++r) {
     const LayerPlan& p = c->plan[layers[r]];
     cudaError_t e = cudaSuccess;
-    if (p.mode == DP_NORM_GHOST && p.norm_tc) {
+    if (p.pergrad) {
+      const int nar = static_cast<int>(p.d_in < p.d_out ? p.d_in : p.d_out);
+      const int bucket = dpk::pergrad_bucket(nar);
+      int b = 0;
+      while ((1 << b) < bucket) ++b;
+      thin[b].push_back(r);
+      if (static_cast<int>(thin[b].size()) == dpk::kPerGradMaxLayers) e = flush_thin(thin[b]);
+    } else if (p.mode == DP_NORM_GHOST && p.norm_tc) {
       grp.push_back(r);
       if (static_cast<int>(grp.size()) == dpk::kGhostMaxLayers) e = flush();
     } else {
@@ -498,6 +603,7 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
       return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
   }
   cudaError_t e = flush();
+  for (int b = 0; b < 6 && e == cudaSuccess; ++b) e = flush_thin(thin[b]);
   if (e != cudaSuccess) return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
   for (int r = 0; r < n; ++r) c->norm_done[layers[r]] = 1;
   return DP_OK;
@@ -546,6 +652,17 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
   // kGemmMaxLayers each); every other layer gets its own kernel.
   std::vector<int> grp;
   dpk::Epilogue ep = make_epilogue(c, flags, 0);
+  // thin layers: one summing launch over their stored per-example gradients
+  std::vector<int> thin;
+  auto flush_thin = [&]() -> cudaError_t {
+    if (thin.empty()) return cudaSuccess;
+    dpk::PerGradSumBatch g = pergrad_sum_batch(c, flags);
+    for (size_t q = 0; q < thin.size(); ++q)
+      fill_pergrad_sum(c, layers[thin[q]], d_out[thin[q]], g.l[q]);
+    g.L = static_cast<int>(thin.size());
+    thin.clear();
+    return dpk::launch_pergrad_sum(g, c->stream);
+  };
   auto flush = [&]() -> cudaError_t {
     if (grp.empty()) return cudaSuccess;
     const void* a[dpk::kGemmMaxLayers];
@@ -577,6 +694,9 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
         e = flush();
       grp.push_back(r);
       if (e == cudaSuccess && static_cast<int>(grp.size()) == dpk::kGemmMaxLayers) e = flush();
+    } else if (!(flags & DP_NOISE_ONLY) && p.pergrad) {
+      thin.push_back(r);
+      if (static_cast<int>(thin.size()) == dpk::kPerGradMaxLayers) e = flush_thin();
     } else {
       e = launch_clipped_sum(c, l, (flags & DP_NOISE_ONLY) ? nullptr : A[r],
                              (flags & DP_NOISE_ONLY) ? nullptr : D[r], d_out[r], flags);
@@ -584,6 +704,7 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
     if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clipped-sum kernel: %s", cudaGetErrorString(e));
   }
   cudaError_t e = flush();
+  if (e == cudaSuccess) e = flush_thin();
   if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clipped-sum kernel: %s", cudaGetErrorString(e));
   return DP_OK;
 }
@@ -662,7 +783,7 @@ dp_status dp_set_noise_key(dp_ctx* c, uint64_t seed, uint64_t step) {
 dp_status dp_layer_path(const dp_ctx* c, int32_t layer, int32_t* norm_tc, int32_t* sum_tc) {
   if (!c || !norm_tc || !sum_tc) return fail(DP_ERR_ARG, "NULL argument");
   if (layer < 0 || layer >= c->L) return fail(DP_ERR_ARG, "layer %d out of range", layer);
-  *norm_tc = c->plan[layer].norm_tc;
+  *norm_tc = c->plan[layer].pergrad ? 2 : c->plan[layer].norm_tc;
   *sum_tc = c->plan[layer].gemm_tc != 0;
   return DP_OK;
 }

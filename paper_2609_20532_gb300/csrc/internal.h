@@ -44,6 +44,46 @@ cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float
 cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, const uint64_t* key,
                              float scale, cudaStream_t s);
 
+// ---- thin layers: per-example gradients stored by the norm pass ----
+constexpr int kThinMax = 32;           // widest narrow side of a thin layer
+constexpr int kPerGradMaxLayers = 32;  // layers per launch
+struct PerGradLayer {
+  const void* X;   // wide operand [B][T][n]
+  const void* Y;   // narrow operand [B][T][r]
+  float* G;        // per-example gradients [B][d_in][d_out]
+  int n, r;        // wide and narrow widths
+  int wide_is_in;  // 1: X = A (n = d_in), 0: X = D (n = d_out)
+  int chunks;      // blocks per example (set by the launcher)
+  int row0;        // partial-sum row of example 0
+  int item0;       // first block of this layer (set by the launcher)
+};
+struct PerGradBatch {
+  PerGradLayer l[kPerGradMaxLayers];
+  float* part;
+  int L, B, T, NP;
+};
+struct PerGradSumLayer {
+  const float* G;   // [B][count]
+  float* out;       // [count]
+  int64_t count;    // d_in * d_out
+  uint64_t p_base;  // global parameter index of element 0
+  int64_t nq;       // quads (set by the launcher)
+  int64_t item0;    // first thread (set by the launcher)
+  int vec;          // float4 path (set by the launcher)
+};
+struct PerGradSumBatch {
+  PerGradSumLayer l[kPerGradMaxLayers];
+  const float* c;
+  const uint64_t* key;
+  float out_scale, sigmaC;
+  int add_noise, accumulate;
+  int L, B;
+};
+int pergrad_bucket(int r);                       // 1, 2, 4, ..., 32, or 0 if too wide
+int pergrad_parts(int64_t d_in, int64_t d_out);  // partials per example
+cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s);
+cudaError_t launch_pergrad_sum(PerGradSumBatch& g, cudaStream_t s);
+
 // ---- noisy gradient + AdamW after the seed release ----
 struct AdamWArgs {
   float lr, beta1, beta2, eps, weight_decay;

@@ -1,0 +1,239 @@
+// Thin layers: one side of the weight at most kThinMax wide (LoRA factors of
+// rank r, small classification heads, bias rows).  For them the per-example
+// gradient g_i = A_i^T D_i of Sec. 2.2 is smaller than the example's inputs,
+// so the norm pass materialises it once in context scratch and the clipped
+// sum reads it back instead of reading A and D a second time:
+//
+//   norm pass   g_i = A_i^T D_i (fp32),  n_i = ||g_i||_F^2 (fixed-order
+//               partials per 256-column slice of the wide side)
+//   sum pass    out = out_scale (sum_i c_i g_i + sigma C z)   (examples in
+//               order, so the result is the same on every run)
+//
+// The wide operand X ([B][T][n], n = the wide width) is read row by row,
+// coalesced; the narrow operand Y ([B][T][r]) is staged in shared memory and
+// broadcast.  Each thread owns VJ consecutive wide columns and all r narrow
+// ones.  One launch serves up to kPerGradMaxLayers layers of the same
+// narrow-width bucket and input type.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "internal.h"
+#include "philox.cuh"
+
+namespace dpk {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int TT = 64;  // positions staged per round
+
+__device__ __forceinline__ float to_float(float x) { return x; }
+__device__ __forceinline__ float to_float(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <int R>
+struct Vj {
+  static constexpr int value = R <= 8 ? 4 : (R <= 16 ? 2 : 1);
+};
+
+__device__ __forceinline__ int find_layer(const PerGradBatch& g, int item) {
+  int l = 0;
+  while (l + 1 < g.L && item >= g.l[l + 1].item0) ++l;
+  return l;
+}
+
+template <typename TIn, int R>
+__global__ void __launch_bounds__(kThreads) k_pergrad_norm(const __grid_constant__ PerGradBatch g) {
+  constexpr int VJ = Vj<R>::value;
+  __shared__ __align__(16) float ys[TT][R];
+  __shared__ float red[kThreads / 32];
+  const int l = find_layer(g, blockIdx.x);
+  const PerGradLayer& P = g.l[l];
+  const int local = static_cast<int>(blockIdx.x) - P.item0;
+  const int i = local / P.chunks, chunk = local - i * P.chunks;
+  const int n = P.n, r = P.r, T = g.T;
+  const TIn* X = static_cast<const TIn*>(P.X) + static_cast<int64_t>(i) * T * n;
+  const TIn* Y = static_cast<const TIn*>(P.Y) + static_cast<int64_t>(i) * T * r;
+  const int j0 = (chunk * kThreads + static_cast<int>(threadIdx.x)) * VJ;
+  float acc[VJ][R];
+#pragma unroll
+  for (int v = 0; v < VJ; ++v)
+#pragma unroll
+    for (int k = 0; k < R; ++k) acc[v][k] = 0.f;
+
+  for (int t0 = 0; t0 < T; t0 += TT) {
+    const int tt = T - t0 < TT ? T - t0 : TT;
+    for (int e = threadIdx.x; e < TT * R; e += kThreads) {
+      const int t = e / R, k = e - (e / R) * R;
+      ys[t][k] = (t < tt && k < r) ? to_float(Y[static_cast<int64_t>(t0 + t) * r + k]) : 0.f;
+    }
+    __syncthreads();
+    if (j0 < n) {
+      const TIn* xrow = X + static_cast<int64_t>(t0) * n + j0;
+#pragma unroll 4
+      for (int t = 0; t < tt; ++t, xrow += n) {
+        float x[VJ];
+#pragma unroll
+        for (int v = 0; v < VJ; ++v) x[v] = (j0 + v < n) ? to_float(xrow[v]) : 0.f;
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+          const float y = ys[t][k];
+#pragma unroll
+          for (int v = 0; v < VJ; ++v) acc[v][k] = fmaf(x[v], y, acc[v][k]);
+        }
+      }
+    }
+    __syncthreads();
+  }
+
+  // g_i rows are [d_in][d_out]: X = A gives G[j][k], X = D gives G[k][j]
+  float* G = P.G + static_cast<int64_t>(i) * n * r;
+  float sq = 0.f;
+#pragma unroll
+  for (int v = 0; v < VJ; ++v) {
+    const int j = j0 + v;
+    if (j >= n) continue;
+#pragma unroll
+    for (int k = 0; k < R; ++k) {
+      if (k >= r) continue;
+      const float val = acc[v][k];
+      sq = fmaf(val, val, sq);
+      if (P.wide_is_in)
+        G[static_cast<int64_t>(j) * r + k] = val;
+      else
+        G[static_cast<int64_t>(k) * n + j] = val;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sq;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+    for (int w = 0; w < kThreads / 32; ++w) s += red[w];
+    g.part[static_cast<int64_t>(P.row0 + i) * g.NP + chunk] = s;
+  }
+}
+
+// out = out_scale (sum_i c_i g_i + sigma C z) over the global quads that
+// overlap each layer's parameters; examples are summed in index order.
+__global__ void __launch_bounds__(kThreads) k_pergrad_sum(const __grid_constant__ PerGradSumBatch g) {
+  int l = 0;
+  while (l + 1 < g.L && static_cast<int64_t>(blockIdx.x) * kThreads >= g.l[l + 1].item0) ++l;
+  const PerGradSumLayer& P = g.l[l];
+  const int64_t local = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x - P.item0;
+  if (local >= P.nq) return;
+  const uint64_t q = (P.p_base >> 2) + static_cast<uint64_t>(local);
+  const int64_t e0 = static_cast<int64_t>(4 * q) - static_cast<int64_t>(P.p_base);
+  const int64_t n = P.count;
+  float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (g.add_noise) z = gauss_quad(g.key[0], g.key[1], q);
+  const float zv[4] = {z.x, z.y, z.z, z.w};
+  const bool vec = P.vec && e0 >= 0 && e0 + 3 < n;
+  float s[4] = {0.f, 0.f, 0.f, 0.f};
+  if (vec) {
+    const float* gp = P.G + e0;
+#pragma unroll 4
+    for (int i = 0; i < g.B; ++i, gp += n) {
+      const float ci = g.c[i];
+      const float4 v = *reinterpret_cast<const float4*>(gp);
+      s[0] = fmaf(ci, v.x, s[0]);
+      s[1] = fmaf(ci, v.y, s[1]);
+      s[2] = fmaf(ci, v.z, s[2]);
+      s[3] = fmaf(ci, v.w, s[3]);
+    }
+  } else {
+    for (int i = 0; i < g.B; ++i) {
+      const float ci = g.c[i];
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const int64_t e = e0 + w;
+        if (e >= 0 && e < n) s[w] = fmaf(ci, P.G[static_cast<int64_t>(i) * n + e], s[w]);
+      }
+    }
+  }
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    const int64_t e = e0 + w;
+    if (e < 0 || e >= n) continue;
+    const float val = g.out_scale * fmaf(g.sigmaC, zv[w], s[w]);
+    P.out[e] = g.accumulate ? P.out[e] + val : val;
+  }
+}
+
+template <typename TIn, int R>
+cudaError_t launch_norm_t(const PerGradBatch& g, int blocks, cudaStream_t s) {
+  k_pergrad_norm<TIn, R><<<blocks, kThreads, 0, s>>>(g);
+  return cudaGetLastError();
+}
+
+template <typename TIn>
+cudaError_t launch_norm_r(const PerGradBatch& g, int R, int blocks, cudaStream_t s) {
+  switch (R) {
+    case 1: return launch_norm_t<TIn, 1>(g, blocks, s);
+    case 2: return launch_norm_t<TIn, 2>(g, blocks, s);
+    case 4: return launch_norm_t<TIn, 4>(g, blocks, s);
+    case 8: return launch_norm_t<TIn, 8>(g, blocks, s);
+    case 16: return launch_norm_t<TIn, 16>(g, blocks, s);
+    case 32: return launch_norm_t<TIn, 32>(g, blocks, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+
+int pergrad_bucket(int r) {
+  int R = 1;
+  while (R < r) R <<= 1;
+  return R <= kThinMax ? R : 0;
+}
+
+int pergrad_parts(int64_t d_in, int64_t d_out) {
+  const int r = static_cast<int>(d_in < d_out ? d_in : d_out);
+  const int64_t n = d_in < d_out ? d_out : d_in;
+  const int R = pergrad_bucket(r);
+  if (R == 0) return 0;
+  const int vj = R <= 8 ? 4 : (R <= 16 ? 2 : 1);
+  return static_cast<int>((n + kThreads * vj - 1) / (kThreads * vj));
+}
+
+cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s) {
+  if (g.L < 1 || g.L > kPerGradMaxLayers) return cudaErrorInvalidValue;
+  int R = 0;
+  int64_t blocks = 0;
+  for (int l = 0; l < g.L; ++l) {
+    PerGradLayer& P = g.l[l];
+    const int Rl = pergrad_bucket(P.r);
+    if (Rl == 0) return cudaErrorInvalidValue;
+    if (Rl > R) R = Rl;
+  }
+  const int vj = R <= 8 ? 4 : (R <= 16 ? 2 : 1);
+  for (int l = 0; l < g.L; ++l) {
+    PerGradLayer& P = g.l[l];
+    P.chunks = static_cast<int>((P.n + kThreads * vj - 1) / (kThreads * vj));
+    P.item0 = static_cast<int>(blocks);
+    blocks += static_cast<int64_t>(g.B) * P.chunks;
+  }
+  if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+  return t == IN_F32 ? launch_norm_r<float>(g, R, static_cast<int>(blocks), s)
+                     : launch_norm_r<__nv_bfloat16>(g, R, static_cast<int>(blocks), s);
+}
+
+cudaError_t launch_pergrad_sum(PerGradSumBatch& g, cudaStream_t s) {
+  if (g.L < 1 || g.L > kPerGradMaxLayers) return cudaErrorInvalidValue;
+  int64_t threads = 0;
+  for (int l = 0; l < g.L; ++l) {
+    PerGradSumLayer& P = g.l[l];
+    P.nq = static_cast<int64_t>(((P.p_base + P.count - 1) >> 2) - (P.p_base >> 2) + 1);
+    P.vec = (P.p_base % 4 == 0) && (P.count % 4 == 0) &&
+            (reinterpret_cast<uintptr_t>(P.G) % 16 == 0);
+    // each layer starts on a block boundary
+    P.item0 = threads;
+    threads += ((P.nq + kThreads - 1) / kThreads) * kThreads;
+  }
+  const int64_t blocks = threads / kThreads;
+  if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+  k_pergrad_sum<<<static_cast<int>(blocks), kThreads, 0, s>>>(g);
+  return cudaGetLastError();
+}
+
+}  // namespace dpk

@@ -31,6 +31,13 @@ def _gpu():
     dp.lib()  # fails loudly if the library was not built
 
 
+def is_thin(d_in, d_out, T, dtype):
+    """The library's rule for layers whose per-example gradients the norm pass
+    stores (include/dp_step.h, dp_clipped_sum_noise)."""
+    elem = 2 if dtype == "bf16" else 4
+    return min(d_in, d_out) <= 32 and 8 * d_in * d_out < T * (d_in + d_out) * elem
+
+
 def oracle_step(w, layers, seed=0, step=0, out_scale=1.0, noise=True, norm="materialised"):
     return O.dp_step([(W.to_f64(A), W.to_f64(D)) for A, D in layers], f32(w.C), f32(w.sigma),
                      seed, step, out_scale=f32(out_scale), noise=noise, norm=norm)
@@ -387,7 +394,7 @@ def test_noise_statistics_on_device():
 TC_CASES = [
     # (layers, B, T): bf16 layers whose clipped sum and norms run on tcgen05
     ([(200, 264)], 3, 64),               # ragged M and N tiles
-    ([(8, 8), (16, 24)], 2, 64),         # tiles far smaller than one MMA
+    ([(40, 48), (48, 56)], 2, 64),       # tiles far smaller than one MMA (not thin)
     ([(520, 1000), (1000, 136)], 2, 128),
     ([(4096, 4096)], 2, 64),             # 512 tiles > SM count: persistent loop
     ([(384, 512)], 5, 192),              # 3 K-blocks per example, T not a power of 2
@@ -413,7 +420,9 @@ def test_tensor_core_paths(case, mode):
                  wid=700 + case)
     layers = W.make_inputs(w, seed=2)
     res = run_gpu_step(w, layers, seed=5, step=1, norm_mode=mode)
-    assert all(n and s for n, s in res["paths"]), res["paths"]
+    for (di, do), path in zip(shapes, res["paths"]):
+        thin = mode != dp.DP_NORM_GHOST and is_thin(di, do, T, "bf16")
+        assert path == ((2, 0) if thin else (1, 1)), (shapes, res["paths"])
     ref = oracle_step(w, layers, seed=5, step=1)
     assert_step_matches(res, ref, "bf16")
 
@@ -425,7 +434,8 @@ def test_small_T_prescaled_clipped_sum(case):
                  wid=750 + case)
     layers = W.make_inputs(w, seed=3)
     res = run_gpu_step(w, layers, seed=8, step=2)
-    assert all(s for _, s in res["paths"]), res["paths"]
+    for (di, do), (npath, spath) in zip(shapes, res["paths"]):
+        assert (npath, spath) == (2, 0) if is_thin(di, do, T, "bf16") else spath, res["paths"]
     ref = oracle_step(w, layers, seed=8, step=2)
     assert_step_matches(res, ref, "bf16")
     nz = run_gpu_step(w, layers, flags=dp.DP_NO_NOISE, audit=False)
@@ -799,3 +809,85 @@ def test_verifier_accepts_gpu_commitment_and_rejects_tampering(name, fam):
     assert r.path in ("hard_reject", "ambiguity") and r.z32 > prm.tau_abs
     if fam == "cifar10":
         assert r.verdict == V.ABORT      # 3 tau_abs > rho_ill = 2 tau_abs
+
+
+# ---------------------------------------------------------------------------
+# thin layers (LoRA factors, heads, bias rows): per-example gradients stored
+# by the norm pass, summed by the clipped-sum pass
+# ---------------------------------------------------------------------------
+
+THIN_CASES = [
+    # (layers, B, T, dtype)
+    ([(256, 8), (8, 520)], 5, 64, "bf16"),        # LoRA-like down / up factors
+    ([(1000, 4), (4, 1000)], 3, 100, "bf16"),     # r = 4, ragged wide side, T % 64 != 0
+    ([(300, 3), (3, 300)], 4, 96, "bf16"),        # odd widths (6-byte bf16 rows)
+    ([(1024, 32), (17, 600)], 2, 256, "f32"),     # widest bucket, r = 17 in it
+    ([(1, 512)], 6, 80, "f32"),                   # a bias row (d_in = 1)
+    ([(256, 8), (264, 136)], 3, 64, "bf16"),      # thin next to a tensor-core layer
+]
+
+
+@pytest.mark.parametrize("case", range(len(THIN_CASES)))
+def test_thin_layers_match_oracle(case):
+    shapes, B, T, dtype = THIN_CASES[case]
+    w = W.custom(f"thin{case}", shapes, B, T, dtype, C=0.3, sigma=0.7, d_std=0.1,
+                 wid=800 + case)
+    layers = W.make_inputs(w)
+    res = run_gpu_step(w, layers, seed=4, step=2, out_scale=1.0 / B)
+    for (i, o), (npath, spath) in zip(shapes, res["paths"]):
+        thin = is_thin(i, o, T, dtype)
+        assert (npath == 2) == thin and (not thin or spath == 0), (shapes, res["paths"])
+    ref = oracle_step(w, layers, seed=4, step=2, out_scale=1.0 / B)
+    assert_step_matches(res, ref, dtype)
+    # the batched calls (one launch per bucket) give the same bits
+    dev = torch.device(DEV)
+    outs = [torch.zeros(i, o, device=dev) for i, o in shapes]
+    cfg = dp.make_config(w.layers, B, T, dtype, w.C, w.sigma, out_scale=1.0 / B, seed=4, step=2)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.run_step(ctx, [A.to(dev) for A, _ in layers], [D.to(dev) for _, D in layers], outs)
+    finally:
+        dp.dp_step_destroy(ctx)
+    for a, b in zip(outs, res["out"]):
+        assert np.array_equal(a.cpu().numpy(), b)
+
+
+def test_thin_accumulate_and_commit_then_noise():
+    """DP_ACCUMULATE and the commit-then-noise order on the stored-gradient path."""
+    w = W.custom("thin_acc", [(512, 8), (8, 512)], 4, 128, "bf16", C=0.2, sigma=0.9,
+                 d_std=0.1, wid=820)
+    layers = W.make_inputs(w)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    one = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    two = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, seed=8, step=3)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.run_step(ctx, Ad, Dd, one)
+        dp.dp_step_init(cfg, ctx=ctx)
+        dp.run_step(ctx, Ad, Dd, two, flags=dp.DP_NO_NOISE)
+        for l in range(2):
+            dp.dp_clipped_sum_noise(ctx, l, None, None, two[l], dp.DP_NOISE_ONLY)
+        acc = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+        for _ in range(2):
+            dp.dp_step_init(cfg, ctx=ctx)
+            dp.run_step(ctx, Ad, Dd, acc, flags=dp.DP_NO_NOISE | dp.DP_ACCUMULATE)
+    finally:
+        dp.dp_step_destroy(ctx)
+    ref = oracle_step(w, layers, noise=False)
+    for a, b, c, r in zip(one, two, acc, ref["out"]):
+        assert rel_err_normwise(b.cpu().numpy(), a.cpu().numpy()) <= 1e-6
+        assert rel_err_normwise(c.cpu().numpy(), 2 * r) <= 2e-3
+
+
+def test_gpt2_medium_lora_workload_full():
+    """The 48 LoRA factor layers of GPT-2-medium (r = 4, B = 64, T = 128)
+    against the full oracle, every norm and every output element."""
+    w = W.get("gpt2m_lora_e2e_bf16")
+    layers = W.make_inputs(w)
+    res = run_gpu_step(w, layers, seed=1, step=7, out_scale=1.0 / w.B)
+    assert all(n == 2 for n, _ in res["paths"])
+    ref = oracle_step(w, layers, seed=1, step=7, out_scale=1.0 / w.B)
+    assert_step_matches(res, ref, "bf16")

@@ -88,6 +88,33 @@ WORKLOADS["llm_ffn_up_bf16"] = Workload("llm_ffn_up_bf16", 5, ((4096, 11008),), 
                                         _normal_all(1), 1.0, math.sqrt(1e-5), 0.5, 1.0,
                                         audit_frac=0.05)
 
+# The paper's LoRA fine-tuning shapes (table of forged-gradient experiment
+# parameters, App. B): GPT-2-medium (24 blocks, d = 1024) with rank-4 adapters
+# on the fused QKV projection 1024 -> 3072, and RoBERTa-large (24 blocks,
+# d = 1024) with rank-8 adapters on the query and value projections.  Each
+# adapter is two dense layers: the down factor (d_in x r, inputs = the
+# block's hidden states, output gradients of width r) and the up factor
+# (r x d_out, inputs of width r).  Seeded N(0,1) activations and N(0,1e-4)
+# output gradients stand in for the real ones; C = 1 and the noise
+# multipliers are the table's.
+def _lora(blocks: int, targets: Sequence[Tuple[int, int]], r: int):
+    out = []
+    for _ in range(blocks):
+        for d_in, d_out in targets:
+            out += [(d_in, r), (r, d_out)]
+    return tuple(out)
+
+
+WORKLOADS["gpt2m_lora_e2e_bf16"] = Workload(
+    "gpt2m_lora_e2e_bf16", 6, _lora(24, [(1024, 3072)], 4), 64, 128, "bf16",
+    _normal_all(48), 1.0, math.sqrt(1e-4), 1.0, 0.6679, audit_frac=0.05)
+WORKLOADS["gpt2m_lora_webnlg_bf16"] = Workload(
+    "gpt2m_lora_webnlg_bf16", 7, _lora(24, [(1024, 3072)], 4), 32, 256, "bf16",
+    _normal_all(48), 1.0, math.sqrt(1e-4), 1.0, 0.6827, audit_frac=0.05)
+WORKLOADS["roberta_l_lora_mnli_bf16"] = Workload(
+    "roberta_l_lora_mnli_bf16", 8, _lora(24, [(1024, 1024), (1024, 1024)], 8), 256, 128,
+    "bf16", _normal_all(96), 1.0, math.sqrt(1e-4), 1.0, 0.6407, audit_frac=0.05)
+
 # one 4096x4096 bf16 layer over B x T
 SWEEP = [Workload(f"sweep_B{b}_T{t}", 100 + 10 * bi + ti, ((4096, 4096),), b, t,
                   "bf16", _normal_all(1), 1.0, 1.0, 1.0, 1.0)
