@@ -385,6 +385,7 @@ cudaError_t launch_layer_norms(dp_ctx* c, int32_t layer, const void* A, const vo
     fill_pergrad(c, layer, A, D, g.l[0]);
     g.L = 1;
     g.part = c->d_part;
+    g.err = c->d_flag;
     g.B = c->B;
     g.T = c->T;
     g.NP = c->NP;
@@ -577,6 +578,7 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
     for (size_t q = 0; q < v.size(); ++q) fill_pergrad(c, layers[v[q]], A[v[q]], D[v[q]], g.l[q]);
     g.L = static_cast<int>(v.size());
     g.part = c->d_part;
+    g.err = c->d_flag;
     g.B = c->B;
     g.T = c->T;
     g.NP = c->NP;

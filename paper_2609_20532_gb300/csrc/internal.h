@@ -53,6 +53,7 @@ struct PerGradLayer {
   float* G;        // per-example gradients [B][d_in][d_out]
   int n, r;        // wide and narrow widths
   int wide_is_in;  // 1: X = A (n = d_in), 0: X = D (n = d_out)
+  int bulk;        // rows of X staged by bulk copies (n * elemsize % 16 == 0)
   int chunks;      // blocks per example (set by the launcher)
   int row0;        // partial-sum row of example 0
   int item0;       // first block of this layer (set by the launcher)
@@ -60,6 +61,7 @@ struct PerGradLayer {
 struct PerGradBatch {
   PerGradLayer l[kPerGradMaxLayers];
   float* part;
+  int* err;  // sticky error word (bounded waits that gave up)
   int L, B, T, NP;
 };
 struct PerGradSumLayer {

@@ -19,6 +19,7 @@
 
 #include "internal.h"
 #include "philox.cuh"
+#include "tc_util.cuh"
 
 namespace dpk {
 
@@ -29,6 +30,46 @@ constexpr int TT = 64;  // positions staged per round
 
 __device__ __forceinline__ float to_float(float x) { return x; }
 __device__ __forceinline__ float to_float(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+// VJ consecutive wide-side values of one row, read once and not kept in L1.
+template <typename TIn, int VJ>
+__device__ __forceinline__ void load_row(const TIn* p, float (&x)[VJ]);
+template <>
+__device__ __forceinline__ void load_row<__nv_bfloat16, 4>(const __nv_bfloat16* p, float (&x)[4]) {
+  const uint2 u = __ldcs(reinterpret_cast<const uint2*>(p));
+  x[0] = __uint_as_float(u.x << 16);
+  x[1] = __uint_as_float(u.x & 0xffff0000u);
+  x[2] = __uint_as_float(u.y << 16);
+  x[3] = __uint_as_float(u.y & 0xffff0000u);
+}
+template <>
+__device__ __forceinline__ void load_row<__nv_bfloat16, 2>(const __nv_bfloat16* p, float (&x)[2]) {
+  const unsigned u = __ldcs(reinterpret_cast<const unsigned*>(p));
+  x[0] = __uint_as_float(u << 16);
+  x[1] = __uint_as_float(u & 0xffff0000u);
+}
+template <>
+__device__ __forceinline__ void load_row<__nv_bfloat16, 1>(const __nv_bfloat16* p, float (&x)[1]) {
+  x[0] = __bfloat162float(p[0]);
+}
+template <>
+__device__ __forceinline__ void load_row<float, 4>(const float* p, float (&x)[4]) {
+  const float4 v = __ldcs(reinterpret_cast<const float4*>(p));
+  x[0] = v.x;
+  x[1] = v.y;
+  x[2] = v.z;
+  x[3] = v.w;
+}
+template <>
+__device__ __forceinline__ void load_row<float, 2>(const float* p, float (&x)[2]) {
+  const float2 v = __ldcs(reinterpret_cast<const float2*>(p));
+  x[0] = v.x;
+  x[1] = v.y;
+}
+template <>
+__device__ __forceinline__ void load_row<float, 1>(const float* p, float (&x)[1]) {
+  x[0] = __ldcs(p);
+}
 
 template <int R>
 struct Vj {
@@ -41,11 +82,72 @@ __device__ __forceinline__ int find_layer(const PerGradBatch& g, int item) {
   return l;
 }
 
+// VJ consecutive values from shared memory.
+template <typename TIn, int VJ>
+__device__ __forceinline__ void load_smem(const TIn* p, float (&x)[VJ]);
+template <>
+__device__ __forceinline__ void load_smem<__nv_bfloat16, 4>(const __nv_bfloat16* p, float (&x)[4]) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  x[0] = __uint_as_float(u.x << 16);
+  x[1] = __uint_as_float(u.x & 0xffff0000u);
+  x[2] = __uint_as_float(u.y << 16);
+  x[3] = __uint_as_float(u.y & 0xffff0000u);
+}
+template <>
+__device__ __forceinline__ void load_smem<__nv_bfloat16, 2>(const __nv_bfloat16* p, float (&x)[2]) {
+  const unsigned u = *reinterpret_cast<const unsigned*>(p);
+  x[0] = __uint_as_float(u << 16);
+  x[1] = __uint_as_float(u & 0xffff0000u);
+}
+template <>
+__device__ __forceinline__ void load_smem<__nv_bfloat16, 1>(const __nv_bfloat16* p, float (&x)[1]) {
+  x[0] = __bfloat162float(p[0]);
+}
+template <>
+__device__ __forceinline__ void load_smem<float, 4>(const float* p, float (&x)[4]) {
+  const float4 v = *reinterpret_cast<const float4*>(p);
+  x[0] = v.x;
+  x[1] = v.y;
+  x[2] = v.z;
+  x[3] = v.w;
+}
+template <>
+__device__ __forceinline__ void load_smem<float, 2>(const float* p, float (&x)[2]) {
+  const float2 v = *reinterpret_cast<const float2*>(p);
+  x[0] = v.x;
+  x[1] = v.y;
+}
+template <>
+__device__ __forceinline__ void load_smem<float, 1>(const float* p, float (&x)[1]) {
+  x[0] = p[0];
+}
+
+template <typename TIn, int R, int VJ>
+__device__ __forceinline__ void fma_row(const float (&x)[VJ], const float* y, float (&acc)[VJ][R]) {
+#pragma unroll
+  for (int k = 0; k < R; ++k) {
+    const float yk = y[k];
+#pragma unroll
+    for (int v = 0; v < VJ; ++v) acc[v][k] = fmaf(x[v], yk, acc[v][k]);
+  }
+}
+
+// Bulk-staged rows: NS ring stages of STAGE_BYTES in dynamic shared memory.
+constexpr int NS = 4;
+constexpr int STAGE_BYTES = 16384;
+constexpr int kPerGradSmem = NS * STAGE_BYTES;
+
 template <typename TIn, int R>
 __global__ void __launch_bounds__(kThreads) k_pergrad_norm(const __grid_constant__ PerGradBatch g) {
   constexpr int VJ = Vj<R>::value;
+  constexpr int SR = STAGE_BYTES / (kThreads * VJ * static_cast<int>(sizeof(TIn)));  // rows / stage
+  static_assert(TT % SR == 0, "stages must tile the staged positions");
+  extern __shared__ __align__(128) uint8_t stage_mem[];
   __shared__ __align__(16) float ys[TT][R];
+  __shared__ uint64_t full[NS];
   __shared__ float red[kThreads / 32];
+  __shared__ int abort_flag;
+  volatile int* abrt = &abort_flag;
   const int l = find_layer(g, blockIdx.x);
   const PerGradLayer& P = g.l[l];
   const int local = static_cast<int>(blockIdx.x) - P.item0;
@@ -53,54 +155,159 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm(const __grid_constant
   const int n = P.n, r = P.r, T = g.T;
   const TIn* X = static_cast<const TIn*>(P.X) + static_cast<int64_t>(i) * T * n;
   const TIn* Y = static_cast<const TIn*>(P.Y) + static_cast<int64_t>(i) * T * r;
-  const int j0 = (chunk * kThreads + static_cast<int>(threadIdx.x)) * VJ;
+  const int c0 = chunk * kThreads * VJ;
+  const int W = n - c0 < kThreads * VJ ? n - c0 : kThreads * VJ;  // columns of this block
+  const int j0 = c0 + static_cast<int>(threadIdx.x) * VJ;
   float acc[VJ][R];
 #pragma unroll
   for (int v = 0; v < VJ; ++v)
 #pragma unroll
     for (int k = 0; k < R; ++k) acc[v][k] = 0.f;
 
-  for (int t0 = 0; t0 < T; t0 += TT) {
-    const int tt = T - t0 < TT ? T - t0 : TT;
+  auto fill_ys = [&](int tb) {
+    const int tt = T - tb < TT ? T - tb : TT;
     for (int e = threadIdx.x; e < TT * R; e += kThreads) {
       const int t = e / R, k = e - (e / R) * R;
-      ys[t][k] = (t < tt && k < r) ? to_float(Y[static_cast<int64_t>(t0 + t) * r + k]) : 0.f;
+      ys[t][k] = (t < tt && k < r) ? to_float(Y[static_cast<int64_t>(tb + t) * r + k]) : 0.f;
+    }
+  };
+
+  if (P.bulk) {
+    // One thread streams the block's rows of X (W contiguous columns per row,
+    // one copy per stage when the block spans the whole row) into the ring;
+    // every thread waits on the stage's barrier, then reads its VJ columns.
+    const uint32_t row_bytes = static_cast<uint32_t>(W) * sizeof(TIn);
+    const int nst = (T + SR - 1) / SR;
+    if (threadIdx.x == 0) {
+      for (int q = 0; q < NS; ++q) tc::mbar_init(&full[q], 1);
+      abort_flag = 0;
+      tc::fence_mbar_init();
     }
     __syncthreads();
-    if (j0 < n) {
-      const TIn* xrow = X + static_cast<int64_t>(t0) * n + j0;
+    int issued = 0;  // meaningful in thread 0
+    auto issue = [&](int st) {
+      const int q = st % NS, r0 = st * SR;
+      const int nr = T - r0 < SR ? T - r0 : SR;
+      uint8_t* dst = stage_mem + q * STAGE_BYTES;
+      tc::mbar_arrive_expect_tx(&full[q], static_cast<uint32_t>(nr) * row_bytes);
+      if (W == n) {
+        tc::bulk_load(dst, X + static_cast<int64_t>(r0) * n, static_cast<uint32_t>(nr) * row_bytes,
+                      &full[q]);
+      } else {
+        for (int rr = 0; rr < nr; ++rr)
+          tc::bulk_load(dst + rr * row_bytes, X + static_cast<int64_t>(r0 + rr) * n + c0,
+                        row_bytes, &full[q]);
+      }
+    };
+    if (threadIdx.x == 0)
+      for (; issued < NS && issued < nst; ++issued) issue(issued);
+    int st = 0;
+    for (; st < nst; ++st) {
+      const int r0 = st * SR;
+      if (r0 % TT == 0) {
+        fill_ys(r0);
+        __syncthreads();
+      }
+      const int q = st % NS;
+      tc::mbar_wait(&full[q], static_cast<uint32_t>(st / NS) & 1u, abrt, g.err);
+      __syncthreads();
+      if (*abrt) break;  // uniform: read after the barrier by every thread
+      const TIn* xs = reinterpret_cast<const TIn*>(stage_mem + q * STAGE_BYTES);
+      const int nr = T - r0 < SR ? T - r0 : SR;
+      const int yb = r0 % TT;
+      if (static_cast<int>(threadIdx.x) * VJ < W) {
+        const TIn* xp = xs + threadIdx.x * VJ;
 #pragma unroll 4
-      for (int t = 0; t < tt; ++t, xrow += n) {
-        float x[VJ];
-#pragma unroll
-        for (int v = 0; v < VJ; ++v) x[v] = (j0 + v < n) ? to_float(xrow[v]) : 0.f;
-#pragma unroll
-        for (int k = 0; k < R; ++k) {
-          const float y = ys[t][k];
-#pragma unroll
-          for (int v = 0; v < VJ; ++v) acc[v][k] = fmaf(x[v], y, acc[v][k]);
+        for (int rr = 0; rr < nr; ++rr, xp += W) {
+          float x[VJ];
+          load_smem<TIn, VJ>(xp, x);
+          fma_row<TIn, R, VJ>(x, &ys[yb + rr][0], acc);
         }
       }
+      __syncthreads();  // the stage is free again
+      if (threadIdx.x == 0 && issued < nst) issue(issued++);
     }
-    __syncthreads();
+    if (st < nst) {
+      // gave up: let every copy issued into the ring land before leaving
+      if (threadIdx.x == 0) {
+        for (int k = st; k < issued; ++k) {
+          const uint64_t t0 = tc::globaltimer_ns();
+          while (!tc::mbar_try_wait(&full[k % NS], static_cast<uint32_t>(k / NS) & 1u))
+            if (tc::globaltimer_ns() - t0 > tc::kWaitLimitNs) break;
+        }
+      }
+      return;
+    }
+  } else {
+    // Rows read straight into registers (widths whose rows are not 16-byte
+    // multiples).
+    const bool vec = j0 + VJ <= n && n % VJ == 0 &&
+                     (reinterpret_cast<uintptr_t>(P.X) % (VJ * sizeof(TIn))) == 0;
+    for (int t0 = 0; t0 < T; t0 += TT) {
+      const int tt = T - t0 < TT ? T - t0 : TT;
+      fill_ys(t0);
+      __syncthreads();
+      const TIn* xrow = X + static_cast<int64_t>(t0) * n + j0;
+      if (vec) {
+#pragma unroll 8
+        for (int t = 0; t < tt; ++t, xrow += n) {
+          float x[VJ];
+          load_row<TIn, VJ>(xrow, x);
+          fma_row<TIn, R, VJ>(x, &ys[t][0], acc);
+        }
+      } else if (j0 < n) {
+#pragma unroll 4
+        for (int t = 0; t < tt; ++t, xrow += n) {
+          float x[VJ];
+#pragma unroll
+          for (int v = 0; v < VJ; ++v) x[v] = (j0 + v < n) ? to_float(xrow[v]) : 0.f;
+          fma_row<TIn, R, VJ>(x, &ys[t][0], acc);
+        }
+      }
+      __syncthreads();
+    }
   }
 
   // g_i rows are [d_in][d_out]: X = A gives G[j][k], X = D gives G[k][j]
   float* G = P.G + static_cast<int64_t>(i) * n * r;
   float sq = 0.f;
 #pragma unroll
-  for (int v = 0; v < VJ; ++v) {
-    const int j = j0 + v;
-    if (j >= n) continue;
+  for (int v = 0; v < VJ; ++v)
+#pragma unroll
+    for (int k = 0; k < R; ++k) sq = fmaf(acc[v][k], acc[v][k], sq);  // padding is zero
+  const bool g16 = (reinterpret_cast<uintptr_t>(G) & 15) == 0;
+  if (P.wide_is_in && R % 4 == 0 && r == R && g16) {
+#pragma unroll
+    for (int v = 0; v < VJ; ++v) {
+      const int j = j0 + v;
+      if (j >= n) continue;
+      float4* dst = reinterpret_cast<float4*>(G + static_cast<int64_t>(j) * r);
+#pragma unroll
+      for (int k4 = 0; k4 < R / 4; ++k4)
+        dst[k4] = make_float4(acc[v][4 * k4], acc[v][4 * k4 + 1], acc[v][4 * k4 + 2],
+                              acc[v][4 * k4 + 3]);
+    }
+  } else if (!P.wide_is_in && VJ == 4 && n % 4 == 0 && g16 && j0 + 3 < n) {
 #pragma unroll
     for (int k = 0; k < R; ++k) {
       if (k >= r) continue;
-      const float val = acc[v][k];
-      sq = fmaf(val, val, sq);
-      if (P.wide_is_in)
-        G[static_cast<int64_t>(j) * r + k] = val;
-      else
-        G[static_cast<int64_t>(k) * n + j] = val;
+      *reinterpret_cast<float4*>(G + static_cast<int64_t>(k) * n + j0) =
+          make_float4(acc[0][k], acc[VJ > 1 ? 1 : 0][k], acc[VJ > 2 ? 2 : 0][k],
+                      acc[VJ > 3 ? 3 : 0][k]);
+    }
+  } else {
+#pragma unroll
+    for (int v = 0; v < VJ; ++v) {
+      const int j = j0 + v;
+      if (j >= n) continue;
+#pragma unroll
+      for (int k = 0; k < R; ++k) {
+        if (k >= r) continue;
+        if (P.wide_is_in)
+          G[static_cast<int64_t>(j) * r + k] = acc[v][k];
+        else
+          G[static_cast<int64_t>(k) * n + j] = acc[v][k];
+      }
     }
   }
 #pragma unroll
@@ -108,9 +315,9 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm(const __grid_constant
   if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = sq;
   __syncthreads();
   if (threadIdx.x == 0) {
-    float s = 0.f;
-    for (int w = 0; w < kThreads / 32; ++w) s += red[w];
-    g.part[static_cast<int64_t>(P.row0 + i) * g.NP + chunk] = s;
+    float s2 = 0.f;
+    for (int w = 0; w < kThreads / 32; ++w) s2 += red[w];
+    g.part[static_cast<int64_t>(P.row0 + i) * g.NP + chunk] = s2;
   }
 }
 
@@ -132,10 +339,10 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_sum(const __grid_constant_
   float s[4] = {0.f, 0.f, 0.f, 0.f};
   if (vec) {
     const float* gp = P.G + e0;
-#pragma unroll 4
+#pragma unroll 8
     for (int i = 0; i < g.B; ++i, gp += n) {
       const float ci = g.c[i];
-      const float4 v = *reinterpret_cast<const float4*>(gp);
+      const float4 v = __ldcs(reinterpret_cast<const float4*>(gp));
       s[0] = fmaf(ci, v.x, s[0]);
       s[1] = fmaf(ci, v.y, s[1]);
       s[2] = fmaf(ci, v.z, s[2]);
@@ -162,7 +369,14 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_sum(const __grid_constant_
 
 template <typename TIn, int R>
 cudaError_t launch_norm_t(const PerGradBatch& g, int blocks, cudaStream_t s) {
-  k_pergrad_norm<TIn, R><<<blocks, kThreads, 0, s>>>(g);
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_pergrad_norm<TIn, R>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kPerGradSmem);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  k_pergrad_norm<TIn, R><<<blocks, kThreads, kPerGradSmem, s>>>(g);
   return cudaGetLastError();
 }
 
@@ -207,9 +421,13 @@ cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s) {
     if (Rl > R) R = Rl;
   }
   const int vj = R <= 8 ? 4 : (R <= 16 ? 2 : 1);
+  const int elem = t == IN_F32 ? 4 : 2;
   for (int l = 0; l < g.L; ++l) {
     PerGradLayer& P = g.l[l];
     P.chunks = static_cast<int>((P.n + kThreads * vj - 1) / (kThreads * vj));
+    // bulk copies need 16-byte aligned rows (the base is 16-byte aligned)
+    P.bulk = (static_cast<int64_t>(P.n) * elem) % 16 == 0 &&
+             (reinterpret_cast<uintptr_t>(P.X) & 15) == 0;
     P.item0 = static_cast<int>(blocks);
     blocks += static_cast<int64_t>(g.B) * P.chunks;
   }
