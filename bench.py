@@ -220,7 +220,7 @@ def run_ours(args, rank, world, local_rank):
     # CUDA graphs are captured on a non-default stream
     stream = torch.cuda.current_stream() if args.eager else torch.cuda.Stream()
     torch.cuda.set_stream(stream)
-    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
+    cfg = dp.make_config(w.specs, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
                          seed=1234 + rank, step=0, audit_capacity=len(idx))
     ctx = dp.dp_step_init(cfg, stream)
     in_bytes = sum(A.numel() * A.element_size() + D.numel() * D.element_size()
@@ -336,7 +336,7 @@ def run_ours(args, rank, world, local_rank):
         return tot / len(ev[kind]) if graph is not None else tot / args.steps
 
     peaks = _peaks()
-    gemm_flops = sum(2.0 * w.B * w.T * i * o for i, o in w.layers)
+    gemm_flops = sum(2.0 * w.B * T_ * i * o for i, o, T_ in w.specs)
     gemm_ms = per_step_ms("gemm")
     gemm_tflops = gemm_flops / (gemm_ms * 1e-3) / 1e12
     in_total = in_bytes
@@ -650,7 +650,7 @@ def run_verifier(args):
     # block_bf16: a whole checked step against the GPU's commitment
     w = W.get("block_bf16")
     layers = W.make_inputs(w, seed=0)
-    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
+    cfg = dp.make_config(w.specs, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
                          audit_capacity=w.B)
     ctx = dp.dp_step_init(cfg)
     outs = [torch.zeros(i, o, device=dev) for i, o in w.layers]

@@ -87,9 +87,16 @@ typedef enum {
     DP_NORM_MATERIALISED = 3
 } dp_norm_mode;
 
+/* One dense layer of the step: weight d_in x d_out, and the positions per
+ * example its A and D carry.  T = 0 takes dp_config.T; a layer applied to one
+ * position only (a classification head on the first token) gives T = 1, and
+ * a bias row is a layer with d_in = 1 whose A holds ones.  All layers share B
+ * and the clip factors: s_i sums every layer of the step. */
 typedef struct {
     int64_t d_in;
     int64_t d_out;
+    int32_t T;          /* positions per example of this layer, 0 = dp_config.T */
+    int32_t reserved;   /* must be 0 */
 } dp_layer;
 
 /* Parameters of Algorithm 2 for one step: batch B (also the aggregation
@@ -97,7 +104,7 @@ typedef struct {
  * the released per-step noise seed (seed, step). */
 typedef struct {
     int32_t B;                 /* examples per step, >= 1 */
-    int32_t T;                 /* positions per example, >= 1 */
+    int32_t T;                 /* positions per example of layers with T = 0, >= 1 */
     int32_t n_layers;          /* L, 1 .. 1024 */
     const dp_layer* layers;    /* host array of L layer shapes; copied by dp_step_init */
     dp_dtype dtype;            /* element type of every A and D */

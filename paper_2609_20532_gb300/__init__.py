@@ -65,7 +65,8 @@ class LibraryNotBuilt(ImportError):
 
 
 class dp_layer(ctypes.Structure):
-    _fields_ = [("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64)]
+    _fields_ = [("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64), ("T", ctypes.c_int32),
+                ("reserved", ctypes.c_int32)]
 
 
 class dp_adamw(ctypes.Structure):
@@ -155,7 +156,10 @@ def _stream(stream) -> Optional[int]:
 def make_config(layers: Sequence[Sequence[int]], B: int, T: int, dtype: str, C: float,
                 sigma: float, out_scale: float = 1.0, seed: int = 0, step: int = 0,
                 norm_mode: int = DP_NORM_AUTO, audit_capacity: int = 0) -> dp_config:
-    arr = (dp_layer * len(layers))(*[dp_layer(int(i), int(o)) for i, o in layers])
+    # a layer is (d_in, d_out) or (d_in, d_out, T); T = 0 takes the config's T
+    arr = (dp_layer * len(layers))(*[dp_layer(int(ly[0]), int(ly[1]),
+                                              int(ly[2]) if len(ly) > 2 else 0, 0)
+                                     for ly in layers])
     cfg = dp_config(B=B, T=T, n_layers=len(layers), layers=arr,
                     dtype=DP_BF16 if dtype == "bf16" else DP_F32, clip_C=C, sigma=sigma,
                     out_scale=out_scale, seed=seed & (2 ** 64 - 1), step=step & (2 ** 64 - 1),

@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <map>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -46,6 +47,7 @@ void set_last_error(const char* msg) { g_err = msg; }
 // Per-layer execution plan, fixed at init from the shapes and the norm mode.
 struct LayerPlan {
   int64_t d_in, d_out;
+  int T;               // positions per example of this layer
   uint64_t p_base;     // global parameter index of element (0, 0)
   dp_norm_mode mode;   // resolved norm mode
   int norm_tc;         // 1: tensor-core norm kernel
@@ -110,6 +112,13 @@ dp_status check_config(const dp_config* cfg) {
     const dp_layer& ly = cfg->layers[l];
     if (ly.d_in < 1 || ly.d_out < 1 || ly.d_in > (1 << 20) || ly.d_out > (1 << 20))
       return fail(DP_ERR_SHAPE, "layer %d: d_in, d_out must be in 1..2^20", l);
+    if (ly.T < 0 || ly.reserved != 0)
+      return fail(DP_ERR_ARG, "layer %d: T must be >= 0 (0 = config T), reserved must be 0", l);
+    const int T = ly.T > 0 ? ly.T : cfg->T;
+    if (static_cast<int64_t>(cfg->B) * T > 0x7fffffffLL)
+      return fail(DP_ERR_SHAPE, "layer %d: B*T exceeds 2^31-1", l);
+    if (cfg->norm_mode == DP_NORM_RANK1 && T != 1)
+      return fail(DP_ERR_SHAPE, "DP_NORM_RANK1 needs T == 1 for every layer");
   }
   if (!(cfg->clip_C > 0.f) || !std::isfinite(cfg->clip_C))
     return fail(DP_ERR_ARG, "clip_C must be finite and > 0");
@@ -118,8 +127,6 @@ dp_status check_config(const dp_config* cfg) {
   if (!std::isfinite(cfg->out_scale)) return fail(DP_ERR_ARG, "out_scale must be finite");
   if (cfg->norm_mode < DP_NORM_AUTO || cfg->norm_mode > DP_NORM_MATERIALISED)
     return fail(DP_ERR_ARG, "unknown norm_mode");
-  if (cfg->norm_mode == DP_NORM_RANK1 && cfg->T != 1)
-    return fail(DP_ERR_SHAPE, "DP_NORM_RANK1 needs T == 1");
   if (cfg->audit_capacity < 0 || cfg->audit_capacity > cfg->B)
     return fail(DP_ERR_ARG, "audit_capacity must be in 0..B");
   return DP_OK;
@@ -140,12 +147,16 @@ dp_norm_mode resolve_mode(dp_norm_mode m, int T, int64_t d_in, int64_t d_out) {
 // a second time: 8 d_in d_out < T (d_in + d_out) elem.  That also makes the
 // materialised norm the cheaper one (T > 4 r), so a forced Gram or rank-1
 // mode keeps the other paths.
-bool use_pergrad(const dp_config* cfg, int64_t d_in, int64_t d_out) {
+int layer_T(const dp_config* cfg, int l) {
+  return cfg->layers[l].T > 0 ? cfg->layers[l].T : cfg->T;
+}
+
+bool use_pergrad(const dp_config* cfg, int T, int64_t d_in, int64_t d_out) {
   if (cfg->norm_mode == DP_NORM_GHOST || cfg->norm_mode == DP_NORM_RANK1) return false;
   const int64_t r = d_in < d_out ? d_in : d_out;
   if (r > dpk::kThinMax) return false;
   const double elem = cfg->dtype == DP_BF16 ? 2.0 : 4.0;
-  return 8.0 * double(d_in) * double(d_out) < double(cfg->T) * double(d_in + d_out) * elem;
+  return 8.0 * double(d_in) * double(d_out) < double(T) * double(d_in + d_out) * elem;
 }
 
 void build_plan(dp_ctx* c, const dp_config* cfg) {
@@ -157,9 +168,11 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
     LayerPlan& p = c->plan[l];
     p.d_in = cfg->layers[l].d_in;
     p.d_out = cfg->layers[l].d_out;
+    p.T = layer_T(cfg, l);
+    const int T = p.T;
     p.p_base = off;
     off += static_cast<uint64_t>(p.d_in) * p.d_out;
-    p.pergrad = use_pergrad(cfg, p.d_in, p.d_out) ? 1 : 0;
+    p.pergrad = use_pergrad(cfg, T, p.d_in, p.d_out) ? 1 : 0;
     p.g_off = 0;
     if (p.pergrad) {
       p.mode = DP_NORM_MATERIALISED;
@@ -171,25 +184,25 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
       if (p.nparts > NP) NP = p.nparts;
       continue;
     }
-    p.mode = resolve_mode(cfg->norm_mode, cfg->T, p.d_in, p.d_out);
+    p.mode = resolve_mode(cfg->norm_mode, T, p.d_in, p.d_out);
     const bool bf16 = cfg->dtype == DP_BF16;
     p.norm_tc = 0;
     if (p.mode == DP_NORM_RANK1) {
       p.nparts = dpk::rank1_parts();
     } else if (p.mode == DP_NORM_GHOST) {
-      p.norm_tc = bf16 && dpk::tc_ghost_supported(cfg->T, p.d_in, p.d_out);
-      p.nparts = p.norm_tc ? dpk::tc_ghost_parts(cfg->T) : dpk::ghost_simt_parts(cfg->T);
+      p.norm_tc = bf16 && dpk::tc_ghost_supported(T, p.d_in, p.d_out);
+      p.nparts = p.norm_tc ? dpk::tc_ghost_parts(T) : dpk::ghost_simt_parts(T);
     } else {
-      p.norm_tc = bf16 && dpk::tc_gemm_supported(cfg->T, p.d_in, p.d_out);
+      p.norm_tc = bf16 && dpk::tc_gemm_supported(T, p.d_in, p.d_out);
       p.nparts = p.norm_tc ? dpk::tc_mat_parts(p.d_in, p.d_out)
                            : dpk::mat_simt_parts(static_cast<int>(p.d_in), static_cast<int>(p.d_out));
     }
     p.gemm_tc = 0;
-    if (bf16 && dpk::tc_gemm_supported(cfg->T, p.d_in, p.d_out)) {
+    if (bf16 && dpk::tc_gemm_supported(T, p.d_in, p.d_out)) {
       p.gemm_tc = 1;
-    } else if (bf16 && dpk::tc_prescaled_supported(cfg->T, p.d_in, p.d_out)) {
+    } else if (bf16 && dpk::tc_prescaled_supported(T, p.d_in, p.d_out)) {
       p.gemm_tc = 2;
-      const int64_t need = dpk::tc_prescaled_scratch_bytes(cfg->B, cfg->T, p.d_in);
+      const int64_t need = dpk::tc_prescaled_scratch_bytes(cfg->B, T, p.d_in);
       if (need > c->prescaled_bytes) c->prescaled_bytes = need;
     }
     if (p.nparts > NP) NP = p.nparts;
@@ -387,7 +400,7 @@ cudaError_t launch_layer_norms(dp_ctx* c, int32_t layer, const void* A, const vo
     g.part = c->d_part;
     g.err = c->d_flag;
     g.B = c->B;
-    g.T = c->T;
+    g.T = p.T;
     g.NP = c->NP;
     return dpk::launch_pergrad_norm(it, g, c->stream);
   }
@@ -396,13 +409,13 @@ cudaError_t launch_layer_norms(dp_ctx* c, int32_t layer, const void* A, const vo
   if (p.mode == DP_NORM_RANK1)
     return dpk::launch_norm_rank1(it, A, D, c->B, din, dout, c->d_part, c->NP, row0, c->stream);
   if (p.mode == DP_NORM_GHOST)
-    return p.norm_tc ? dpk::tc_launch_ghost(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
+    return p.norm_tc ? dpk::tc_launch_ghost(A, D, c->B, p.T, din, dout, c->d_part, c->NP, row0,
                                             c->d_flag, c->stream)
-                     : dpk::launch_norm_ghost_simt(it, A, D, c->B, c->T, din, dout, c->d_part,
+                     : dpk::launch_norm_ghost_simt(it, A, D, c->B, p.T, din, dout, c->d_part,
                                                    c->NP, row0, c->stream);
-  return p.norm_tc ? dpk::tc_launch_mat_norm(A, D, c->B, c->T, din, dout, c->d_part, c->NP, row0,
+  return p.norm_tc ? dpk::tc_launch_mat_norm(A, D, c->B, p.T, din, dout, c->d_part, c->NP, row0,
                                              c->d_flag, c->stream)
-                   : dpk::launch_norm_mat_simt(it, A, D, c->B, c->T, din, dout, c->d_part, c->NP,
+                   : dpk::launch_norm_mat_simt(it, A, D, c->B, p.T, din, dout, c->d_part, c->NP,
                                                row0, c->stream);
 }
 
@@ -448,13 +461,13 @@ cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const vo
   }
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
   if (p.gemm_tc == 1)
-    return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep, c->d_flag,
+    return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, p.T, din, dout, d_out, ep, c->d_flag,
                                   c->stream);
   if (p.gemm_tc == 2)
-    return dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, c->T, din, dout, d_out, ep,
+    return dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, p.T, din, dout, d_out, ep,
                                             c->d_flag, c->d_prescaled, c->stream);
   return dpk::launch_gemm_simt(c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, A, D, c->d_c,
-                               c->B, c->T, din, dout, d_out, ep, c->stream);
+                               c->B, p.T, din, dout, d_out, ep, c->stream);
 }
 
 }  // namespace
@@ -470,7 +483,8 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     bool same = c->B == cfg->B && c->T == cfg->T && c->L == cfg->n_layers &&
                 c->dtype == cfg->dtype;
     for (int l = 0; same && l < c->L; ++l)
-      same = c->plan[l].d_in == cfg->layers[l].d_in && c->plan[l].d_out == cfg->layers[l].d_out;
+      same = c->plan[l].d_in == cfg->layers[l].d_in && c->plan[l].d_out == cfg->layers[l].d_out &&
+             c->plan[l].T == layer_T(cfg, l);
     if (!same) return fail(DP_ERR_SHAPE, "re-key with different shapes; destroy and re-create");
     // The norm mode may change; the partial buffer must still be large enough.
     std::vector<LayerPlan> old = c->plan;
@@ -564,14 +578,14 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
       row0[q] = l * c->B;
     }
     cudaError_t e = dpk::tc_launch_ghost_batch(static_cast<int>(grp.size()), a, d, din, dout, row0,
-                                               c->B, c->T, c->d_part, c->NP, c->d_flag,
-                                               c->stream);
+                                               c->B, c->plan[layers[grp[0]]].T, c->d_part, c->NP,
+                                               c->d_flag, c->stream);
     grp.clear();
     return e;
   };
-  // Thin layers share launches too, one list per narrow-width bucket.
+  // Thin layers share launches too, one list per (narrow-width bucket, T).
   const dpk::InType it = c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32;
-  std::vector<int> thin[6];
+  std::map<std::pair<int, int>, std::vector<int>> thin;
   auto flush_thin = [&](std::vector<int>& v) -> cudaError_t {
     if (v.empty()) return cudaSuccess;
     dpk::PerGradBatch g{};
@@ -580,7 +594,7 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
     g.part = c->d_part;
     g.err = c->d_flag;
     g.B = c->B;
-    g.T = c->T;
+    g.T = c->plan[layers[v[0]]].T;
     g.NP = c->NP;
     v.clear();
     return dpk::launch_pergrad_norm(it, g, c->stream);
@@ -590,12 +604,11 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
     cudaError_t e = cudaSuccess;
     if (p.pergrad) {
       const int nar = static_cast<int>(p.d_in < p.d_out ? p.d_in : p.d_out);
-      const int bucket = dpk::pergrad_bucket(nar);
-      int b = 0;
-      while ((1 << b) < bucket) ++b;
-      thin[b].push_back(r);
-      if (static_cast<int>(thin[b].size()) == dpk::kPerGradMaxLayers) e = flush_thin(thin[b]);
+      std::vector<int>& v = thin[std::make_pair(dpk::pergrad_bucket(nar), p.T)];
+      v.push_back(r);
+      if (static_cast<int>(v.size()) == dpk::kPerGradMaxLayers) e = flush_thin(v);
     } else if (p.mode == DP_NORM_GHOST && p.norm_tc) {
+      if (!grp.empty() && c->plan[layers[grp[0]]].T != p.T) e = flush();
       grp.push_back(r);
       if (static_cast<int>(grp.size()) == dpk::kGhostMaxLayers) e = flush();
     } else {
@@ -605,7 +618,8 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
       return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
   }
   cudaError_t e = flush();
-  for (int b = 0; b < 6 && e == cudaSuccess; ++b) e = flush_thin(thin[b]);
+  for (auto it2 = thin.begin(); it2 != thin.end() && e == cudaSuccess; ++it2)
+    e = flush_thin(it2->second);
   if (e != cudaSuccess) return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
   for (int r = 0; r < n; ++r) c->norm_done[layers[r]] = 1;
   return DP_OK;
@@ -683,7 +697,8 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
       pb[q] = p.p_base;
     }
     cudaError_t e = dpk::tc_launch_clipsum_batch(static_cast<int>(grp.size()), a, d, o, din, dout,
-                                                 pb, c->d_c, c->B, c->T, ep, c->d_flag, c->stream);
+                                                 pb, c->d_c, c->B, c->plan[layers[grp[0]]].T, ep,
+                                                 c->d_flag, c->stream);
     grp.clear();
     return e;
   };
@@ -692,7 +707,8 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
     const LayerPlan& p = c->plan[l];
     cudaError_t e = cudaSuccess;
     if (!(flags & DP_NOISE_ONLY) && p.gemm_tc == 1) {
-      if (!grp.empty() && !dpk::tc_clipsum_same_launch(c->plan[layers[grp[0]]].d_in, p.d_in))
+      if (!grp.empty() && (!dpk::tc_clipsum_same_launch(c->plan[layers[grp[0]]].d_in, p.d_in) ||
+                           c->plan[layers[grp[0]]].T != p.T))
         e = flush();
       grp.push_back(r);
       if (e == cudaSuccess && static_cast<int>(grp.size()) == dpk::kGemmMaxLayers) e = flush();

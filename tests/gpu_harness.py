@@ -33,7 +33,7 @@ def run_gpu_step(w: W.Workload, layers, seed=0, step=0, out_scale=1.0, flags=0,
     outs = [torch.zeros(i, o, device=dev, dtype=torch.float32) for i, o in w.layers]
     s_dev = torch.empty(w.B, device=dev)
     c_dev = torch.empty(w.B, device=dev)
-    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=out_scale,
+    cfg = dp.make_config(w.specs, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=out_scale,
                          seed=seed, step=step, norm_mode=norm_mode, audit_capacity=w.B)
     ctx = dp.dp_step_init(cfg)
     try:

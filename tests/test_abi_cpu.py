@@ -51,7 +51,7 @@ def _init_status(L, cfg):
 
 @pytest.mark.parametrize("kw,status", [
     (dict(B=0), 2), (dict(T=0), 2), (dict(layers=[(0, 4)]), 2),
-    (dict(layers=[(1 << 21, 4)]), 2), (dict(layers=[(8, 8)] * 1025), 2),
+    (dict(layers=[(1 << 21, 4)]), 2), (dict(layers=[(8, 8)] * 1025), 2), (dict(layers=[(8, 8, -1)]), 1),
     (dict(C=0.0), 1), (dict(C=float("inf")), 1), (dict(sigma=-1.0), 1),
     (dict(sigma=float("nan")), 1), (dict(out_scale=float("inf")), 1),
     (dict(norm_mode=7), 1), (dict(norm_mode=dp.DP_NORM_RANK1, T=4), 2),

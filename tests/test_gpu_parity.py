@@ -891,3 +891,55 @@ def test_gpt2_medium_lora_workload_full():
     assert all(n == 2 for n, _ in res["paths"])
     ref = oracle_step(w, layers, seed=1, step=7, out_scale=1.0 / w.B)
     assert_step_matches(res, ref, "bf16")
+
+
+# ---------------------------------------------------------------------------
+# layers with their own T: a classification head and bias rows on the first
+# token next to LoRA factors over the whole sequence
+# ---------------------------------------------------------------------------
+
+MIXED_T_CASES = [
+    # (layers (d_in, d_out, T), a_dist, dtype)
+    ([(256, 8, 64), (8, 256, 64), (64, 32, 1), (1, 32, 1), (264, 136, 64), (40, 48, 3)],
+     ("normal", "normal", "normal", "ones", "normal", "normal"), "bf16"),
+    ([(128, 4, 96), (4, 300, 96), (300, 5, 1), (1, 5, 1)],
+     ("normal", "normal", "normal", "ones"), "f32"),
+]
+
+
+@pytest.mark.parametrize("case", range(len(MIXED_T_CASES)))
+def test_per_layer_T_matches_oracle(case):
+    specs, a_dist, dtype = MIXED_T_CASES[case]
+    w = W.custom(f"mixT{case}", specs, 6, 64, dtype, C=0.3, sigma=0.8, d_std=0.1,
+                 wid=850 + case, a_dist=a_dist)
+    layers = W.make_inputs(w)
+    assert [A.shape[1] for A, _ in layers] == [t for _, _, t in specs]
+    res = run_gpu_step(w, layers, seed=6, step=4, out_scale=1.0 / w.B)
+    ref = oracle_step(w, layers, seed=6, step=4, out_scale=1.0 / w.B)
+    assert_step_matches(res, ref, dtype)
+    dev = torch.device(DEV)
+    outs = [torch.zeros(i, o, device=dev) for i, o, _ in specs]
+    cfg = dp.make_config(w.specs, w.B, w.T, dtype, w.C, w.sigma, out_scale=1.0 / w.B, seed=6,
+                         step=4)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.run_step(ctx, [A.to(dev) for A, _ in layers], [D.to(dev) for _, D in layers], outs)
+    finally:
+        dp.dp_step_destroy(ctx)
+    for a, b in zip(outs, res["out"]):
+        assert np.array_equal(a.cpu().numpy(), b)
+
+
+def test_roberta_adapters_with_head_reduced():
+    """Two blocks of RoBERTa-style rank-8 query/value adapters (T = 128) and
+    the 3-class head with its biases on the first token (T = 1), B = 64."""
+    specs = [(1024, 8, 128), (8, 1024, 128)] * 4 + [(1024, 1024, 1), (1, 1024, 1),
+                                                     (1024, 3, 1), (1, 3, 1)]
+    a_dist = ("normal",) * 8 + ("normal", "ones", "normal", "ones")
+    w = W.custom("rob_head", specs, 64, 128, "bf16", C=1.0, sigma=0.6407, d_std=0.01,
+                 wid=860, a_dist=a_dist)
+    layers = W.make_inputs(w)
+    res = run_gpu_step(w, layers, seed=2, step=9, out_scale=1.0 / w.B)
+    assert [n for n, _ in res["paths"][:8]] == [2] * 8
+    ref = oracle_step(w, layers, seed=2, step=9, out_scale=1.0 / w.B)
+    assert_step_matches(res, ref, "bf16")

@@ -47,13 +47,23 @@ class Workload:
     C: float
     sigma: float
     audit_frac: float = 0.0
+    layer_T: Tuple[int, ...] = ()  # per-layer positions (empty: every layer has T)
 
     @property
     def n_params(self) -> int:
         return sum(i * o for i, o in self.layers)
 
+    def T_of(self, layer: int) -> int:
+        return self.layer_T[layer] if self.layer_T else self.T
+
+    @property
+    def specs(self) -> Tuple[Tuple[int, int, int], ...]:
+        """(d_in, d_out, T) of every layer, as the C ABI's dp_layer takes them."""
+        return tuple((i, o, self.T_of(l)) for l, (i, o) in enumerate(self.layers))
+
     def describe(self) -> str:
-        dims = ",".join(f"{i}x{o}" for i, o in self.layers)
+        dims = ",".join(f"{i}x{o}" if self.T_of(l) == self.T else f"{i}x{o}@T{self.T_of(l)}"
+                        for l, (i, o) in enumerate(self.layers))
         return f"{self.name}: layers[{dims}] B={self.B} T={self.T} {self.dtype}"
 
 
@@ -114,6 +124,14 @@ WORKLOADS["gpt2m_lora_webnlg_bf16"] = Workload(
 WORKLOADS["roberta_l_lora_mnli_bf16"] = Workload(
     "roberta_l_lora_mnli_bf16", 8, _lora(24, [(1024, 1024), (1024, 1024)], 8), 256, 128,
     "bf16", _normal_all(96), 1.0, math.sqrt(1e-4), 1.0, 0.6407, audit_frac=0.05)
+# ... with the trainable classification head of a 3-class task (MNLI): dense
+# 1024 x 1024 and its bias, out_proj 1024 x 3 and its bias, all applied to the
+# first token only (T = 1); a bias row is a layer with d_in = 1 and ones as A
+_HEAD = ((1024, 1024), (1, 1024), (1024, 3), (1, 3))
+WORKLOADS["roberta_l_lora_head_mnli_bf16"] = Workload(
+    "roberta_l_lora_head_mnli_bf16", 9, _lora(24, [(1024, 1024), (1024, 1024)], 8) + _HEAD,
+    256, 128, "bf16", _normal_all(96) + ("normal", "ones", "normal", "ones"), 1.0,
+    math.sqrt(1e-4), 1.0, 0.6407, audit_frac=0.05, layer_T=(128,) * 96 + (1, 1, 1, 1))
 
 # one 4096x4096 bf16 layer over B x T
 SWEEP = [Workload(f"sweep_B{b}_T{t}", 100 + 10 * bi + ti, ((4096, 4096),), b, t,
@@ -130,13 +148,16 @@ def get(name: str) -> Workload:
     raise KeyError(name)
 
 
-def custom(name: str, layers: Sequence[Tuple[int, int]], B: int, T: int, dtype: str,
+def custom(name: str, layers: Sequence[Sequence[int]], B: int, T: int, dtype: str,
            C: float = 1.0, sigma: float = 1.0, a_std: float = 1.0, d_std: float = 1.0,
            wid: int = 999, a_dist=None) -> Workload:
-    """An ad-hoc workload (tests use these for ragged and edge shapes)."""
+    """An ad-hoc workload (tests use these for ragged and edge shapes).  A
+    layer is (d_in, d_out) or (d_in, d_out, T)."""
     a_dist = tuple(a_dist) if a_dist else _normal_all(len(layers))
-    return Workload(name, wid, tuple(tuple(x) for x in layers), B, T, dtype,
-                    a_dist, a_std, d_std, C, sigma)
+    lt = tuple(int(x[2]) if len(x) > 2 else T for x in layers)
+    return Workload(name, wid, tuple((int(x[0]), int(x[1])) for x in layers), B, T, dtype,
+                    a_dist, a_std, d_std, C, sigma,
+                    layer_T=lt if any(t != T for t in lt) else ())
 
 
 def _draw(rng: np.random.Generator, dist: str, shape, std: float) -> np.ndarray:
@@ -147,6 +168,8 @@ def _draw(rng: np.random.Generator, dist: str, shape, std: float) -> np.ndarray:
     elif dist == "relu_normal":
         x = rng.standard_normal(shape, dtype=np.float32)
         np.maximum(x, np.float32(0.0), out=x)
+    elif dist == "ones":  # the input of a bias row
+        return np.ones(shape, dtype=np.float32)
     else:
         raise ValueError(dist)
     if std != 1.0:
@@ -171,10 +194,11 @@ def make_layer(w: Workload, layer: int, seed: int = 0, B: int | None = None):
     batch, so callers that sample examples pass the full B)."""
     B = w.B if B is None else B
     d_in, d_out = w.layers[layer]
+    T = w.T_of(layer)
     ra = np.random.default_rng(np.random.SeedSequence([seed, w.wid, layer, 0]))
     rd = np.random.default_rng(np.random.SeedSequence([seed, w.wid, layer, 1]))
-    A = _draw(ra, w.a_dist[layer], (B, w.T, d_in), w.a_std)
-    D = _draw(rd, "normal", (B, w.T, d_out), w.d_std)
+    A = _draw(ra, w.a_dist[layer], (B, T, d_in), w.a_std)
+    D = _draw(rd, "normal", (B, T, d_out), w.d_std)
     return _to_dtype(A, w.dtype), _to_dtype(D, w.dtype)
 
 
