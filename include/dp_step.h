@@ -186,7 +186,8 @@ dp_status dp_clip_factors(dp_ctx* ctx, float* d_sqnorm_out, float* d_clip_out);
  * flags: DP_NO_NOISE, DP_NOISE_ONLY, DP_ACCUMULATE (see above).
  * d_out: device fp32 [d_in][d_out], 16-byte aligned, owned by the caller.
  * Thin layers.  When one side of a layer is at most 32 wide (LoRA factors,
- *   small heads, bias rows) and 8 d_in d_out < T (d_in + d_out) elemsize,
+ *   small heads, bias rows) and either T = 1 or 8 d_in d_out < T (d_in +
+ *   d_out) elemsize (and the norm mode is AUTO or MATERIALISED),
  *   dp_layer_norms stores the layer's per-example gradients G_{i,l} in the
  *   context (B d_in d_out floats), and this call sums those in example order
  *   instead of reading A and D again.  Its A and D must be the arrays given

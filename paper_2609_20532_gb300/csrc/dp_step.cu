@@ -144,9 +144,11 @@ dp_norm_mode resolve_mode(dp_norm_mode m, int T, int64_t d_in, int64_t d_out) {
 
 // A thin layer (narrow side <= kThinMax) stores its per-example gradients
 // when writing and reading them back moves fewer bytes than reading A and D
-// a second time: 8 d_in d_out < T (d_in + d_out) elem.  That also makes the
-// materialised norm the cheaper one (T > 4 r), so a forced Gram or rank-1
-// mode keeps the other paths.
+// a second time, 8 d_in d_out < T (d_in + d_out) elem, which also makes the
+// materialised norm the cheaper one (T > 4 r); and always at T = 1, where
+// such a layer (a bias row, a head with few outputs) is too small for bytes
+// to matter and its clipped sum would otherwise be a latency-bound K = B
+// loop of its own.  A forced Gram or rank-1 mode keeps the other paths.
 int layer_T(const dp_config* cfg, int l) {
   return cfg->layers[l].T > 0 ? cfg->layers[l].T : cfg->T;
 }
@@ -155,6 +157,7 @@ bool use_pergrad(const dp_config* cfg, int T, int64_t d_in, int64_t d_out) {
   if (cfg->norm_mode == DP_NORM_GHOST || cfg->norm_mode == DP_NORM_RANK1) return false;
   const int64_t r = d_in < d_out ? d_in : d_out;
   if (r > dpk::kThinMax) return false;
+  if (T == 1) return true;
   const double elem = cfg->dtype == DP_BF16 ? 2.0 : 4.0;
   return 8.0 * double(d_in) * double(d_out) < double(T) * double(d_in + d_out) * elem;
 }

@@ -70,8 +70,9 @@ struct PerGradSumLayer {
   int64_t count;    // d_in * d_out
   uint64_t p_base;  // global parameter index of element 0
   int64_t nq;       // quads (set by the launcher)
-  int64_t item0;    // first thread (set by the launcher)
+  int64_t item0;    // first block (set by the launcher)
   int vec;          // float4 path (set by the launcher)
+  int split;        // threads per quad over the examples (set by the launcher)
 };
 struct PerGradSumBatch {
   PerGradSumLayer l[kPerGradMaxLayers];

@@ -19,6 +19,7 @@
 
 #include "internal.h"
 #include "philox.cuh"
+#include "tc.h"
 #include "tc_util.cuh"
 
 namespace dpk {
@@ -322,42 +323,66 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm(const __grid_constant
 }
 
 // out = out_scale (sum_i c_i g_i + sigma C z) over the global quads that
-// overlap each layer's parameters; examples are summed in index order.
+// overlap each layer's parameters.  A layer with few parameters splits its
+// examples over `split` threads per quad (split from the layer's own size,
+// so a batched launch rounds exactly like a single one): each thread sums a
+// contiguous range of examples in order, and the ranges are added in order.
 __global__ void __launch_bounds__(kThreads) k_pergrad_sum(const __grid_constant__ PerGradSumBatch g) {
+  __shared__ float4 red[kThreads];
   int l = 0;
-  while (l + 1 < g.L && static_cast<int64_t>(blockIdx.x) * kThreads >= g.l[l + 1].item0) ++l;
+  while (l + 1 < g.L && static_cast<int64_t>(blockIdx.x) >= g.l[l + 1].item0) ++l;
   const PerGradSumLayer& P = g.l[l];
-  const int64_t local = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x - P.item0;
-  if (local >= P.nq) return;
-  const uint64_t q = (P.p_base >> 2) + static_cast<uint64_t>(local);
+  const int split = P.split;
+  const int qpb = kThreads / split;  // quads per block
+  const int qi = static_cast<int>(threadIdx.x) % qpb, sp = static_cast<int>(threadIdx.x) / qpb;
+  const int64_t local = (static_cast<int64_t>(blockIdx.x) - P.item0) * qpb + qi;
+  const bool live = local < P.nq;
+  const uint64_t q = (P.p_base >> 2) + static_cast<uint64_t>(live ? local : 0);
   const int64_t e0 = static_cast<int64_t>(4 * q) - static_cast<int64_t>(P.p_base);
   const int64_t n = P.count;
-  float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (g.add_noise) z = gauss_quad(g.key[0], g.key[1], q);
-  const float zv[4] = {z.x, z.y, z.z, z.w};
-  const bool vec = P.vec && e0 >= 0 && e0 + 3 < n;
+  const int i0 = static_cast<int>((static_cast<int64_t>(g.B) * sp) / split);
+  const int i1 = static_cast<int>((static_cast<int64_t>(g.B) * (sp + 1)) / split);
   float s[4] = {0.f, 0.f, 0.f, 0.f};
-  if (vec) {
-    const float* gp = P.G + e0;
+  if (live) {
+    const bool vec = P.vec && e0 >= 0 && e0 + 3 < n;
+    if (vec) {
+      const float* gp = P.G + static_cast<int64_t>(i0) * n + e0;
 #pragma unroll 8
-    for (int i = 0; i < g.B; ++i, gp += n) {
-      const float ci = g.c[i];
-      const float4 v = __ldcs(reinterpret_cast<const float4*>(gp));
-      s[0] = fmaf(ci, v.x, s[0]);
-      s[1] = fmaf(ci, v.y, s[1]);
-      s[2] = fmaf(ci, v.z, s[2]);
-      s[3] = fmaf(ci, v.w, s[3]);
-    }
-  } else {
-    for (int i = 0; i < g.B; ++i) {
-      const float ci = g.c[i];
+      for (int i = i0; i < i1; ++i, gp += n) {
+        const float ci = g.c[i];
+        const float4 v = __ldcs(reinterpret_cast<const float4*>(gp));
+        s[0] = fmaf(ci, v.x, s[0]);
+        s[1] = fmaf(ci, v.y, s[1]);
+        s[2] = fmaf(ci, v.z, s[2]);
+        s[3] = fmaf(ci, v.w, s[3]);
+      }
+    } else {
+      for (int i = i0; i < i1; ++i) {
+        const float ci = g.c[i];
 #pragma unroll
-      for (int w = 0; w < 4; ++w) {
-        const int64_t e = e0 + w;
-        if (e >= 0 && e < n) s[w] = fmaf(ci, P.G[static_cast<int64_t>(i) * n + e], s[w]);
+        for (int w = 0; w < 4; ++w) {
+          const int64_t e = e0 + w;
+          if (e >= 0 && e < n) s[w] = fmaf(ci, P.G[static_cast<int64_t>(i) * n + e], s[w]);
+        }
       }
     }
   }
+  if (split > 1) {  // uniform per block
+    red[threadIdx.x] = make_float4(s[0], s[1], s[2], s[3]);
+    __syncthreads();
+    if (sp != 0) return;
+    for (int k = 1; k < split; ++k) {
+      const float4 o = red[k * qpb + qi];
+      s[0] += o.x;
+      s[1] += o.y;
+      s[2] += o.z;
+      s[3] += o.w;
+    }
+  }
+  if (!live) return;
+  float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (g.add_noise) z = gauss_quad(g.key[0], g.key[1], q);
+  const float zv[4] = {z.x, z.y, z.z, z.w};
 #pragma unroll
   for (int w = 0; w < 4; ++w) {
     const int64_t e = e0 + w;
@@ -438,17 +463,22 @@ cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s) {
 
 cudaError_t launch_pergrad_sum(PerGradSumBatch& g, cudaStream_t s) {
   if (g.L < 1 || g.L > kPerGradMaxLayers) return cudaErrorInvalidValue;
-  int64_t threads = 0;
+  const int64_t target = static_cast<int64_t>(device_sm_count()) * kThreads;  // ~one wave
+  int64_t blocks = 0;
   for (int l = 0; l < g.L; ++l) {
     PerGradSumLayer& P = g.l[l];
     P.nq = static_cast<int64_t>(((P.p_base + P.count - 1) >> 2) - (P.p_base >> 2) + 1);
     P.vec = (P.p_base % 4 == 0) && (P.count % 4 == 0) &&
             (reinterpret_cast<uintptr_t>(P.G) % 16 == 0);
-    // each layer starts on a block boundary
-    P.item0 = threads;
-    threads += ((P.nq + kThreads - 1) / kThreads) * kThreads;
+    // split the examples while the layer alone is short of a wave and every
+    // range keeps at least 16 examples
+    int split = 1;
+    while (split < 8 && P.nq * split * 2 <= target && g.B / (split * 2) >= 16) split *= 2;
+    P.split = split;
+    P.item0 = blocks;  // in blocks
+    const int qpb = kThreads / split;
+    blocks += (P.nq + qpb - 1) / qpb;
   }
-  const int64_t blocks = threads / kThreads;
   if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
   k_pergrad_sum<<<static_cast<int>(blocks), kThreads, 0, s>>>(g);
   return cudaGetLastError();
