@@ -181,7 +181,8 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
       p.mode = DP_NORM_MATERIALISED;
       p.norm_tc = 0;
       p.gemm_tc = 0;
-      p.nparts = dpk::pergrad_parts(p.d_in, p.d_out);
+      p.nparts = dpk::pergrad_parts(cfg->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, p.d_in,
+                                    p.d_out);
       p.g_off = grads;
       grads += static_cast<int64_t>(cfg->B) * p.d_in * p.d_out;
       if (p.nparts > NP) NP = p.nparts;

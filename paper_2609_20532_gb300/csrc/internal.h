@@ -83,7 +83,7 @@ struct PerGradSumBatch {
   int L, B;
 };
 int pergrad_bucket(int r);                       // 1, 2, 4, ..., 32, or 0 if too wide
-int pergrad_parts(int64_t d_in, int64_t d_out);  // partials per example
+int pergrad_parts(InType t, int64_t d_in, int64_t d_out);  // partials per example
 cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s);
 cudaError_t launch_pergrad_sum(PerGradSumBatch& g, cudaStream_t s);
 

@@ -322,6 +322,238 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm(const __grid_constant
   }
 }
 
+// ---------------------------------------------------------------------------
+// bf16 thin layers on warp tensor-core MMAs.  Per example the contraction is
+// tiny (N = r <= 32, K = T) and the pass is bound by HBM, but on CUDA cores
+// the multiply-adds and bf16 unpacking spend more issue slots than the bytes
+// take to arrive; one m16n8k16 MMA does 2048 multiply-adds in one
+// instruction.  A block covers one example and kMmaCols wide columns; each
+// of its 8 warps owns 4 m-tiles of 16 wide columns against all NT n-tiles of
+// 8 narrow columns.  A stage is one k16 step: 16 rows of the wide operand at
+// a padded stride (the 8 rows one ldmatrix reads fall in distinct banks) and
+// the same 16 rows of the narrow operand, zero-padded to 8 NT columns.
+// ---------------------------------------------------------------------------
+constexpr int kMmaCols = 512;
+constexpr int kMmaSR = 16;
+constexpr int kMmaXStride = kMmaCols * 2 + 16;  // bytes per staged wide row
+
+template <int NT>
+struct MmaCfg {
+  static constexpr int YW = 8 * NT;            // staged narrow width
+  static constexpr int Y_STRIDE = YW * 2;      // bytes per staged narrow row
+  static constexpr int X_BYTES = kMmaSR * kMmaXStride;
+  static constexpr int Y_BYTES = kMmaSR * Y_STRIDE;
+  static constexpr int STAGE = ((X_BYTES + Y_BYTES + 127) / 128) * 128;
+  static constexpr int SMEM = NS * STAGE;
+};
+
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t (&a)[4]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(a[0]), "=r"(a[1]), "=r"(a[2]), "=r"(a[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x2_trans(uint32_t addr, uint32_t (&b)[2]) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.trans.shared.b16 {%0, %1}, [%2];"
+               : "=r"(b[0]), "=r"(b[1])
+               : "r"(addr));
+}
+__device__ __forceinline__ void mma_16816(float (&c)[4], const uint32_t (&a)[4],
+                                          const uint32_t (&b)[2]) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+      "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b[0]), "r"(b[1]));
+}
+
+// One (layer, example, column slice) work item of a launch.
+struct MmaItem {
+  const __nv_bfloat16* X;  // the example's wide rows, at this slice's first column
+  const __nv_bfloat16* Y;  // the example's narrow rows
+  float* G;                // the example's gradient
+  int n, r, W, wide_is_in, row, slot;
+};
+
+__device__ __forceinline__ MmaItem mma_item(const PerGradBatch& g, int item) {
+  const int l = find_layer(g, item);
+  const PerGradLayer& P = g.l[l];
+  const int local = item - P.item0;
+  const int i = local / P.chunks, chunk = local - i * P.chunks;
+  MmaItem it;
+  it.n = P.n;
+  it.r = P.r;
+  const int c0 = chunk * kMmaCols;
+  it.W = P.n - c0 < kMmaCols ? P.n - c0 : kMmaCols;
+  it.X = static_cast<const __nv_bfloat16*>(P.X) + static_cast<int64_t>(i) * g.T * P.n + c0;
+  it.Y = static_cast<const __nv_bfloat16*>(P.Y) + static_cast<int64_t>(i) * g.T * P.r;
+  it.G = P.G + static_cast<int64_t>(i) * P.n * P.r;
+  it.wide_is_in = P.wide_is_in;
+  it.row = P.row0 + i;
+  it.slot = chunk;
+  return it;
+}
+
+// One block per item; its stage ring runs over the item's T rows.
+template <int NT>
+__global__ void __launch_bounds__(kThreads) k_pergrad_norm_mma(const __grid_constant__ PerGradBatch g) {
+  using Cf = MmaCfg<NT>;
+  extern __shared__ __align__(128) uint8_t stage_mem[];
+  __shared__ uint64_t full[NS];
+  __shared__ float red[kThreads / 32];
+  __shared__ int abort_flag;
+  volatile int* abrt = &abort_flag;
+  const int warp = static_cast<int>(threadIdx.x) >> 5, lane = static_cast<int>(threadIdx.x) & 31;
+  const int T = g.T;
+  const int nst = (T + kMmaSR - 1) / kMmaSR;
+  const MmaItem it = mma_item(g, static_cast<int>(blockIdx.x));
+  const bool yb = it.r == Cf::YW;  // narrow rows arrive by copy (no padding needed)
+  float acc[4][NT][4];
+#pragma unroll
+  for (int mt = 0; mt < 4; ++mt)
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.f;
+
+  if (threadIdx.x == 0) {
+    for (int q = 0; q < NS; ++q) tc::mbar_init(&full[q], 1);
+    abort_flag = 0;
+    tc::fence_mbar_init();
+  }
+  __syncthreads();
+  int issued = 0;  // thread 0
+  const uint32_t row_bytes = static_cast<uint32_t>(it.W) * 2;
+  auto issue = [&](int st) {
+    const int q = st % NS, r0 = st * kMmaSR;
+    const int nr = T - r0 < kMmaSR ? T - r0 : kMmaSR;
+    uint8_t* xs = stage_mem + q * Cf::STAGE;
+    tc::mbar_arrive_expect_tx(&full[q], static_cast<uint32_t>(nr) * row_bytes +
+                                            (yb ? static_cast<uint32_t>(nr * it.r * 2) : 0u));
+    for (int rr = 0; rr < nr; ++rr)
+      tc::bulk_load(xs + rr * kMmaXStride, it.X + static_cast<int64_t>(r0 + rr) * it.n, row_bytes,
+                    &full[q]);
+    if (yb)
+      tc::bulk_load(xs + Cf::X_BYTES, it.Y + static_cast<int64_t>(r0) * it.r, nr * it.r * 2,
+                    &full[q]);
+  };
+  if (threadIdx.x == 0)
+    for (; issued < NS && issued < nst; ++issued) issue(issued);
+
+  // narrow rows that no copy brings (padded widths): each thread holds its
+  // elements of the next stage in registers, loaded a stage ahead
+  constexpr int YPT = (kMmaSR * Cf::YW + kThreads - 1) / kThreads;
+  __nv_bfloat16 ypre[YPT];
+  auto load_y = [&](int st) {
+    if (yb || st >= nst) return;
+    const int rn0 = st * kMmaSR;
+#pragma unroll
+    for (int u = 0; u < YPT; ++u) {
+      const int e = static_cast<int>(threadIdx.x) + u * kThreads;
+      const int t = e / Cf::YW, k = e - (e / Cf::YW) * Cf::YW;
+      ypre[u] = (e < kMmaSR * Cf::YW && rn0 + t < T && k < it.r)
+                    ? it.Y[static_cast<int64_t>(rn0 + t) * it.r + k]
+                    : __float2bfloat16_rn(0.f);
+    }
+  };
+  load_y(0);
+
+  const uint32_t sbase = tc::smem_u32(stage_mem);
+  const int mat = lane >> 3, mrow = lane & 7;
+  const int gq = lane >> 2, tq = lane & 3;
+  int st = 0;
+  for (; st < nst; ++st) {
+    const int q = st % NS, r0 = st * kMmaSR;
+    const int nr = T - r0 < kMmaSR ? T - r0 : kMmaSR;
+    uint8_t* xs = stage_mem + q * Cf::STAGE;
+    __nv_bfloat16* ysm = reinterpret_cast<__nv_bfloat16*>(xs + Cf::X_BYTES);
+    // parts no copy writes: rows past T, and narrow rows that need padding
+    if (nr < kMmaSR) {
+      const int words = (kMmaSR - nr) * (kMmaXStride / 4);
+      uint32_t* z = reinterpret_cast<uint32_t*>(xs + nr * kMmaXStride);
+      for (int e = threadIdx.x; e < words; e += kThreads) z[e] = 0u;
+    }
+    if (!yb) {
+#pragma unroll
+      for (int u = 0; u < YPT; ++u) {
+        const int e = static_cast<int>(threadIdx.x) + u * kThreads;
+        if (e < kMmaSR * Cf::YW) ysm[e] = ypre[u];
+      }
+    } else if (nr < kMmaSR) {
+      for (int e = threadIdx.x; e < kMmaSR * Cf::YW; e += kThreads)
+        if (e / Cf::YW >= nr) ysm[e] = __float2bfloat16_rn(0.f);  // rows past T
+    }
+    load_y(st + 1);
+    tc::mbar_wait(&full[q], static_cast<uint32_t>(st / NS) & 1u, abrt, g.err);
+    __syncthreads();
+    if (*abrt) break;
+    const uint32_t xa = sbase + q * Cf::STAGE;
+    const uint32_t ya = xa + Cf::X_BYTES;
+    uint32_t b[NT][2];
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+      ldsm_x2_trans(ya + (lane & 15) * Cf::Y_STRIDE + nt * 16, b[nt]);
+#pragma unroll
+    for (int mt = 0; mt < 4; ++mt) {
+      const int m0 = warp * 64 + mt * 16;
+      if (m0 >= it.W) continue;
+      uint32_t a[4];
+      ldsm_x4_trans(xa + ((mat >> 1) * 8 + mrow) * kMmaXStride + (m0 + (mat & 1) * 8) * 2, a);
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) mma_16816(acc[mt][nt], a, b[nt]);
+    }
+    __syncthreads();  // the stage is free again
+    if (threadIdx.x == 0 && issued < nst) {
+      // rows this block wrote into the slot (padding, staged narrow rows)
+      // may be overwritten by the copies: order them before the async proxy
+      tc::fence_proxy_async_smem();
+      issue(issued++);
+    }
+  }
+  if (st < nst) {
+    if (threadIdx.x == 0) {
+      // gave up: let every copy issued into the ring land before leaving
+      for (int k = st; k < issued; ++k) {
+        const uint64_t t0 = tc::globaltimer_ns();
+        while (!tc::mbar_try_wait(&full[k % NS], static_cast<uint32_t>(k / NS) & 1u))
+          if (tc::globaltimer_ns() - t0 > tc::kWaitLimitNs) break;
+      }
+    }
+    return;
+  }
+
+  // C fragment: c0, c1 at (row g, cols 2t, 2t+1), c2, c3 at row g + 8
+  const int c0 = it.slot * kMmaCols;
+  float sq = 0.f;
+#pragma unroll
+  for (int mt = 0; mt < 4; ++mt) {
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int mm = warp * 64 + mt * 16 + gq + (e >> 1) * 8;
+        const int k = nt * 8 + 2 * tq + (e & 1);
+        if (mm >= it.W || k >= it.r) continue;
+        const int m = c0 + mm;
+        const float v = acc[mt][nt][e];
+        sq = fmaf(v, v, sq);
+        if (it.wide_is_in)
+          it.G[static_cast<int64_t>(m) * it.r + k] = v;
+        else
+          it.G[static_cast<int64_t>(k) * it.n + m] = v;
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, o);
+  if (lane == 0) red[warp] = sq;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float s2 = 0.f;
+    for (int w = 0; w < kThreads / 32; ++w) s2 += red[w];
+    g.part[static_cast<int64_t>(it.row) * g.NP + it.slot] = s2;
+  }
+}
+
 // out = out_scale (sum_i c_i g_i + sigma C z) over the global quads that
 // overlap each layer's parameters.  A layer with few parameters splits its
 // examples over `split` threads per quad (split from the layer's own size,
@@ -426,30 +658,50 @@ int pergrad_bucket(int r) {
   return R <= kThinMax ? R : 0;
 }
 
-int pergrad_parts(int64_t d_in, int64_t d_out) {
+// bf16 layers whose wide rows are whole 16-byte vectors take the MMA kernel,
+// except narrow widths of 4 or less: padded to an 8-wide n-tile they waste
+// half of every MMA, and the multiply-add kernel keeps up with HBM there.
+bool pergrad_mma(InType t, int64_t n, int r) { return t == IN_BF16 && n % 8 == 0 && r > 4; }
+
+int pergrad_parts(InType t, int64_t d_in, int64_t d_out) {
   const int r = static_cast<int>(d_in < d_out ? d_in : d_out);
   const int64_t n = d_in < d_out ? d_out : d_in;
   const int R = pergrad_bucket(r);
   if (R == 0) return 0;
+  if (pergrad_mma(t, n, r)) return static_cast<int>((n + kMmaCols - 1) / kMmaCols);
   const int vj = R <= 8 ? 4 : (R <= 16 ? 2 : 1);
   return static_cast<int>((n + kThreads * vj - 1) / (kThreads * vj));
 }
 
-cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s) {
-  if (g.L < 1 || g.L > kPerGradMaxLayers) return cudaErrorInvalidValue;
+template <int NT>
+cudaError_t launch_mma_t(const PerGradBatch& g, int blocks, cudaStream_t s) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(k_pergrad_norm_mma<NT>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         MmaCfg<NT>::SMEM);
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  k_pergrad_norm_mma<NT><<<blocks, kThreads, MmaCfg<NT>::SMEM, s>>>(g);
+  return cudaGetLastError();
+}
+
+// One launch of the layers of g that share a path (all on MMAs or none).
+cudaError_t launch_norm_group(InType t, PerGradBatch& g, bool mma, cudaStream_t s) {
   int R = 0;
-  int64_t blocks = 0;
   for (int l = 0; l < g.L; ++l) {
-    PerGradLayer& P = g.l[l];
-    const int Rl = pergrad_bucket(P.r);
+    const int Rl = pergrad_bucket(g.l[l].r);
     if (Rl == 0) return cudaErrorInvalidValue;
     if (Rl > R) R = Rl;
   }
   const int vj = R <= 8 ? 4 : (R <= 16 ? 2 : 1);
   const int elem = t == IN_F32 ? 4 : 2;
+  int64_t blocks = 0;
   for (int l = 0; l < g.L; ++l) {
     PerGradLayer& P = g.l[l];
-    P.chunks = static_cast<int>((P.n + kThreads * vj - 1) / (kThreads * vj));
+    P.chunks = mma ? static_cast<int>((P.n + kMmaCols - 1) / kMmaCols)
+                   : static_cast<int>((P.n + kThreads * vj - 1) / (kThreads * vj));
     // bulk copies need 16-byte aligned rows (the base is 16-byte aligned)
     P.bulk = (static_cast<int64_t>(P.n) * elem) % 16 == 0 &&
              (reinterpret_cast<uintptr_t>(P.X) & 15) == 0;
@@ -457,8 +709,33 @@ cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s) {
     blocks += static_cast<int64_t>(g.B) * P.chunks;
   }
   if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
-  return t == IN_F32 ? launch_norm_r<float>(g, R, static_cast<int>(blocks), s)
-                     : launch_norm_r<__nv_bfloat16>(g, R, static_cast<int>(blocks), s);
+  const int nb = static_cast<int>(blocks);
+  if (mma) {
+    const int NT = R <= 8 ? 1 : (R <= 16 ? 2 : 4);
+    return NT == 1 ? launch_mma_t<1>(g, nb, s) : NT == 2 ? launch_mma_t<2>(g, nb, s)
+                                                         : launch_mma_t<4>(g, nb, s);
+  }
+  return t == IN_F32 ? launch_norm_r<float>(g, R, nb, s) : launch_norm_r<__nv_bfloat16>(g, R, nb, s);
+}
+
+cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s) {
+  if (g.L < 1 || g.L > kPerGradMaxLayers) return cudaErrorInvalidValue;
+  // split the batch by path, keeping each layer's partial rows and slots
+  PerGradBatch part[2];
+  for (int m = 0; m < 2; ++m) {
+    part[m] = g;
+    part[m].L = 0;
+  }
+  for (int l = 0; l < g.L; ++l) {
+    const int m = pergrad_mma(t, g.l[l].n, g.l[l].r) ? 1 : 0;
+    part[m].l[part[m].L++] = g.l[l];
+  }
+  for (int m = 0; m < 2; ++m) {
+    if (part[m].L == 0) continue;
+    cudaError_t e = launch_norm_group(t, part[m], m == 1, s);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_pergrad_sum(PerGradSumBatch& g, cudaStream_t s) {

@@ -825,6 +825,9 @@ THIN_CASES = [
     ([(1024, 32), (17, 600)], 2, 256, "f32"),     # widest bucket, r = 17 in it
     ([(1, 512)], 6, 80, "f32"),                   # a bias row (d_in = 1)
     ([(256, 8), (264, 136)], 3, 64, "bf16"),      # thin next to a tensor-core layer
+    ([(1000, 12), (24, 1000)], 3, 101, "bf16"),   # MMA kernel, padded n-tiles, ragged chunk and T
+    ([(16, 1536), (2048, 32)], 2, 150, "bf16"),   # MMA kernel, copied narrow rows, 3 and 4 chunks
+    ([(1001, 6)], 3, 40, "bf16"),                 # bf16 r > 4 with unaligned rows: multiply-adds
 ]
 
 

@@ -124,6 +124,11 @@ WORKLOADS["gpt2m_lora_webnlg_bf16"] = Workload(
 WORKLOADS["roberta_l_lora_mnli_bf16"] = Workload(
     "roberta_l_lora_mnli_bf16", 8, _lora(24, [(1024, 1024), (1024, 1024)], 8), 256, 128,
     "bf16", _normal_all(96), 1.0, math.sqrt(1e-4), 1.0, 0.6407, audit_frac=0.05)
+# one RoBERTa-large block's query and value adapters alone (profiling case for
+# the thin-layer kernels: 270 MB of inputs, larger than L2)
+WORKLOADS["roberta_l_lora_block_bf16"] = Workload(
+    "roberta_l_lora_block_bf16", 10, _lora(1, [(1024, 1024), (1024, 1024)], 8), 256, 128,
+    "bf16", _normal_all(4), 1.0, math.sqrt(1e-4), 1.0, 0.6407, audit_frac=0.05)
 # ... with the trainable classification head of a 3-class task (MNLI): dense
 # 1024 x 1024 and its bias, out_proj 1024 x 3 and its bias, all applied to the
 # first token only (T = 1); a bias row is a layer with d_in = 1 and ones as A
