@@ -327,8 +327,31 @@ def run_ours(args, rank, world, local_rank):
         torch.cuda.synchronize()
         ms_no_audit = e_a.elapsed_time(e_b) / args.steps
 
-    if graph is not None:  # per-kernel split from one eager timed step
-        step(args.warmup + args.steps, timed=True)
+    if graph is not None:
+        # per-kernel split: the step's stages captured as separate graphs and
+        # replayed back to back with an event between stages, so the host
+        # work of each call (planning, marshalling) stays out of the times
+        stages = (lambda: dp.dp_step_init(cfg, stream, ctx),
+                  lambda: dp.dp_layer_norms_batch(ctx, layer_ids, A_d, D_d),
+                  lambda: dp.dp_clip_factors(ctx),
+                  lambda: dp.dp_clipped_sum_noise_batch(ctx, layer_ids, A_d, D_d, outs, 0))
+        stage_graphs = []
+        for fn in stages:
+            g_ = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g_, stream=stream):
+                fn()
+            stage_graphs.append(g_)
+        torch.cuda.synchronize()
+        ev = {k: [] for k in ev}
+        for t in range(args.warmup + args.steps):
+            es = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+            for g_, e_ in zip(stage_graphs, es):
+                g_.replay()
+                e_.record(stream)
+            if t >= args.warmup:
+                ev["norm"].append((None, es[0], es[1]))
+                ev["clip"].append((0, es[1], es[2]))
+                ev["gemm"].append((None, es[2], es[3]))
         torch.cuda.synchronize()
 
     def per_step_ms(kind, layer=None):

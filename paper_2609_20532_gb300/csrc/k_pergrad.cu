@@ -334,7 +334,9 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm(const __grid_constant
 // the same 16 rows of the narrow operand, zero-padded to 8 NT columns.
 // ---------------------------------------------------------------------------
 constexpr int kMmaCols = 512;
-constexpr int kMmaSR = 16;
+constexpr int kMmaSR = 16;  // rows per stage, a multiple of 16 (one k16 step each)
+constexpr int kMmaNS = 2;   // stages in the ring
+constexpr int kMmaThreads = kMmaCols / 64 * 32;  // a warp owns 64 wide columns
 constexpr int kMmaXStride = kMmaCols * 2 + 16;  // bytes per staged wide row
 
 template <int NT>
@@ -344,7 +346,9 @@ struct MmaCfg {
   static constexpr int X_BYTES = kMmaSR * kMmaXStride;
   static constexpr int Y_BYTES = kMmaSR * Y_STRIDE;
   static constexpr int STAGE = ((X_BYTES + Y_BYTES + 127) / 128) * 128;
-  static constexpr int SMEM = NS * STAGE;
+  static constexpr int SMEM = kMmaNS * STAGE;
+  static_assert(kMmaSR % 16 == 0, "a stage is whole k16 steps");
+  static_assert(SMEM <= 227 * 1024, "stage ring exceeds shared memory");
 };
 
 __device__ __forceinline__ void ldsm_x4_trans(uint32_t addr, uint32_t (&a)[4]) {
@@ -395,11 +399,11 @@ __device__ __forceinline__ MmaItem mma_item(const PerGradBatch& g, int item) {
 
 // One block per item; its stage ring runs over the item's T rows.
 template <int NT>
-__global__ void __launch_bounds__(kThreads) k_pergrad_norm_mma(const __grid_constant__ PerGradBatch g) {
+__global__ void __launch_bounds__(kMmaThreads) k_pergrad_norm_mma(const __grid_constant__ PerGradBatch g) {
   using Cf = MmaCfg<NT>;
   extern __shared__ __align__(128) uint8_t stage_mem[];
-  __shared__ uint64_t full[NS];
-  __shared__ float red[kThreads / 32];
+  __shared__ uint64_t full[kMmaNS];
+  __shared__ float red[kMmaThreads / 32];
   __shared__ int abort_flag;
   volatile int* abrt = &abort_flag;
   const int warp = static_cast<int>(threadIdx.x) >> 5, lane = static_cast<int>(threadIdx.x) & 31;
@@ -416,7 +420,7 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm_mma(const __grid_cons
       for (int e = 0; e < 4; ++e) acc[mt][nt][e] = 0.f;
 
   if (threadIdx.x == 0) {
-    for (int q = 0; q < NS; ++q) tc::mbar_init(&full[q], 1);
+    for (int q = 0; q < kMmaNS; ++q) tc::mbar_init(&full[q], 1);
     abort_flag = 0;
     tc::fence_mbar_init();
   }
@@ -424,7 +428,7 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm_mma(const __grid_cons
   int issued = 0;  // thread 0
   const uint32_t row_bytes = static_cast<uint32_t>(it.W) * 2;
   auto issue = [&](int st) {
-    const int q = st % NS, r0 = st * kMmaSR;
+    const int q = st % kMmaNS, r0 = st * kMmaSR;
     const int nr = T - r0 < kMmaSR ? T - r0 : kMmaSR;
     uint8_t* xs = stage_mem + q * Cf::STAGE;
     tc::mbar_arrive_expect_tx(&full[q], static_cast<uint32_t>(nr) * row_bytes +
@@ -437,18 +441,18 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm_mma(const __grid_cons
                     &full[q]);
   };
   if (threadIdx.x == 0)
-    for (; issued < NS && issued < nst; ++issued) issue(issued);
+    for (; issued < kMmaNS && issued < nst; ++issued) issue(issued);
 
   // narrow rows that no copy brings (padded widths): each thread holds its
   // elements of the next stage in registers, loaded a stage ahead
-  constexpr int YPT = (kMmaSR * Cf::YW + kThreads - 1) / kThreads;
+  constexpr int YPT = (kMmaSR * Cf::YW + kMmaThreads - 1) / kMmaThreads;
   __nv_bfloat16 ypre[YPT];
   auto load_y = [&](int st) {
     if (yb || st >= nst) return;
     const int rn0 = st * kMmaSR;
 #pragma unroll
     for (int u = 0; u < YPT; ++u) {
-      const int e = static_cast<int>(threadIdx.x) + u * kThreads;
+      const int e = static_cast<int>(threadIdx.x) + u * kMmaThreads;
       const int t = e / Cf::YW, k = e - (e / Cf::YW) * Cf::YW;
       ypre[u] = (e < kMmaSR * Cf::YW && rn0 + t < T && k < it.r)
                     ? it.Y[static_cast<int64_t>(rn0 + t) * it.r + k]
@@ -462,7 +466,7 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm_mma(const __grid_cons
   const int gq = lane >> 2, tq = lane & 3;
   int st = 0;
   for (; st < nst; ++st) {
-    const int q = st % NS, r0 = st * kMmaSR;
+    const int q = st % kMmaNS, r0 = st * kMmaSR;
     const int nr = T - r0 < kMmaSR ? T - r0 : kMmaSR;
     uint8_t* xs = stage_mem + q * Cf::STAGE;
     __nv_bfloat16* ysm = reinterpret_cast<__nv_bfloat16*>(xs + Cf::X_BYTES);
@@ -470,36 +474,41 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm_mma(const __grid_cons
     if (nr < kMmaSR) {
       const int words = (kMmaSR - nr) * (kMmaXStride / 4);
       uint32_t* z = reinterpret_cast<uint32_t*>(xs + nr * kMmaXStride);
-      for (int e = threadIdx.x; e < words; e += kThreads) z[e] = 0u;
+      for (int e = threadIdx.x; e < words; e += kMmaThreads) z[e] = 0u;
     }
     if (!yb) {
 #pragma unroll
       for (int u = 0; u < YPT; ++u) {
-        const int e = static_cast<int>(threadIdx.x) + u * kThreads;
+        const int e = static_cast<int>(threadIdx.x) + u * kMmaThreads;
         if (e < kMmaSR * Cf::YW) ysm[e] = ypre[u];
       }
     } else if (nr < kMmaSR) {
-      for (int e = threadIdx.x; e < kMmaSR * Cf::YW; e += kThreads)
+      for (int e = threadIdx.x; e < kMmaSR * Cf::YW; e += kMmaThreads)
         if (e / Cf::YW >= nr) ysm[e] = __float2bfloat16_rn(0.f);  // rows past T
     }
     load_y(st + 1);
-    tc::mbar_wait(&full[q], static_cast<uint32_t>(st / NS) & 1u, abrt, g.err);
+    tc::mbar_wait(&full[q], static_cast<uint32_t>(st / kMmaNS) & 1u, abrt, g.err);
     __syncthreads();
     if (*abrt) break;
     const uint32_t xa = sbase + q * Cf::STAGE;
     const uint32_t ya = xa + Cf::X_BYTES;
-    uint32_t b[NT][2];
 #pragma unroll
-    for (int nt = 0; nt < NT; ++nt)
-      ldsm_x2_trans(ya + (lane & 15) * Cf::Y_STRIDE + nt * 16, b[nt]);
+    for (int kk = 0; kk < kMmaSR / 16; ++kk) {
+      uint32_t b[NT][2];
 #pragma unroll
-    for (int mt = 0; mt < 4; ++mt) {
-      const int m0 = warp * 64 + mt * 16;
-      if (m0 >= it.W) continue;
-      uint32_t a[4];
-      ldsm_x4_trans(xa + ((mat >> 1) * 8 + mrow) * kMmaXStride + (m0 + (mat & 1) * 8) * 2, a);
+      for (int nt = 0; nt < NT; ++nt)
+        ldsm_x2_trans(ya + (kk * 16 + (lane & 15)) * Cf::Y_STRIDE + nt * 16, b[nt]);
 #pragma unroll
-      for (int nt = 0; nt < NT; ++nt) mma_16816(acc[mt][nt], a, b[nt]);
+      for (int mt = 0; mt < 4; ++mt) {
+        const int m0 = warp * 64 + mt * 16;
+        if (m0 >= it.W) continue;
+        uint32_t a[4];
+        ldsm_x4_trans(xa + (kk * 16 + (mat >> 1) * 8 + mrow) * kMmaXStride +
+                          (m0 + (mat & 1) * 8) * 2,
+                      a);
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) mma_16816(acc[mt][nt], a, b[nt]);
+      }
     }
     __syncthreads();  // the stage is free again
     if (threadIdx.x == 0 && issued < nst) {
@@ -514,7 +523,7 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm_mma(const __grid_cons
       // gave up: let every copy issued into the ring land before leaving
       for (int k = st; k < issued; ++k) {
         const uint64_t t0 = tc::globaltimer_ns();
-        while (!tc::mbar_try_wait(&full[k % NS], static_cast<uint32_t>(k / NS) & 1u))
+        while (!tc::mbar_try_wait(&full[k % kMmaNS], static_cast<uint32_t>(k / kMmaNS) & 1u))
           if (tc::globaltimer_ns() - t0 > tc::kWaitLimitNs) break;
       }
     }
@@ -549,7 +558,7 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm_mma(const __grid_cons
   __syncthreads();
   if (threadIdx.x == 0) {
     float s2 = 0.f;
-    for (int w = 0; w < kThreads / 32; ++w) s2 += red[w];
+    for (int w = 0; w < kMmaThreads / 32; ++w) s2 += red[w];
     g.part[static_cast<int64_t>(it.row) * g.NP + it.slot] = s2;
   }
 }
@@ -658,10 +667,10 @@ int pergrad_bucket(int r) {
   return R <= kThinMax ? R : 0;
 }
 
-// bf16 layers whose wide rows are whole 16-byte vectors take the MMA kernel,
-// except narrow widths of 4 or less: padded to an 8-wide n-tile they waste
-// half of every MMA, and the multiply-add kernel keeps up with HBM there.
-bool pergrad_mma(InType t, int64_t n, int r) { return t == IN_BF16 && n % 8 == 0 && r > 4; }
+// bf16 layers whose wide rows are whole 16-byte vectors take the MMA kernel
+// (narrow widths below 8 are zero-padded to one n-tile; the pass stays bound
+// by the wide rows' bytes).
+bool pergrad_mma(InType t, int64_t n, int r) { return t == IN_BF16 && n % 8 == 0 && r > 0; }
 
 int pergrad_parts(InType t, int64_t d_in, int64_t d_out) {
   const int r = static_cast<int>(d_in < d_out ? d_in : d_out);
@@ -683,7 +692,7 @@ cudaError_t launch_mma_t(const PerGradBatch& g, int blocks, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  k_pergrad_norm_mma<NT><<<blocks, kThreads, MmaCfg<NT>::SMEM, s>>>(g);
+  k_pergrad_norm_mma<NT><<<blocks, kMmaThreads, MmaCfg<NT>::SMEM, s>>>(g);
   return cudaGetLastError();
 }
 

@@ -242,23 +242,30 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
 }
 
 // ---------------------------------------------------------------------------
-// Cross-layer sum and clip factors (one thread per example, fixed order)
+// Cross-layer sum and clip factors.  One warp per example: lane j adds the
+// layers j, j + 32, ... (each layer's partials in slot order), then a fixed
+// butterfly adds the 32 lane sums, so the order never depends on timing.
 // ---------------------------------------------------------------------------
 __global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
                        const int* __restrict__ nparts, float C, float* __restrict__ layer_sq,
                        float* __restrict__ s_out, float* __restrict__ c_out,
                        float* __restrict__ user_s, float* __restrict__ user_c, int* flag) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= B) return;
+  const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = static_cast<int>(threadIdx.x) & 31;
+  if (w >= B) return;  // the whole warp leaves together
+  const int i = static_cast<int>(w);
   float s = 0.f;
-  for (int l = 0; l < L; ++l) {
-    const float* p = part + static_cast<int64_t>(l * B + i) * NP;
+  for (int l = lane; l < L; l += 32) {
+    const float* p = part + (static_cast<int64_t>(l) * B + i) * NP;
     float n = 0.f;
     const int np = nparts[l];
     for (int q = 0; q < np; ++q) n += p[q];
-    layer_sq[l * B + i] = n;
+    layer_sq[static_cast<int64_t>(l) * B + i] = n;
     s += n;
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if (lane != 0) return;
   float c;
   if (!isfinite(s)) {
     atomicOr(flag, 1);
@@ -451,8 +458,8 @@ cudaError_t launch_norm_mat_simt(InType t, const void* A, const void* D, int B, 
 cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_nparts, float C,
                         float* layer_sq, float* s_out, float* c_out, float* user_s, float* user_c,
                         int* flag, cudaStream_t s) {
-  k_clip<<<(B + 127) / 128, 128, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out,
-                                         user_s, user_c, flag);
+  k_clip<<<(B + 7) / 8, 256, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out,
+                                      user_s, user_c, flag);
   return cudaGetLastError();
 }
 
