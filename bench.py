@@ -150,6 +150,16 @@ def _traffic(kernel_key, units, path=None):
     return d["captured_dram_bytes"] * units / d["captured_units"]
 
 
+def _data_desc(w):
+    """The input recipe of a workload in words (seeded, synthetic)."""
+    names = {"normal": f"N(0,{w.a_std ** 2:g})", "uniform": "U[0,1)",
+             "relu_normal": "ReLU-sparse N(0,1)", "ones": "ones (bias rows)"}
+    acts = "/".join(names[d] for d in dict.fromkeys(w.a_dist))
+    prec = "rounded to bf16" if w.dtype == "bf16" else "fp32"
+    return (f"synthetic: seeded {acts} activations, N(0,{w.d_std ** 2:.3g}) output grads, "
+            f"{prec}")
+
+
 def cpu_baseline_sample(w, seed=0):
     """The fp64 oracle, as it stands, on a bounded sample of the workload:
     example 0 through every layer (materialised norms, clip factor, its
@@ -229,16 +239,20 @@ def run_ours(args, rank, world, local_rank):
     rec_bytes = len(idx) * dp.dp_audit_record_bytes(L)
 
     ev = {k: [] for k in ("norm", "clip", "gemm")}
+    stage_launches = {}  # kernels each stage of the last step issued (the library's count)
 
     layer_ids = list(range(L))
 
     def step(t, timed=False):
         cfg.step = t
+        n0 = dp.dp_kernel_launches()
         dp.dp_step_init(cfg, stream, ctx)
+        n1 = dp.dp_kernel_launches()
         if timed:
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-        dp.dp_layer_norms_batch(ctx, layer_ids, A_d, D_d)   # every layer, one launch
+        dp.dp_layer_norms_batch(ctx, layer_ids, A_d, D_d)   # every layer, one call
+        n2 = dp.dp_kernel_launches()
         if timed:
             e1.record(stream)
             ev["norm"].append((None, e0, e1))
@@ -246,17 +260,23 @@ def run_ours(args, rank, world, local_rank):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
         dp.dp_clip_factors(ctx)
+        n3 = dp.dp_kernel_launches()
         if timed:
             e1.record(stream)
             ev["clip"].append((0, e0, e1))
         if timed:
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-        dp.dp_clipped_sum_noise_batch(ctx, layer_ids, A_d, D_d, outs, 0)  # every layer, one launch
+        dp.dp_clipped_sum_noise_batch(ctx, layer_ids, A_d, D_d, outs, 0)  # every layer, one call
+        n4 = dp.dp_kernel_launches()
         if timed:
             e1.record(stream)
             ev["gemm"].append((None, e0, e1))
-        return dp.dp_audit_emit(ctx, idx, L)
+        rec = dp.dp_audit_emit(ctx, idx, L)
+        n5 = dp.dp_kernel_launches()
+        stage_launches.update(init=n1 - n0, norm=n2 - n1, clip=n3 - n2, gemm=n4 - n3,
+                              audit=n5 - n4, step=n5 - n0)
+        return rec
 
     def barrier():
         if world > 1:
@@ -295,6 +315,7 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize()
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     marks = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    host_launches0 = dp.dp_kernel_launches()
     with ClockSampler(local_rank) as clk:
         start.record(stream)
         for t in range(args.steps):
@@ -308,6 +329,12 @@ def run_ours(args, rank, world, local_rank):
         marks[args.steps].record(stream)
         stop.record(stream)
         torch.cuda.synchronize()
+    # kernels of the timed region: those issued from the host during it, plus
+    # the graph's (captured once, replayed each step)
+    timed_launches = dp.dp_kernel_launches() - host_launches0
+    if graph is not None:
+        timed_launches += args.steps * sum(stage_launches[k]
+                                           for k in ("init", "norm", "clip", "gemm"))
     barrier()
     torch.cuda.synchronize()
     ms = max_over_ranks(start.elapsed_time(stop), world, dev)
@@ -373,10 +400,10 @@ def run_ours(args, rank, world, local_rank):
                          "frac_bf16_peak": gemm_tflops / peaks["bf16_tflops"],
                          "frac_bf16_sustained": (gemm_tflops / peaks["bf16_tflops_sustained"]
                                                  if peaks.get("bf16_tflops_sustained") else None),
-                         "launches_per_step": 1},
+                         "launches_per_step": stage_launches["gemm"]},
         "layer_norms": {"ms_per_step": norm_ms, "gbs_inputs_read_once": norm_gbs,
                         "frac_hbm": norm_gbs / peaks["hbm_gbs"], "traffic": norm_traffic,
-                        "launches_per_step": 1},
+                        "launches_per_step": stage_launches["norm"]},
         "clip": {"ms_per_step": per_step_ms("clip")},
     }
     # thin layers (norm path 2): the norm pass reads the inputs and writes
@@ -389,7 +416,6 @@ def run_ours(args, rank, world, local_rank):
     # HBM roofline when most input bytes belong to thin layers (LoRA
     # adapters, with or without a small head)
     all_thin = thin_in * 2 >= in_total
-    n_thin = sum(thin)
     if any(thin):
         grads = 4.0 * w.B * sum(i * o for (i, o), t in zip(w.layers, thin) if t)
         p_all = 4.0 * sum(i * o for i, o in w.layers)
@@ -400,12 +426,12 @@ def run_ours(args, rank, world, local_rank):
                 "ms_per_step": norm_ms, "path": "stored per-example gradients",
                 "bytes": norm_bytes, "gbs": norm_bytes / (norm_ms * 1e-3) / 1e9,
                 "frac_hbm": norm_bytes / (norm_ms * 1e-3) / 1e9 / peaks["hbm_gbs"],
-                "launches_per_step": -(-n_thin // 32) + (L - n_thin)}
+                "launches_per_step": stage_launches["norm"]}
             kernels["clipsum_gemm"] = {
                 "ms_per_step": gemm_ms, "path": "stored per-example gradients",
                 "bytes": sum_bytes, "gbs": sum_bytes / (gemm_ms * 1e-3) / 1e9,
                 "frac_hbm": sum_bytes / (gemm_ms * 1e-3) / 1e9 / peaks["hbm_gbs"],
-                "launches_per_step": -(-n_thin // 32) + (L - n_thin)}
+                "launches_per_step": stage_launches["gemm"]}
 
     # standalone noise add over every layer (the DP_NOISE_ONLY call that adds
     # the released seed's noise to a committed sum): 8 bytes per parameter
@@ -521,15 +547,6 @@ def run_ours(args, rank, world, local_rank):
         v, dt, desc = cpu_baseline_sample(w)
         cpu = {"value": v, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": desc,
                "seconds": dt}
-    # launches of one step of a mostly-thin workload: key, clip, audit; thin
-    # layers one launch per 32 in each pass; every other layer one norm
-    # launch and one clipped-sum launch (two for a bf16 layer with T < 32 on
-    # tensor cores: the pre-scale and the GEMM)
-    launches_thin_step = 3 + 2 * -(-n_thin // 32)
-    for (i, o, T_), t in zip(w.specs, thin):
-        if not t:
-            pre = w.dtype == "bf16" and T_ < 32 and i % 8 == 0 and o % 8 == 0
-            launches_thin_step += 1 + (2 if pre else 1)
     dominant = "clipsum_gemm"
     roofline = {"kernel": dominant, "bound": "tensor", "achieved": gemm_tflops,
                 "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
@@ -545,7 +562,7 @@ def run_ours(args, rank, world, local_rank):
         "warmup": args.warmup, "ms_per_step": ms_step, "ms_per_step_median": ms_median,
         "ms_per_step_no_audit": ms_no_audit, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
-        "data": "synthetic: seeded N(0,1) activations, N(0,1e-5) output grads, rounded to bf16",
+        "data": _data_desc(w),
         "config": {"workload": w.describe(), "layers": [list(x) for x in w.layers], "B": w.B,
                    "T": w.T, "C": w.C, "sigma": w.sigma, "out_scale": "1/B",
                    "audit_examples": len(idx),
@@ -556,9 +573,10 @@ def run_ours(args, rank, world, local_rank):
         "kernels": kernels,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        # per step: key + flag reset, norms (all layers), clip, clipped sums
-        # (all layers), audit gather
-        "gpu_launches": args.steps * (5 if not all_thin else launches_thin_step),
+        # the library's own launch count over the timed region (key + flag
+        # reset, norms, clip, clipped sums, audit gather of every step)
+        "gpu_launches": timed_launches,
+        "launches_per_stage": dict(stage_launches),
         "clocks": clk.summary(),
     }
     print(json.dumps(line), flush=True)

@@ -302,6 +302,14 @@ const char* dp_last_error(void);
 /* Name of a status code. */
 const char* dp_status_string(dp_status s);
 
+/* Number of CUDA kernels this library has issued in this process, counted on
+ * the host as each launch is made, by every call above and the test exports
+ * below (dp_layer_sqnorms_noalloc is not counted).  A launch made while the
+ * stream is being captured into a CUDA graph counts once, at capture; graph
+ * replays do not call the library and are not counted.  Thread-safe.
+ * Errors: DP_ERR_ARG if count_out is NULL.                                 */
+dp_status dp_kernel_launches(int64_t* count_out);
+
 /* ---- test exports (not part of the step API) ---------------------------
  * They expose the generator the noise uses so tests can compare it with the
  * oracle: raw Philox4x32-10 blocks and the Gaussian numbers z_p.

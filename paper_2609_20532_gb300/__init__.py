@@ -27,8 +27,8 @@ __all__ = [
     "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
     "dp_audit_emit", "audit_dtype", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_layer_path",
     "dp_set_noise_key", "dp_step_destroy",
-    "dp_last_error", "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
-    "EXPORTED_SYMBOLS",
+    "dp_last_error", "dp_kernel_launches", "dp_debug_philox", "dp_debug_gaussian",
+    "dp_layer_sqnorms_noalloc", "EXPORTED_SYMBOLS",
 ]
 
 HERE = os.path.dirname(os.path.abspath(__file__))
@@ -48,7 +48,7 @@ EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "d
                     "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
                     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode",
                     "dp_layer_path", "dp_set_noise_key", "dp_step_destroy", "dp_last_error",
-                    "dp_status_string",
+                    "dp_status_string", "dp_kernel_launches",
                     "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
                     "dp_noise_adamw"]
 
@@ -113,6 +113,7 @@ def lib() -> ctypes.CDLL:
         "dp_step_destroy": ([vp], None),
         "dp_last_error": ([], ctypes.c_char_p),
         "dp_status_string": ([i32], ctypes.c_char_p),
+        "dp_kernel_launches": ([ctypes.POINTER(i64)], i32),
         "dp_debug_philox": ([u64, u64, u64, i64, vp, vp], i32),
         "dp_debug_gaussian": ([u64, u64, u64, i64, vp, vp], i32),
         "dp_layer_sqnorms_noalloc": ([vp, vp, i32, i32, i64, i64, i32, vp, vp], i32),
@@ -251,6 +252,13 @@ def dp_step_destroy(ctx: Optional[int]) -> None:
 
 def dp_last_error() -> str:
     return lib().dp_last_error().decode()
+
+
+def dp_kernel_launches() -> int:
+    """Kernels the library has issued in this process (host-side count)."""
+    n = ctypes.c_int64(0)
+    _check(lib().dp_kernel_launches(ctypes.byref(n)))
+    return n.value
 
 
 def dp_debug_philox(seed: int, step: int, first_quad: int, n_quads: int, out, stream=None):

@@ -835,6 +835,12 @@ const char* dp_status_string(dp_status s) {
   return "DP_ERR_UNKNOWN";
 }
 
+dp_status dp_kernel_launches(int64_t* count_out) {
+  if (!count_out) return fail(DP_ERR_ARG, "count_out is NULL");
+  *count_out = dpk::launch_count();
+  return DP_OK;
+}
+
 dp_status dp_debug_philox(uint64_t seed, uint64_t step, uint64_t first_quad, int64_t n_quads,
                           uint32_t* d_out, void* stream) {
   if (n_quads < 0) return fail(DP_ERR_ARG, "n_quads < 0");

@@ -108,6 +108,11 @@ cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, int* fl
 cudaError_t launch_set_key(uint64_t seed, uint64_t step, uint64_t* key, int* flag,
                            cudaStream_t s);
 
+// ---- launch count: every launcher calls note_launch() once per kernel it
+// issues (process-wide, thread-safe), read back by dp_kernel_launches() ----
+void note_launch();
+int64_t launch_count();
+
 // ---- error message of the calling thread, read back by dp_last_error() ----
 void set_last_error(const char* msg);
 

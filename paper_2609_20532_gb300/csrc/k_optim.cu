@@ -85,6 +85,7 @@ cudaError_t launch_noise_adamw(float* grad, float* theta, float* m, float* v, in
   const int64_t nq = static_cast<int64_t>(((p_base + n - 1) >> 2) - (p_base >> 2) + 1);
   int64_t blocks = (nq + 255) / 256;
   const int64_t cap = 152 * 8;
+  note_launch();
   if (blocks > cap) blocks = cap;
   k_noise_adamw<<<static_cast<int>(blocks), 256, 0, s>>>(grad, theta, m, v, n, p_base, key,
                                                          noise_scale, add_noise, write_grad, h);

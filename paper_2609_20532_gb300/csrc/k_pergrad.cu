@@ -642,6 +642,7 @@ cudaError_t launch_norm_t(const PerGradBatch& g, int blocks, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
+  note_launch();
   k_pergrad_norm<TIn, R><<<blocks, kThreads, kPerGradSmem, s>>>(g);
   return cudaGetLastError();
 }
@@ -692,6 +693,7 @@ cudaError_t launch_mma_t(const PerGradBatch& g, int blocks, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
+  note_launch();
   k_pergrad_norm_mma<NT><<<blocks, kMmaThreads, MmaCfg<NT>::SMEM, s>>>(g);
   return cudaGetLastError();
 }
@@ -765,6 +767,7 @@ cudaError_t launch_pergrad_sum(PerGradSumBatch& g, cudaStream_t s) {
     const int qpb = kThreads / split;
     blocks += (P.nq + qpb - 1) / qpb;
   }
+  note_launch();
   if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
   k_pergrad_sum<<<static_cast<int>(blocks), kThreads, 0, s>>>(g);
   return cudaGetLastError();

@@ -415,6 +415,7 @@ int mat_simt_parts(int d_in, int d_out) {
 
 cudaError_t launch_norm_rank1(InType t, const void* A, const void* D, int B, int d_in, int d_out,
                               float* part, int NP, int row0, cudaStream_t s) {
+  note_launch();
   if (t == IN_F32)
     k_norm_rank1<float><<<B, 256, 0, s>>>(static_cast<const float*>(A),
                                            static_cast<const float*>(D), d_in, d_out, part, NP,
@@ -429,6 +430,7 @@ cudaError_t launch_norm_rank1(InType t, const void* A, const void* D, int B, int
 cudaError_t launch_norm_ghost_simt(InType t, const void* A, const void* D, int B, int T, int d_in,
                                    int d_out, float* part, int NP, int row0, cudaStream_t s) {
   const dim3 grid(ghost_simt_parts(T), B);
+  note_launch();
   if (t == IN_F32)
     k_norm_ghost_simt<float><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
                                                    static_cast<const float*>(D), T, d_in, d_out,
@@ -444,6 +446,7 @@ cudaError_t launch_norm_mat_simt(InType t, const void* A, const void* D, int B, 
                                  int d_out, float* part, int NP, int row0, cudaStream_t s) {
   const dim3 grid((d_out + SB - 1) / SB, (d_in + SB - 1) / SB, B);
   Epilogue ep{};
+  note_launch();
   if (t == IN_F32)
     k_gemm_simt<float, true, SB><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
                                                        static_cast<const float*>(D), nullptr, T,
@@ -458,6 +461,7 @@ cudaError_t launch_norm_mat_simt(InType t, const void* A, const void* D, int B, 
 cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_nparts, float C,
                         float* layer_sq, float* s_out, float* c_out, float* user_s, float* user_c,
                         int* flag, cudaStream_t s) {
+  note_launch();
   k_clip<<<(B + 7) / 8, 256, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out,
                                       user_s, user_c, flag);
   return cudaGetLastError();
@@ -467,6 +471,7 @@ template <int TB>
 void launch_gemm_simt_tb(InType t, const void* A, const void* D, const float* c, int B, int T,
                          int d_in, int d_out, float* out, const Epilogue& ep, cudaStream_t s) {
   const dim3 grid((d_out + TB - 1) / TB, (d_in + TB - 1) / TB, 1);
+  note_launch();
   if (t == IN_F32)
     k_gemm_simt<float, false, TB><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
                                                         static_cast<const float*>(D), c, T, B,
@@ -492,6 +497,7 @@ cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, const uint6
                              float scale, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const int64_t nq = static_cast<int64_t>(((p_base + n - 1) >> 2) - (p_base >> 2) + 1);
+  note_launch();
   k_noise_add<<<grid_for(nq, 256), 256, 0, s>>>(out, n, p_base, key, scale);
   return cudaGetLastError();
 }
@@ -500,24 +506,28 @@ cudaError_t launch_audit(const int* idx, int n, int L, int B, const float* layer
                          const float* s_vec, const float* c_vec, const int* flag, float* rec,
                          int* flag_out, cudaStream_t s) {
   const int blocks = n > 0 ? (n + 127) / 128 : 1;
+  note_launch();
   k_audit<<<blocks, 128, 0, s>>>(idx, n, L, B, layer_sq, s_vec, c_vec, flag, rec, flag_out);
   return cudaGetLastError();
 }
 
 cudaError_t launch_set_key(uint64_t seed, uint64_t step, uint64_t* key, int* flag,
                            cudaStream_t s) {
+  note_launch();
   k_set_key<<<1, 1, 0, s>>>(seed, step, key, flag);
   return cudaGetLastError();
 }
 
 cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, int* flag,
                             cudaStream_t s) {
+  note_launch();
   k_load_key<<<1, 1, 0, s>>>(host_key_dev, key, flag);
   return cudaGetLastError();
 }
 
 cudaError_t launch_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
                                 uint32_t* out, cudaStream_t s) {
+  note_launch();
   if (nq <= 0) return cudaSuccess;
   k_debug_philox<<<grid_for(nq, 256), 256, 0, s>>>(seed, step, q0, nq, out);
   return cudaGetLastError();
@@ -525,6 +535,7 @@ cudaError_t launch_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64
 
 cudaError_t launch_debug_gauss(uint64_t seed, uint64_t step, uint64_t p0, int64_t n, float* out,
                                cudaStream_t s) {
+  note_launch();
   if (n <= 0) return cudaSuccess;
   k_debug_gauss<<<grid_for(n, 256), 256, 0, s>>>(seed, step, p0, n, out);
   return cudaGetLastError();

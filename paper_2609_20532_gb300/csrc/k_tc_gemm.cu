@@ -534,9 +534,11 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
     }
     const int pairs = tiles < max_pairs ? tiles : max_pairs;
     cfg.gridDim = dim3(2 * pairs);
+    note_launch();
     return cudaLaunchKernelEx(&cfg, k_gemm_tc<NORM, PAIR>, g);
   } else {
     const int grid = tiles < sms ? tiles : sms;
+    note_launch();
     k_gemm_tc<NORM, PAIR><<<grid, GEMM_THREADS, C::SMEM_BYTES, s>>>(g);
     return cudaGetLastError();
   }
@@ -628,6 +630,7 @@ cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const floa
   const int64_t nvec = 2 * R * (d_in / 8);
   int64_t blocks = (nvec + 255) / 256;
   const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
+  note_launch();
   if (blocks > cap) blocks = cap;
   k_prescale_hilo<<<static_cast<int>(blocks), 256, 0, s>>>(
       static_cast<const __nv_bfloat16*>(A), c, T, BT, R, d_in, A2);

@@ -347,6 +347,7 @@ cudaError_t tc_launch_ghost_batch(int L, const void* const* A, const void* const
   const int items = L * B * (g.n_full + g.n_half);
   const int sms = device_sm_count();
   const int grid = items < sms ? items : sms;
+  note_launch();
   k_ghost_tc<<<grid, GHOST_THREADS, SMEM_BYTES, s>>>(g);
   return cudaGetLastError();
 }

@@ -5,11 +5,19 @@
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "tc.h"
 
 namespace dpk {
+
+namespace {
+std::atomic<int64_t> g_launches{0};
+}  // namespace
+
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+int64_t launch_count() { return g_launches.load(std::memory_order_relaxed); }
 
 namespace {
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {

@@ -98,3 +98,14 @@ def test_misc_exports(L):
     assert L.dp_debug_gaussian(0, 0, 0, -1, None, None) == 1
     # zero-length requests launch nothing
     assert L.dp_debug_philox(0, 0, 0, 0, None, None) == 0
+
+
+def test_kernel_launch_count_is_a_host_query(L):
+    """dp_kernel_launches reads a host counter: no device is touched, a NULL
+    output is rejected, and calls that fail on the host launch nothing."""
+    n0 = dp.dp_kernel_launches()
+    assert isinstance(n0, int) and n0 >= 0
+    assert L.dp_kernel_launches(None) == 1
+    st, h = _init_status(L, _cfg(B=0))
+    assert st == 2 and not h
+    assert dp.dp_kernel_launches() == n0

@@ -623,6 +623,54 @@ def test_cuda_graph_replay_matches_eager_steps():
         dp.dp_step_destroy(ctx)
 
 
+def test_launch_counts_of_a_step():
+    """The library's own launch count: 33 thin layers of one width bucket and
+    T take two norm launches and two clipped-sum launches (32 layers per
+    launch), the re-key, clip and audit one each, a call refused on the host
+    none; a captured step counts its kernels once, at capture, and replays
+    add nothing."""
+    w = W.custom("launch33", [(64, 8)] * 33, 4, 64, "bf16", C=0.5, sigma=0.5, wid=870)
+    assert is_thin(64, 8, w.T, w.dtype)
+    layers = W.make_inputs(w)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    outs = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    ids = list(range(len(layers)))
+    n = dp.dp_kernel_launches
+    s = torch.cuda.Stream()
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, audit_capacity=w.B)
+    ctx = dp.dp_step_init(cfg, s)
+    try:
+        with torch.cuda.stream(s):
+            counts = []
+            for call in (lambda: dp.dp_step_init(cfg, s, ctx),
+                         lambda: dp.dp_layer_norms_batch(ctx, ids, Ad, Dd),
+                         lambda: dp.dp_clip_factors(ctx),
+                         lambda: dp.dp_clipped_sum_noise_batch(ctx, ids, Ad, Dd, outs, 0),
+                         lambda: dp.dp_audit_emit(ctx, range(w.B), len(layers))):
+                c0 = n()
+                call()
+                counts.append(n() - c0)
+            assert counts == [1, 2, 1, 2, 1]
+            c0 = n()
+            with pytest.raises(dp.DPError):
+                dp.dp_clip_factors(ctx)          # twice in one step: refused on the host
+            assert n() == c0
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=s):
+                dp.dp_step_init(cfg, s, ctx)
+                dp.run_step(ctx, Ad, Dd, outs)
+            assert n() - c0 == 6
+            c0 = n()
+            for _ in range(3):
+                graph.replay()
+            s.synchronize()
+            assert n() == c0
+    finally:
+        dp.dp_step_destroy(ctx)
+
+
 # ---------------------------------------------------------------------------
 # the GPU's update after the seed release (Algorithm 2, OptStep = AdamW, App. A)
 # ---------------------------------------------------------------------------
