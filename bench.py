@@ -426,11 +426,13 @@ def run_ours(args, rank, world, local_rank):
                 "ms_per_step": norm_ms, "path": "stored per-example gradients",
                 "bytes": norm_bytes, "gbs": norm_bytes / (norm_ms * 1e-3) / 1e9,
                 "frac_hbm": norm_bytes / (norm_ms * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                "traffic": _traffic("pergrad_norm", norm_bytes),
                 "launches_per_step": stage_launches["norm"]}
             kernels["clipsum_gemm"] = {
                 "ms_per_step": gemm_ms, "path": "stored per-example gradients",
                 "bytes": sum_bytes, "gbs": sum_bytes / (gemm_ms * 1e-3) / 1e9,
                 "frac_hbm": sum_bytes / (gemm_ms * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                "traffic": _traffic("pergrad_sum", sum_bytes),
                 "launches_per_step": stage_launches["gemm"]}
 
     # standalone noise add over every layer (the DP_NOISE_ONLY call that adds
@@ -556,7 +558,7 @@ def run_ours(args, rank, world, local_rank):
         k = kernels["layer_norms"]
         roofline = {"kernel": "pergrad_norm", "bound": "hbm", "achieved": k["gbs"],
                     "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": k["frac_hbm"],
-                    "traffic": None, "peak_src": f"{peaks['src']} HBM copy"}
+                    "traffic": k["traffic"], "peak_src": f"{peaks['src']} HBM copy"}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "ms_per_step_median": ms_median,
