@@ -55,6 +55,8 @@ struct LayerPlan {
   int gemm_tc;         // 0: CUDA-core clipped sum, 1: tcgen05, 2: tcgen05 on a pre-scaled operand
   int pergrad;         // 1: thin layer, per-example gradients stored by the norm pass
   int64_t g_off;       // offset (floats) of its [B][d_in][d_out] gradients in d_grads
+  int split;           // tensor-core clipped sum: example ranges per tile (tc_gemm_split)
+  int64_t s_off;       // offset (floats) of its [split][d_in][d_out] partials in d_split
 };
 
 struct dp_ctx {
@@ -91,6 +93,8 @@ struct dp_ctx {
   int64_t prescaled_bytes = 0;
   float* d_grads = nullptr;     // per-example gradients of thin layers
   int64_t grads_floats = 0;
+  float* d_split = nullptr;     // partial sums of tensor-core layers whose batch is split
+  int64_t split_floats = 0;
   size_t part_bytes = 0;
   // per-step state
   std::vector<char> norm_done;
@@ -165,7 +169,7 @@ bool use_pergrad(const dp_config* cfg, int T, int64_t d_in, int64_t d_out) {
 void build_plan(dp_ctx* c, const dp_config* cfg) {
   c->plan.resize(cfg->n_layers);
   uint64_t off = 0;
-  int64_t grads = 0;
+  int64_t grads = 0, splits = 0;
   int NP = 1;
   for (int l = 0; l < cfg->n_layers; ++l) {
     LayerPlan& p = c->plan[l];
@@ -177,6 +181,8 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
     off += static_cast<uint64_t>(p.d_in) * p.d_out;
     p.pergrad = use_pergrad(cfg, T, p.d_in, p.d_out) ? 1 : 0;
     p.g_off = 0;
+    p.split = 1;
+    p.s_off = 0;
     if (p.pergrad) {
       p.mode = DP_NORM_MATERIALISED;
       p.norm_tc = 0;
@@ -204,6 +210,11 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
     p.gemm_tc = 0;
     if (bf16 && dpk::tc_gemm_supported(T, p.d_in, p.d_out)) {
       p.gemm_tc = 1;
+      p.split = dpk::tc_gemm_split(cfg->B, T, p.d_in, p.d_out);
+      if (p.split > 1) {
+        p.s_off = splits;
+        splits += static_cast<int64_t>(p.split) * p.d_in * p.d_out;
+      }
     } else if (bf16 && dpk::tc_prescaled_supported(T, p.d_in, p.d_out)) {
       p.gemm_tc = 2;
       const int64_t need = dpk::tc_prescaled_scratch_bytes(cfg->B, T, p.d_in);
@@ -213,6 +224,7 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
   }
   c->NP = NP;
   c->grads_floats = grads;
+  c->split_floats = splits;
 }
 
 void free_scratch(dp_ctx* c) {
@@ -227,8 +239,10 @@ void free_scratch(dp_ctx* c) {
   cudaFreeHost(c->h_flag);
   cudaFree(c->d_prescaled);
   cudaFree(c->d_grads);
+  cudaFree(c->d_split);
   c->d_prescaled = nullptr;
   c->d_grads = nullptr;
+  c->d_split = nullptr;
   cudaFree(c->d_key);
   cudaFreeHost(c->h_key);
   c->d_key = nullptr;
@@ -263,6 +277,7 @@ dp_status alloc_scratch(dp_ctx* c) {
   DP_ALLOC(c->d_flag, sizeof(int));
   if (c->prescaled_bytes > 0) DP_ALLOC(c->d_prescaled, static_cast<size_t>(c->prescaled_bytes));
   if (c->grads_floats > 0) DP_ALLOC(c->d_grads, sizeof(float) * static_cast<size_t>(c->grads_floats));
+  if (c->split_floats > 0) DP_ALLOC(c->d_split, sizeof(float) * static_cast<size_t>(c->split_floats));
   DP_ALLOC(c->d_key, 2 * sizeof(uint64_t));
 #undef DP_ALLOC
   if (cudaHostAlloc(reinterpret_cast<void**>(&c->h_idx), sizeof(int) * (cap > 0 ? cap : 1),
@@ -465,7 +480,8 @@ cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const vo
   }
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
   if (p.gemm_tc == 1)
-    return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, p.T, din, dout, d_out, ep, c->d_flag,
+    return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, p.T, din, dout, d_out,
+                                  p.split > 1 ? c->d_split + p.s_off : nullptr, ep, c->d_flag,
                                   c->stream);
   if (p.gemm_tc == 2)
     return dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, p.T, din, dout, d_out, ep,
@@ -495,16 +511,19 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     const int oldNP = c->NP;
     const int64_t old_pre = c->prescaled_bytes;
     const int64_t old_grads = c->grads_floats;
+    const int64_t old_splits = c->split_floats;
     build_plan(c, cfg);
     c->prescaled_bytes = old_pre;  // shapes are unchanged, so is the pre-scale need
-    if (c->NP > oldNP || c->grads_floats > old_grads) {
+    if (c->NP > oldNP || c->grads_floats > old_grads || c->split_floats > old_splits) {
       c->plan = old;
       c->NP = oldNP;
       c->grads_floats = old_grads;
+      c->split_floats = old_splits;
       return fail(DP_ERR_SHAPE, "norm_mode change needs more scratch; destroy and re-create");
     }
     c->NP = oldNP;  // keep the allocated stride
     c->grads_floats = old_grads;
+    c->split_floats = old_splits;
     set_scalars(c, cfg, cuda_stream);
     if (!same_parts(old, c->plan)) {
       st = upload_plan(c);
@@ -688,6 +707,7 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
     const void* a[dpk::kGemmMaxLayers];
     const void* d[dpk::kGemmMaxLayers];
     float* o[dpk::kGemmMaxLayers];
+    float* part[dpk::kGemmMaxLayers];
     int din[dpk::kGemmMaxLayers], dout[dpk::kGemmMaxLayers];
     uint64_t pb[dpk::kGemmMaxLayers];
     for (size_t q = 0; q < grp.size(); ++q) {
@@ -696,13 +716,14 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
       a[q] = A[r];
       d[q] = D[r];
       o[q] = d_out[r];
+      part[q] = p.split > 1 ? c->d_split + p.s_off : nullptr;
       din[q] = static_cast<int>(p.d_in);
       dout[q] = static_cast<int>(p.d_out);
       pb[q] = p.p_base;
     }
-    cudaError_t e = dpk::tc_launch_clipsum_batch(static_cast<int>(grp.size()), a, d, o, din, dout,
-                                                 pb, c->d_c, c->B, c->plan[layers[grp[0]]].T, ep,
-                                                 c->d_flag, c->stream);
+    cudaError_t e = dpk::tc_launch_clipsum_batch(static_cast<int>(grp.size()), a, d, o, part, din,
+                                                 dout, pb, c->d_c, c->B, c->plan[layers[grp[0]]].T,
+                                                 ep, c->d_flag, c->stream);
     grp.clear();
     return e;
   };

@@ -79,12 +79,13 @@ struct Cfg {
 struct GemmArgs {
   CUtensorMap mapA[kGemmMaxLayers];
   CUtensorMap mapD[kGemmMaxLayers];
-  CUtensorMap mapO[kGemmMaxLayers];  // fp32 outputs, 32 x 32 boxes
+  CUtensorMap mapO[kGemmMaxLayers];  // fp32 outputs, 32 x 32 boxes ([split][d_in][d_out] when split)
   float* out[kGemmMaxLayers];
   uint64_t p_base[kGemmMaxLayers];  // global parameter index of element (0, 0)
   int d_in[kGemmMaxLayers], d_out[kGemmMaxLayers];
   int n_m[kGemmMaxLayers], n_n[kGemmMaxLayers];
-  int tile_start[kGemmMaxLayers + 1];
+  int split[kGemmMaxLayers];  // example ranges per tile (1: the whole batch)
+  int tile_start[kGemmMaxLayers + 1];  // first work item of each layer
   int L;
   const float* c;  // clip factors [B]; nullptr: all ones (pre-scaled operand)
   float* part;     // materialised-norm partials (L == 1)
@@ -97,6 +98,28 @@ struct GemmArgs {
   float out_scale, sigmaC;
   int add_noise, accumulate;
 };
+
+// One work item: a tile of layer l over the examples [e0, e1) of range s.
+// Items are range-major within a layer, so the items in flight at once are
+// different tiles of the same examples and share their operand rows in L2.
+struct GemmItem {
+  int l, lt, s, e0, e1;
+};
+
+__device__ __forceinline__ GemmItem gemm_item(const GemmArgs& g, int item) {
+  GemmItem w;
+  int l = 0;
+  while (item >= g.tile_start[l + 1]) ++l;
+  const int li = item - g.tile_start[l];
+  const int tiles = g.n_m[l] * g.n_n[l];
+  const int S = g.split[l];
+  w.l = l;
+  w.s = li / tiles;
+  w.lt = li - w.s * tiles;
+  w.e0 = static_cast<int>(static_cast<int64_t>(g.B) * w.s / S);
+  w.e1 = static_cast<int>(static_cast<int64_t>(g.B) * (w.s + 1) / S);
+  return w;
+}
 
 // Bounded wait used only at teardown (ignores the abort flag).
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* err) {
@@ -248,14 +271,13 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       uint32_t phase = 0;
       uint32_t uses[STAGES] = {};
       for (int tile = unit; tile < n_tiles; tile += n_units) {
-        int l = 0;
-        while (tile >= g.tile_start[l + 1]) ++l;
-        const int lt = tile - g.tile_start[l];
+        const GemmItem w = gemm_item(g, tile);
+        const int l = w.l;
         int mt, nt;
-        tile_mn(lt, g.n_m[l], g.n_n[l], mt, nt);
+        tile_mn(w.lt, g.n_m[l], g.n_n[l], mt, nt);
         const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
         const int n0 = nt * BN + (PAIR ? static_cast<int>(rank) * (BN / 2) : 0);
-        for (int ex = 0; ex < g.B; ++ex) {
+        for (int ex = w.e0; ex < w.e1; ++ex) {
           for (int kb = 0; kb < kpe; ++kb) {
             if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
             uint8_t* sa = smem + stage * C::STAGE_BYTES;
@@ -286,7 +308,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       uint32_t phase = 0;
       int it = 0;
       for (int tile = unit; tile < n_tiles; tile += n_units) {
-        for (int ex = 0; ex < g.B; ++ex, ++it) {
+        const GemmItem w = gemm_item(g, tile);
+        for (int ex = w.e0; ex < w.e1; ++ex, ++it) {
           const int buf = it & 1;
           const uint32_t tph = (it >> 1) & 1;
           if (!mbar_wait(&tempty_bar[buf], tph ^ 1, abrt, g.err)) goto mma_done;
@@ -344,10 +367,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int qpe = (32 + g.B - 1) / g.B;
     const uint64_t seed = g.add_noise ? g.key[0] : 0, step = g.add_noise ? g.key[1] : 0;
     for (int tile = unit; tile < n_tiles; tile += n_units) {
-      int l = 0;
-      while (tile >= g.tile_start[l + 1]) ++l;
-      const int lt = tile - g.tile_start[l];
+      const GemmItem w = gemm_item(g, tile);
+      const int l = w.l, lt = w.lt;
       const int d_in = g.d_in[l], d_out = g.d_out[l];
+      // a split tile stores its partial sum unscaled and without noise; the
+      // reduce pass adds the ranges in order, then the noise
+      const bool part_out = g.split[l] > 1;
       int mt, nt;
       tile_mn(lt, g.n_m[l], g.n_n[l], mt, nt);
       const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
@@ -360,17 +385,19 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 #pragma unroll
         for (int i = 0; i < 128; ++i) S[i] = 0.f;
       }
-      for (int ex = 0; ex < g.B; ++ex, ++it) {
+      for (int ex = w.e0; ex < w.e1; ++ex, ++it) {
         if constexpr (!NORM) {
-          if (g.add_noise && j < d_in) {
+          if (g.add_noise && !part_out && j < d_in) {
             const int q_lo = ex * qpe;
             const int q_hi = q_lo + qpe < 32 ? q_lo + qpe : 32;
 #pragma unroll 1
             for (int q = q_lo; q < q_hi; ++q) {
-              // p_base and d_out are multiples of 8 on this path, so the four
-              // parameters prow+k .. +3 form exactly one Philox quad
+              // d_out is a multiple of 8 on this path, so the four parameters
+              // prow+k .. +3 sit in one output row; they form one Philox quad
+              // when p_base is a multiple of 4, else they straddle two (a
+              // layer after one whose size is not a multiple of 4)
               if (k0 + 4 * q >= d_out) break;
-              const float4 z = gauss_quad(seed, step, (prow + k0 + 4 * q) >> 2);
+              const float4 z = gauss4_at(seed, step, prow + k0 + 4 * q);
               add_noise_slot<0, 32>(S, q, z, g.sigmaC);
             }
           }
@@ -425,17 +452,20 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           __syncwarp();
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
+            const float sc = part_out ? 1.f : g.out_scale;
             float4 v;
-            v.x = g.out_scale * S[32 * c4 + 4 * k + 0];
-            v.y = g.out_scale * S[32 * c4 + 4 * k + 1];
-            v.z = g.out_scale * S[32 * c4 + 4 * k + 2];
-            v.w = g.out_scale * S[32 * c4 + 4 * k + 3];
+            v.x = sc * S[32 * c4 + 4 * k + 0];
+            v.y = sc * S[32 * c4 + 4 * k + 1];
+            v.z = sc * S[32 * c4 + 4 * k + 2];
+            v.w = sc * S[32 * c4 + 4 * k + 3];
             *reinterpret_cast<float4*>(stg + lane * 128 + ((k ^ (lane & 7)) << 4)) = v;
           }
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
-            if (g.accumulate)
+            if (part_out)
+              tma_store_3d(&g.mapO[l], stg, k0 + 32 * c4, y, w.s);
+            else if (g.accumulate)
               tma_reduce_add_2d(&g.mapO[l], stg, k0 + 32 * c4, y);
             else
               tma_store_2d(&g.mapO[l], stg, k0 + 32 * c4, y);
@@ -505,7 +535,8 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
   for (int l = 0; l < g.L; ++l) {
     g.n_m[l] = (g.d_in[l] + C::TILE_M - 1) / C::TILE_M;
     g.n_n[l] = (g.d_out[l] + BN - 1) / BN;
-    g.tile_start[l + 1] = g.tile_start[l] + g.n_m[l] * g.n_n[l];
+    if (g.split[l] < 1) g.split[l] = 1;
+    g.tile_start[l + 1] = g.tile_start[l] + g.n_m[l] * g.n_n[l] * g.split[l];
   }
   const int tiles = g.tile_start[g.L];
   const int sms = device_sm_count();
@@ -605,7 +636,81 @@ __global__ void k_prescale_hilo(const __nv_bfloat16* __restrict__ A, const float
 
 int64_t prescale_rows(int B, int T) { return ((static_cast<int64_t>(B) * T + BK - 1) / BK) * BK; }
 
+// out = out_scale (sum over ranges s of part[s] + sigma C z) for the split
+// layers of a launch, one thread per 4 consecutive parameters, the ranges
+// added in order.  On the tensor-core path d_in * d_out is a multiple of 64,
+// so every group of 4 is whole and 16-byte aligned; its noise is one Philox
+// quad, or two when p_base is not a multiple of 4.
+struct SplitReduceLayer {
+  const float* part;
+  float* out;
+  int64_t count;    // d_in * d_out
+  uint64_t p_base;  // global parameter index of element 0
+  int64_t q0;       // first thread of this layer in the launch
+  int split;
+};
+struct SplitReduceBatch {
+  SplitReduceLayer l[kGemmMaxLayers];
+  int L;
+  const uint64_t* key;
+  float out_scale, sigmaC;
+  int add_noise, accumulate;
+};
+
+__global__ void __launch_bounds__(256) k_split_reduce(const __grid_constant__ SplitReduceBatch g) {
+  const int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  int l = 0;
+  while (l + 1 < g.L && q >= g.l[l + 1].q0) ++l;
+  const SplitReduceLayer& P = g.l[l];
+  const int64_t e = (q - P.q0) * 4;
+  if (q < P.q0 || e >= P.count) return;
+  float4 s = __ldcs(reinterpret_cast<const float4*>(P.part + e));
+  for (int k = 1; k < P.split; ++k) {
+    const float4 v = __ldcs(reinterpret_cast<const float4*>(P.part + k * P.count + e));
+    s.x += v.x;
+    s.y += v.y;
+    s.z += v.z;
+    s.w += v.w;
+  }
+  float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (g.add_noise) z = gauss4_at(g.key[0], g.key[1], P.p_base + e);
+  float4 v;
+  v.x = g.out_scale * fmaf(g.sigmaC, z.x, s.x);
+  v.y = g.out_scale * fmaf(g.sigmaC, z.y, s.y);
+  v.z = g.out_scale * fmaf(g.sigmaC, z.z, s.z);
+  v.w = g.out_scale * fmaf(g.sigmaC, z.w, s.w);
+  float4* o = reinterpret_cast<float4*>(P.out + e);
+  if (g.accumulate) {
+    const float4 a = *o;
+    v.x += a.x;
+    v.y += a.y;
+    v.z += a.z;
+    v.w += a.w;
+  }
+  *o = v;
+}
+
 }  // namespace
+
+// Example ranges per tile of a layer's clipped sum or materialised norm.  A
+// layer with fewer tiles than the GPU has units splits its batch so that the
+// items fill the units, each range keeping at least 8 K-blocks of work.  The
+// count depends only on the layer's own shape (and the device's SM count),
+// so a layer rounds the same in a batched launch and in a launch of its own.
+int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out) {
+  const bool pair = use_pair(d_in);
+  const int64_t tile_m = pair ? 2 * BM : BM;
+  const int64_t tiles = ((d_in + tile_m - 1) / tile_m) * ((d_out + BN - 1) / BN);
+  const int64_t units = pair ? device_sm_count() / 2 : device_sm_count();
+  if (tiles >= units || B < 2) return 1;
+  const int64_t kpe = (T + BK - 1) / BK;
+  int64_t S = (units + tiles - 1) / tiles;
+  const int64_t by_work = static_cast<int64_t>(B) * kpe / 8;
+  if (S > by_work) S = by_work;
+  if (S > B) S = B;
+  if (S > kGemmMaxSplit) S = kGemmMaxSplit;
+  return S < 1 ? 1 : static_cast<int>(S);
+}
 
 // Direct path: T a multiple of 64, or T >= 32 (3-D padding wastes at most half).
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out) {
@@ -672,6 +777,7 @@ cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d
   g.T = T;
   g.d_in[0] = d_in;
   g.d_out[0] = d_out;
+  g.split[0] = tc_gemm_split(B, T, d_in, d_out);
   g.NP = NP;
   g.row0 = row0;
   if (!make_input_maps(A, D, g, 0)) return cudaErrorInvalidValue;
@@ -679,9 +785,9 @@ cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d
 }
 
 cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
-                                    float* const* out, const int* d_in, const int* d_out,
-                                    const uint64_t* p_base, const float* c, int B, int T,
-                                    const Epilogue& ep, int* err, cudaStream_t s) {
+                                    float* const* out, float* const* part, const int* d_in,
+                                    const int* d_out, const uint64_t* p_base, const float* c,
+                                    int B, int T, const Epilogue& ep, int* err, cudaStream_t s) {
   if (L < 1 || L > kGemmMaxLayers) return cudaErrorInvalidValue;
   const bool pair = use_pair(d_in[0]);
   GemmArgs g{};
@@ -691,22 +797,49 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
   g.B = B;
   g.T = T;
   set_epilogue(g, ep);
+  SplitReduceBatch r{};
+  int64_t threads = 0;
   for (int l = 0; l < L; ++l) {
     if (use_pair(d_in[l]) != pair) return cudaErrorInvalidValue;  // caller groups by tile shape
     g.d_in[l] = d_in[l];
     g.d_out[l] = d_out[l];
     g.out[l] = out[l];
     g.p_base[l] = p_base[l];
-    if (!make_input_maps(A[l], D[l], g, l) || !make_tma_f32_out(&g.mapO[l], out[l], d_in[l], d_out[l]))
+    g.split[l] = tc_gemm_split(B, T, d_in[l], d_out[l]);
+    if (!make_input_maps(A[l], D[l], g, l)) return cudaErrorInvalidValue;
+    if (g.split[l] > 1) {
+      if (!part || !part[l] || (reinterpret_cast<uintptr_t>(part[l]) & 15) != 0 ||
+          !make_tma_f32_split(&g.mapO[l], part[l], g.split[l], d_in[l], d_out[l]))
+        return cudaErrorInvalidValue;
+      SplitReduceLayer& R = r.l[r.L++];
+      R.part = part[l];
+      R.out = out[l];
+      R.count = static_cast<int64_t>(d_in[l]) * d_out[l];
+      R.p_base = p_base[l];
+      R.q0 = threads;
+      R.split = g.split[l];
+      threads += R.count / 4;
+    } else if (!make_tma_f32_out(&g.mapO[l], out[l], d_in[l], d_out[l])) {
       return cudaErrorInvalidValue;
+    }
   }
-  return launch_any<false>(g, s);
+  cudaError_t e = launch_any<false>(g, s);
+  if (e != cudaSuccess || r.L == 0) return e;
+  r.key = ep.key;
+  r.out_scale = ep.out_scale;
+  r.sigmaC = ep.sigmaC;
+  r.add_noise = ep.add_noise;
+  r.accumulate = ep.accumulate;
+  note_launch();
+  k_split_reduce<<<static_cast<int>((threads + 255) / 256), 256, 0, s>>>(r);
+  return cudaGetLastError();
 }
 
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
-                              int d_in, int d_out, float* out, const Epilogue& ep, int* err,
-                              cudaStream_t s) {
-  return tc_launch_clipsum_batch(1, &A, &D, &out, &d_in, &d_out, &ep.p_base, c, B, T, ep, err, s);
+                              int d_in, int d_out, float* out, float* part, const Epilogue& ep,
+                              int* err, cudaStream_t s) {
+  return tc_launch_clipsum_batch(1, &A, &D, &out, &part, &d_in, &d_out, &ep.p_base, c, B, T, ep,
+                                 err, s);
 }
 
 bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_in_b) {

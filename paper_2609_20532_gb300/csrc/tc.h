@@ -24,19 +24,25 @@ cudaError_t tc_launch_ghost_batch(int L, const void* const* A, const void* const
 // per-example norm that shares its main loop.  One clipped-sum launch can
 // serve up to kGemmMaxLayers layers whose tiles have the same shape
 // (tc_clipsum_same_launch).
+// A layer with few tiles splits its examples into tc_gemm_split ranges: the
+// clipped sum then writes one partial per range into the caller's scratch
+// (split * d_in * d_out fp32, 16-byte aligned) and a reduce pass adds them in
+// order with the noise; the materialised norm needs no scratch.
 constexpr int kGemmMaxLayers = 8;
+constexpr int kGemmMaxSplit = 32;
+int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out);
 bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_in_b);
 cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
-                                    float* const* out, const int* d_in, const int* d_out,
-                                    const uint64_t* p_base, const float* c, int B, int T,
-                                    const Epilogue& ep, int* err, cudaStream_t s);
+                                    float* const* out, float* const* part, const int* d_in,
+                                    const int* d_out, const uint64_t* p_base, const float* c,
+                                    int B, int T, const Epilogue& ep, int* err, cudaStream_t s);
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out);
 int tc_mat_parts(int64_t d_in, int64_t d_out);
 cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d_in, int d_out,
                                float* part, int NP, int row0, int* err, cudaStream_t s);
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
-                              int d_in, int d_out, float* out, const Epilogue& ep, int* err,
-                              cudaStream_t s);
+                              int d_in, int d_out, float* out, float* part, const Epilogue& ep,
+                              int* err, cudaStream_t s);
 
 // Clipped sum for short examples (T < 32): c_i folded into a bf16 hi+lo
 // split of A in scratch (tc_prescaled_scratch_bytes), then one plain GEMM.
@@ -55,6 +61,8 @@ bool make_tma_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* d
                    const uint64_t* strides_bytes, const uint32_t* box);
 // fp32 output map over [rows][cols], box 32 x 32 (128-byte rows), 128-byte swizzle.
 bool make_tma_f32_out(CUtensorMap* m, void* base, uint64_t rows, uint64_t cols);
+// fp32 map over [split][rows][cols] partial sums, box 32 x 32 x 1, 128-byte swizzle.
+bool make_tma_f32_split(CUtensorMap* m, void* base, int split, uint64_t rows, uint64_t cols);
 int device_sm_count();
 
 }  // namespace dpk

@@ -67,6 +67,18 @@ bool make_tma_f32_out(CUtensorMap* m, void* base, uint64_t rows, uint64_t cols) 
             CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool make_tma_f32_split(CUtensorMap* m, void* base, int split, uint64_t rows, uint64_t cols) {
+  auto fn = encode_fn();
+  if (!fn || split < 1) return false;
+  cuuint64_t d[3] = {cols, rows, static_cast<cuuint64_t>(split)};
+  cuuint64_t st[2] = {cols * 4, rows * cols * 4};
+  cuuint32_t b[3] = {32, 32, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, d, st, b, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int device_sm_count() {
   int dev = 0, n = 0;
   cudaGetDevice(&dev);

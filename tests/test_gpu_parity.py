@@ -623,6 +623,80 @@ def test_cuda_graph_replay_matches_eager_steps():
         dp.dp_step_destroy(ctx)
 
 
+SPLIT_CASES = [
+    # (layers, B, T): tensor-core layers with few output tiles and many
+    # examples, so each tile's examples are split into ranges and reduced
+    ([(256, 64)], 64, 256),                 # one CTA-pair tile, 32 ranges
+    ([(576, 64), (1152, 128)], 48, 100),    # conv-like widths, T % 64 != 0, 12 ranges
+]
+
+
+@pytest.mark.parametrize("mode", [dp.DP_NORM_AUTO, dp.DP_NORM_MATERIALISED])
+@pytest.mark.parametrize("case", range(len(SPLIT_CASES)))
+def test_split_batch_tensor_core_layers(case, mode):
+    """Few tiles, many examples: the clipped sum splits each tile's examples
+    into ranges, stores their partial sums and adds them in order with the
+    noise (a second launch); the materialised norm splits the same way."""
+    shapes, B, T = SPLIT_CASES[case]
+    w = W.custom(f"split{case}", shapes, B, T, "bf16", C=0.2, sigma=0.6, d_std=0.1,
+                 wid=880 + case)
+    assert not any(is_thin(i, o, T, "bf16") for i, o in shapes)
+    layers = W.make_inputs(w)
+    res = run_gpu_step(w, layers, seed=8, step=3, out_scale=1.0 / B, norm_mode=mode)
+    assert all(sum_tc == 1 for _, sum_tc in res["paths"])
+    ref = oracle_step(w, layers, seed=8, step=3, out_scale=1.0 / B)
+    assert_step_matches(res, ref, "bf16")
+    # the split path runs (GEMM + reduce) and DP_ACCUMULATE adds exactly
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    cfg = dp.make_config(w.layers, B, T, "bf16", w.C, w.sigma, out_scale=1.0 / B,
+                         norm_mode=mode)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.dp_layer_norms_batch(ctx, list(range(len(shapes))), Ad, Dd)
+        dp.dp_clip_factors(ctx)
+        once = torch.zeros(shapes[0], device=dev)
+        twice = torch.zeros(shapes[0], device=dev)
+        n0 = dp.dp_kernel_launches()
+        dp.dp_clipped_sum_noise(ctx, 0, Ad[0], Dd[0], once, dp.DP_NO_NOISE)
+        assert dp.dp_kernel_launches() - n0 == 2
+        for _ in range(2):
+            dp.dp_clipped_sum_noise(ctx, 0, Ad[0], Dd[0], twice, dp.DP_NO_NOISE | dp.DP_ACCUMULATE)
+        torch.cuda.synchronize()
+        assert torch.equal(twice, 2 * once)
+    finally:
+        dp.dp_step_destroy(ctx)
+
+
+ODD_BASE_CASES = [
+    # (layers, B, T): a tensor-core layer whose first global parameter index
+    # is not a multiple of 4, so its noise groups straddle two Philox quads
+    ([(1, 3), (264, 136)], 6, 64),      # direct tiles, p_base = 3
+    ([(1, 5), (256, 64)], 64, 256),     # split ranges + reduce, p_base = 5
+    ([(1, 3), (256, 256)], 16, 8),      # pre-scaled operand (T < 32), p_base = 3
+]
+
+
+@pytest.mark.parametrize("case", range(len(ODD_BASE_CASES)))
+def test_tensor_core_layer_after_odd_sized_layer(case):
+    shapes, B, T = ODD_BASE_CASES[case]
+    w = W.custom(f"oddbase{case}", shapes, B, T, "bf16", C=0.3, sigma=0.9, d_std=0.1,
+                 wid=890 + case, a_dist=("ones", "normal"))
+    layers = W.make_inputs(w)
+    res = run_gpu_step(w, layers, seed=9, step=7, out_scale=1.0 / B)
+    assert res["paths"][1][1] == 1 and is_thin(*shapes[0], T, "bf16")
+    ref = oracle_step(w, layers, seed=9, step=7, out_scale=1.0 / B)
+    assert_step_matches(res, ref, "bf16")
+    # the noise part alone equals the oracle's noise to 1e-6
+    noiseless = run_gpu_step(w, layers, seed=9, step=7, out_scale=1.0 / B, flags=dp.DP_NO_NOISE,
+                             audit=False)
+    z = O.gaussian_noise(9, 7, 0, sum(i * o for i, o in shapes))
+    got = np.concatenate([(a - b).ravel() for a, b in zip(res["out"], noiseless["out"])])
+    want = z * (float(np.float32(w.C)) * float(np.float32(w.sigma)) / B)
+    assert np.max(np.abs(got - want)) <= 1e-5 * np.max(np.abs(want))
+
+
 def test_launch_counts_of_a_step():
     """The library's own launch count: 33 thin layers of one width bucket and
     T take two norm launches and two clipped-sum launches (32 layers per
