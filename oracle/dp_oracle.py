@@ -24,6 +24,10 @@ What is computed (paper: Sec. 2.2 "DP-SGD", and the GPU loop of Algorithm 2):
 * output ``out_l = out_scale * (S_l + sigma*C*z_l)``; ``out_scale = 1/B`` is the
   paper's average ``(1/|B_t|)(sum + z)`` of Sec. 2.2, ``out_scale = 1`` the
   plain sum;
+* per-example weight gradients of 2-D convolutions (the CIFAR-10 WideResNet
+  of App. B) from the definition of the convolution, and the patch rows
+  (unfold) that turn a convolution into the dense form above; the step on
+  per-example gradients given directly (:func:`dp_step_from_grads`);
 * audit records (example, per-layer squared norms, total, clip factor) for a
   caller-chosen subset of examples, the material a CPU checker recomputes when
   it partially re-executes a step (Sec. 7, "recomputes, or partially
@@ -57,6 +61,13 @@ Pins (tests/test_oracle_pins.py, all ``-m "not gpu"``):
   b1 = b2 = 0 special cases where the step is lr (g/(|g| + eps) + wd theta)
   (tests/golden/adamw_hand.json, worked by hand); g = 0 leaves theta
   changed by weight decay only.
+* conv2d_weight_grads: a pure-Python six-fold loop on tiny inputs; PyTorch's
+  independent ``torch.nn.grad.conv2d_weight`` per example (NCHW, strides and
+  padding); a 1x1 stride-1 convolution is the dense layer on the pixels.
+* conv2d_unfold: ``torch.nn.functional.unfold`` with its (c, ki, kj) column
+  order permuted; hand-placed values including the zero padding; its dense
+  product equals conv2d_weight_grads.
+* dp_step_from_grads: equals dp_step on dense layers.
 * gaussian_noise: sample mean / variance / Kolmogorov-Smirnov against
   N(0, 1); per-coordinate std of the averaged noise against the sigma*C/B
   column printed in the paper's attack-parameter table (App. B.1).
@@ -83,6 +94,10 @@ __all__ = [
     "sincospi",
     "gaussian_noise",
     "dp_step",
+    "dp_step_from_grads",
+    "conv2d_out_hw",
+    "conv2d_weight_grads",
+    "conv2d_unfold",
     "audit_records",
     "adamw_step",
     "noise_adamw",
@@ -356,6 +371,107 @@ def dp_step(layers, C: float, sigma: float, seed: int, step: int,
         out.append(out_scale * o)
         offset += S.size
     return {"n": n, "s": s, "c": c, "S": S_list, "out": out}
+
+
+def dp_step_from_grads(grads, C: float, sigma: float, seed: int, step: int,
+                       out_scale: float = 1.0, noise: bool = True):
+    """The same step on per-example gradients given directly.
+
+    grads: sequence of [B, ...] arrays, one per layer (any layer kind whose
+    per-example gradient is known, e.g. :func:`conv2d_weight_grads`); each
+    layer's parameters are its trailing dimensions in C order, which fixes
+    their global noise indices.  n_{l,i} = ||G_{l,i}||^2, then clip, clipped
+    sum and noise exactly as :func:`dp_step` (Sec. 2.2, Algorithm 2).
+    """
+    grads = [_as_f64(G) for G in grads]
+    B = grads[0].shape[0]
+    if any(G.shape[0] != B for G in grads):
+        raise ValueError("every layer needs the same B")
+    n = np.stack([np.sum(G.reshape(B, -1) ** 2, axis=1) for G in grads])
+    s, c = clip_factors(n, C)
+    S_list, out = [], []
+    offset = 0
+    for G in grads:
+        S = np.tensordot(c, G, axes=(0, 0))
+        S_list.append(S)
+        o = S.copy()
+        if noise:
+            z = gaussian_noise(seed, step, offset, S.size).reshape(S.shape)
+            o = o + sigma * C * z
+        out.append(out_scale * o)
+        offset += S.size
+    return {"n": n, "s": s, "c": c, "S": S_list, "out": out}
+
+
+# ---------------------------------------------------------------------------
+# 2-D convolution layers (the CIFAR-10 WideResNet of App. B)
+# ---------------------------------------------------------------------------
+# A convolution without bias, NHWC activations x [H, W, C_in] and weight
+# W [kh, kw, C_in, C_out]:
+#   y[h, w, o] = sum_{ki, kj, c} xp[h*sh + ki, w*sw + kj, c] * W[ki, kj, c, o]
+# where xp is x with pad rows / columns of zeros on every side.  Its weight
+# gradient for one example is the sum over output positions of the input
+# patch times the output gradient.
+
+def conv2d_out_hw(H: int, W: int, kh: int, kw: int, stride=(1, 1), pad=(0, 0)):
+    """(H_out, W_out) of the convolution above."""
+    sh, sw = stride
+    ph, pw = pad
+    Ho = (H + 2 * ph - kh) // sh + 1
+    Wo = (W + 2 * pw - kw) // sw + 1
+    if Ho < 1 or Wo < 1:
+        raise ValueError("kernel larger than the padded input")
+    return Ho, Wo
+
+
+def _padded(X, pad):
+    ph, pw = pad
+    return np.pad(X, ((0, 0), (ph, ph), (pw, pw), (0, 0)))
+
+
+def conv2d_weight_grads(X, Dy, kh: int, kw: int, stride=(1, 1), pad=(0, 0)) -> np.ndarray:
+    """Per-example weight gradients G_i[ki, kj, c, o] = sum_{h, w}
+    xp_i[h*sh + ki, w*sw + kj, c] * dy_i[h, w, o].
+
+    X: [B, H, W, C_in], Dy: [B, H_out, W_out, C_out] -> [B, kh, kw, C_in, C_out].
+    One contraction per kernel tap (ki, kj) over the output positions.
+    """
+    X = _as_f64(X)
+    Dy = _as_f64(Dy)
+    B, H, W_, Cin = X.shape
+    Ho, Wo = conv2d_out_hw(H, W_, kh, kw, stride, pad)
+    if Dy.shape[:3] != (B, Ho, Wo):
+        raise ValueError("Dy must be [B, H_out, W_out, C_out]")
+    sh, sw = stride
+    Xp = _padded(X, pad)
+    G = np.zeros((B, kh, kw, Cin, Dy.shape[3]))
+    for ki in range(kh):
+        for kj in range(kw):
+            tap = Xp[:, ki:ki + sh * (Ho - 1) + 1:sh, kj:kj + sw * (Wo - 1) + 1:sw, :]
+            G[:, ki, kj] = np.einsum("bhwc,bhwo->bco", tap, Dy)
+    return G
+
+
+def conv2d_unfold(X, kh: int, kw: int, stride=(1, 1), pad=(0, 0)) -> np.ndarray:
+    """Input patches as rows: A[i, h*W_out + w, (ki*kw + kj)*C_in + c] =
+    xp_i[h*sh + ki, w*sw + kj, c]  ->  [B, H_out*W_out, kh*kw*C_in].
+
+    With it a convolution's weight gradient is the dense A_i^T D_i of
+    :func:`per_example_grads` with D_i = dy_i as [H_out*W_out, C_out], laid out
+    [(ki, kj, c), o].  The values are copies of inputs and zeros, so the
+    result is exact in any precision.
+    """
+    X = np.asarray(X)
+    B, H, W_, Cin = X.shape
+    Ho, Wo = conv2d_out_hw(H, W_, kh, kw, stride, pad)
+    sh, sw = stride
+    Xp = _padded(X, pad)
+    A = np.empty((B, Ho, Wo, kh, kw, Cin), dtype=X.dtype)
+    for ki in range(kh):
+        for kj in range(kw):
+            A[:, :, :, ki, kj, :] = Xp[:, ki:ki + sh * (Ho - 1) + 1:sh,
+                                       kj:kj + sw * (Wo - 1) + 1:sw, :]
+    return A.reshape(B, Ho * Wo, kh * kw * Cin)
 
 
 def audit_records(n, s, c, idx):

@@ -537,3 +537,167 @@ def test_planted_adamw_mistakes_are_caught():
     assert not check_adamw_golden(no_bias_correction)
     assert not check_adamw_golden(coupled_decay)
     assert not check_adamw_golden(eps_inside_sqrt)
+
+
+# ---------------------------------------------------------------------------
+# 2-D convolutions (CIFAR-10 WideResNet of App. B)
+# ---------------------------------------------------------------------------
+
+CONV_GEOMS = [
+    # (B, H, W, C_in, C_out, kh, kw, stride, pad)
+    (2, 5, 6, 3, 4, 3, 3, (1, 1), (1, 1)),
+    (2, 7, 5, 2, 3, 3, 3, (2, 2), (1, 1)),
+    (1, 6, 6, 4, 2, 1, 1, (2, 2), (0, 0)),
+    (2, 4, 5, 2, 3, 2, 3, (1, 2), (0, 1)),
+]
+
+
+def _conv_inputs(geom, seed=0):
+    B, H, W_, Cin, Cout, kh, kw, st, pd = geom
+    Ho, Wo = O.conv2d_out_hw(H, W_, kh, kw, st, pd)
+    r = np.random.default_rng(seed)
+    return r.standard_normal((B, H, W_, Cin)), r.standard_normal((B, Ho, Wo, Cout))
+
+
+def brute_force_conv_grads(X, Dy, kh, kw, stride, pad):
+    """Pure-Python loops over examples, taps, channels and output positions,
+    reading padded positions as zero."""
+    B, H, W_, Cin = X.shape
+    _, Ho, Wo, Cout = Dy.shape
+    Xl, Dl = X.tolist(), Dy.tolist()
+    G = [[[[[0.0] * Cout for _ in range(Cin)] for _ in range(kw)] for _ in range(kh)]
+         for _ in range(B)]
+    for i in range(B):
+        for ki in range(kh):
+            for kj in range(kw):
+                for h in range(Ho):
+                    for w in range(Wo):
+                        y = h * stride[0] + ki - pad[0]
+                        x = w * stride[1] + kj - pad[1]
+                        if not (0 <= y < H and 0 <= x < W_):
+                            continue
+                        for c in range(Cin):
+                            a = Xl[i][y][x][c]
+                            for o in range(Cout):
+                                G[i][ki][kj][c][o] += a * Dl[i][h][w][o]
+    return np.array(G)
+
+
+def check_conv_grads(fn):
+    """fn(X, Dy, kh, kw, stride, pad) against brute force and PyTorch's own
+    weight-gradient routine, one example at a time."""
+    import torch
+    for g in CONV_GEOMS:
+        B, H, W_, Cin, Cout, kh, kw, st, pd = g
+        X, Dy = _conv_inputs(g, seed=B + H)
+        G = fn(X, Dy, kh, kw, st, pd)
+        if G.shape != (B, kh, kw, Cin, Cout):
+            return False
+        if not np.allclose(G, brute_force_conv_grads(X, Dy, kh, kw, st, pd), rtol=1e-12, atol=1e-12):
+            return False
+        for i in range(B):
+            x = torch.from_numpy(X[i:i + 1]).permute(0, 3, 1, 2)
+            dy = torch.from_numpy(Dy[i:i + 1]).permute(0, 3, 1, 2)
+            gw = torch.nn.grad.conv2d_weight(x, (Cout, Cin, kh, kw), dy, stride=st, padding=pd)
+            if not np.allclose(G[i], gw.permute(2, 3, 1, 0).numpy(), rtol=1e-10, atol=1e-10):
+                return False
+    return True
+
+
+def check_unfold(fn):
+    """fn(X, kh, kw, stride, pad) against torch.nn.functional.unfold (columns
+    (c, ki, kj), permuted to (ki, kj, c)) and hand-placed values."""
+    import torch
+    for g in CONV_GEOMS:
+        B, H, W_, Cin, Cout, kh, kw, st, pd = g
+        X, _ = _conv_inputs(g, seed=3)
+        A = fn(X, kh, kw, st, pd)
+        Ho, Wo = O.conv2d_out_hw(H, W_, kh, kw, st, pd)
+        u = torch.nn.functional.unfold(torch.from_numpy(X).permute(0, 3, 1, 2), (kh, kw),
+                                       padding=pd, stride=st)          # [B, C*kh*kw, L]
+        u = u.reshape(B, Cin, kh, kw, Ho * Wo).permute(0, 4, 2, 3, 1).reshape(B, Ho * Wo, -1)
+        if A.shape != u.shape or not np.array_equal(A, u.numpy()):
+            return False
+    # hand-placed: X[0, y, x, c] = 100 y + 10 x + c on a 3x3x2 image, 3x3
+    # kernel, pad 1: output position (0, 0) reads rows -1..1 and columns -1..1
+    X = np.array([[[[100 * y + 10 * x + c for c in range(2)] for x in range(3)] for y in range(3)]],
+                 dtype=np.float64)
+    A = fn(X, 3, 3, (1, 1), (1, 1))
+    row = A[0, 0].reshape(3, 3, 2)
+    want = np.zeros((3, 3, 2))
+    for ki in range(3):
+        for kj in range(3):
+            y, x = ki - 1, kj - 1
+            if 0 <= y < 3 and 0 <= x < 3:
+                want[ki, kj] = [100 * y + 10 * x, 100 * y + 10 * x + 1]
+    return bool(np.array_equal(row, want) and A[0, 4].reshape(3, 3, 2)[1, 1, 1] == 111)
+
+
+def test_conv2d_weight_grads_pins():
+    assert check_conv_grads(O.conv2d_weight_grads)
+
+
+def test_conv2d_unfold_pins():
+    assert check_unfold(O.conv2d_unfold)
+
+
+def test_unfold_product_is_the_conv_gradient():
+    for g in CONV_GEOMS:
+        B, H, W_, Cin, Cout, kh, kw, st, pd = g
+        X, Dy = _conv_inputs(g, seed=7)
+        A = O.conv2d_unfold(X, kh, kw, st, pd)
+        G = O.per_example_grads(A, Dy.reshape(B, -1, Cout))
+        np.testing.assert_allclose(G.reshape(B, kh, kw, Cin, Cout),
+                                   O.conv2d_weight_grads(X, Dy, kh, kw, st, pd), rtol=0, atol=1e-12)
+
+
+def test_1x1_conv_is_the_dense_layer_on_pixels():
+    r = np.random.default_rng(11)
+    X, Dy = r.standard_normal((3, 4, 5, 6)), r.standard_normal((3, 4, 5, 7))
+    G = O.conv2d_weight_grads(X, Dy, 1, 1)
+    np.testing.assert_allclose(G[:, 0, 0], O.per_example_grads(X.reshape(3, 20, 6), Dy.reshape(3, 20, 7)),
+                               rtol=0, atol=1e-12)
+
+
+def test_step_from_grads_equals_dense_step():
+    r = np.random.default_rng(12)
+    layers = [(r.standard_normal((5, 4, 6)), r.standard_normal((5, 4, 3))),
+              (r.standard_normal((5, 4, 3)), 0.1 * r.standard_normal((5, 4, 2)))]
+    a = O.dp_step(layers, 0.7, 1.3, seed=5, step=2, out_scale=0.2)
+    b = O.dp_step_from_grads([O.per_example_grads(A, D) for A, D in layers], 0.7, 1.3, seed=5,
+                             step=2, out_scale=0.2)
+    for k in ("n", "s", "c"):
+        np.testing.assert_allclose(a[k], b[k], rtol=1e-13, atol=0)
+    for x, y in zip(a["out"], b["out"]):
+        np.testing.assert_allclose(x, y, rtol=1e-12, atol=1e-15)
+
+
+def test_planted_conv_mistakes_are_caught():
+    # a true convolution (kernel flipped) instead of the cross-correlation
+    def flipped(X, Dy, kh, kw, st, pd):
+        return O.conv2d_weight_grads(X, Dy, kh, kw, st, pd)[:, ::-1, ::-1]
+    assert not check_conv_grads(flipped)
+
+    # stride ignored in the input taps
+    def no_stride(X, Dy, kh, kw, st, pd):
+        Xp = np.pad(X, ((0, 0), (pd[0], pd[0]), (pd[1], pd[1]), (0, 0)))
+        Ho, Wo = Dy.shape[1:3]
+        G = np.zeros((X.shape[0], kh, kw, X.shape[3], Dy.shape[3]))
+        for ki in range(kh):
+            for kj in range(kw):
+                G[:, ki, kj] = np.einsum("bhwc,bhwo->bco", Xp[:, ki:ki + Ho, kj:kj + Wo], Dy)
+        return G
+    assert not check_conv_grads(no_stride)
+
+    # padding applied on one side only
+    def one_side(X, Dy, kh, kw, st, pd):
+        Xs = np.pad(X, ((0, 0), (2 * pd[0], 0), (2 * pd[1], 0), (0, 0)))
+        return O.conv2d_weight_grads(Xs, Dy, kh, kw, st, (0, 0))
+    assert not check_conv_grads(one_side)
+
+    # unfold columns in (c, ki, kj) order
+    def unfold_c_major(X, kh, kw, st, pd):
+        A = O.conv2d_unfold(X, kh, kw, st, pd)
+        B, T, K = A.shape
+        return A.reshape(B, T, kh, kw, -1).transpose(0, 1, 4, 2, 3).reshape(B, T, K)
+    assert not check_unfold(unfold_c_major)
