@@ -302,6 +302,44 @@ const char* dp_last_error(void);
 /* Name of a status code. */
 const char* dp_status_string(dp_status s);
 
+/* ---- 2-D convolutions (the CIFAR-10 WideResNet of App. B) ---------------
+ * A convolution without bias over NHWC activations (a cross-correlation):
+ *   y[h][w][o] = sum_{ki, kj, c} xp[h*stride_h + ki][w*stride_w + kj][c] * W[ki][kj][c][o]
+ * where xp is the input with pad_h rows and pad_w columns of zeros on each
+ * side.  Its per-example weight gradient sum_{h,w} patch(h,w)^T dy[h][w] is
+ * the dense A_i^T D_i of a layer {d_in = K, d_out = C_out, T} with
+ *   T = H_out * W_out, H_out = (H + 2 pad_h - kh) / stride_h + 1 (W_out alike),
+ *   K = kh * kw * C_in,
+ *   A_i[h*W_out + w][(ki*kw + kj)*C_in + c] = xp_i[h*stride_h + ki][w*stride_w + kj][c]
+ *     (the patch rows dp_conv2d_unfold writes),
+ *   D_i = dy_i [H_out][W_out][C_out] read as [T][C_out],
+ * so the layer's output is laid out [kh][kw][C_in][C_out] (HWIO), row-major.
+ * A convolution enters a step as that dense layer: unfold, then pass the
+ * patch rows as its A to dp_layer_norms and dp_clipped_sum_noise.          */
+typedef struct {
+    int32_t H, W;                /* input height and width, >= 1 */
+    int32_t C_in;                /* input channels, >= 1 */
+    int32_t kh, kw;              /* kernel height and width, >= 1 */
+    int32_t stride_h, stride_w;  /* >= 1 */
+    int32_t pad_h, pad_w;        /* zero rows / columns on each side, >= 0 */
+} dp_conv2d;
+
+/* T = H_out * W_out and K = kh * kw * C_in of a convolution (host only).
+ * Errors: DP_ERR_ARG (NULL argument), DP_ERR_SHAPE (a size < 1 or pad < 0,
+ * a kernel larger than the padded input, T above 2^31 - 1, K above 2^20). */
+dp_status dp_conv2d_dims(const dp_conv2d* conv, int32_t* T_out, int64_t* K_out);
+
+/* Patch rows of B examples: x [B][H][W][C_in] -> a_out [B][T][K], both of
+ * element type dtype, device arrays owned by the caller, 16-byte aligned and
+ * not overlapping.  Values are copied and padding positions written as zero,
+ * so the result is exact.  Asynchronous on stream (a cudaStream_t; NULL = the
+ * legacy default stream); no context is needed.
+ * Errors: DP_ERR_ARG (NULL, misaligned or overlapping arrays, B < 1),
+ * DP_ERR_SHAPE (as dp_conv2d_dims, or B * T above 2^31 - 1), DP_ERR_DTYPE,
+ * DP_ERR_CUDA. */
+dp_status dp_conv2d_unfold(const dp_conv2d* conv, int32_t B, dp_dtype dtype, const void* x,
+                           void* a_out, void* stream);
+
 /* Number of CUDA kernels this library has issued in this process, counted on
  * the host as each launch is made, by every call above and the test exports
  * below (dp_layer_sqnorms_noalloc is not counted).  A launch made while the

@@ -28,7 +28,8 @@ __all__ = [
     "dp_audit_emit", "audit_dtype", "dp_audit_record_bytes", "dp_layer_norm_mode", "dp_layer_path",
     "dp_set_noise_key", "dp_step_destroy",
     "dp_last_error", "dp_kernel_launches", "dp_debug_philox", "dp_debug_gaussian",
-    "dp_layer_sqnorms_noalloc", "EXPORTED_SYMBOLS",
+    "dp_layer_sqnorms_noalloc", "dp_conv2d", "make_conv", "dp_conv2d_dims", "dp_conv2d_unfold",
+    "EXPORTED_SYMBOLS",
 ]
 
 HERE = os.path.dirname(os.path.abspath(__file__))
@@ -48,7 +49,8 @@ EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "d
                     "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
                     "dp_audit_emit", "dp_audit_record_bytes", "dp_layer_norm_mode",
                     "dp_layer_path", "dp_set_noise_key", "dp_step_destroy", "dp_last_error",
-                    "dp_status_string", "dp_kernel_launches",
+                    "dp_status_string", "dp_kernel_launches", "dp_conv2d_dims",
+                    "dp_conv2d_unfold",
                     "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
                     "dp_noise_adamw"]
 
@@ -67,6 +69,12 @@ class LibraryNotBuilt(ImportError):
 class dp_layer(ctypes.Structure):
     _fields_ = [("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64), ("T", ctypes.c_int32),
                 ("reserved", ctypes.c_int32)]
+
+
+class dp_conv2d(ctypes.Structure):
+    _fields_ = [("H", ctypes.c_int32), ("W", ctypes.c_int32), ("C_in", ctypes.c_int32),
+                ("kh", ctypes.c_int32), ("kw", ctypes.c_int32), ("stride_h", ctypes.c_int32),
+                ("stride_w", ctypes.c_int32), ("pad_h", ctypes.c_int32), ("pad_w", ctypes.c_int32)]
 
 
 class dp_adamw(ctypes.Structure):
@@ -114,6 +122,8 @@ def lib() -> ctypes.CDLL:
         "dp_last_error": ([], ctypes.c_char_p),
         "dp_status_string": ([i32], ctypes.c_char_p),
         "dp_kernel_launches": ([ctypes.POINTER(i64)], i32),
+        "dp_conv2d_dims": ([ctypes.POINTER(dp_conv2d), ctypes.POINTER(i32), ctypes.POINTER(i64)], i32),
+        "dp_conv2d_unfold": ([ctypes.POINTER(dp_conv2d), i32, i32, vp, vp, vp], i32),
         "dp_debug_philox": ([u64, u64, u64, i64, vp, vp], i32),
         "dp_debug_gaussian": ([u64, u64, u64, i64, vp, vp], i32),
         "dp_layer_sqnorms_noalloc": ([vp, vp, i32, i32, i64, i64, i32, vp, vp], i32),
@@ -269,6 +279,24 @@ def dp_debug_philox(seed: int, step: int, first_quad: int, n_quads: int, out, st
 def dp_debug_gaussian(seed: int, step: int, first_index: int, n: int, out, stream=None):
     _check(lib().dp_debug_gaussian(seed & (2 ** 64 - 1), step & (2 ** 64 - 1),
                                    first_index & (2 ** 64 - 1), n, _ptr(out), _stream(stream)))
+
+
+def make_conv(H: int, W: int, C_in: int, kh: int, kw: int, stride=(1, 1), pad=(0, 0)) -> dp_conv2d:
+    return dp_conv2d(H=H, W=W, C_in=C_in, kh=kh, kw=kw, stride_h=stride[0], stride_w=stride[1],
+                     pad_h=pad[0], pad_w=pad[1])
+
+
+def dp_conv2d_dims(conv: dp_conv2d):
+    """(T, K) of a convolution: T = H_out * W_out, K = kh * kw * C_in."""
+    T, K = ctypes.c_int32(0), ctypes.c_int64(0)
+    _check(lib().dp_conv2d_dims(ctypes.byref(conv), ctypes.byref(T), ctypes.byref(K)))
+    return T.value, K.value
+
+
+def dp_conv2d_unfold(conv: dp_conv2d, B: int, dtype: str, x, a_out, stream=None) -> None:
+    """Patch rows a_out [B][T][K] of the NHWC input x [B][H][W][C_in]."""
+    _check(lib().dp_conv2d_unfold(ctypes.byref(conv), B, DP_BF16 if dtype == "bf16" else DP_F32,
+                                  _ptr(x), _ptr(a_out), _stream(stream)))
 
 
 def dp_layer_sqnorms_noalloc(A, D, B: int, T: int, d_in: int, d_out: int, dtype: str, out,

@@ -38,6 +38,8 @@ dp_status fail(dp_status st, const char* fmt, ...) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+constexpr int64_t kMaxDim = 1 << 20;  // largest d_in, d_out (and convolution K)
+
 }  // namespace
 
 namespace dpk {
@@ -114,7 +116,7 @@ dp_status check_config(const dp_config* cfg) {
   if (cfg->dtype != DP_F32 && cfg->dtype != DP_BF16) return fail(DP_ERR_DTYPE, "unknown dtype");
   for (int l = 0; l < cfg->n_layers; ++l) {
     const dp_layer& ly = cfg->layers[l];
-    if (ly.d_in < 1 || ly.d_out < 1 || ly.d_in > (1 << 20) || ly.d_out > (1 << 20))
+    if (ly.d_in < 1 || ly.d_out < 1 || ly.d_in > kMaxDim || ly.d_out > kMaxDim)
       return fail(DP_ERR_SHAPE, "layer %d: d_in, d_out must be in 1..2^20", l);
     if (ly.T < 0 || ly.reserved != 0)
       return fail(DP_ERR_ARG, "layer %d: T must be >= 0 (0 = config T), reserved must be 0", l);
@@ -854,6 +856,57 @@ const char* dp_status_string(dp_status s) {
     case DP_ERR_UNSUPPORTED: return "DP_ERR_UNSUPPORTED";
   }
   return "DP_ERR_UNKNOWN";
+}
+
+namespace {
+dp_status conv_geom(const dp_conv2d* v, dpk::ConvGeom* g) {
+  if (!v) return fail(DP_ERR_ARG, "conv is NULL");
+  if (v->H < 1 || v->W < 1 || v->C_in < 1 || v->kh < 1 || v->kw < 1 || v->stride_h < 1 ||
+      v->stride_w < 1 || v->pad_h < 0 || v->pad_w < 0)
+    return fail(DP_ERR_SHAPE, "convolution sizes must be >= 1 and pads >= 0");
+  const int64_t hp = static_cast<int64_t>(v->H) + 2 * static_cast<int64_t>(v->pad_h);
+  const int64_t wp = static_cast<int64_t>(v->W) + 2 * static_cast<int64_t>(v->pad_w);
+  if (v->kh > hp || v->kw > wp) return fail(DP_ERR_SHAPE, "kernel larger than the padded input");
+  const int64_t ho = (hp - v->kh) / v->stride_h + 1, wo = (wp - v->kw) / v->stride_w + 1;
+  const int64_t K = static_cast<int64_t>(v->kh) * v->kw * v->C_in;
+  if (ho * wo > 0x7fffffffLL) return fail(DP_ERR_SHAPE, "H_out * W_out above 2^31 - 1");
+  if (K > kMaxDim) return fail(DP_ERR_SHAPE, "kh * kw * C_in above 2^20");
+  *g = dpk::ConvGeom{v->H, v->W, v->C_in, v->kh, v->kw, v->stride_h, v->stride_w,
+                     v->pad_h, v->pad_w, static_cast<int>(ho), static_cast<int>(wo)};
+  return DP_OK;
+}
+}  // namespace
+
+dp_status dp_conv2d_dims(const dp_conv2d* conv, int32_t* T_out, int64_t* K_out) {
+  if (!T_out || !K_out) return fail(DP_ERR_ARG, "NULL output");
+  dpk::ConvGeom g{};
+  dp_status st = conv_geom(conv, &g);
+  if (st != DP_OK) return st;
+  *T_out = g.H_out * g.W_out;
+  *K_out = static_cast<int64_t>(g.kh) * g.kw * g.C_in;
+  return DP_OK;
+}
+
+dp_status dp_conv2d_unfold(const dp_conv2d* conv, int32_t B, dp_dtype dtype, const void* x,
+                           void* a_out, void* stream) {
+  dpk::ConvGeom g{};
+  dp_status st = conv_geom(conv, &g);
+  if (st != DP_OK) return st;
+  if (B < 1) return fail(DP_ERR_ARG, "B must be >= 1");
+  if (dtype != DP_F32 && dtype != DP_BF16) return fail(DP_ERR_DTYPE, "unknown dtype %d", dtype);
+  if (!x || !a_out) return fail(DP_ERR_ARG, "x or a_out is NULL");
+  if (!aligned16(x) || !aligned16(a_out)) return fail(DP_ERR_ARG, "x and a_out must be 16-byte aligned");
+  if (static_cast<int64_t>(B) * g.H_out * g.W_out > 0x7fffffffLL)
+    return fail(DP_ERR_SHAPE, "B * H_out * W_out above 2^31 - 1");
+  const int64_t elem = dtype == DP_F32 ? 4 : 2;
+  const int64_t xb = static_cast<int64_t>(B) * g.H * g.W * g.C_in * elem;
+  const int64_t ab = static_cast<int64_t>(B) * g.H_out * g.W_out * g.kh * g.kw * g.C_in * elem;
+  const char* xp = static_cast<const char*>(x);
+  const char* ap = static_cast<const char*>(a_out);
+  if (xp < ap + ab && ap < xp + xb) return fail(DP_ERR_ARG, "x and a_out overlap");
+  DP_CUDA(dpk::launch_conv_unfold(dtype == DP_F32 ? dpk::IN_F32 : dpk::IN_BF16, x, a_out, g, B,
+                                  static_cast<cudaStream_t>(stream)));
+  return DP_OK;
 }
 
 dp_status dp_kernel_launches(int64_t* count_out) {

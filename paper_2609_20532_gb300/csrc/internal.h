@@ -108,6 +108,14 @@ cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, int* fl
 cudaError_t launch_set_key(uint64_t seed, uint64_t step, uint64_t* key, int* flag,
                            cudaStream_t s);
 
+// ---- patch rows of a 2-D convolution over NHWC activations (k_conv.cu) ----
+struct ConvGeom {
+  int H, W, C_in, kh, kw, stride_h, stride_w, pad_h, pad_w;
+  int H_out, W_out;
+};
+cudaError_t launch_conv_unfold(InType t, const void* x, void* a, const ConvGeom& g, int B,
+                               cudaStream_t s);
+
 // ---- launch count: every launcher calls note_launch() once per kernel it
 // issues (process-wide, thread-safe), read back by dp_kernel_launches() ----
 void note_launch();

@@ -20,6 +20,50 @@ def f32(x: float) -> float:
     return float(np.float32(x))
 
 
+def conv_struct(w: W.Workload, l: int):
+    """The library's description of layer l's convolution (None if dense)."""
+    cv = w.conv_of(l)
+    if not cv:
+        return None
+    H, W_, cin, kh, kw, st, pd = cv
+    return dp.make_conv(H, W_, cin, kh, kw, (st, st), (pd, pd))
+
+
+def device_inputs(w: W.Workload, layers, dev="cuda:0"):
+    """A and D of every layer on the device; a convolution's A becomes its
+    patch rows through dp_conv2d_unfold (the library's kernel)."""
+    Ad, Dd = [], []
+    for l, (A, D) in enumerate(layers):
+        x = A.to(dev)
+        conv = conv_struct(w, l)
+        if conv is not None:
+            T, K = dp.dp_conv2d_dims(conv)
+            a = torch.empty((w.B, T, K), dtype=x.dtype, device=dev)
+            dp.dp_conv2d_unfold(conv, w.B, w.dtype, x, a)
+            x = a
+        Ad.append(x)
+        Dd.append(D.to(dev))
+    return Ad, Dd
+
+
+def oracle_grads(w: W.Workload, layers):
+    """fp64 per-example gradients of every layer from the oracle: a dense
+    layer's A_i^T D_i, a convolution's from its definition (not through the
+    patch rows), laid out [B, d_in, d_out] as the library's outputs are."""
+    G = []
+    for l, (A, D) in enumerate(layers):
+        cv = w.conv_of(l)
+        if cv:
+            H, W_, cin, kh, kw, st, pd = cv
+            Ho, Wo = O.conv2d_out_hw(H, W_, kh, kw, (st, st), (pd, pd))
+            Dy = W.to_f64(D).reshape(w.B, Ho, Wo, -1)
+            g = O.conv2d_weight_grads(W.to_f64(A), Dy, kh, kw, (st, st), (pd, pd))
+            G.append(g.reshape(w.B, kh * kw * cin, -1))
+        else:
+            G.append(O.per_example_grads(W.to_f64(A), W.to_f64(D)))
+    return G
+
+
 def run_gpu_step(w: W.Workload, layers, seed=0, step=0, out_scale=1.0, flags=0,
                  norm_mode=dp.DP_NORM_AUTO, audit=True):
     """Run norms -> clip -> clipped sum (+noise) on cuda:0.
@@ -28,8 +72,7 @@ def run_gpu_step(w: W.Workload, layers, seed=0, step=0, out_scale=1.0, flags=0,
     (from the audit records of every example), out (list of fp32 numpy) and
     the chosen norm modes."""
     dev = torch.device("cuda:0")
-    Ad = [A.to(dev) for A, _ in layers]
-    Dd = [D.to(dev) for _, D in layers]
+    Ad, Dd = device_inputs(w, layers, dev)
     outs = [torch.zeros(i, o, device=dev, dtype=torch.float32) for i, o in w.layers]
     s_dev = torch.empty(w.B, device=dev)
     c_dev = torch.empty(w.B, device=dev)

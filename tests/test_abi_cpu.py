@@ -109,3 +109,19 @@ def test_kernel_launch_count_is_a_host_query(L):
     st, h = _init_status(L, _cfg(B=0))
     assert st == 2 and not h
     assert dp.dp_kernel_launches() == n0
+
+
+def test_conv2d_dims_on_host(L):
+    """dp_conv2d_dims: T and K of a convolution, and its host-side refusals."""
+    from oracle import dp_oracle as O
+    for H, W_, C, kh, kw, st, pd in [(32, 32, 3, 3, 3, (1, 1), (1, 1)), (32, 32, 64, 1, 1, (2, 2), (0, 0)),
+                                     (9, 7, 8, 2, 3, (1, 2), (0, 1)), (3, 3, 8, 3, 3, (1, 1), (0, 0))]:
+        T, K = dp.dp_conv2d_dims(dp.make_conv(H, W_, C, kh, kw, st, pd))
+        Ho, Wo = O.conv2d_out_hw(H, W_, kh, kw, st, pd)
+        assert (T, K) == (Ho * Wo, kh * kw * C)
+    for bad in [dp.make_conv(0, 8, 3, 3, 3), dp.make_conv(8, 8, 3, 3, 3, (0, 1)),
+                dp.make_conv(8, 8, 3, 3, 3, (1, 1), (-1, 0)), dp.make_conv(2, 2, 3, 5, 5),
+                dp.make_conv(8, 8, 1 << 18, 3, 3)]:
+        with pytest.raises(dp.DPError) as ei:
+            dp.dp_conv2d_dims(bad)
+        assert ei.value.status == 2

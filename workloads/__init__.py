@@ -13,7 +13,10 @@ Recipe (stated once, used everywhere):
     workload's dtype (fp32: unchanged; bf16: one RNE rounding);
   * "N(0, v)" in a workload description is read as variance v (std sqrt(v));
     "ReLU-sparse N(0,1)" is max(0, x) with x ~ N(0,1) (about half exact zeros);
-  * layouts: A [B, T, d_in], D [B, T, d_out], row-major, example-major.
+  * layouts: A [B, T, d_in], D [B, T, d_out], row-major, example-major; for
+    a convolution layer A is its NHWC input [B, H, W, C_in] (the patch rows
+    the layer's dense form needs are built from it by each side on its own)
+    and D its output gradient [B, H_out * W_out, C_out].
 
 The paper trains LoRA adapters of GPT-2 / RoBERTa, an MLP on Purchase and a
 WideResNet on CIFAR-10 (App. B); none of those datasets or checkpoints is
@@ -48,6 +51,9 @@ class Workload:
     sigma: float
     audit_frac: float = 0.0
     layer_T: Tuple[int, ...] = ()  # per-layer positions (empty: every layer has T)
+    # per layer: None for a dense layer, else the convolution
+    # (H, W, C_in, kh, kw, stride, pad) whose dense form is layers[l]
+    convs: Tuple = ()
 
     @property
     def n_params(self) -> int:
@@ -56,14 +62,22 @@ class Workload:
     def T_of(self, layer: int) -> int:
         return self.layer_T[layer] if self.layer_T else self.T
 
+    def conv_of(self, layer: int):
+        return self.convs[layer] if self.convs else None
+
     @property
     def specs(self) -> Tuple[Tuple[int, int, int], ...]:
         """(d_in, d_out, T) of every layer, as the C ABI's dp_layer takes them."""
         return tuple((i, o, self.T_of(l)) for l, (i, o) in enumerate(self.layers))
 
     def describe(self) -> str:
-        dims = ",".join(f"{i}x{o}" if self.T_of(l) == self.T else f"{i}x{o}@T{self.T_of(l)}"
-                        for l, (i, o) in enumerate(self.layers))
+        def one(l, i, o):
+            cv = self.conv_of(l)
+            if cv:
+                H, W_, cin, kh, kw, st, pd = cv
+                return f"conv{kh}x{kw}s{st}:{H}x{W_}x{cin}->{o}"
+            return f"{i}x{o}" if self.T_of(l) == self.T else f"{i}x{o}@T{self.T_of(l)}"
+        dims = ",".join(one(l, i, o) for l, (i, o) in enumerate(self.layers))
         return f"{self.name}: layers[{dims}] B={self.B} T={self.T} {self.dtype}"
 
 
@@ -138,6 +152,55 @@ WORKLOADS["roberta_l_lora_head_mnli_bf16"] = Workload(
     256, 128, "bf16", _normal_all(96) + ("normal", "ones", "normal", "ones"), 1.0,
     math.sqrt(1e-4), 1.0, 0.6407, audit_frac=0.05, layer_T=(128,) * 96 + (1, 1, 1, 1))
 
+def conv_out(H: int, k: int, stride: int, pad: int) -> int:
+    return (H + 2 * pad - k) // stride + 1
+
+
+def _conv_net(specs, head=()):
+    """Dense forms, per-layer T and geometries of a list of convolutions
+    (H, C_in, C_out, k, stride) on square inputs with pad k // 2, followed by
+    dense head layers (d_in, d_out, T)."""
+    layers, Ts, convs = [], [], []
+    for H, cin, cout, k, st in specs:
+        pad = k // 2
+        Ho = conv_out(H, k, st, pad)
+        layers.append((k * k * cin, cout))
+        Ts.append(Ho * Ho)
+        convs.append((H, H, cin, k, k, st, pad))
+    for d_in, d_out, T in head:
+        layers.append((d_in, d_out))
+        Ts.append(T)
+        convs.append(None)
+    return tuple(layers), tuple(Ts), tuple(convs)
+
+
+# WideResNet-16-4 on CIFAR-10 (App. B): 32x32x3 images, a 3x3 stem to 16
+# channels, three groups of two basic blocks of widths 64, 128, 256 (the
+# first block of groups 2 and 3 strides by 2; a 1x1 convolution is the
+# shortcut where the width changes), then the 256 -> 10 classifier and its
+# bias on the pooled features (T = 1).  The normalisation layers' scale and
+# shift are not part of it: their per-example gradients are per-channel dot
+# products, not dense products.  Batch 2048 in one pass (the paper's batch;
+# it trains it as 4 micro-batches of 512), C = 1, sigma from the
+# accountant for epsilon = 2, delta = 1e-5, 5000 steps at q = 2048/40000.
+_WRN = [(32, 3, 16, 3, 1),
+        (32, 16, 64, 3, 1), (32, 64, 64, 3, 1), (32, 16, 64, 1, 1),
+        (32, 64, 64, 3, 1), (32, 64, 64, 3, 1),
+        (32, 64, 128, 3, 2), (16, 128, 128, 3, 1), (32, 64, 128, 1, 2),
+        (16, 128, 128, 3, 1), (16, 128, 128, 3, 1),
+        (16, 128, 256, 3, 2), (8, 256, 256, 3, 1), (16, 128, 256, 1, 2),
+        (8, 256, 256, 3, 1), (8, 256, 256, 3, 1)]
+_wl, _wT, _wc = _conv_net(_WRN, head=((256, 10, 1), (1, 10, 1)))
+WORKLOADS["wrn16_4_cifar10_bf16"] = Workload(
+    "wrn16_4_cifar10_bf16", 11, _wl, 2048, 1024, "bf16",
+    ("normal",) + ("relu_normal",) * 16 + ("ones",), 1.0, math.sqrt(1e-4), 1.0, 9.11,
+    audit_frac=0.05, layer_T=_wT, convs=_wc)
+# its first group alone at the paper's micro-batch of 512 (profiling case)
+_gl, _gT, _gc = _conv_net(_WRN[1:6])
+WORKLOADS["wrn16_4_group1_bf16"] = Workload(
+    "wrn16_4_group1_bf16", 12, _gl, 512, 1024, "bf16", ("relu_normal",) * 5, 1.0,
+    math.sqrt(1e-4), 1.0, 9.11, audit_frac=0.05, layer_T=_gT, convs=_gc)
+
 # one 4096x4096 bf16 layer over B x T
 SWEEP = [Workload(f"sweep_B{b}_T{t}", 100 + 10 * bi + ti, ((4096, 4096),), b, t,
                   "bf16", _normal_all(1), 1.0, 1.0, 1.0, 1.0)
@@ -163,6 +226,26 @@ def custom(name: str, layers: Sequence[Sequence[int]], B: int, T: int, dtype: st
     return Workload(name, wid, tuple((int(x[0]), int(x[1])) for x in layers), B, T, dtype,
                     a_dist, a_std, d_std, C, sigma,
                     layer_T=lt if any(t != T for t in lt) else ())
+
+
+def custom_conv(name: str, convs: Sequence[Sequence[int]], B: int, dtype: str, C: float = 1.0,
+                sigma: float = 1.0, d_std: float = 1.0, wid: int = 999, a_dist=None,
+                head: Sequence[Sequence[int]] = ()) -> Workload:
+    """An ad-hoc convolution workload: convolutions (H, W, C_in, C_out, kh,
+    kw, stride, pad), then dense head layers (d_in, d_out, T)."""
+    layers, Ts, cv = [], [], []
+    for H, W_, cin, cout, kh, kw, st, pd in convs:
+        Ho, Wo = (H + 2 * pd - kh) // st + 1, (W_ + 2 * pd - kw) // st + 1
+        layers.append((kh * kw * cin, cout))
+        Ts.append(Ho * Wo)
+        cv.append((H, W_, cin, kh, kw, st, pd))
+    for d_in, d_out, T in head:
+        layers.append((d_in, d_out))
+        Ts.append(T)
+        cv.append(None)
+    a_dist = tuple(a_dist) if a_dist else _normal_all(len(layers))
+    return Workload(name, wid, tuple(layers), B, max(Ts), dtype, a_dist, 1.0, d_std, C, sigma,
+                    layer_T=tuple(Ts), convs=tuple(cv))
 
 
 def _draw(rng: np.random.Generator, dist: str, shape, std: float) -> np.ndarray:
@@ -202,7 +285,9 @@ def make_layer(w: Workload, layer: int, seed: int = 0, B: int | None = None):
     T = w.T_of(layer)
     ra = np.random.default_rng(np.random.SeedSequence([seed, w.wid, layer, 0]))
     rd = np.random.default_rng(np.random.SeedSequence([seed, w.wid, layer, 1]))
-    A = _draw(ra, w.a_dist[layer], (B, T, d_in), w.a_std)
+    cv = w.conv_of(layer)
+    a_shape = (B, cv[0], cv[1], cv[2]) if cv else (B, T, d_in)
+    A = _draw(ra, w.a_dist[layer], a_shape, w.a_std)
     D = _draw(rd, "normal", (B, T, d_out), w.d_std)
     return _to_dtype(A, w.dtype), _to_dtype(D, w.dtype)
 
