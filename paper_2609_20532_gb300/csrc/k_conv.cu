@@ -20,6 +20,7 @@ namespace {
 
 constexpr int kConvThreads = 256;
 constexpr int kConvRowElems = 4096;  // output units a block takes per row group
+constexpr int kConvUPT = 4;          // units a thread loads before it stores them
 
 // One output unit = V consecutive elements of a row (V = 16 bytes' worth
 // when C_in allows it, else 1).  U = units per row = kh*kw*C_in / V.
@@ -31,22 +32,94 @@ __global__ void __launch_bounds__(kConvThreads)
   const int rpb = kConvRowElems / U > 0 ? kConvRowElems / U : 1;  // rows per group
   const int64_t groups = (rows + rpb - 1) / rpb;
   const int T = g.H_out * g.W_out;
+  // rows < 2^31 (checked on the host), so row and position indices are 32-bit
   for (int64_t grp = blockIdx.x; grp < groups; grp += gridDim.x) {
-    const int64_t r0 = grp * rpb;
+    const int r0 = static_cast<int>(grp * rpb);
     const int n = static_cast<int>((rows - r0 < rpb ? rows - r0 : rpb) * U);
-    for (int e = threadIdx.x; e < n; e += kConvThreads) {
-      const int dr = e / U, u = e - dr * U;
-      const int64_t row = r0 + dr;
-      const int i = static_cast<int>(row / T), t = static_cast<int>(row - static_cast<int64_t>(i) * T);
-      const int ho = t / g.W_out, wo = t - ho * g.W_out;
-      const int tap = u / cu, cc = u - tap * cu;
-      const int ki = tap / g.kw, kj = tap - ki * g.kw;
-      const int y = ho * g.stride_h + ki - g.pad_h;
-      const int xx = wo * g.stride_w + kj - g.pad_w;
-      Unit v{};
-      if (y >= 0 && y < g.H && xx >= 0 && xx < g.W)
-        v = x[((static_cast<int64_t>(i) * g.H + y) * g.W + xx) * cu + cc];
-      __stcs(a + row * U + u, v);
+    for (int e0 = threadIdx.x; e0 < n; e0 += kConvThreads * kConvUPT) {
+      Unit v[kConvUPT];
+      int64_t dst[kConvUPT];
+#pragma unroll
+      for (int j = 0; j < kConvUPT; ++j) {
+        const int e = e0 + j * kConvThreads;
+        dst[j] = -1;
+        v[j] = Unit{};
+        if (e >= n) continue;
+        const int dr = e / U, u = e - dr * U;
+        const int row = r0 + dr;
+        const int i = row / T, t = row - i * T;
+        const int ho = t / g.W_out, wo = t - ho * g.W_out;
+        const int tap = u / cu, cc = u - tap * cu;
+        const int ki = tap / g.kw, kj = tap - ki * g.kw;
+        const int y = ho * g.stride_h + ki - g.pad_h;
+        const int xx = wo * g.stride_w + kj - g.pad_w;
+        dst[j] = static_cast<int64_t>(row) * U + u;
+        if (y >= 0 && y < g.H && xx >= 0 && xx < g.W)
+          v[j] = x[((static_cast<int64_t>(i) * g.H + y) * g.W + xx) * cu + cc];
+      }
+#pragma unroll
+      for (int j = 0; j < kConvUPT; ++j)
+        if (dst[j] >= 0) __stcs(a + dst[j], v[j]);
+    }
+  }
+}
+
+// Row-walking form for rows of at most kConvTab units: a table in shared
+// memory gives every unit of a row its tap offsets and channel unit, and
+// each warp copies a contiguous run of rows, lanes over the row's units, so
+// the loop does no division; (example, h, w) advance by increments.
+constexpr int kConvTab = 4096;
+constexpr int kConvWarps = kConvThreads / 32;
+
+template <typename Unit>
+__global__ void __launch_bounds__(kConvThreads)
+    k_conv_unfold_rows(const Unit* __restrict__ x, Unit* __restrict__ a, ConvGeom g, int rows,
+                       int cu) {
+  extern __shared__ int tab[];  // [3][U]: row offset, column offset, channel unit
+  const int U = g.kh * g.kw * cu;
+  for (int u = threadIdx.x; u < U; u += kConvThreads) {
+    const int tap = u / cu, ki = tap / g.kw;
+    tab[u] = ki - g.pad_h;
+    tab[U + u] = tap - ki * g.kw - g.pad_w;
+    tab[2 * U + u] = u - tap * cu;
+  }
+  __syncthreads();
+  const int lane = static_cast<int>(threadIdx.x) & 31;
+  const int64_t warp = static_cast<int64_t>(blockIdx.x) * kConvWarps + (threadIdx.x >> 5);
+  const int64_t nwarps = static_cast<int64_t>(gridDim.x) * kConvWarps;
+  int row = static_cast<int>(rows * warp / nwarps);
+  const int row_end = static_cast<int>(rows * (warp + 1) / nwarps);
+  if (row >= row_end) return;
+  const int T = g.H_out * g.W_out;
+  int i = row / T;
+  const int t = row - i * T;
+  int ho = t / g.W_out, wo = t - ho * g.W_out;
+  for (; row < row_end; ++row) {
+    const int y0 = ho * g.stride_h, x0 = wo * g.stride_w;
+    const Unit* xi = x + static_cast<int64_t>(i) * g.H * g.W * cu;
+    Unit* ar = a + static_cast<int64_t>(row) * U;
+    for (int u0 = lane; u0 < U; u0 += 32 * kConvUPT) {
+      Unit v[kConvUPT];
+#pragma unroll
+      for (int j = 0; j < kConvUPT; ++j) {
+        const int u = u0 + 32 * j;
+        v[j] = Unit{};
+        if (u < U) {
+          const int y = y0 + tab[u], xx = x0 + tab[U + u];
+          if (y >= 0 && y < g.H && xx >= 0 && xx < g.W)
+            v[j] = xi[(static_cast<int64_t>(y) * g.W + xx) * cu + tab[2 * U + u]];
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < kConvUPT; ++j)
+        if (u0 + 32 * j < U) __stcs(ar + u0 + 32 * j, v[j]);
+    }
+    if (++wo == g.W_out) {
+      wo = 0;
+      if (++ho == g.H_out) {
+        ho = 0;
+        ++i;
+      }
     }
   }
 }
@@ -56,6 +129,27 @@ cudaError_t launch_unfold_t(const void* x, void* a, const ConvGeom& g, int B, in
                             cudaStream_t s) {
   const int64_t rows = static_cast<int64_t>(B) * g.H_out * g.W_out;
   const int U = g.kh * g.kw * cu;
+  if (U <= kConvTab) {
+    const int smem = 3 * U * static_cast<int>(sizeof(int));
+    if (smem > 48 * 1024) {
+      static bool attr_set = false;
+      if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(k_conv_unfold_rows<Unit>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             3 * kConvTab * static_cast<int>(sizeof(int)));
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+      }
+    }
+    const int64_t warps_needed = rows;  // at least one row per warp
+    const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
+    int64_t grid = (warps_needed + kConvWarps - 1) / kConvWarps;
+    if (grid > cap) grid = cap;
+    note_launch();
+    k_conv_unfold_rows<Unit><<<static_cast<int>(grid), kConvThreads, smem, s>>>(
+        static_cast<const Unit*>(x), static_cast<Unit*>(a), g, static_cast<int>(rows), cu);
+    return cudaGetLastError();
+  }
   const int rpb = kConvRowElems / U > 0 ? kConvRowElems / U : 1;
   const int64_t groups = (rows + rpb - 1) / rpb;
   const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;

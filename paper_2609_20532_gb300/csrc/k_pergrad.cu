@@ -241,31 +241,68 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_norm(const __grid_constant
     }
   } else {
     // Rows read straight into registers (widths whose rows are not 16-byte
-    // multiples).
-    const bool vec = j0 + VJ <= n && n % VJ == 0 &&
+    // multiples).  A block narrower than its threads splits the positions
+    // over S groups of tpr threads (group s takes t = s, s + S, ...) and adds
+    // the groups' sums in order at the end.
+    const int tpr = (W + VJ - 1) / VJ;
+    const int S = tpr < kThreads ? kThreads / tpr : 1;
+    const int s = static_cast<int>(threadIdx.x) / tpr;
+    const int jj0 = c0 + (static_cast<int>(threadIdx.x) - s * tpr) * VJ;
+    const bool active = s < S && jj0 < n;
+    const bool vec = jj0 + VJ <= n && n % VJ == 0 &&
                      (reinterpret_cast<uintptr_t>(P.X) % (VJ * sizeof(TIn))) == 0;
     for (int t0 = 0; t0 < T; t0 += TT) {
       const int tt = T - t0 < TT ? T - t0 : TT;
       fill_ys(t0);
       __syncthreads();
-      const TIn* xrow = X + static_cast<int64_t>(t0) * n + j0;
-      if (vec) {
+      const TIn* xrow = X + static_cast<int64_t>(t0 + s) * n + jj0;
+      const int64_t step = static_cast<int64_t>(S) * n;
+      if (active && vec) {
 #pragma unroll 8
-        for (int t = 0; t < tt; ++t, xrow += n) {
+        for (int t = s; t < tt; t += S, xrow += step) {
           float x[VJ];
           load_row<TIn, VJ>(xrow, x);
           fma_row<TIn, R, VJ>(x, &ys[t][0], acc);
         }
-      } else if (j0 < n) {
+      } else if (active) {
 #pragma unroll 4
-        for (int t = 0; t < tt; ++t, xrow += n) {
+        for (int t = s; t < tt; t += S, xrow += step) {
           float x[VJ];
 #pragma unroll
-          for (int v = 0; v < VJ; ++v) x[v] = (j0 + v < n) ? to_float(xrow[v]) : 0.f;
+          for (int v = 0; v < VJ; ++v) x[v] = (jj0 + v < n) ? to_float(xrow[v]) : 0.f;
           fma_row<TIn, R, VJ>(x, &ys[t][0], acc);
         }
       }
       __syncthreads();
+    }
+    if (S > 1) {
+      // groups 1.. hand their sums to group 0 through the (unused) staging
+      // memory: S * tpr <= kThreads slots of VJ * R floats (at most 32 KB)
+      float* part = reinterpret_cast<float*>(stage_mem);
+      float* mine = part + static_cast<int64_t>(threadIdx.x) * VJ * R;
+      if (s > 0 && s < S) {
+#pragma unroll
+        for (int v = 0; v < VJ; ++v)
+#pragma unroll
+          for (int k = 0; k < R; ++k) mine[v * R + k] = acc[v][k];
+      }
+      __syncthreads();
+      if (s == 0) {
+        for (int q = 1; q < S; ++q) {
+          const float* o = part + static_cast<int64_t>(q * tpr + threadIdx.x) * VJ * R;
+#pragma unroll
+          for (int v = 0; v < VJ; ++v)
+#pragma unroll
+            for (int k = 0; k < R; ++k) acc[v][k] += o[v * R + k];
+        }
+      } else {
+        // the sums now live in group 0 (and these threads' columns j0 are
+        // past the layer's width, so they store nothing)
+#pragma unroll
+        for (int v = 0; v < VJ; ++v)
+#pragma unroll
+          for (int k = 0; k < R; ++k) acc[v][k] = 0.f;
+      }
     }
   }
 
