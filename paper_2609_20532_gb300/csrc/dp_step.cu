@@ -734,7 +734,8 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
     const LayerPlan& p = c->plan[l];
     cudaError_t e = cudaSuccess;
     if (!(flags & DP_NOISE_ONLY) && p.gemm_tc == 1) {
-      if (!grp.empty() && (!dpk::tc_clipsum_same_launch(c->plan[layers[grp[0]]].d_in, p.d_in) ||
+      const LayerPlan& p0 = c->plan[layers[grp.empty() ? r : grp[0]]];
+      if (!grp.empty() && (!dpk::tc_clipsum_same_launch(p0.d_in, p0.d_out, p.d_in, p.d_out) ||
                            c->plan[layers[grp[0]]].T != p.T))
         e = flush();
       grp.push_back(r);

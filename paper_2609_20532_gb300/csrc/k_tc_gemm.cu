@@ -56,13 +56,14 @@ constexpr int NUM_EPI_WARPS = 8;
 constexpr int FIRST_EPI_WARP = 4;
 constexpr int GEMM_THREADS = 128 + 32 * NUM_EPI_WARPS;
 constexpr int REGS_CTRL = 48, REGS_EPI = 224;
-constexpr uint32_t TMEM_COLS = 512;
 constexpr uint32_t LBO = CHUNK, SBO = 1024;
 
-template <bool PAIR>
+// NB: tile width in output columns (N of the MMA), 256, or 128 for layers
+// with d_out <= 128 (no MMA work on columns past the layer).
+template <bool PAIR, int NB>
 struct Cfg {
   static constexpr int STAGES = PAIR ? 6 : 4;
-  static constexpr int B_COLS = PAIR ? BN / 2 : BN;         // D columns staged per CTA
+  static constexpr int B_COLS = PAIR ? NB / 2 : NB;         // D columns staged per CTA
   static constexpr int A_STAGE = BM * BK * 2;               // 16 KB
   static constexpr int B_STAGE = B_COLS * BK * 2;           // 16 / 32 KB
   static constexpr int STAGE_BYTES = A_STAGE + B_STAGE;     // 32 / 48 KB
@@ -70,7 +71,9 @@ struct Cfg {
   // pipeline stages, then one 4 KB store-staging block per epilogue warp
   static constexpr int STAGING = STAGES * STAGE_BYTES;
   static constexpr int SMEM_BYTES = STAGING + NUM_EPI_WARPS * 4096 + 1024;
-  static constexpr uint32_t IDESC = idesc_bf16_f32(TILE_M, BN, /*a_mn=*/1, /*b_mn=*/1);
+  static constexpr uint32_t IDESC = idesc_bf16_f32(TILE_M, NB, /*a_mn=*/1, /*b_mn=*/1);
+  static constexpr uint32_t TMEM_COLS = 2 * NB;             // two accumulator buffers
+  static constexpr int HALF = NB / 2;                       // columns per epilogue thread
 };
 
 // One launch serves up to kGemmMaxLayers layers of a step (same B and T):
@@ -134,11 +137,11 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* 
 
 // TMA loads of one stage: A rows m0.. (two 64-column chunks) and the D
 // columns this CTA stages, for K block kb of example ex.
-template <bool PAIR>
+template <bool PAIR, int NB>
 __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, uint64_t* full,
                                                   bool leader, uint8_t* sa, uint8_t* sb, int m0,
                                                   int n0, int ex, int kb) {
-  using C = Cfg<PAIR>;
+  using C = Cfg<PAIR, NB>;
   const CUtensorMap* mapA = &g.mapA[layer];
   const CUtensorMap* mapD = &g.mapD[layer];
   const int arow = ex * g.T + kb * BK;                       // row of [B*T, d]
@@ -182,8 +185,8 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
 // S[4t .. 4t+3] += s * z for the warp-uniform quad slot q in [T0, T0 + N):
 // a binary tree of uniform branches down to static register indices, so the
 // accumulator stays in registers and each quad costs a few branches.
-template <int T0, int N>
-__device__ __forceinline__ void add_noise_slot(float (&S)[128], int q, float4 z, float s) {
+template <int T0, int N, int SZ>
+__device__ __forceinline__ void add_noise_slot(float (&S)[SZ], int q, float4 z, float s) {
   if constexpr (N == 1) {
     S[4 * T0 + 0] = fmaf(s, z.x, S[4 * T0 + 0]);
     S[4 * T0 + 1] = fmaf(s, z.y, S[4 * T0 + 1]);
@@ -191,9 +194,9 @@ __device__ __forceinline__ void add_noise_slot(float (&S)[128], int q, float4 z,
     S[4 * T0 + 3] = fmaf(s, z.w, S[4 * T0 + 3]);
   } else {
     if (q < T0 + N / 2)
-      add_noise_slot<T0, N / 2>(S, q, z, s);
+      add_noise_slot<T0, N / 2, SZ>(S, q, z, s);
     else
-      add_noise_slot<T0 + N / 2, N / 2>(S, q, z, s);
+      add_noise_slot<T0 + N / 2, N / 2, SZ>(S, q, z, s);
   }
 }
 
@@ -211,10 +214,10 @@ __device__ __forceinline__ void tile_mn(int t, int n_m, int n_n, int& mt, int& n
   nt = r / gm;
 }
 
-template <bool NORM, bool PAIR>
+template <bool NORM, bool PAIR, int NB>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_gemm_tc(const __grid_constant__ GemmArgs g) {
-  using C = Cfg<PAIR>;
+  using C = Cfg<PAIR, NB>;
   constexpr int STAGES = C::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -253,9 +256,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   }
   if (warp == 1) {
     if constexpr (PAIR)
-      tmem_alloc_pair(&tmem_slot, TMEM_COLS);
+      tmem_alloc_pair(&tmem_slot, C::TMEM_COLS);
     else
-      tmem_alloc(&tmem_slot, TMEM_COLS);
+      tmem_alloc(&tmem_slot, C::TMEM_COLS);
   }
   tc_fence_before();
   __syncthreads();
@@ -264,7 +267,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   const uint32_t tmem_base = tmem_slot;
 
   if (warp < FIRST_EPI_WARP) {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(REGS_CTRL));
+    // the 256-wide tile's epilogue holds 128 accumulators per thread and
+    // takes registers from the control warps; the 128-wide one fits the
+    // uniform allocation
+    if constexpr (NB == 256) asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(REGS_CTRL));
     if (warp == 0 && lane == 0) {
       // ---------------- TMA producer (both CTAs of a pair) ----------------
       int stage = 0;
@@ -276,13 +282,13 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         int mt, nt;
         tile_mn(w.lt, g.n_m[l], g.n_n[l], mt, nt);
         const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
-        const int n0 = nt * BN + (PAIR ? static_cast<int>(rank) * (BN / 2) : 0);
+        const int n0 = nt * NB + (PAIR ? static_cast<int>(rank) * (NB / 2) : 0);
         for (int ex = w.e0; ex < w.e1; ++ex) {
           for (int kb = 0; kb < kpe; ++kb) {
             if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
             uint8_t* sa = smem + stage * C::STAGE_BYTES;
             uint8_t* sb = sa + C::A_STAGE;
-            issue_stage_loads<PAIR>(g, l, &full_bar[stage], leader, sa, sb, m0, n0, ex, kb);
+            issue_stage_loads<PAIR, NB>(g, l, &full_bar[stage], leader, sa, sb, m0, n0, ex, kb);
             ++uses[stage];
             if (++stage == STAGES) {
               stage = 0;
@@ -314,7 +320,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           const uint32_t tph = (it >> 1) & 1;
           if (!mbar_wait(&tempty_bar[buf], tph ^ 1, abrt, g.err)) goto mma_done;
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + buf * BN;
+          const uint32_t d_tmem = tmem_base + buf * NB;
           for (int kb = 0; kb < kpe; ++kb) {
             if (!mbar_wait(&full_bar[stage], phase, abrt, g.err)) goto mma_done;
             tc_fence_after();
@@ -352,7 +358,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         mma_commit(&done_bar);
     }
   } else {
-    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REGS_EPI));
+    if constexpr (NB == 256) asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REGS_EPI));
     // ---------------- fold / epilogue warps ----------------
     const int ew = warp - FIRST_EPI_WARP;
     const int quad = warp & 3;         // TMEM lane quadrant this warp may access
@@ -360,11 +366,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int row = quad * 32 + lane;  // tile row held by this thread
     const uint32_t t_lane = static_cast<uint32_t>(quad * 32) << 16;
     int it = 0;
-    // The tile's noise (32 Philox quads per thread) is generated in slices
-    // of qpe quads while the tensor core works on each example and added
+    // The tile's noise (QPT groups of 4 per thread) is generated in slices
+    // of qpe groups while the tensor core works on each example and added
     // into the register accumulator (sum and noise commute), so the tile end
     // only scales and stores.
-    const int qpe = (32 + g.B - 1) / g.B;
+    constexpr int QPT = C::HALF / 4;
+    const int qpe = (QPT + g.B - 1) / g.B;
     const uint64_t seed = g.add_noise ? g.key[0] : 0, step = g.add_noise ? g.key[1] : 0;
     for (int tile = unit; tile < n_tiles; tile += n_units) {
       const GemmItem w = gemm_item(g, tile);
@@ -376,20 +383,20 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       int mt, nt;
       tile_mn(lt, g.n_m[l], g.n_n[l], mt, nt);
       const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
-      const int n0 = nt * BN;
+      const int n0 = nt * NB;
       const int j = m0 + row;
-      const int k0 = n0 + half * 128;
+      const int k0 = n0 + half * C::HALF;
       const uint64_t prow = g.p_base[l] + static_cast<uint64_t>(j) * d_out;
-      float S[128];
+      float S[C::HALF];
       if constexpr (!NORM) {
 #pragma unroll
-        for (int i = 0; i < 128; ++i) S[i] = 0.f;
+        for (int i = 0; i < C::HALF; ++i) S[i] = 0.f;
       }
       for (int ex = w.e0; ex < w.e1; ++ex, ++it) {
         if constexpr (!NORM) {
           if (g.add_noise && !part_out && j < d_in) {
             const int q_lo = ex * qpe;
-            const int q_hi = q_lo + qpe < 32 ? q_lo + qpe : 32;
+            const int q_hi = q_lo + qpe < QPT ? q_lo + qpe : QPT;
 #pragma unroll 1
             for (int q = q_lo; q < q_hi; ++q) {
               // d_out is a multiple of 8 on this path, so the four parameters
@@ -398,7 +405,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
               // layer after one whose size is not a multiple of 4)
               if (k0 + 4 * q >= d_out) break;
               const float4 z = gauss4_at(seed, step, prow + k0 + 4 * q);
-              add_noise_slot<0, 32>(S, q, z, g.sigmaC);
+              add_noise_slot<0, QPT, C::HALF>(S, q, z, g.sigmaC);
             }
           }
         }
@@ -406,11 +413,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         const uint32_t tph = (it >> 1) & 1;
         if (!mbar_wait(&tfull_bar[buf], tph, abrt, g.err)) goto epi_done;
         tc_fence_after();
-        const uint32_t tcol = t_lane + buf * BN + half * 128;
+        const uint32_t tcol = t_lane + buf * NB + half * C::HALF;
         float sq = 0.f;
         const float ci = NORM ? 0.f : (g.c ? g.c[ex] : 1.f);
 #pragma unroll
-        for (int ch = 0; ch < 2; ++ch) {
+        for (int ch = 0; ch < C::HALF / 64; ++ch) {
           uint32_t v[64];
           tmem_ld64(tmem_base + tcol + ch * 64, v);
 #pragma unroll
@@ -447,7 +454,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         uint8_t* stg = smem + C::STAGING + ew * 4096;
         const int y = m0 + quad * 32;
 #pragma unroll
-        for (int c4 = 0; c4 < 4; ++c4) {
+        for (int c4 = 0; c4 < C::HALF / 32; ++c4) {
           if (lane == 0) bulk_wait_read_all();  // previous block has been read
           __syncwarp();
 #pragma unroll
@@ -489,9 +496,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     if (lane == 0) drain_wait(&done_bar, 0, g.err);
     __syncwarp();
     if constexpr (PAIR)
-      tmem_dealloc_pair(tmem_base, TMEM_COLS);
+      tmem_dealloc_pair(tmem_base, C::TMEM_COLS);
     else
-      tmem_dealloc(tmem_base, TMEM_COLS);
+      tmem_dealloc(tmem_base, C::TMEM_COLS);
   }
 }
 
@@ -519,22 +526,34 @@ bool make_map_3d(CUtensorMap* m, const void* base, uint64_t cols, uint64_t T, ui
 
 // CTA pairs for every layer wider than one 128-row tile.
 bool use_pair(int64_t d_in) { return d_in > BM; }
+// Tile width: 128 columns for layers with d_out <= 128, else 256.
+int gemm_nb(int64_t d_out) { return d_out <= 128 ? 128 : BN; }
 
-template <bool NORM, bool PAIR>
+template <bool NORM, bool PAIR, int NB>
 cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
-  using C = Cfg<PAIR>;
+  using C = Cfg<PAIR, NB>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<NORM, PAIR>,
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<NORM, PAIR, NB>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
+    if constexpr (NB == 256) {
+      // setmaxnreg moves registers within what the block was launched with:
+      // the split must fit the compiled count, else the raise never returns
+      cudaFuncAttributes fa{};
+      e = cudaFuncGetAttributes(&fa, k_gemm_tc<NORM, PAIR, NB>);
+      if (e != cudaSuccess) return e;
+      if (fa.numRegs * GEMM_THREADS < 4 * 32 * REGS_CTRL + NUM_EPI_WARPS * 32 * REGS_EPI ||
+          fa.numRegs > REGS_EPI)
+        return cudaErrorInvalidConfiguration;
+    }
     attr_set = true;
   }
   g.tile_start[0] = 0;
   for (int l = 0; l < g.L; ++l) {
     g.n_m[l] = (g.d_in[l] + C::TILE_M - 1) / C::TILE_M;
-    g.n_n[l] = (g.d_out[l] + BN - 1) / BN;
+    g.n_n[l] = (g.d_out[l] + NB - 1) / NB;
     if (g.split[l] < 1) g.split[l] = 1;
     g.tile_start[l + 1] = g.tile_start[l] + g.n_m[l] * g.n_n[l] * g.split[l];
   }
@@ -557,7 +576,8 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
     if (max_pairs == 0) {
       cfg.gridDim = dim3(sms);
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<NORM, PAIR>, &cfg) != cudaSuccess || n < 1) {
+      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<NORM, PAIR, NB>, &cfg) != cudaSuccess ||
+          n < 1) {
         cudaGetLastError();
         n = sms / 2;
       }
@@ -566,11 +586,11 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
     const int pairs = tiles < max_pairs ? tiles : max_pairs;
     cfg.gridDim = dim3(2 * pairs);
     note_launch();
-    return cudaLaunchKernelEx(&cfg, k_gemm_tc<NORM, PAIR>, g);
+    return cudaLaunchKernelEx(&cfg, k_gemm_tc<NORM, PAIR, NB>, g);
   } else {
     const int grid = tiles < sms ? tiles : sms;
     note_launch();
-    k_gemm_tc<NORM, PAIR><<<grid, GEMM_THREADS, C::SMEM_BYTES, s>>>(g);
+    k_gemm_tc<NORM, PAIR, NB><<<grid, GEMM_THREADS, C::SMEM_BYTES, s>>>(g);
     return cudaGetLastError();
   }
 }
@@ -590,7 +610,12 @@ bool make_input_maps(const void* A, const void* D, GemmArgs& g, int l) {
 
 template <bool NORM>
 cudaError_t launch_any(GemmArgs& g, cudaStream_t s) {
-  return use_pair(g.d_in[0]) ? launch_gemm<NORM, true>(g, s) : launch_gemm<NORM, false>(g, s);
+  // every layer of a launch shares the tile shape (use_pair, gemm_nb)
+  if (gemm_nb(g.d_out[0]) == 128)
+    return use_pair(g.d_in[0]) ? launch_gemm<NORM, true, 128>(g, s)
+                               : launch_gemm<NORM, false, 128>(g, s);
+  return use_pair(g.d_in[0]) ? launch_gemm<NORM, true, BN>(g, s)
+                             : launch_gemm<NORM, false, BN>(g, s);
 }
 
 void set_epilogue(GemmArgs& g, const Epilogue& ep) {
@@ -693,23 +718,35 @@ __global__ void __launch_bounds__(256) k_split_reduce(const __grid_constant__ Sp
 }  // namespace
 
 // Example ranges per tile of a layer's clipped sum or materialised norm.  A
-// layer with fewer tiles than the GPU has units splits its batch so that the
-// items fill the units, each range keeping at least 8 K-blocks of work.  The
-// count depends only on the layer's own shape (and the device's SM count),
-// so a layer rounds the same in a batched launch and in a launch of its own.
+// layer with fewer tiles than the GPU has units splits its batch into S
+// ranges, S chosen to fill whole rounds of the units (the largest fraction
+// tiles*S / (rounds * units), the smallest S on a tie), each range keeping
+// at least 8 K-blocks of work.  S depends only on the layer's own shape (and
+// the device's SM count), so a layer rounds the same in a batched launch and
+// in a launch of its own.
 int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out) {
   const bool pair = use_pair(d_in);
   const int64_t tile_m = pair ? 2 * BM : BM;
-  const int64_t tiles = ((d_in + tile_m - 1) / tile_m) * ((d_out + BN - 1) / BN);
+  const int64_t nb = gemm_nb(d_out);
+  const int64_t tiles = ((d_in + tile_m - 1) / tile_m) * ((d_out + nb - 1) / nb);
   const int64_t units = pair ? device_sm_count() / 2 : device_sm_count();
   if (tiles >= units || B < 2) return 1;
   const int64_t kpe = (T + BK - 1) / BK;
-  int64_t S = (units + tiles - 1) / tiles;
-  const int64_t by_work = static_cast<int64_t>(B) * kpe / 8;
-  if (S > by_work) S = by_work;
-  if (S > B) S = B;
-  if (S > kGemmMaxSplit) S = kGemmMaxSplit;
-  return S < 1 ? 1 : static_cast<int>(S);
+  int64_t smax = static_cast<int64_t>(B) * kpe / 8;
+  if (smax > B) smax = B;
+  if (smax > kGemmMaxSplit) smax = kGemmMaxSplit;
+  int64_t best = 1;
+  double best_eff = 0.0;
+  for (int64_t S = 1; S <= smax; ++S) {
+    const int64_t items = tiles * S;
+    const int64_t rounds = (items + units - 1) / units;
+    const double eff = static_cast<double>(items) / static_cast<double>(rounds * units);
+    if (eff > best_eff + 1e-9) {
+      best_eff = eff;
+      best = S;
+    }
+  }
+  return static_cast<int>(best);
 }
 
 // Direct path: T a multiple of 64, or T >= 32 (3-D padding wastes at most half).
@@ -763,7 +800,8 @@ cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const floa
 int tc_mat_parts(int64_t d_in, int64_t d_out) {
   const int64_t tile_m = use_pair(d_in) ? 2 * BM : BM;
   const int64_t ctas_per_tile = use_pair(d_in) ? 2 : 1;
-  return static_cast<int>(((d_in + tile_m - 1) / tile_m) * ((d_out + BN - 1) / BN) *
+  const int64_t nb = gemm_nb(d_out);
+  return static_cast<int>(((d_in + tile_m - 1) / tile_m) * ((d_out + nb - 1) / nb) *
                           ctas_per_tile * NUM_EPI_WARPS);
 }
 
@@ -790,6 +828,7 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
                                     int B, int T, const Epilogue& ep, int* err, cudaStream_t s) {
   if (L < 1 || L > kGemmMaxLayers) return cudaErrorInvalidValue;
   const bool pair = use_pair(d_in[0]);
+  const int nb = gemm_nb(d_out[0]);
   GemmArgs g{};
   g.L = L;
   g.c = c;
@@ -800,7 +839,8 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
   SplitReduceBatch r{};
   int64_t threads = 0;
   for (int l = 0; l < L; ++l) {
-    if (use_pair(d_in[l]) != pair) return cudaErrorInvalidValue;  // caller groups by tile shape
+    // the caller groups layers by tile shape
+    if (use_pair(d_in[l]) != pair || gemm_nb(d_out[l]) != nb) return cudaErrorInvalidValue;
     g.d_in[l] = d_in[l];
     g.d_out[l] = d_out[l];
     g.out[l] = out[l];
@@ -842,8 +882,8 @@ cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int 
                                  err, s);
 }
 
-bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_in_b) {
-  return use_pair(d_in_a) == use_pair(d_in_b);
+bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_out_a, int64_t d_in_b, int64_t d_out_b) {
+  return use_pair(d_in_a) == use_pair(d_in_b) && gemm_nb(d_out_a) == gemm_nb(d_out_b);
 }
 
 }  // namespace dpk

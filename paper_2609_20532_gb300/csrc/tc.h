@@ -29,9 +29,9 @@ cudaError_t tc_launch_ghost_batch(int L, const void* const* A, const void* const
 // (split * d_in * d_out fp32, 16-byte aligned) and a reduce pass adds them in
 // order with the noise; the materialised norm needs no scratch.
 constexpr int kGemmMaxLayers = 8;
-constexpr int kGemmMaxSplit = 32;
+constexpr int kGemmMaxSplit = 256;
 int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out);
-bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_in_b);
+bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_out_a, int64_t d_in_b, int64_t d_out_b);
 cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
                                     float* const* out, float* const* part, const int* d_in,
                                     const int* d_out, const uint64_t* p_base, const float* c,
