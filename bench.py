@@ -234,35 +234,32 @@ def run_ours(args, rank, world, local_rank):
     w = W.get(args.workload)
     L = len(w.layers)
     layers = W.make_inputs(w, seed=rank)
-    X_d = [A.to(dev) for A, _ in layers]     # a convolution's A is its NHWC input
+    # a convolution is declared as such: its A is the NHWC input and the
+    # library forms the patch rows (in place in the tensor-core kernels, or
+    # in context scratch)
+    A_d = [A.to(dev) for A, _ in layers]
     D_d = [D.to(dev) for _, D in layers]
-    # convolutions: the step unfolds each input into patch rows (its dense A)
     convs = {}
     for l in range(L):
         cv = w.conv_of(l)
         if cv:
             H, W_, cin, kh, kw, st, pd = cv
             convs[l] = dp.make_conv(H, W_, cin, kh, kw, (st, st), (pd, pd))
-    A_d = [torch.empty((w.B, w.T_of(l), w.layers[l][0]), dtype=X_d[l].dtype, device=dev)
-           if l in convs else X_d[l] for l in range(L)]
-
-    def unfold(X_list, A_list):
-        for l, conv in convs.items():
-            dp.dp_conv2d_unfold(conv, w.B, w.dtype, X_list[l], A_list[l], stream)
     outs = [torch.empty(i, o, device=dev, dtype=torch.float32) for i, o in w.layers]
     idx = W.audit_indices(w, seed=rank)
     # CUDA graphs are captured on a non-default stream
     stream = torch.cuda.current_stream() if args.eager else torch.cuda.Stream()
     torch.cuda.set_stream(stream)
     cfg = dp.make_config(w.specs, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
-                         seed=1234 + rank, step=0, audit_capacity=len(idx))
+                         seed=1234 + rank, step=0, audit_capacity=len(idx),
+                         convs=[convs.get(l) for l in range(L)] if convs else None)
     ctx = dp.dp_step_init(cfg, stream)
     in_bytes = sum(A.numel() * A.element_size() + D.numel() * D.element_size()
                    for A, D in layers)
     out_bytes = sum(o.numel() * 4 for o in outs)
     rec_bytes = len(idx) * dp.dp_audit_record_bytes(L)
 
-    ev = {k: [] for k in ("unfold", "norm", "clip", "gemm")}
+    ev = {k: [] for k in ("norm", "clip", "gemm")}
     stage_launches = {}  # kernels each stage of the last step issued (the library's count)
 
     layer_ids = list(range(L))
@@ -271,14 +268,6 @@ def run_ours(args, rank, world, local_rank):
         cfg.step = t
         n0 = dp.dp_kernel_launches()
         dp.dp_step_init(cfg, stream, ctx)
-        n_i = dp.dp_kernel_launches()
-        if timed and convs:
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-        unfold(X_d, A_d)
-        if timed and convs:
-            e1.record(stream)
-            ev["unfold"].append((None, e0, e1))
         n1 = dp.dp_kernel_launches()
         if timed:
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -306,7 +295,7 @@ def run_ours(args, rank, world, local_rank):
             ev["gemm"].append((None, e0, e1))
         rec = dp.dp_audit_emit(ctx, idx, L)
         n5 = dp.dp_kernel_launches()
-        stage_launches.update(init=n_i - n0, unfold=n1 - n_i, norm=n2 - n1, clip=n3 - n2, gemm=n4 - n3,
+        stage_launches.update(init=n1 - n0, norm=n2 - n1, clip=n3 - n2, gemm=n4 - n3,
                               audit=n5 - n4, step=n5 - n0)
         return rec
 
@@ -327,7 +316,6 @@ def run_ours(args, rank, world, local_rank):
             graph = torch.cuda.CUDAGraph()
             with torch.cuda.graph(graph, stream=stream):
                 dp.dp_step_init(cfg, stream, ctx)
-                unfold(X_d, A_d)
                 dp.dp_layer_norms_batch(ctx, layer_ids, A_d, D_d)
                 dp.dp_clip_factors(ctx)
                 dp.dp_clipped_sum_noise_batch(ctx, layer_ids, A_d, D_d, outs, 0)
@@ -367,7 +355,7 @@ def run_ours(args, rank, world, local_rank):
     timed_launches = dp.dp_kernel_launches() - host_launches0
     if graph is not None:
         timed_launches += args.steps * sum(stage_launches[k]
-                                           for k in ("init", "unfold", "norm", "clip", "gemm"))
+                                           for k in ("init", "norm", "clip", "gemm"))
     barrier()
     torch.cuda.synchronize()
     ms = max_over_ranks(start.elapsed_time(stop), world, dev)
@@ -392,8 +380,6 @@ def run_ours(args, rank, world, local_rank):
         # replayed back to back with an event between stages, so the host
         # work of each call (planning, marshalling) stays out of the times
         stages = [("init", lambda: dp.dp_step_init(cfg, stream, ctx))]
-        if convs:
-            stages.append(("unfold", lambda: unfold(X_d, A_d)))
         stages += [("norm", lambda: dp.dp_layer_norms_batch(ctx, layer_ids, A_d, D_d)),
                    ("clip", lambda: dp.dp_clip_factors(ctx)),
                    ("gemm", lambda: dp.dp_clipped_sum_noise_batch(ctx, layer_ids, A_d, D_d,
@@ -470,30 +456,24 @@ def run_ours(args, rank, world, local_rank):
                 "traffic": _traffic("pergrad_sum", sum_bytes),
                 "launches_per_step": stage_launches["gemm"]}
 
-    # convolutions: the unfold reads each input and writes its patch rows; the
-    # norm and clipped-sum passes then read the dense form (patch rows + D)
-    # of every layer that does not store per-example gradients, else the
-    # stored gradients.  The dominant stage's HBM rate is the roofline.
+    # convolutions: the norm and clipped-sum passes read each layer's NHWC
+    # input (or dense A) and D; thin layers also write and read back their
+    # per-example gradients.  Patch rows formed in scratch are implementation
+    # traffic, not counted.  The slower stage's HBM rate is the roofline.
     conv_dom = None
     if convs:
-        elem = 2 if w.dtype == "bf16" else 4
-        unf_ms = per_step_ms("unfold")
-        unf_bytes = sum(X_d[l].numel() * elem + A_d[l].numel() * elem for l in convs)
         grads = 4.0 * w.B * sum(i * o for (i, o), t in zip(w.layers, thin) if t)
-        dense = sum(w.B * T_ * (i + o) * elem for i, o, T_ in w.specs)
         p_all = 4.0 * sum(i * o for i, o in w.layers)
-        norm_bytes = dense + grads
-        sum_bytes = sum(w.B * T_ * (i + o) * elem for (i, o, T_), t in zip(w.specs, thin)
-                        if not t) + grads + p_all
-        for name, ms_, b in (("unfold", unf_ms, unf_bytes), ("layer_norms", norm_ms, norm_bytes),
-                             ("clipsum_gemm", gemm_ms, sum_bytes)):
+        io = [A.numel() * A.element_size() + D.numel() * D.element_size() for A, D in layers]
+        norm_bytes = sum(io) + grads
+        sum_bytes = sum(b_ for b_, t in zip(io, thin) if not t) + grads + p_all
+        for name, ms_, b in (("layer_norms", norm_ms, norm_bytes), ("clipsum_gemm", gemm_ms, sum_bytes)):
             k = kernels.setdefault(name, {})
             k.update({"ms_per_step": ms_, "bytes": b, "gbs": b / (ms_ * 1e-3) / 1e9,
                       "frac_hbm": b / (ms_ * 1e-3) / 1e9 / peaks["hbm_gbs"],
                       "launches_per_step": stage_launches[
-                          {"unfold": "unfold", "layer_norms": "norm", "clipsum_gemm": "gemm"}[name]]})
-        conv_dom = max(("unfold", "layer_norms", "clipsum_gemm"),
-                       key=lambda n: kernels[n]["ms_per_step"])
+                          {"layer_norms": "norm", "clipsum_gemm": "gemm"}[name]]})
+        conv_dom = max(("layer_norms", "clipsum_gemm"), key=lambda n: kernels[n]["ms_per_step"])
 
     # standalone noise add over every layer (the DP_NOISE_ONLY call that adds
     # the released seed's noise to a committed sum): 8 bytes per parameter
@@ -544,7 +524,7 @@ def run_ours(args, rank, world, local_rank):
         D_h = [D.pin_memory() for _, D in layers]
         O_h = [[torch.empty(o.shape, dtype=torch.float32).pin_memory() for o in outs]
                for _ in range(2)]
-        A_b = [X_d, [torch.empty_like(x) for x in X_d]]   # host copies land as given
+        A_b = [A_d, [torch.empty_like(a) for a in A_d]]
         D_b = [D_d, [torch.empty_like(d) for d in D_d]]
         O_b = [outs, [torch.empty_like(o) for o in outs]]
         s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
@@ -569,12 +549,9 @@ def run_ours(args, rank, world, local_rank):
             stream.wait_event(ev_back[b])
             cfg.step = t
             dp.dp_step_init(cfg, stream, ctx)
-            # convolutions read the patch rows (one scratch set, stream-ordered)
-            dense = [A_d[l] if l in convs else A_b[b][l] for l in range(L)]
-            unfold(A_b[b], dense)
-            dp.dp_layer_norms_batch(ctx, layer_ids, dense, D_b[b])
+            dp.dp_layer_norms_batch(ctx, layer_ids, A_b[b], D_b[b])
             dp.dp_clip_factors(ctx)
-            dp.dp_clipped_sum_noise_batch(ctx, layer_ids, dense, D_b[b], O_b[b], 0)
+            dp.dp_clipped_sum_noise_batch(ctx, layer_ids, A_b[b], D_b[b], O_b[b], 0)
             ev_used[b].record(stream)
             ev_sum[b].record(stream)
             with torch.cuda.stream(s_out):

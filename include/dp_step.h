@@ -87,16 +87,49 @@ typedef enum {
     DP_NORM_MATERIALISED = 3
 } dp_norm_mode;
 
+/* ---- 2-D convolutions (the CIFAR-10 WideResNet of App. B) ---------------
+ * A convolution without bias over NHWC activations (a cross-correlation):
+ *   y[h][w][o] = sum_{ki, kj, c} xp[h*stride_h + ki][w*stride_w + kj][c] * W[ki][kj][c][o]
+ * where xp is the input with pad_h rows and pad_w columns of zeros on each
+ * side.  Its per-example weight gradient sum_{h,w} patch(h,w)^T dy[h][w] is
+ * the dense A_i^T D_i of a layer {d_in = K, d_out = C_out, T} with
+ *   T = H_out * W_out, H_out = (H + 2 pad_h - kh) / stride_h + 1 (W_out alike),
+ *   K = kh * kw * C_in,
+ *   A_i[h*W_out + w][(ki*kw + kj)*C_in + c] = xp_i[h*stride_h + ki][w*stride_w + kj][c]
+ *     (the patch rows dp_conv2d_unfold writes),
+ *   D_i = dy_i [H_out][W_out][C_out] read as [T][C_out],
+ * so the layer's output is laid out [kh][kw][C_in][C_out] (HWIO), row-major.
+ * A convolution enters a step in either of two ways:
+ *   - as a DP_LAYER_CONV2D layer (dp_layer.kind) with its geometry in
+ *     dp_config.convs: its A argument is then the NHWC input x [B][H][W][C_in]
+ *     itself, and the library forms the patch rows, on the fly inside the
+ *     tensor-core kernels where the shape allows (bf16, C_in a multiple of
+ *     64, T a multiple of 64, W_out dividing 64 or 64 dividing W_out), else
+ *     in context scratch when the layer's norms are computed;
+ *   - as a dense layer whose A is the caller's dp_conv2d_unfold output.    */
+typedef struct {
+    int32_t H, W;                /* input height and width, >= 1 */
+    int32_t C_in;                /* input channels, >= 1 */
+    int32_t kh, kw;              /* kernel height and width, >= 1 */
+    int32_t stride_h, stride_w;  /* >= 1 */
+    int32_t pad_h, pad_w;        /* zero rows / columns on each side, >= 0 */
+} dp_conv2d;
+
 /* One dense layer of the step: weight d_in x d_out, and the positions per
  * example its A and D carry.  T = 0 takes dp_config.T; a layer applied to one
  * position only (a classification head on the first token) gives T = 1, and
  * a bias row is a layer with d_in = 1 whose A holds ones.  All layers share B
  * and the clip factors: s_i sums every layer of the step. */
+#define DP_LAYER_DENSE  0
+#define DP_LAYER_CONV2D 1
+
 typedef struct {
     int64_t d_in;
     int64_t d_out;
     int32_t T;          /* positions per example of this layer, 0 = dp_config.T */
-    int32_t reserved;   /* must be 0 */
+    int32_t kind;       /* DP_LAYER_DENSE, or DP_LAYER_CONV2D: a convolution whose
+                           geometry is dp_config.convs[l], with d_in = kh*kw*C_in
+                           and T = H_out*W_out (or 0, which takes H_out*W_out) */
 } dp_layer;
 
 /* Parameters of Algorithm 2 for one step: batch B (also the aggregation
@@ -115,6 +148,8 @@ typedef struct {
     uint64_t step;             /* step index t; upper Philox counter words */
     dp_norm_mode norm_mode;    /* applies to every layer (AUTO picks per layer) */
     int32_t audit_capacity;    /* max records per dp_audit_emit call, 0 .. B */
+    const dp_conv2d* convs;    /* host array of L geometries, read for DP_LAYER_CONV2D
+                                  layers only (NULL when there are none); copied */
 } dp_config;
 
 /* Flags of dp_clipped_sum_noise. */
@@ -143,7 +178,8 @@ typedef struct {
  *   after the commitment (Algorithm 3, Derive/release) before a
  *   DP_NOISE_ONLY call.
  * Limits: B * T <= 2^31 - 1; every d_in, d_out in 1 .. 2^20; the device must
- *   be compute capability 10.3.
+ *   be compute capability 10.3.  A DP_LAYER_CONV2D layer needs a valid
+ *   geometry (as dp_conv2d_dims) with d_in = kh*kw*C_in and T = H_out*W_out.
  * Errors: DP_ERR_ARG, DP_ERR_SHAPE, DP_ERR_DTYPE, DP_ERR_UNSUPPORTED,
  *   DP_ERR_OOM, DP_ERR_CUDA. On failure of a create, *ctx stays NULL. */
 dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream);
@@ -151,7 +187,9 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream);
 /* Per-example squared gradient norms of one layer (Sec. 2.2 clipping
  * equation: ||g_t(x_i)||_2^2 restricted to layer l):
  *   n_{l,i} = ||A_{i,l}^T D_{i,l}||_F^2,  i = 0 .. B-1,
- * kept in the context.  A: [B][T][d_in], D: [B][T][d_out] device arrays.
+ * kept in the context.  A: [B][T][d_in], D: [B][T][d_out] device arrays; for a
+ * DP_LAYER_CONV2D layer A is the NHWC input [B][H][W][C_in] and D the output
+ * gradient [B][H_out][W_out][C_out].
  * Errors: DP_ERR_ARG (null / misaligned), DP_ERR_ORDER (after
  * dp_clip_factors of this step), DP_ERR_CUDA. */
 dp_status dp_layer_norms(dp_ctx* ctx, int32_t layer, const void* A, const void* D);
@@ -302,27 +340,7 @@ const char* dp_last_error(void);
 /* Name of a status code. */
 const char* dp_status_string(dp_status s);
 
-/* ---- 2-D convolutions (the CIFAR-10 WideResNet of App. B) ---------------
- * A convolution without bias over NHWC activations (a cross-correlation):
- *   y[h][w][o] = sum_{ki, kj, c} xp[h*stride_h + ki][w*stride_w + kj][c] * W[ki][kj][c][o]
- * where xp is the input with pad_h rows and pad_w columns of zeros on each
- * side.  Its per-example weight gradient sum_{h,w} patch(h,w)^T dy[h][w] is
- * the dense A_i^T D_i of a layer {d_in = K, d_out = C_out, T} with
- *   T = H_out * W_out, H_out = (H + 2 pad_h - kh) / stride_h + 1 (W_out alike),
- *   K = kh * kw * C_in,
- *   A_i[h*W_out + w][(ki*kw + kj)*C_in + c] = xp_i[h*stride_h + ki][w*stride_w + kj][c]
- *     (the patch rows dp_conv2d_unfold writes),
- *   D_i = dy_i [H_out][W_out][C_out] read as [T][C_out],
- * so the layer's output is laid out [kh][kw][C_in][C_out] (HWIO), row-major.
- * A convolution enters a step as that dense layer: unfold, then pass the
- * patch rows as its A to dp_layer_norms and dp_clipped_sum_noise.          */
-typedef struct {
-    int32_t H, W;                /* input height and width, >= 1 */
-    int32_t C_in;                /* input channels, >= 1 */
-    int32_t kh, kw;              /* kernel height and width, >= 1 */
-    int32_t stride_h, stride_w;  /* >= 1 */
-    int32_t pad_h, pad_w;        /* zero rows / columns on each side, >= 0 */
-} dp_conv2d;
+
 
 /* T = H_out * W_out and K = kh * kw * C_in of a convolution (host only).
  * Errors: DP_ERR_ARG (NULL argument), DP_ERR_SHAPE (a size < 1 or pad < 0,

@@ -22,6 +22,7 @@ __all__ = [
     "DP_OK", "DP_F32", "DP_BF16",
     "DP_NORM_AUTO", "DP_NORM_RANK1", "DP_NORM_GHOST", "DP_NORM_MATERIALISED",
     "DP_NO_NOISE", "DP_NOISE_ONLY", "DP_ACCUMULATE", "DP_WRITE_GRAD", "dp_adamw", "dp_noise_adamw",
+    "DP_LAYER_DENSE", "DP_LAYER_CONV2D",
     "dp_layer", "dp_config", "make_config",
     "dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "dp_clip_factors",
     "dp_clipped_sum_noise", "dp_clipped_sum_noise_batch",
@@ -39,6 +40,7 @@ DP_OK = 0
 DP_F32, DP_BF16 = 0, 1
 DP_NORM_AUTO, DP_NORM_RANK1, DP_NORM_GHOST, DP_NORM_MATERIALISED = 0, 1, 2, 3
 DP_NO_NOISE, DP_NOISE_ONLY, DP_ACCUMULATE, DP_WRITE_GRAD = 0x1, 0x2, 0x4, 0x8
+DP_LAYER_DENSE, DP_LAYER_CONV2D = 0, 1
 
 STATUS_NAMES = {0: "DP_OK", 1: "DP_ERR_ARG", 2: "DP_ERR_SHAPE", 3: "DP_ERR_DTYPE",
                 4: "DP_ERR_ORDER", 5: "DP_ERR_NONFINITE", 6: "DP_ERR_CUDA",
@@ -66,15 +68,15 @@ class LibraryNotBuilt(ImportError):
     pass
 
 
-class dp_layer(ctypes.Structure):
-    _fields_ = [("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64), ("T", ctypes.c_int32),
-                ("reserved", ctypes.c_int32)]
-
-
 class dp_conv2d(ctypes.Structure):
     _fields_ = [("H", ctypes.c_int32), ("W", ctypes.c_int32), ("C_in", ctypes.c_int32),
                 ("kh", ctypes.c_int32), ("kw", ctypes.c_int32), ("stride_h", ctypes.c_int32),
                 ("stride_w", ctypes.c_int32), ("pad_h", ctypes.c_int32), ("pad_w", ctypes.c_int32)]
+
+
+class dp_layer(ctypes.Structure):
+    _fields_ = [("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64), ("T", ctypes.c_int32),
+                ("kind", ctypes.c_int32)]
 
 
 class dp_adamw(ctypes.Structure):
@@ -88,7 +90,7 @@ class dp_config(ctypes.Structure):
                 ("clip_C", ctypes.c_float), ("sigma", ctypes.c_float),
                 ("out_scale", ctypes.c_float), ("seed", ctypes.c_uint64),
                 ("step", ctypes.c_uint64), ("norm_mode", ctypes.c_int32),
-                ("audit_capacity", ctypes.c_int32)]
+                ("audit_capacity", ctypes.c_int32), ("convs", ctypes.POINTER(dp_conv2d))]
 
 
 _LIB = None
@@ -166,16 +168,26 @@ def _stream(stream) -> Optional[int]:
 
 def make_config(layers: Sequence[Sequence[int]], B: int, T: int, dtype: str, C: float,
                 sigma: float, out_scale: float = 1.0, seed: int = 0, step: int = 0,
-                norm_mode: int = DP_NORM_AUTO, audit_capacity: int = 0) -> dp_config:
-    # a layer is (d_in, d_out) or (d_in, d_out, T); T = 0 takes the config's T
+                norm_mode: int = DP_NORM_AUTO, audit_capacity: int = 0,
+                convs: Optional[Sequence[Optional[dp_conv2d]]] = None) -> dp_config:
+    """A layer is (d_in, d_out) or (d_in, d_out, T); T = 0 takes the config's
+    T.  convs, when given, has one entry per layer: a dp_conv2d makes that
+    layer a DP_LAYER_CONV2D layer (its A is then the NHWC input), None keeps
+    it dense."""
+    kinds = [DP_LAYER_CONV2D if convs is not None and convs[i] is not None else DP_LAYER_DENSE
+             for i in range(len(layers))]
     arr = (dp_layer * len(layers))(*[dp_layer(int(ly[0]), int(ly[1]),
-                                              int(ly[2]) if len(ly) > 2 else 0, 0)
-                                     for ly in layers])
+                                              int(ly[2]) if len(ly) > 2 else 0, kinds[i])
+                                     for i, ly in enumerate(layers)])
+    carr = None
+    if convs is not None and any(k == DP_LAYER_CONV2D for k in kinds):
+        carr = (dp_conv2d * len(layers))(*[cv if cv is not None else dp_conv2d() for cv in convs])
     cfg = dp_config(B=B, T=T, n_layers=len(layers), layers=arr,
                     dtype=DP_BF16 if dtype == "bf16" else DP_F32, clip_C=C, sigma=sigma,
                     out_scale=out_scale, seed=seed & (2 ** 64 - 1), step=step & (2 ** 64 - 1),
-                    norm_mode=norm_mode, audit_capacity=audit_capacity)
-    cfg._keep = arr  # keep the layer array alive with the struct
+                    norm_mode=norm_mode, audit_capacity=audit_capacity,
+                    convs=ctypes.cast(carr, ctypes.POINTER(dp_conv2d)) if carr is not None else None)
+    cfg._keep = (arr, carr)  # keep the arrays alive with the struct
     return cfg
 
 

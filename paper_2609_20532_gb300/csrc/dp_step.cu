@@ -40,6 +40,23 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 constexpr int64_t kMaxDim = 1 << 20;  // largest d_in, d_out (and convolution K)
 
+dp_status conv_geom(const dp_conv2d* v, dpk::ConvGeom* g) {
+  if (!v) return fail(DP_ERR_ARG, "conv is NULL");
+  if (v->H < 1 || v->W < 1 || v->C_in < 1 || v->kh < 1 || v->kw < 1 || v->stride_h < 1 ||
+      v->stride_w < 1 || v->pad_h < 0 || v->pad_w < 0)
+    return fail(DP_ERR_SHAPE, "convolution sizes must be >= 1 and pads >= 0");
+  const int64_t hp = static_cast<int64_t>(v->H) + 2 * static_cast<int64_t>(v->pad_h);
+  const int64_t wp = static_cast<int64_t>(v->W) + 2 * static_cast<int64_t>(v->pad_w);
+  if (v->kh > hp || v->kw > wp) return fail(DP_ERR_SHAPE, "kernel larger than the padded input");
+  const int64_t ho = (hp - v->kh) / v->stride_h + 1, wo = (wp - v->kw) / v->stride_w + 1;
+  const int64_t K = static_cast<int64_t>(v->kh) * v->kw * v->C_in;
+  if (ho * wo > 0x7fffffffLL) return fail(DP_ERR_SHAPE, "H_out * W_out above 2^31 - 1");
+  if (K > kMaxDim) return fail(DP_ERR_SHAPE, "kh * kw * C_in above 2^20");
+  *g = dpk::ConvGeom{v->H, v->W, v->C_in, v->kh, v->kw, v->stride_h, v->stride_w,
+                     v->pad_h, v->pad_w, static_cast<int>(ho), static_cast<int>(wo)};
+  return DP_OK;
+}
+
 }  // namespace
 
 namespace dpk {
@@ -59,6 +76,13 @@ struct LayerPlan {
   int64_t g_off;       // offset (floats) of its [B][d_in][d_out] gradients in d_grads
   int split;           // tensor-core clipped sum: example ranges per tile (tc_gemm_split)
   int64_t s_off;       // offset (floats) of its [split][d_in][d_out] partials in d_split
+  // convolutions (kind DP_LAYER_CONV2D; A is the NHWC input)
+  int kind;            // dp_layer.kind as given
+  int conv;            // 1: a convolution whose patch rows differ from its input
+  dpk::ConvGeom cg;    // its geometry
+  int implicit;        // 1: the tensor-core kernels read its patch rows from A directly
+  int unfold;          // 1: its patch rows are formed in d_unf when its norms are computed
+  int64_t u_off;       // byte offset of those patch rows in d_unf
 };
 
 struct dp_ctx {
@@ -97,6 +121,8 @@ struct dp_ctx {
   int64_t grads_floats = 0;
   float* d_split = nullptr;     // partial sums of tensor-core layers whose batch is split
   int64_t split_floats = 0;
+  uint8_t* d_unf = nullptr;     // patch rows of convolutions formed in scratch
+  int64_t unf_bytes = 0;
   size_t part_bytes = 0;
   // per-step state
   std::vector<char> norm_done;
@@ -118,9 +144,21 @@ dp_status check_config(const dp_config* cfg) {
     const dp_layer& ly = cfg->layers[l];
     if (ly.d_in < 1 || ly.d_out < 1 || ly.d_in > kMaxDim || ly.d_out > kMaxDim)
       return fail(DP_ERR_SHAPE, "layer %d: d_in, d_out must be in 1..2^20", l);
-    if (ly.T < 0 || ly.reserved != 0)
-      return fail(DP_ERR_ARG, "layer %d: T must be >= 0 (0 = config T), reserved must be 0", l);
-    const int T = ly.T > 0 ? ly.T : cfg->T;
+    if (ly.T < 0) return fail(DP_ERR_ARG, "layer %d: T must be >= 0 (0 = config T)", l);
+    if (ly.kind != DP_LAYER_DENSE && ly.kind != DP_LAYER_CONV2D)
+      return fail(DP_ERR_ARG, "layer %d: unknown kind %d", l, ly.kind);
+    int T = ly.T > 0 ? ly.T : cfg->T;
+    if (ly.kind == DP_LAYER_CONV2D) {
+      if (!cfg->convs) return fail(DP_ERR_ARG, "layer %d is a convolution but convs is NULL", l);
+      dpk::ConvGeom g{};
+      dp_status st = conv_geom(&cfg->convs[l], &g);
+      if (st != DP_OK) return st;
+      if (ly.d_in != static_cast<int64_t>(g.kh) * g.kw * g.C_in)
+        return fail(DP_ERR_SHAPE, "layer %d: d_in must be kh*kw*C_in", l);
+      if (ly.T != 0 && ly.T != g.H_out * g.W_out)
+        return fail(DP_ERR_SHAPE, "layer %d: T must be H_out*W_out (or 0)", l);
+      T = g.H_out * g.W_out;
+    }
     if (static_cast<int64_t>(cfg->B) * T > 0x7fffffffLL)
       return fail(DP_ERR_SHAPE, "layer %d: B*T exceeds 2^31-1", l);
     if (cfg->norm_mode == DP_NORM_RANK1 && T != 1)
@@ -156,6 +194,11 @@ dp_norm_mode resolve_mode(dp_norm_mode m, int T, int64_t d_in, int64_t d_out) {
 // to matter and its clipped sum would otherwise be a latency-bound K = B
 // loop of its own.  A forced Gram or rank-1 mode keeps the other paths.
 int layer_T(const dp_config* cfg, int l) {
+  if (cfg->layers[l].kind == DP_LAYER_CONV2D) {  // geometry checked by check_config
+    dpk::ConvGeom g{};
+    conv_geom(&cfg->convs[l], &g);
+    return g.H_out * g.W_out;
+  }
   return cfg->layers[l].T > 0 ? cfg->layers[l].T : cfg->T;
 }
 
@@ -171,7 +214,7 @@ bool use_pergrad(const dp_config* cfg, int T, int64_t d_in, int64_t d_out) {
 void build_plan(dp_ctx* c, const dp_config* cfg) {
   c->plan.resize(cfg->n_layers);
   uint64_t off = 0;
-  int64_t grads = 0, splits = 0;
+  int64_t grads = 0, splits = 0, unf = 0;
   int NP = 1;
   for (int l = 0; l < cfg->n_layers; ++l) {
     LayerPlan& p = c->plan[l];
@@ -185,6 +228,26 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
     p.g_off = 0;
     p.split = 1;
     p.s_off = 0;
+    p.kind = cfg->layers[l].kind;
+    p.conv = p.kind == DP_LAYER_CONV2D ? 1 : 0;
+    p.cg = dpk::ConvGeom{};
+    p.implicit = 0;
+    p.unfold = 0;
+    p.u_off = 0;
+    if (p.conv) {
+      conv_geom(&cfg->convs[l], &p.cg);
+      // a 1x1, stride-1, unpadded convolution's input already is its patch rows
+      const bool identity = p.cg.kh == 1 && p.cg.kw == 1 && p.cg.stride_h == 1 &&
+                            p.cg.stride_w == 1 && p.cg.pad_h == 0 && p.cg.pad_w == 0;
+      if (identity) p.conv = 0;
+    }
+    auto need_unfold = [&]() {
+      p.unfold = 1;
+      p.u_off = unf;
+      const int64_t bytes = static_cast<int64_t>(cfg->B) * T * p.d_in *
+                            (cfg->dtype == DP_BF16 ? 2 : 4);
+      unf += (bytes + 255) / 256 * 256;
+    };
     if (p.pergrad) {
       p.mode = DP_NORM_MATERIALISED;
       p.norm_tc = 0;
@@ -194,6 +257,7 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
       p.g_off = grads;
       grads += static_cast<int64_t>(cfg->B) * p.d_in * p.d_out;
       if (p.nparts > NP) NP = p.nparts;
+      if (p.conv) need_unfold();
       continue;
     }
     p.mode = resolve_mode(cfg->norm_mode, T, p.d_in, p.d_out);
@@ -217,16 +281,26 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
         p.s_off = splits;
         splits += static_cast<int64_t>(p.split) * p.d_in * p.d_out;
       }
+      // a convolution read in place: the materialised norm (the Gram kernel
+      // has no implicit loads) unless the caller forced the Gram form
+      if (p.conv && cfg->norm_mode != DP_NORM_GHOST && dpk::tc_conv_implicit_ok(p.cg, T)) {
+        p.implicit = 1;
+        p.mode = DP_NORM_MATERIALISED;
+        p.norm_tc = 1;
+        p.nparts = dpk::tc_mat_parts(p.d_in, p.d_out);
+      }
     } else if (bf16 && dpk::tc_prescaled_supported(T, p.d_in, p.d_out)) {
       p.gemm_tc = 2;
       const int64_t need = dpk::tc_prescaled_scratch_bytes(cfg->B, T, p.d_in);
       if (need > c->prescaled_bytes) c->prescaled_bytes = need;
     }
+    if (p.conv && !p.implicit) need_unfold();
     if (p.nparts > NP) NP = p.nparts;
   }
   c->NP = NP;
   c->grads_floats = grads;
   c->split_floats = splits;
+  c->unf_bytes = unf;
 }
 
 void free_scratch(dp_ctx* c) {
@@ -242,9 +316,11 @@ void free_scratch(dp_ctx* c) {
   cudaFree(c->d_prescaled);
   cudaFree(c->d_grads);
   cudaFree(c->d_split);
+  cudaFree(c->d_unf);
   c->d_prescaled = nullptr;
   c->d_grads = nullptr;
   c->d_split = nullptr;
+  c->d_unf = nullptr;
   cudaFree(c->d_key);
   cudaFreeHost(c->h_key);
   c->d_key = nullptr;
@@ -280,6 +356,7 @@ dp_status alloc_scratch(dp_ctx* c) {
   if (c->prescaled_bytes > 0) DP_ALLOC(c->d_prescaled, static_cast<size_t>(c->prescaled_bytes));
   if (c->grads_floats > 0) DP_ALLOC(c->d_grads, sizeof(float) * static_cast<size_t>(c->grads_floats));
   if (c->split_floats > 0) DP_ALLOC(c->d_split, sizeof(float) * static_cast<size_t>(c->split_floats));
+  if (c->unf_bytes > 0) DP_ALLOC(c->d_unf, static_cast<size_t>(c->unf_bytes));
   DP_ALLOC(c->d_key, 2 * sizeof(uint64_t));
 #undef DP_ALLOC
   if (cudaHostAlloc(reinterpret_cast<void**>(&c->h_idx), sizeof(int) * (cap > 0 ? cap : 1),
@@ -379,6 +456,19 @@ dp_status check_norm_args(dp_ctx* c, int32_t layer, const void* A, const void* D
   return DP_OK;
 }
 
+// The A the dense kernels read for a layer: a convolution's patch rows in
+// context scratch when they are formed there, else the caller's array.
+const void* dense_A(const dp_ctx* c, int32_t layer, const void* A) {
+  const LayerPlan& p = c->plan[layer];
+  return p.unfold ? static_cast<const void*>(c->d_unf + p.u_off) : A;
+}
+
+cudaError_t unfold_layer(dp_ctx* c, int32_t layer, const void* X) {
+  const LayerPlan& p = c->plan[layer];
+  return dpk::launch_conv_unfold(c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, X,
+                                 c->d_unf + p.u_off, p.cg, c->B, c->stream);
+}
+
 void fill_pergrad(const dp_ctx* c, int32_t layer, const void* A, const void* D,
                   dpk::PerGradLayer& P) {
   const LayerPlan& p = c->plan[layer];
@@ -435,7 +525,7 @@ cudaError_t launch_layer_norms(dp_ctx* c, int32_t layer, const void* A, const vo
                      : dpk::launch_norm_ghost_simt(it, A, D, c->B, p.T, din, dout, c->d_part,
                                                    c->NP, row0, c->stream);
   return p.norm_tc ? dpk::tc_launch_mat_norm(A, D, c->B, p.T, din, dout, c->d_part, c->NP, row0,
-                                             c->d_flag, c->stream)
+                                             c->d_flag, c->stream, p.implicit ? &p.cg : nullptr)
                    : dpk::launch_norm_mat_simt(it, A, D, c->B, p.T, din, dout, c->d_part, c->NP,
                                                row0, c->stream);
 }
@@ -480,11 +570,12 @@ cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const vo
     g.L = 1;
     return dpk::launch_pergrad_sum(g, c->stream);
   }
+  A = dense_A(c, layer, A);
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
   if (p.gemm_tc == 1)
     return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, p.T, din, dout, d_out,
                                   p.split > 1 ? c->d_split + p.s_off : nullptr, ep, c->d_flag,
-                                  c->stream);
+                                  c->stream, p.implicit ? &p.cg : nullptr);
   if (p.gemm_tc == 2)
     return dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, p.T, din, dout, d_out, ep,
                                             c->d_flag, c->d_prescaled, c->stream);
@@ -504,9 +595,15 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     dp_ctx* c = *ctx;
     bool same = c->B == cfg->B && c->T == cfg->T && c->L == cfg->n_layers &&
                 c->dtype == cfg->dtype;
-    for (int l = 0; same && l < c->L; ++l)
+    for (int l = 0; same && l < c->L; ++l) {
       same = c->plan[l].d_in == cfg->layers[l].d_in && c->plan[l].d_out == cfg->layers[l].d_out &&
-             c->plan[l].T == layer_T(cfg, l);
+             c->plan[l].T == layer_T(cfg, l) && c->plan[l].kind == cfg->layers[l].kind;
+      if (same && cfg->layers[l].kind == DP_LAYER_CONV2D) {
+        dpk::ConvGeom g{};
+        conv_geom(&cfg->convs[l], &g);
+        same = std::memcmp(&g, &c->plan[l].cg, sizeof g) == 0 || !c->plan[l].conv;
+      }
+    }
     if (!same) return fail(DP_ERR_SHAPE, "re-key with different shapes; destroy and re-create");
     // The norm mode may change; the partial buffer must still be large enough.
     std::vector<LayerPlan> old = c->plan;
@@ -514,18 +611,22 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     const int64_t old_pre = c->prescaled_bytes;
     const int64_t old_grads = c->grads_floats;
     const int64_t old_splits = c->split_floats;
+    const int64_t old_unf = c->unf_bytes;
     build_plan(c, cfg);
     c->prescaled_bytes = old_pre;  // shapes are unchanged, so is the pre-scale need
-    if (c->NP > oldNP || c->grads_floats > old_grads || c->split_floats > old_splits) {
+    if (c->NP > oldNP || c->grads_floats > old_grads || c->split_floats > old_splits ||
+        c->unf_bytes > old_unf) {
       c->plan = old;
       c->NP = oldNP;
       c->grads_floats = old_grads;
       c->split_floats = old_splits;
+      c->unf_bytes = old_unf;
       return fail(DP_ERR_SHAPE, "norm_mode change needs more scratch; destroy and re-create");
     }
     c->NP = oldNP;  // keep the allocated stride
     c->grads_floats = old_grads;
     c->split_floats = old_splits;
+    c->unf_bytes = old_unf;
     set_scalars(c, cfg, cuda_stream);
     if (!same_parts(old, c->plan)) {
       st = upload_plan(c);
@@ -568,7 +669,8 @@ dp_status dp_layer_norms(dp_ctx* c, int32_t layer, const void* A, const void* D)
   if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
   dp_status st = check_norm_args(c, layer, A, D);
   if (st != DP_OK) return st;
-  cudaError_t e = launch_layer_norms(c, layer, A, D);
+  cudaError_t e = c->plan[layer].unfold ? unfold_layer(c, layer, A) : cudaSuccess;
+  if (e == cudaSuccess) e = launch_layer_norms(c, layer, dense_A(c, layer, A), D);
   if (e != cudaSuccess) return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
   c->norm_done[layer] = 1;
   return DP_OK;
@@ -586,6 +688,16 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
     if (seen[layers[r]]) return fail(DP_ERR_ARG, "layer %d listed twice", layers[r]);
     seen[layers[r]] = 1;
   }
+  // convolutions whose patch rows are formed in scratch: form them first;
+  // from here on A is what the dense kernels read
+  std::vector<const void*> Ad(n);
+  for (int r = 0; r < n; ++r) {
+    if (c->plan[layers[r]].unfold) {
+      cudaError_t e = unfold_layer(c, layers[r], A[r]);
+      if (e != cudaSuccess) return fail(DP_ERR_CUDA, "unfold kernel: %s", cudaGetErrorString(e));
+    }
+    Ad[r] = dense_A(c, layers[r], A[r]);
+  }
   // Gram-form tensor-core layers share launches (up to kGhostMaxLayers each);
   // every other layer gets its own kernel.
   std::vector<int> grp;
@@ -596,7 +708,7 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
     int din[dpk::kGhostMaxLayers], dout[dpk::kGhostMaxLayers], row0[dpk::kGhostMaxLayers];
     for (size_t q = 0; q < grp.size(); ++q) {
       const int r = grp[q], l = layers[r];
-      a[q] = A[r];
+      a[q] = Ad[r];
       d[q] = D[r];
       din[q] = static_cast<int>(c->plan[l].d_in);
       dout[q] = static_cast<int>(c->plan[l].d_out);
@@ -614,7 +726,7 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
   auto flush_thin = [&](std::vector<int>& v) -> cudaError_t {
     if (v.empty()) return cudaSuccess;
     dpk::PerGradBatch g{};
-    for (size_t q = 0; q < v.size(); ++q) fill_pergrad(c, layers[v[q]], A[v[q]], D[v[q]], g.l[q]);
+    for (size_t q = 0; q < v.size(); ++q) fill_pergrad(c, layers[v[q]], Ad[v[q]], D[v[q]], g.l[q]);
     g.L = static_cast<int>(v.size());
     g.part = c->d_part;
     g.err = c->d_flag;
@@ -637,7 +749,7 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
       grp.push_back(r);
       if (static_cast<int>(grp.size()) == dpk::kGhostMaxLayers) e = flush();
     } else {
-      e = launch_layer_norms(c, layers[r], A[r], D[r]);
+      e = launch_layer_norms(c, layers[r], Ad[r], D[r]);
     }
     if (e != cudaSuccess)
       return fail(DP_ERR_CUDA, "norm kernel launch: %s", cudaGetErrorString(e));
@@ -710,22 +822,24 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
     const void* d[dpk::kGemmMaxLayers];
     float* o[dpk::kGemmMaxLayers];
     float* part[dpk::kGemmMaxLayers];
+    const dpk::ConvGeom* cg[dpk::kGemmMaxLayers];
     int din[dpk::kGemmMaxLayers], dout[dpk::kGemmMaxLayers];
     uint64_t pb[dpk::kGemmMaxLayers];
     for (size_t q = 0; q < grp.size(); ++q) {
       const int r = grp[q];
       const LayerPlan& p = c->plan[layers[r]];
-      a[q] = A[r];
+      a[q] = dense_A(c, layers[r], A[r]);
       d[q] = D[r];
       o[q] = d_out[r];
       part[q] = p.split > 1 ? c->d_split + p.s_off : nullptr;
+      cg[q] = p.implicit ? &p.cg : nullptr;
       din[q] = static_cast<int>(p.d_in);
       dout[q] = static_cast<int>(p.d_out);
       pb[q] = p.p_base;
     }
     cudaError_t e = dpk::tc_launch_clipsum_batch(static_cast<int>(grp.size()), a, d, o, part, din,
                                                  dout, pb, c->d_c, c->B, c->plan[layers[grp[0]]].T,
-                                                 ep, c->d_flag, c->stream);
+                                                 ep, c->d_flag, c->stream, cg);
     grp.clear();
     return e;
   };
@@ -859,24 +973,6 @@ const char* dp_status_string(dp_status s) {
   return "DP_ERR_UNKNOWN";
 }
 
-namespace {
-dp_status conv_geom(const dp_conv2d* v, dpk::ConvGeom* g) {
-  if (!v) return fail(DP_ERR_ARG, "conv is NULL");
-  if (v->H < 1 || v->W < 1 || v->C_in < 1 || v->kh < 1 || v->kw < 1 || v->stride_h < 1 ||
-      v->stride_w < 1 || v->pad_h < 0 || v->pad_w < 0)
-    return fail(DP_ERR_SHAPE, "convolution sizes must be >= 1 and pads >= 0");
-  const int64_t hp = static_cast<int64_t>(v->H) + 2 * static_cast<int64_t>(v->pad_h);
-  const int64_t wp = static_cast<int64_t>(v->W) + 2 * static_cast<int64_t>(v->pad_w);
-  if (v->kh > hp || v->kw > wp) return fail(DP_ERR_SHAPE, "kernel larger than the padded input");
-  const int64_t ho = (hp - v->kh) / v->stride_h + 1, wo = (wp - v->kw) / v->stride_w + 1;
-  const int64_t K = static_cast<int64_t>(v->kh) * v->kw * v->C_in;
-  if (ho * wo > 0x7fffffffLL) return fail(DP_ERR_SHAPE, "H_out * W_out above 2^31 - 1");
-  if (K > kMaxDim) return fail(DP_ERR_SHAPE, "kh * kw * C_in above 2^20");
-  *g = dpk::ConvGeom{v->H, v->W, v->C_in, v->kh, v->kw, v->stride_h, v->stride_w,
-                     v->pad_h, v->pad_w, static_cast<int>(ho), static_cast<int>(wo)};
-  return DP_OK;
-}
-}  // namespace
 
 dp_status dp_conv2d_dims(const dp_conv2d* conv, int32_t* T_out, int64_t* K_out) {
   if (!T_out || !K_out) return fail(DP_ERR_ARG, "NULL output");

@@ -88,6 +88,8 @@ struct GemmArgs {
   int d_in[kGemmMaxLayers], d_out[kGemmMaxLayers];
   int n_m[kGemmMaxLayers], n_n[kGemmMaxLayers];
   int split[kGemmMaxLayers];  // example ranges per tile (1: the whole batch)
+  int conv[kGemmMaxLayers];   // 1: mapA is the NHWC input of a convolution (patch rows on the fly)
+  ConvGeom cg[kGemmMaxLayers];
   int tile_start[kGemmMaxLayers + 1];  // first work item of each layer
   int L;
   const float* c;  // clip factors [B]; nullptr: all ones (pre-scaled operand)
@@ -135,12 +137,44 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* 
   }
 }
 
+// A convolution's two A chunks of a tile: 64 channels of one kernel tap
+// each, fixed for the whole work item.  cc: first channel (C_in for a chunk
+// past K: a box wholly out of range, read as zeros); dx, dy: the tap's
+// offset from the output position, padding included.
+struct ConvTaps {
+  int cc[2], dx[2], dy[2];
+};
+
+__device__ __forceinline__ ConvTaps conv_taps(const ConvGeom& v, int m0) {
+  ConvTaps t;
+#pragma unroll
+  for (int q = 0; q < 2; ++q) {
+    const int mm = m0 + 64 * q;
+    int tap = mm / v.C_in, cc = mm - tap * v.C_in;
+    if (tap >= v.kh * v.kw) {
+      tap = 0;
+      cc = v.C_in;
+    }
+    const int ki = tap / v.kw;
+    t.cc[q] = cc;
+    t.dx[q] = (tap - ki * v.kw) - v.pad_w;
+    t.dy[q] = ki - v.pad_h;
+  }
+  return t;
+}
+
 // TMA loads of one stage: A rows m0.. (two 64-column chunks) and the D
-// columns this CTA stages, for K block kb of example ex.
-template <bool PAIR, int NB>
+// columns this CTA stages, for K block kb of example ex.  For a convolution
+// an A chunk is 64 channels of one kernel tap at 64 output positions
+// starting at output row ho0, column wo0: one 4-D box [1 image][rows]
+// [columns][64 channels] of the NHWC input at the tap's offset, whose
+// out-of-range pixels (the zero padding) read as zeros.  The producer thread
+// issues every stage, so nothing here divides.
+template <bool PAIR, int NB, bool CONV>
 __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, uint64_t* full,
                                                   bool leader, uint8_t* sa, uint8_t* sb, int m0,
-                                                  int n0, int ex, int kb) {
+                                                  int n0, int ex, int kb, const ConvTaps& ct,
+                                                  int ho0, int wo0) {
   using C = Cfg<PAIR, NB>;
   const CUtensorMap* mapA = &g.mapA[layer];
   const CUtensorMap* mapD = &g.mapD[layer];
@@ -151,7 +185,13 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
     // both CTAs' loads complete on the leader's full barrier
     const uint32_t fb = mapa_shared(smem_u32(full), 0);
     if (leader) mbar_arrive_expect_tx(full, 2 * C::STAGE_BYTES);
-    if (g.pad3d) {
+    if (CONV && g.conv[layer]) {
+      tma_load_4d_pair(mapA, fb, sa, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
+      tma_load_4d_pair(mapA, fb, sa + CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
+#pragma unroll
+      for (int q = 0; q < C::B_COLS / 64; ++q)
+        tma_load_2d_pair(mapD, fb, sb + q * CHUNK, n0 + 64 * q, drow);
+    } else if (g.pad3d) {
       tma_load_3d_pair(mapA, fb, sa, m0, trow, ex);
       tma_load_3d_pair(mapA, fb, sa + CHUNK, m0 + 64, trow, ex);
 #pragma unroll
@@ -166,7 +206,13 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
     }
   } else {
     mbar_arrive_expect_tx(full, C::STAGE_BYTES);
-    if (g.pad3d) {
+    if (CONV && g.conv[layer]) {
+      tma_load_4d(mapA, full, sa, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
+      tma_load_4d(mapA, full, sa + CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
+#pragma unroll
+      for (int q = 0; q < C::B_COLS / 64; ++q)
+        tma_load_2d(mapD, full, sb + q * CHUNK, n0 + 64 * q, drow);
+    } else if (g.pad3d) {
       tma_load_3d(mapA, full, sa, m0, trow, ex);
       tma_load_3d(mapA, full, sa + CHUNK, m0 + 64, trow, ex);
 #pragma unroll
@@ -214,7 +260,10 @@ __device__ __forceinline__ void tile_mn(int t, int n_m, int n_n, int& mt, int& n
   nt = r / gm;
 }
 
-template <bool NORM, bool PAIR, int NB>
+// CONV: some layer of the launch is a convolution read in place (the
+// producer forms its patch rows from 4-D boxes); the dense instantiations
+// carry none of that per-stage work.
+template <bool NORM, bool PAIR, int NB, bool CONV>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     k_gemm_tc(const __grid_constant__ GemmArgs g) {
   using C = Cfg<PAIR, NB>;
@@ -225,6 +274,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   __shared__ uint64_t full_bar[STAGES], empty_bar[STAGES], tfull_bar[2], tempty_bar[2], done_bar;
   __shared__ uint32_t tmem_slot;
   __shared__ int abort_flag;
+  __shared__ ConvTaps s_taps;  // the producer's current convolution taps
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t rank = PAIR ? cluster_ctarank() : 0;
@@ -283,12 +333,31 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         tile_mn(w.lt, g.n_m[l], g.n_n[l], mt, nt);
         const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
         const int n0 = nt * NB + (PAIR ? static_cast<int>(rank) * (NB / 2) : 0);
+        // convolution: the tile's taps (kept in shared memory: this warp runs
+        // on few registers), and how a K block advances the output position
+        // (whole rows when W_out divides 64, else 64 columns)
+        int rows_per_kb = 0, wout = 1;
+        if (CONV && g.conv[l]) {
+          s_taps = conv_taps(g.cg[l], m0);
+          wout = g.cg[l].W_out;
+          rows_per_kb = wout <= BK ? BK / wout : 0;
+        }
         for (int ex = w.e0; ex < w.e1; ++ex) {
+          int ho0 = 0, wo0 = 0;
           for (int kb = 0; kb < kpe; ++kb) {
             if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
             uint8_t* sa = smem + stage * C::STAGE_BYTES;
             uint8_t* sb = sa + C::A_STAGE;
-            issue_stage_loads<PAIR, NB>(g, l, &full_bar[stage], leader, sa, sb, m0, n0, ex, kb);
+            issue_stage_loads<PAIR, NB, CONV>(g, l, &full_bar[stage], leader, sa, sb, m0, n0, ex,
+                                              kb, s_taps, ho0, wo0);
+            if constexpr (CONV) {
+              if (rows_per_kb) {
+                ho0 += rows_per_kb;
+              } else if (wout > 1 && (wo0 += BK) == wout) {
+                wo0 = 0;
+                ++ho0;
+              }
+            }
             ++uses[stage];
             if (++stage == STAGES) {
               stage = 0;
@@ -529,12 +598,12 @@ bool use_pair(int64_t d_in) { return d_in > BM; }
 // Tile width: 128 columns for layers with d_out <= 128, else 256.
 int gemm_nb(int64_t d_out) { return d_out <= 128 ? 128 : BN; }
 
-template <bool NORM, bool PAIR, int NB>
+template <bool NORM, bool PAIR, int NB, bool CONV>
 cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
   using C = Cfg<PAIR, NB>;
   static bool attr_set = false;
   if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<NORM, PAIR, NB>,
+    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<NORM, PAIR, NB, CONV>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          C::SMEM_BYTES);
     if (e != cudaSuccess) return e;
@@ -542,7 +611,7 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
       // setmaxnreg moves registers within what the block was launched with:
       // the split must fit the compiled count, else the raise never returns
       cudaFuncAttributes fa{};
-      e = cudaFuncGetAttributes(&fa, k_gemm_tc<NORM, PAIR, NB>);
+      e = cudaFuncGetAttributes(&fa, k_gemm_tc<NORM, PAIR, NB, CONV>);
       if (e != cudaSuccess) return e;
       if (fa.numRegs * GEMM_THREADS < 4 * 32 * REGS_CTRL + NUM_EPI_WARPS * 32 * REGS_EPI ||
           fa.numRegs > REGS_EPI)
@@ -576,7 +645,7 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
     if (max_pairs == 0) {
       cfg.gridDim = dim3(sms);
       int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<NORM, PAIR, NB>, &cfg) != cudaSuccess ||
+      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<NORM, PAIR, NB, CONV>, &cfg) != cudaSuccess ||
           n < 1) {
         cudaGetLastError();
         n = sms / 2;
@@ -586,11 +655,11 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
     const int pairs = tiles < max_pairs ? tiles : max_pairs;
     cfg.gridDim = dim3(2 * pairs);
     note_launch();
-    return cudaLaunchKernelEx(&cfg, k_gemm_tc<NORM, PAIR, NB>, g);
+    return cudaLaunchKernelEx(&cfg, k_gemm_tc<NORM, PAIR, NB, CONV>, g);
   } else {
     const int grid = tiles < sms ? tiles : sms;
     note_launch();
-    k_gemm_tc<NORM, PAIR, NB><<<grid, GEMM_THREADS, C::SMEM_BYTES, s>>>(g);
+    k_gemm_tc<NORM, PAIR, NB, CONV><<<grid, GEMM_THREADS, C::SMEM_BYTES, s>>>(g);
     return cudaGetLastError();
   }
 }
@@ -598,8 +667,28 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
 // Maps over the caller's [B][T][d] arrays of layer slot l: 2-D [B*T, d] when
 // T is a multiple of the K block, else 3-D with each example's positions
 // padded to it.
-bool make_input_maps(const void* A, const void* D, GemmArgs& g, int l) {
+bool make_input_maps(const void* A, const void* D, GemmArgs& g, int l,
+                     const ConvGeom* conv = nullptr) {
   g.pad3d = (g.T % BK) != 0;
+  g.conv[l] = 0;
+  if (conv) {
+    // the NHWC input [B][H][W][C_in]; a box is 64 output positions of one
+    // tap: whole output rows when W_out divides 64, else a run of 64 in a row
+    if (!tc_conv_implicit_ok(*conv, g.T)) return false;
+    const ConvGeom& v = *conv;
+    g.conv[l] = 1;
+    g.cg[l] = v;
+    const uint64_t c = static_cast<uint64_t>(v.C_in);
+    const uint64_t dims[4] = {c, static_cast<uint64_t>(v.W), static_cast<uint64_t>(v.H),
+                              static_cast<uint64_t>(g.B)};
+    const uint64_t strides[3] = {c * 2, c * v.W * 2, c * v.W * v.H * 2};
+    const uint32_t rows = v.W_out <= BK ? static_cast<uint32_t>(BK / v.W_out) : 1u;
+    const uint32_t cols = v.W_out <= BK ? static_cast<uint32_t>(v.W_out) : static_cast<uint32_t>(BK);
+    const uint32_t box[4] = {64, cols, rows, 1};
+    const uint64_t rows_all = static_cast<uint64_t>(g.B) * g.T;
+    return make_tma_bf16(&g.mapA[l], A, 4, dims, strides, box) &&
+           make_map_2d(&g.mapD[l], D, g.d_out[l], rows_all, BK);
+  }
   if (g.pad3d)
     return make_map_3d(&g.mapA[l], A, g.d_in[l], g.T, g.B, BK) &&
            make_map_3d(&g.mapD[l], D, g.d_out[l], g.T, g.B, BK);
@@ -610,12 +699,19 @@ bool make_input_maps(const void* A, const void* D, GemmArgs& g, int l) {
 
 template <bool NORM>
 cudaError_t launch_any(GemmArgs& g, cudaStream_t s) {
-  // every layer of a launch shares the tile shape (use_pair, gemm_nb)
-  if (gemm_nb(g.d_out[0]) == 128)
-    return use_pair(g.d_in[0]) ? launch_gemm<NORM, true, 128>(g, s)
-                               : launch_gemm<NORM, false, 128>(g, s);
-  return use_pair(g.d_in[0]) ? launch_gemm<NORM, true, BN>(g, s)
-                             : launch_gemm<NORM, false, BN>(g, s);
+  // every layer of a launch shares the tile shape (use_pair, gemm_nb); a
+  // convolution read in place always has pairs (tc_conv_implicit_ok)
+  bool conv = false;
+  for (int l = 0; l < g.L; ++l) conv = conv || g.conv[l];
+  const bool pair = use_pair(g.d_in[0]);
+  if (conv && !pair) return cudaErrorInvalidValue;
+  if (gemm_nb(g.d_out[0]) == 128) {
+    if (conv) return launch_gemm<NORM, true, 128, true>(g, s);
+    return pair ? launch_gemm<NORM, true, 128, false>(g, s)
+                : launch_gemm<NORM, false, 128, false>(g, s);
+  }
+  if (conv) return launch_gemm<NORM, true, BN, true>(g, s);
+  return pair ? launch_gemm<NORM, true, BN, false>(g, s) : launch_gemm<NORM, false, BN, false>(g, s);
 }
 
 void set_epilogue(GemmArgs& g, const Epilogue& ep) {
@@ -749,6 +845,17 @@ int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out) {
   return static_cast<int>(best);
 }
 
+// Patch rows on the fly: 64-channel chunks never straddle a tap (C_in a
+// multiple of 64), K blocks are whole boxes of output positions (T a
+// multiple of 64, W_out dividing 64 or 64 dividing W_out), unit strides.
+bool tc_conv_implicit_ok(const ConvGeom& g, int T) {
+  if (g.C_in % 64 != 0 || T % BK != 0 || T != g.H_out * g.W_out) return false;
+  if (!use_pair(static_cast<int64_t>(g.kh) * g.kw * g.C_in)) return false;
+  if (g.stride_h != 1 || g.stride_w != 1) return false;
+  if (g.W_out <= BK) return BK % g.W_out == 0;
+  return g.W_out % BK == 0;
+}
+
 // Direct path: T a multiple of 64, or T >= 32 (3-D padding wastes at most half).
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out) {
   return (T % BK == 0 || T >= 32) && d_in % 8 == 0 && d_out % 8 == 0 && tma_encode_available();
@@ -806,7 +913,8 @@ int tc_mat_parts(int64_t d_in, int64_t d_out) {
 }
 
 cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d_in, int d_out,
-                               float* part, int NP, int row0, int* err, cudaStream_t s) {
+                               float* part, int NP, int row0, int* err, cudaStream_t s,
+                               const ConvGeom* conv) {
   GemmArgs g{};
   g.L = 1;
   g.part = part;
@@ -818,14 +926,15 @@ cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d
   g.split[0] = tc_gemm_split(B, T, d_in, d_out);
   g.NP = NP;
   g.row0 = row0;
-  if (!make_input_maps(A, D, g, 0)) return cudaErrorInvalidValue;
+  if (!make_input_maps(A, D, g, 0, conv)) return cudaErrorInvalidValue;
   return launch_any<true>(g, s);
 }
 
 cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
                                     float* const* out, float* const* part, const int* d_in,
                                     const int* d_out, const uint64_t* p_base, const float* c,
-                                    int B, int T, const Epilogue& ep, int* err, cudaStream_t s) {
+                                    int B, int T, const Epilogue& ep, int* err, cudaStream_t s,
+                                    const ConvGeom* const* conv) {
   if (L < 1 || L > kGemmMaxLayers) return cudaErrorInvalidValue;
   const bool pair = use_pair(d_in[0]);
   const int nb = gemm_nb(d_out[0]);
@@ -846,7 +955,7 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
     g.out[l] = out[l];
     g.p_base[l] = p_base[l];
     g.split[l] = tc_gemm_split(B, T, d_in[l], d_out[l]);
-    if (!make_input_maps(A[l], D[l], g, l)) return cudaErrorInvalidValue;
+    if (!make_input_maps(A[l], D[l], g, l, conv ? conv[l] : nullptr)) return cudaErrorInvalidValue;
     if (g.split[l] > 1) {
       if (!part || !part[l] || (reinterpret_cast<uintptr_t>(part[l]) & 15) != 0 ||
           !make_tma_f32_split(&g.mapO[l], part[l], g.split[l], d_in[l], d_out[l]))
@@ -877,9 +986,9 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
 
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
                               int d_in, int d_out, float* out, float* part, const Epilogue& ep,
-                              int* err, cudaStream_t s) {
+                              int* err, cudaStream_t s, const ConvGeom* conv) {
   return tc_launch_clipsum_batch(1, &A, &D, &out, &part, &d_in, &d_out, &ep.p_base, c, B, T, ep,
-                                 err, s);
+                                 err, s, &conv);
 }
 
 bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_out_a, int64_t d_in_b, int64_t d_out_b) {

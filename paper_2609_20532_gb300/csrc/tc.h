@@ -32,17 +32,22 @@ constexpr int kGemmMaxLayers = 8;
 constexpr int kGemmMaxSplit = 256;
 int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out);
 bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_out_a, int64_t d_in_b, int64_t d_out_b);
+// conv (per layer, NULL for a dense layer): A is then the NHWC input and the
+// kernels read its patch rows directly (tc_conv_implicit_ok must hold).
 cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
                                     float* const* out, float* const* part, const int* d_in,
                                     const int* d_out, const uint64_t* p_base, const float* c,
-                                    int B, int T, const Epilogue& ep, int* err, cudaStream_t s);
+                                    int B, int T, const Epilogue& ep, int* err, cudaStream_t s,
+                                    const ConvGeom* const* conv = nullptr);
+bool tc_conv_implicit_ok(const ConvGeom& g, int T);
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out);
 int tc_mat_parts(int64_t d_in, int64_t d_out);
 cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d_in, int d_out,
-                               float* part, int NP, int row0, int* err, cudaStream_t s);
+                               float* part, int NP, int row0, int* err, cudaStream_t s,
+                               const ConvGeom* conv = nullptr);
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
                               int d_in, int d_out, float* out, float* part, const Epilogue& ep,
-                              int* err, cudaStream_t s);
+                              int* err, cudaStream_t s, const ConvGeom* conv = nullptr);
 
 // Clipped sum for short examples (T < 32): c_i folded into a bf16 hi+lo
 // split of A in scratch (tc_prescaled_scratch_bytes), then one plain GEMM.
@@ -56,9 +61,11 @@ cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const floa
 // Host helpers shared by the tensor-core launchers (tc_host.cu).
 bool tma_encode_available();
 // bf16 tensor map, 128-byte swizzle, zero fill out of bounds; dims[0] innermost,
-// strides_bytes[r] is the byte stride of dimension r+1.
+// strides_bytes[r] is the byte stride of dimension r+1; estrides (NULL: all 1)
+// the traversal strides.
 bool make_tma_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
-                   const uint64_t* strides_bytes, const uint32_t* box);
+                   const uint64_t* strides_bytes, const uint32_t* box,
+                   const uint32_t* estrides = nullptr);
 // fp32 output map over [rows][cols], box 32 x 32 (128-byte rows), 128-byte swizzle.
 bool make_tma_f32_out(CUtensorMap* m, void* base, uint64_t rows, uint64_t cols);
 // fp32 map over [split][rows][cols] partial sums, box 32 x 32 x 1, 128-byte swizzle.

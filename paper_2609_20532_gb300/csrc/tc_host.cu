@@ -38,7 +38,7 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 bool tma_encode_available() { return encode_fn() != nullptr; }
 
 bool make_tma_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* dims,
-                   const uint64_t* strides_bytes, const uint32_t* box) {
+                   const uint64_t* strides_bytes, const uint32_t* box, const uint32_t* estrides) {
   auto fn = encode_fn();
   if (!fn || rank < 1 || rank > 5) return false;
   cuuint64_t d[5], st[4];
@@ -46,7 +46,7 @@ bool make_tma_bf16(CUtensorMap* m, const void* base, int rank, const uint64_t* d
   for (int r = 0; r < rank; ++r) {
     d[r] = dims[r];
     b[r] = box[r];
-    es[r] = 1;
+    es[r] = estrides ? estrides[r] : 1;
     if (r + 1 < rank) st[r] = strides_bytes[r];
   }
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), d, st, b, es,

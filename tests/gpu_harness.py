@@ -29,14 +29,16 @@ def conv_struct(w: W.Workload, l: int):
     return dp.make_conv(H, W_, cin, kh, kw, (st, st), (pd, pd))
 
 
-def device_inputs(w: W.Workload, layers, dev="cuda:0"):
-    """A and D of every layer on the device; a convolution's A becomes its
-    patch rows through dp_conv2d_unfold (the library's kernel)."""
+def device_inputs(w: W.Workload, layers, dev="cuda:0", conv_mode="explicit"):
+    """A and D of every layer on the device.  conv_mode "explicit": a
+    convolution's A becomes its patch rows through dp_conv2d_unfold; "library":
+    it stays the NHWC input and the step forms the patch rows itself (the
+    layer is declared DP_LAYER_CONV2D, see conv_structs)."""
     Ad, Dd = [], []
     for l, (A, D) in enumerate(layers):
         x = A.to(dev)
         conv = conv_struct(w, l)
-        if conv is not None:
+        if conv is not None and conv_mode == "explicit":
             T, K = dp.dp_conv2d_dims(conv)
             a = torch.empty((w.B, T, K), dtype=x.dtype, device=dev)
             dp.dp_conv2d_unfold(conv, w.B, w.dtype, x, a)
@@ -64,20 +66,28 @@ def oracle_grads(w: W.Workload, layers):
     return G
 
 
+def conv_structs(w: W.Workload, conv_mode: str):
+    """make_config's convs argument: the geometries in "library" mode."""
+    if conv_mode != "library" or not w.convs:
+        return None
+    return [conv_struct(w, l) for l in range(len(w.layers))]
+
+
 def run_gpu_step(w: W.Workload, layers, seed=0, step=0, out_scale=1.0, flags=0,
-                 norm_mode=dp.DP_NORM_AUTO, audit=True):
+                 norm_mode=dp.DP_NORM_AUTO, audit=True, conv_mode="explicit"):
     """Run norms -> clip -> clipped sum (+noise) on cuda:0.
 
     layers: list of (A, D) CPU tensors.  Returns dict with n [L,B], s, c
     (from the audit records of every example), out (list of fp32 numpy) and
     the chosen norm modes."""
     dev = torch.device("cuda:0")
-    Ad, Dd = device_inputs(w, layers, dev)
+    Ad, Dd = device_inputs(w, layers, dev, conv_mode)
     outs = [torch.zeros(i, o, device=dev, dtype=torch.float32) for i, o in w.layers]
     s_dev = torch.empty(w.B, device=dev)
     c_dev = torch.empty(w.B, device=dev)
     cfg = dp.make_config(w.specs, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=out_scale,
-                         seed=seed, step=step, norm_mode=norm_mode, audit_capacity=w.B)
+                         seed=seed, step=step, norm_mode=norm_mode, audit_capacity=w.B,
+                         convs=conv_structs(w, conv_mode))
     ctx = dp.dp_step_init(cfg)
     try:
         for l in range(len(layers)):

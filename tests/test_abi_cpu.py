@@ -125,3 +125,30 @@ def test_conv2d_dims_on_host(L):
         with pytest.raises(dp.DPError) as ei:
             dp.dp_conv2d_dims(bad)
         assert ei.value.status == 2
+
+
+def test_conv_layer_config_checked_on_host(L):
+    """DP_LAYER_CONV2D layers: geometry present and consistent with d_in, T."""
+    cv = dp.make_conv(8, 8, 16, 3, 3, (1, 1), (1, 1))      # T = 64, K = 144
+    ok = dp.make_config([(144, 32)], 2, 1, "bf16", 1.0, 1.0, convs=[cv])
+    assert ok.layers[0].kind == dp.DP_LAYER_CONV2D
+    for layers, convs, status in [
+        ([(144, 32)], None, None),                 # dense: fine without geometry
+        ([(143, 32)], [cv], 2),                    # d_in is not kh*kw*C_in
+        ([(144, 32, 63)], [cv], 2),                # T is not H_out*W_out
+        ([(144, 32)], [dp.make_conv(2, 2, 16, 5, 5)], 2),
+    ]:
+        cfg = dp.make_config(layers, 2, 1, "bf16", 1.0, 1.0, convs=convs)
+        st, h = _init_status(L, cfg)
+        if status is None:
+            assert st in (0, 6, 9), st   # no GPU here: the host checks passed
+            if h:
+                L.dp_step_destroy(h)
+        else:
+            assert st == status and not h
+    bad = dp.make_config([(144, 32)], 2, 1, "bf16", 1.0, 1.0)
+    bad.layers[0].kind = 7
+    assert _init_status(L, bad)[0] == 1
+    nogeom = dp.make_config([(144, 32)], 2, 1, "bf16", 1.0, 1.0)
+    nogeom.layers[0].kind = dp.DP_LAYER_CONV2D
+    assert _init_status(L, nogeom)[0] == 1

@@ -91,11 +91,21 @@ CONV_NETS = [
       (16, 16, 16, 64, 1, 1, 2, 0)],    # 1x1 shortcut: thin, warp MMAs
      [(64, 10, 1), (1, 10, 1)], 8, "bf16"),
     ([(6, 6, 4, 8, 3, 3, 1, 1), (6, 6, 8, 8, 3, 3, 2, 1)], [(8, 3, 1)], 5, "f32"),
+    # channels in multiples of 64: patch rows read in place by the tensor-core
+    # kernels (W_out = 16, 8 and 128), a 1x1 identity, a strided convolution
+    # (patch rows in scratch)
+    ([(16, 16, 64, 64, 3, 3, 1, 1),       # T = 256, W_out = 16
+      (8, 8, 128, 128, 3, 3, 1, 1),       # T = 64, W_out = 8
+      (4, 128, 64, 64, 3, 3, 1, 1),       # W_out = 128: boxes are half rows
+      (16, 16, 64, 128, 1, 1, 1, 0),      # 1x1 stride 1: the input is the patch rows
+      (16, 16, 64, 128, 3, 3, 2, 1)],     # stride 2
+     [], 6, "bf16"),
 ]
 
 
+@pytest.mark.parametrize("conv_mode", ["explicit", "library"])
 @pytest.mark.parametrize("case", range(len(CONV_NETS)))
-def test_conv_net_step_matches_oracle(case):
+def test_conv_net_step_matches_oracle(case, conv_mode):
     convs, head, B, dtype = CONV_NETS[case]
     dists = ("normal",) + ("relu_normal",) * (len(convs) - 1) + ("normal",) * len(head)
     if head and head[-1][0] == 1:
@@ -103,10 +113,42 @@ def test_conv_net_step_matches_oracle(case):
     w = W.custom_conv(f"convnet{case}", convs, B, dtype, C=0.5, sigma=0.8, d_std=0.05,
                       wid=950 + case, a_dist=dists, head=head)
     layers = W.make_inputs(w)
-    res = run_gpu_step(w, layers, seed=3, step=11, out_scale=1.0 / B)
+    res = run_gpu_step(w, layers, seed=3, step=11, out_scale=1.0 / B, conv_mode=conv_mode)
     ref = oracle_conv_step(w, layers, seed=3, step=11, out_scale=1.0 / B)
     ref["out"] = [o.reshape(i, d) for o, (i, d) in zip(ref["out"], w.layers)]
     assert_step_matches(res, ref, dtype)
+
+
+@pytest.mark.parametrize("conv,launches", [
+    ((16, 16, 64, 64, 3, 3, 1, 1), 1),    # read in place: the norm kernel alone
+    ((16, 16, 64, 128, 3, 3, 2, 1), 2),   # strided: unfold into scratch, then the norm
+    ((16, 16, 64, 128, 1, 1, 1, 0), 1),   # 1x1 identity: the input is the patch rows
+])
+def test_library_conv_paths_and_launches(conv, launches):
+    """A DP_LAYER_CONV2D layer: how many kernels its norm call issues shows
+    whether its patch rows are read in place, and its outputs match the
+    caller-unfolded dense layer within the bf16 tolerance."""
+    w = W.custom_conv("libconv", [conv], 4, "bf16", C=0.5, sigma=0.5, d_std=0.05, wid=970,
+                      a_dist=("relu_normal",))
+    layers = W.make_inputs(w)
+    H, W_, cin, cout, kh, kw, st, pd = conv
+    cv = dp.make_conv(H, W_, cin, kh, kw, (st, st), (pd, pd))
+    cfg = dp.make_config(w.specs, w.B, w.T, "bf16", w.C, w.sigma, audit_capacity=w.B, convs=[cv])
+    ctx = dp.dp_step_init(cfg)
+    try:
+        x, d = layers[0][0].to(DEV), layers[0][1].to(DEV)
+        n0 = dp.dp_kernel_launches()
+        dp.dp_layer_norms(ctx, 0, x, d)
+        assert dp.dp_kernel_launches() - n0 == launches
+        dp.dp_clip_factors(ctx)
+        out = torch.zeros(w.layers[0], device=DEV)
+        dp.dp_clipped_sum_noise(ctx, 0, x, d, out, dp.DP_NO_NOISE)
+        recs = dp.dp_audit_emit(ctx, range(w.B), 1)
+    finally:
+        dp.dp_step_destroy(ctx)
+    ref = oracle_conv_step(w, layers, noise=False)
+    assert rel_err_elementwise(recs["layer_sqnorm"].astype(np.float64).T, ref["n"]) <= TOL["bf16"]
+    assert rel_err_normwise(out.cpu().numpy(), ref["out"][0].reshape(w.layers[0])) <= TOL["bf16"]
 
 
 def test_wrn16_4_full_size_sampled():
@@ -118,7 +160,7 @@ def test_wrn16_4_full_size_sampled():
     w = W.get("wrn16_4_cifar10_bf16")
     layers = W.make_inputs(w)
     tol = TOL[w.dtype]
-    res = run_gpu_step(w, layers, seed=1, step=5, out_scale=1.0 / w.B)
+    res = run_gpu_step(w, layers, seed=1, step=5, out_scale=1.0 / w.B, conv_mode="library")
     rng = np.random.default_rng(77)
     ex = np.sort(rng.choice(w.B, size=3, replace=False))
     sub = [(A[ex], D[ex]) for A, D in layers]
@@ -134,7 +176,7 @@ def test_wrn16_4_full_size_sampled():
     # nothing clipped: the commitment is the plain sum over the batch
     wbig = W.Workload(w.name, w.wid, w.layers, w.B, w.T, w.dtype, w.a_dist, w.a_std, w.d_std,
                       1e30, w.sigma, layer_T=w.layer_T, convs=w.convs)
-    big = run_gpu_step(wbig, layers, flags=dp.DP_NO_NOISE, audit=False)
+    big = run_gpu_step(wbig, layers, flags=dp.DP_NO_NOISE, audit=False, conv_mode="library")
     assert np.all(big["c"] == 1.0)
     for l, (A, D) in enumerate(layers):
         d_in, d_out = w.layers[l]
