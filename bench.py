@@ -150,6 +150,32 @@ def _traffic(kernel_key, units, path=None):
     return d["captured_dram_bytes"] * units / d["captured_units"]
 
 
+def _stage_ms(fn, stream, args, use_graph):
+    """Median device time of one call of fn: captured in a CUDA graph and
+    replayed back to back with an event pair around each replay (so host
+    work stays out), or, in eager mode, timed call by call."""
+    import torch
+    reps = args.warmup + args.steps
+    if use_graph:
+        g_ = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_, stream=stream):
+            fn()
+        torch.cuda.synchronize()
+        run = g_.replay
+    else:
+        run = fn
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(reps)]
+    for a, b in evs:
+        a.record(stream)
+        run()
+        b.record(stream)
+        if not use_graph:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
+    return statistics.median(a.elapsed_time(b) for a, b in evs[args.warmup:])
+
+
 def _data_desc(w):
     """The input recipe of a workload in words (seeded, synthetic)."""
     names = {"normal": f"N(0,{w.a_std ** 2:g})", "uniform": "U[0,1)",
@@ -476,38 +502,29 @@ def run_ours(args, rank, world, local_rank):
         conv_dom = max(("layer_norms", "clipsum_gemm"), key=lambda n: kernels[n]["ms_per_step"])
 
     # standalone noise add over every layer (the DP_NOISE_ONLY call that adds
-    # the released seed's noise to a committed sum): 8 bytes per parameter
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    nts = []
-    for r in range(args.warmup + args.steps):
-        e0.record(stream)
-        for l in range(L):
-            dp.dp_clipped_sum_noise(ctx, l, None, None, outs[l], dp.DP_NOISE_ONLY)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        if r >= args.warmup:
-            nts.append(e0.elapsed_time(e1))
-    noise_ms = statistics.median(nts)
+    # the released seed's noise to a committed sum): 8 bytes per parameter,
+    # all layers in one batched call
+    n_noise0 = dp.dp_kernel_launches()
+    dp.dp_clipped_sum_noise_batch(ctx, list(range(L)), None, None, outs, dp.DP_NOISE_ONLY)
+    noise_launches = dp.dp_kernel_launches() - n_noise0
+    noise_ms = _stage_ms(lambda: dp.dp_clipped_sum_noise_batch(ctx, list(range(L)), None, None,
+                                                               outs, dp.DP_NOISE_ONLY),
+                         stream, args, graph is not None)
     noise_gbs = 8.0 * w.n_params / (noise_ms * 1e-3) / 1e9
     kernels["noise_add"] = {"ms_per_step": noise_ms, "gbs": noise_gbs,
-                            "frac_hbm": noise_gbs / peaks["hbm_gbs"], "launches": L,
+                            "frac_hbm": noise_gbs / peaks["hbm_gbs"], "launches": noise_launches,
                             "bytes": 8 * w.n_params}
 
     # the released update: noisy gradient + AdamW on theta, m, v in place
     # (read g, theta, m, v; write theta, m, v): 28 bytes per parameter
     opt = [[torch.zeros(i, o, device=dev) for i, o in w.layers] for _ in range(3)]
-    ats = []
-    for r in range(args.warmup + args.steps):
-        e0.record(stream)
+
+    def adamw_all():
         for l in range(L):
             dp.dp_noise_adamw(ctx, l, outs[l], opt[0][l], opt[1][l], opt[2][l], 1e-4, 0.9,
-                              0.999, 1e-8, 0.01, r + 1)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        if r >= args.warmup:
-            ats.append(e0.elapsed_time(e1))
+                              0.999, 1e-8, 0.01, 1)
+    adamw_ms = _stage_ms(adamw_all, stream, args, graph is not None)
     del opt
-    adamw_ms = statistics.median(ats)
     adamw_gbs = 28.0 * w.n_params / (adamw_ms * 1e-3) / 1e9
     kernels["noise_adamw"] = {"ms_per_step": adamw_ms, "gbs": adamw_gbs,
                               "frac_hbm": adamw_gbs / peaks["hbm_gbs"], "launches": L,

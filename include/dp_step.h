@@ -239,7 +239,9 @@ dp_status dp_clipped_sum_noise(dp_ctx* ctx, int32_t layer, const void* A, const 
  * layer indices, each at most once, and their A, D and d_out pointers; A
  * and D may be NULL with DP_NOISE_ONLY).  Equivalent to dp_clipped_sum_noise
  * on each; tensor-core layers share kernel launches, so the last round of
- * output tiles of one layer overlaps the next layer's.  Errors: as
+ * output tiles of one layer overlaps the next layer's, and with
+ * DP_NOISE_ONLY every listed layer's noise is added in one launch (per 32
+ * layers).  Errors: as
  * dp_clipped_sum_noise; nothing is launched if any argument is invalid. */
 dp_status dp_clipped_sum_noise_batch(dp_ctx* ctx, int32_t n, const int32_t* layers,
                                      const void* const* A, const void* const* D,

@@ -561,9 +561,16 @@ cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const vo
                                float* d_out, uint32_t flags) {
   const LayerPlan& p = c->plan[layer];
   const dpk::Epilogue ep = make_epilogue(c, flags, p.p_base);
-  if (flags & DP_NOISE_ONLY)
-    return dpk::launch_noise_add(d_out, p.d_in * p.d_out, p.p_base, c->d_key,
-                                 c->out_scale * ep.sigmaC, c->stream);
+  if (flags & DP_NOISE_ONLY) {
+    dpk::NoiseAddBatch nb{};
+    nb.key = c->d_key;
+    nb.scale = c->out_scale * ep.sigmaC;
+    nb.out[0] = d_out;
+    nb.n[0] = p.d_in * p.d_out;
+    nb.p_base[0] = p.p_base;
+    nb.L = 1;
+    return dpk::launch_noise_add(nb, c->stream);
+  }
   if (p.pergrad) {
     dpk::PerGradSumBatch g = pergrad_sum_batch(c, flags);
     fill_pergrad_sum(c, layer, d_out, g.l[0]);
@@ -805,6 +812,24 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
   // kGemmMaxLayers each); every other layer gets its own kernel.
   std::vector<int> grp;
   dpk::Epilogue ep = make_epilogue(c, flags, 0);
+  // noise only: every listed layer in one launch (up to kNoiseMaxLayers each)
+  if (flags & DP_NOISE_ONLY) {
+    dpk::NoiseAddBatch nb{};
+    nb.key = c->d_key;
+    nb.scale = c->out_scale * (c->sigma * c->C);
+    for (int r = 0; r < n; ++r) {
+      const LayerPlan& p = c->plan[layers[r]];
+      nb.out[nb.L] = d_out[r];
+      nb.n[nb.L] = p.d_in * p.d_out;
+      nb.p_base[nb.L] = p.p_base;
+      if (++nb.L == dpk::kNoiseMaxLayers || r == n - 1) {
+        cudaError_t e = dpk::launch_noise_add(nb, c->stream);
+        if (e != cudaSuccess) return fail(DP_ERR_CUDA, "noise kernel: %s", cudaGetErrorString(e));
+        nb.L = 0;
+      }
+    }
+    return DP_OK;
+  }
   // thin layers: one summing launch over their stored per-example gradients
   std::vector<int> thin;
   auto flush_thin = [&]() -> cudaError_t {

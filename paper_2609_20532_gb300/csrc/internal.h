@@ -40,9 +40,21 @@ cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_np
 cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float* c, int B, int T,
                              int d_in, int d_out, float* out, const Epilogue& ep, cudaStream_t s);
 
-// ---- standalone noise add: out[e] += scale * z_{p_base + e}, e < n ----
-cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, const uint64_t* key,
-                             float scale, cudaStream_t s);
+// ---- standalone noise add: out_l[e] += scale * z_{p_base_l + e}, e < n_l ----
+// One launch serves up to kNoiseMaxLayers layers; each block takes a
+// contiguous chunk of kNoiseChunk Philox quads of one layer.
+constexpr int kNoiseMaxLayers = 32;
+constexpr int kNoiseChunk = 4096;
+struct NoiseAddBatch {
+  float* out[kNoiseMaxLayers];
+  int64_t n[kNoiseMaxLayers];
+  uint64_t p_base[kNoiseMaxLayers];
+  int64_t block0[kNoiseMaxLayers + 1];  // first block of each layer (set by the launcher)
+  const uint64_t* key;
+  float scale;
+  int L;
+};
+cudaError_t launch_noise_add(NoiseAddBatch& b, cudaStream_t s);
 
 // ---- thin layers: per-example gradients stored by the norm pass ----
 constexpr int kThinMax = 32;           // widest narrow side of a thin layer

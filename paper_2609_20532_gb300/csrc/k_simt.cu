@@ -282,46 +282,55 @@ __global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
 // ---------------------------------------------------------------------------
 // Standalone noise add: out[e] += scale * z_{p_base + e}
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) k_noise_add(float* __restrict__ out, int64_t n,
-                                                   uint64_t p_base,
-                                                   const uint64_t* __restrict__ key, float scale) {
-  const uint64_t seed = key[0], step = key[1];
-  // quads that overlap [p_base, p_base + n)
-  const uint64_t q_first = p_base >> 2;
-  const uint64_t q_last = (p_base + n - 1) >> 2;
-  const int64_t nq = static_cast<int64_t>(q_last - q_first + 1);
-  const bool vec = ((p_base & 3) == 0) && ((reinterpret_cast<uintptr_t>(out) & 15) == 0);
-  // Two quads per iteration, a grid-stride apart: two independent Philox /
-  // Box-Muller chains give the scheduler instruction-level parallelism.
-  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < nq;
-       g += 2 * stride) {
-    const bool has_b = g + stride < nq;
-    const float4 za = gauss_quad(seed, step, q_first + g);
-    const float4 zb = gauss_quad(seed, step, q_first + (has_b ? g + stride : g));
+// out[e] += scale * z for the four parameters of quad q (e0 = 4q - p_base,
+// possibly negative for the first quad of an unaligned layer).
+__device__ __forceinline__ void noise_store(float* __restrict__ out, int64_t e0, int64_t n,
+                                            bool vec, float scale, float4 z) {
+  if (vec && e0 + 3 < n) {
+    float4* o = reinterpret_cast<float4*>(out + e0);
+    float4 v = *o;
+    v.x = fmaf(scale, z.x, v.x);
+    v.y = fmaf(scale, z.y, v.y);
+    v.z = fmaf(scale, z.z, v.z);
+    v.w = fmaf(scale, z.w, v.w);
+    *o = v;
+  } else {
+    const float zv[4] = {z.x, z.y, z.z, z.w};
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      if (h == 1 && !has_b) break;
-      const uint64_t q = q_first + g + h * stride;
-      const float4 z = h == 0 ? za : zb;
-      const int64_t e0 = static_cast<int64_t>(4 * q) - static_cast<int64_t>(p_base);
-      if (vec && e0 + 3 < n) {
-        float4* o = reinterpret_cast<float4*>(out + e0);
-        float4 v = *o;
-        v.x = fmaf(scale, z.x, v.x);
-        v.y = fmaf(scale, z.y, v.y);
-        v.z = fmaf(scale, z.z, v.z);
-        v.w = fmaf(scale, z.w, v.w);
-        *o = v;
-      } else {
-        const float zv[4] = {z.x, z.y, z.z, z.w};
-#pragma unroll
-        for (int w = 0; w < 4; ++w) {
-          const int64_t e = e0 + w;
-          if (e >= 0 && e < n) out[e] = fmaf(scale, zv[w], out[e]);
-        }
-      }
+    for (int w = 0; w < 4; ++w) {
+      const int64_t e = e0 + w;
+      if (e >= 0 && e < n) out[e] = fmaf(scale, zv[w], out[e]);
     }
+  }
+}
+
+// Each block adds the noise of one contiguous chunk of kNoiseChunk quads of
+// one layer (the quads that overlap [p_base, p_base + n)).  Threads take two
+// quads 256 apart per iteration: two independent Philox / Box-Muller chains
+// give the scheduler instruction-level parallelism, and the chunk keeps the
+// index arithmetic in 32 bits.
+__global__ void __launch_bounds__(256) k_noise_add(const __grid_constant__ NoiseAddBatch b) {
+  int l = 0;
+  while (l + 1 < b.L && static_cast<int64_t>(blockIdx.x) >= b.block0[l + 1]) ++l;
+  const uint64_t seed = b.key[0], step = b.key[1];
+  float* __restrict__ out = b.out[l];
+  const int64_t n = b.n[l];
+  const uint64_t p_base = b.p_base[l];
+  const uint64_t q_first = p_base >> 2;
+  const int64_t nq = static_cast<int64_t>(((p_base + n - 1) >> 2) - q_first + 1);
+  const int64_t c0 = (static_cast<int64_t>(blockIdx.x) - b.block0[l]) * kNoiseChunk;
+  const int64_t rem = nq - c0;
+  const int cnt = rem < kNoiseChunk ? static_cast<int>(rem) : kNoiseChunk;
+  const uint64_t q0 = q_first + c0;
+  const int64_t e_base = static_cast<int64_t>(4 * q0) - static_cast<int64_t>(p_base);
+  const bool vec = (p_base & 3) == 0;
+  for (int j = threadIdx.x; j < cnt; j += 512) {
+    const bool has_b = j + 256 < cnt;
+    const int jb = has_b ? j + 256 : j;
+    const float4 za = gauss_quad(seed, step, q0 + j);
+    const float4 zb = gauss_quad(seed, step, q0 + jb);
+    noise_store(out, e_base + 4 * j, n, vec, b.scale, za);
+    if (has_b) noise_store(out, e_base + 4 * jb, n, vec, b.scale, zb);
   }
 }
 
@@ -493,12 +502,20 @@ cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float
   return cudaGetLastError();
 }
 
-cudaError_t launch_noise_add(float* out, int64_t n, uint64_t p_base, const uint64_t* key,
-                             float scale, cudaStream_t s) {
-  if (n <= 0) return cudaSuccess;
-  const int64_t nq = static_cast<int64_t>(((p_base + n - 1) >> 2) - (p_base >> 2) + 1);
+cudaError_t launch_noise_add(NoiseAddBatch& b, cudaStream_t s) {
+  int64_t blocks = 0;
+  for (int l = 0; l < b.L; ++l) {
+    b.block0[l] = blocks;
+    if (b.n[l] <= 0) continue;
+    const int64_t nq =
+        static_cast<int64_t>(((b.p_base[l] + b.n[l] - 1) >> 2) - (b.p_base[l] >> 2) + 1);
+    blocks += (nq + kNoiseChunk - 1) / kNoiseChunk;
+  }
+  b.block0[b.L] = blocks;
+  if (blocks == 0) return cudaSuccess;
+  if (blocks > 0x7FFFFFFF) return cudaErrorInvalidValue;
   note_launch();
-  k_noise_add<<<grid_for(nq, 256), 256, 0, s>>>(out, n, p_base, key, scale);
+  k_noise_add<<<static_cast<unsigned>(blocks), 256, 0, s>>>(b);
   return cudaGetLastError();
 }
 

@@ -387,6 +387,44 @@ def test_noise_statistics_on_device():
     assert abs(x.var() / sd ** 2 - 1) <= 5 * math.sqrt(2 / n)
 
 
+def test_noise_only_batch_one_launch():
+    """DP_NOISE_ONLY over several layers in one batched call: one launch, the
+    same bits as per-layer calls, and scale * z of the oracle to 1e-6.  The
+    layer sizes are not multiples of 4, so most layers start inside a Philox
+    quad, and the largest spans several 4096-quad blocks with a ragged end."""
+    shapes = [(3, 5), (64, 33), (7, 1), (300, 257), (1, 3), (128, 128)]
+    w = W.custom("noise_batch", shapes, 2, 1, "f32", C=0.7, sigma=1.3, wid=611)
+    dev = torch.device(DEV)
+    scale = 0.25
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=scale,
+                         seed=(1 << 63) + 5, step=11)
+    ctx = dp.dp_step_init(cfg)
+    g = torch.Generator().manual_seed(3)
+    init = [torch.randn(i, o, generator=g) for i, o in shapes]
+    one = [x.clone().to(dev) for x in init]
+    per = [x.clone().to(dev) for x in init]
+    zero = [torch.zeros(i, o, device=dev) for i, o in shapes]
+    try:
+        n0 = dp.dp_kernel_launches()
+        dp.dp_clipped_sum_noise_batch(ctx, list(range(len(shapes))), None, None, one,
+                                      dp.DP_NOISE_ONLY)
+        assert dp.dp_kernel_launches() - n0 == 1
+        for l in range(len(shapes)):
+            dp.dp_clipped_sum_noise(ctx, l, None, None, per[l], dp.DP_NOISE_ONLY)
+        # listed out of order: each layer still takes its own global indices
+        dp.dp_clipped_sum_noise_batch(ctx, list(range(len(shapes)))[::-1], None, None,
+                                      zero[::-1], dp.DP_NOISE_ONLY)
+    finally:
+        dp.dp_step_destroy(ctx)
+    torch.cuda.synchronize()
+    for a, b in zip(one, per):
+        assert torch.equal(a, b)
+    z = O.gaussian_noise((1 << 63) + 5, 11, 0, sum(i * o for i, o in shapes))
+    want = z * (scale * float(np.float32(w.sigma)) * float(np.float32(w.C)))
+    got = np.concatenate([x.double().cpu().numpy().ravel() for x in zero])
+    assert rel_err_elementwise(got, want) <= 1e-6
+
+
 # ---------------------------------------------------------------------------
 # tensor-core paths: ragged tiles, persistence across many tiles, both norms
 # ---------------------------------------------------------------------------
