@@ -151,11 +151,10 @@ def _traffic(kernel_key, units, path=None):
 
 
 def _stage_ms(fn, stream, args, use_graph):
-    """Median device time of one call of fn: captured in a CUDA graph and
-    replayed back to back with an event pair around each replay (so host
-    work stays out), or, in eager mode, timed call by call."""
+    """Device time of one call of fn: captured in a CUDA graph (or, in eager
+    mode, called directly), run W times untimed and then K times back to
+    back between two events on the stream; returns the mean over the K."""
     import torch
-    reps = args.warmup + args.steps
     if use_graph:
         g_ = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g_, stream=stream):
@@ -164,16 +163,15 @@ def _stage_ms(fn, stream, args, use_graph):
         run = g_.replay
     else:
         run = fn
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(reps)]
-    for a, b in evs:
-        a.record(stream)
+    for _ in range(args.warmup):
         run()
-        b.record(stream)
-        if not use_graph:
-            torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(args.steps):
+        run()
+    b.record(stream)
     torch.cuda.synchronize()
-    return statistics.median(a.elapsed_time(b) for a, b in evs[args.warmup:])
+    return a.elapsed_time(b) / args.steps
 
 
 def _data_desc(w):
@@ -504,6 +502,12 @@ def run_ours(args, rank, world, local_rank):
     # standalone noise add over every layer (the DP_NOISE_ONLY call that adds
     # the released seed's noise to a committed sum): 8 bytes per parameter,
     # all layers in one batched call
+    # The standalone kernels are timed alone: after the GEMM-heavy loops
+    # above the SM clock sits below its maximum for about a second (the
+    # noise add measured 0.28 ms right after 1 s of GEMM launches against
+    # 0.24 ms on an idle GPU), so the GPU idles for 1 s first.
+    torch.cuda.synchronize()
+    time.sleep(1.0)
     n_noise0 = dp.dp_kernel_launches()
     dp.dp_clipped_sum_noise_batch(ctx, list(range(L)), None, None, outs, dp.DP_NOISE_ONLY)
     noise_launches = dp.dp_kernel_launches() - n_noise0
