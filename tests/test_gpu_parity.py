@@ -495,6 +495,21 @@ def test_workload_paths_use_tensor_cores():
             assert p == ((2, 0) if is_thin(i, o, w.T, w.dtype) else (expect, expect)), (name, paths)
 
 
+@pytest.mark.parametrize("T", [200, 300, 450, 512, 640, 800, 1000, 1100, 2000])
+def test_gram_strips_cover_every_block_pair(T):
+    """Tensor-core Gram norms at 2 to 16 blocks of 128 positions: the strips
+    must cover every block pair of the upper triangle once (diagonal pairs
+    weighted 1, the others 2), with ragged last blocks."""
+    shapes = [(64, 72), (136, 32)]
+    w = W.custom(f"gram{T}", shapes, 2, T, "bf16", C=1e6, sigma=0.0, wid=960 + T % 97)
+    layers = W.make_inputs(w, seed=1)
+    res = run_gpu_step(w, layers, norm_mode=dp.DP_NORM_GHOST, flags=dp.DP_NO_NOISE, audit=True)
+    assert res["modes"] == [dp.DP_NORM_GHOST] * 2 and all(p[0] == 1 for p in res["paths"])
+    for l, (A, D) in enumerate(layers):
+        ref = O.layer_sqnorms_materialised(W.to_f64(A), W.to_f64(D))
+        assert rel_err_elementwise(res["n"][l], ref) <= TOL["bf16"]
+
+
 def test_ghost_and_materialised_agree_on_block_workload():
     w = W.get("block_bf16")
     layers = W.make_inputs(w)
