@@ -517,7 +517,8 @@ def run_ours(args, rank, world, local_rank):
     noise_gbs = 8.0 * w.n_params / (noise_ms * 1e-3) / 1e9
     kernels["noise_add"] = {"ms_per_step": noise_ms, "gbs": noise_gbs,
                             "frac_hbm": noise_gbs / peaks["hbm_gbs"], "launches": noise_launches,
-                            "bytes": 8 * w.n_params}
+                            "bytes": 8 * w.n_params,
+                            "traffic": _traffic("noise_add", 8.0 * w.n_params)}
 
     # the released update: noisy gradient + AdamW on theta, m, v in place
     # (read g, theta, m, v; write theta, m, v): 28 bytes per parameter
