@@ -493,8 +493,10 @@ def run_ours(args, rank, world, local_rank):
         sum_bytes = sum(b_ for b_, t in zip(io, thin) if not t) + grads + p_all
         for name, ms_, b in (("layer_norms", norm_ms, norm_bytes), ("clipsum_gemm", gemm_ms, sum_bytes)):
             k = kernels.setdefault(name, {})
+            # no ncu capture of these launches: traffic unknown
             k.update({"ms_per_step": ms_, "bytes": b, "gbs": b / (ms_ * 1e-3) / 1e9,
                       "frac_hbm": b / (ms_ * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                      "traffic": None,
                       "launches_per_step": stage_launches[
                           {"layer_norms": "norm", "clipsum_gemm": "gemm"}[name]]})
         conv_dom = max(("layer_norms", "clipsum_gemm"), key=lambda n: kernels[n]["ms_per_step"])
