@@ -79,7 +79,10 @@ typedef enum { DP_F32 = 0, DP_BF16 = 1 } dp_dtype;
  * MATERIALISED: the d_in x d_out gradient is formed tile by tile on chip,
  *   squared and summed; it is never written to memory.
  * AUTO: RANK1 when T == 1, else whichever of GHOST / MATERIALISED has the
- *   smaller arithmetic cost (T <= 2 d_in d_out / (d_in + d_out) picks GHOST). */
+ *   smaller arithmetic cost (T <= 2 d_in d_out / (d_in + d_out) picks GHOST),
+ *   except that a bf16 layer wider than 65536 on either side takes
+ *   MATERIALISED on tensor cores instead of GHOST on CUDA cores (see
+ *   dp_layer_path). */
 typedef enum {
     DP_NORM_AUTO = 0,
     DP_NORM_RANK1 = 1,
@@ -299,11 +302,15 @@ dp_status dp_set_noise_key(dp_ctx* ctx, uint64_t seed, uint64_t step);
 
 /* Which kernels serve a layer: *norm_tc = 1 if its per-example norms run on
  * the tcgen05 tensor cores (0: CUDA cores), *sum_tc = 1 if its clipped sum
- * does.  For bf16 layers the Gram norm always does; the clipped sum and the
- * materialised norm do when T is a multiple of 64 or T >= 32 (each example
- * padded to 64 positions), and for T < 32 the clipped sum runs on a
- * pre-scaled copy of A (c_i folded into a bf16 hi + lo pair held in context
- * scratch).  fp32 layers never use tensor cores.  Thin layers whose
+ * does.  For bf16 layers the Gram norm does when d_in, d_out <= 65536; the
+ * clipped sum and the materialised norm do when T is a multiple of 64 or
+ * T >= 32 (each example padded to 64 positions) and T <= 65536, and for
+ * T < 32 the clipped sum runs on a pre-scaled copy of A (c_i folded into a
+ * bf16 hi + lo pair held in context scratch) when 2 B T <= 65536 (rounded
+ * up to 64).  The bounds are accuracy bounds: a tensor-core fp32
+ * accumulator drifts low by about 1.6 * 2^-24 per 16-long step of its
+ * reduction, so longer reductions run on CUDA cores.  fp32 layers never use
+ * tensor cores.  Thin layers whose
  * per-example gradients are stored by the norm pass (see
  * dp_clipped_sum_noise) report *norm_tc = 2 and *sum_tc = 0: both passes run
  * on CUDA cores. */

@@ -253,7 +253,7 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
       p.norm_tc = 0;
       p.gemm_tc = 0;
       p.nparts = dpk::pergrad_parts(cfg->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, p.d_in,
-                                    p.d_out);
+                                    p.d_out, T);
       p.g_off = grads;
       grads += static_cast<int64_t>(cfg->B) * p.d_in * p.d_out;
       if (p.nparts > NP) NP = p.nparts;
@@ -262,6 +262,12 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
     }
     p.mode = resolve_mode(cfg->norm_mode, T, p.d_in, p.d_out);
     const bool bf16 = cfg->dtype == DP_BF16;
+    // the cost model picked the Gram form, but a side wider than the tensor
+    // cores' accumulation bound keeps it off them: the materialised form on
+    // tensor cores (reductions of length T) beats the Gram form on CUDA cores
+    if (cfg->norm_mode == DP_NORM_AUTO && p.mode == DP_NORM_GHOST && bf16 &&
+        !dpk::tc_ghost_supported(T, p.d_in, p.d_out) && dpk::tc_gemm_supported(T, p.d_in, p.d_out))
+      p.mode = DP_NORM_MATERIALISED;
     p.norm_tc = 0;
     if (p.mode == DP_NORM_RANK1) {
       p.nparts = dpk::rank1_parts();
@@ -289,7 +295,7 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
         p.norm_tc = 1;
         p.nparts = dpk::tc_mat_parts(p.d_in, p.d_out);
       }
-    } else if (bf16 && dpk::tc_prescaled_supported(T, p.d_in, p.d_out)) {
+    } else if (bf16 && dpk::tc_prescaled_supported(cfg->B, T, p.d_in, p.d_out)) {
       p.gemm_tc = 2;
       const int64_t need = dpk::tc_prescaled_scratch_bytes(cfg->B, T, p.d_in);
       if (need > c->prescaled_bytes) c->prescaled_bytes = need;

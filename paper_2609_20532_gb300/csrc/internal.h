@@ -7,6 +7,14 @@ namespace dpk {
 
 enum InType { IN_F32 = 0, IN_BF16 = 1 };
 
+// Longest reduction one tensor-core fp32 accumulator takes over its K
+// dimension (features of a Gram, positions of an example's product): the
+// accumulation drifts low by about 1.6 * 2^-24 per K = 16 step (measured on
+// GB300: -3.1e-4 for a 65536-feature Gram norm, -6.2e-3 for 2^20), so 2^16
+// keeps each factor of a norm below 4e-4.  Longer reductions run on CUDA
+// cores, whose round-to-nearest fp32 sums do not drift.
+constexpr int64_t kTcMaxAccum = 1 << 16;
+
 // How the output tile of a clipped-sum kernel is written.
 struct Epilogue {
   const uint64_t* key;  // device words {seed, step}: read by the kernel, so a
@@ -95,7 +103,7 @@ struct PerGradSumBatch {
   int L, B;
 };
 int pergrad_bucket(int r);                       // 1, 2, 4, ..., 32, or 0 if too wide
-int pergrad_parts(InType t, int64_t d_in, int64_t d_out);  // partials per example
+int pergrad_parts(InType t, int64_t d_in, int64_t d_out, int T);  // partials per example
 cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s);
 cudaError_t launch_pergrad_sum(PerGradSumBatch& g, cudaStream_t s);
 

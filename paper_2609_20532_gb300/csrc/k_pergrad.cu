@@ -707,15 +707,18 @@ int pergrad_bucket(int r) {
 
 // bf16 layers whose wide rows are whole 16-byte vectors take the MMA kernel
 // (narrow widths below 8 are zero-padded to one n-tile; the pass stays bound
-// by the wide rows' bytes).
-bool pergrad_mma(InType t, int64_t n, int r) { return t == IN_BF16 && n % 8 == 0 && r > 0; }
+// by the wide rows' bytes), as long as an example's T positions stay within
+// the accumulation bound of the MMA's fp32 accumulators.
+bool pergrad_mma(InType t, int64_t n, int r, int T) {
+  return t == IN_BF16 && n % 8 == 0 && r > 0 && T <= kTcMaxAccum;
+}
 
-int pergrad_parts(InType t, int64_t d_in, int64_t d_out) {
+int pergrad_parts(InType t, int64_t d_in, int64_t d_out, int T) {
   const int r = static_cast<int>(d_in < d_out ? d_in : d_out);
   const int64_t n = d_in < d_out ? d_out : d_in;
   const int R = pergrad_bucket(r);
   if (R == 0) return 0;
-  if (pergrad_mma(t, n, r)) return static_cast<int>((n + kMmaCols - 1) / kMmaCols);
+  if (pergrad_mma(t, n, r, T)) return static_cast<int>((n + kMmaCols - 1) / kMmaCols);
   const int vj = R <= 8 ? 4 : (R <= 16 ? 2 : 1);
   return static_cast<int>((n + kThreads * vj - 1) / (kThreads * vj));
 }
@@ -775,7 +778,7 @@ cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s) {
     part[m].L = 0;
   }
   for (int l = 0; l < g.L; ++l) {
-    const int m = pergrad_mma(t, g.l[l].n, g.l[l].r) ? 1 : 0;
+    const int m = pergrad_mma(t, g.l[l].n, g.l[l].r, g.T) ? 1 : 0;
     part[m].l[part[m].L++] = g.l[l];
   }
   for (int m = 0; m < 2; ++m) {

@@ -857,12 +857,16 @@ bool tc_conv_implicit_ok(const ConvGeom& g, int T) {
 }
 
 // Direct path: T a multiple of 64, or T >= 32 (3-D padding wastes at most half).
+// (an example's product accumulates over its T positions in TMEM: T <= kTcMaxAccum)
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out) {
-  return (T % BK == 0 || T >= 32) && d_in % 8 == 0 && d_out % 8 == 0 && tma_encode_available();
+  return (T % BK == 0 || T >= 32) && T <= kTcMaxAccum && d_in % 8 == 0 && d_out % 8 == 0 &&
+         tma_encode_available();
 }
 
-bool tc_prescaled_supported(int T, int64_t d_in, int64_t d_out) {
-  return T < 32 && d_in % 8 == 0 && d_out % 8 == 0 && tma_encode_available();
+// (the whole batch, 2 B T rows of hi + lo, accumulates in one TMEM tile)
+bool tc_prescaled_supported(int B, int T, int64_t d_in, int64_t d_out) {
+  return T < 32 && 2 * prescale_rows(B, T) <= kTcMaxAccum && d_in % 8 == 0 && d_out % 8 == 0 &&
+         tma_encode_available();
 }
 
 int64_t tc_prescaled_scratch_bytes(int B, int T, int64_t d_in) {

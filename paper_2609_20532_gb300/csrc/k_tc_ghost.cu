@@ -307,7 +307,8 @@ int half_strips(int nb) { return (nb + 1) / 2; }
 
 bool tc_ghost_supported(int T, int64_t d_in, int64_t d_out) {
   (void)T;
-  return d_in % 8 == 0 && d_out % 8 == 0 && tma_encode_available();
+  return d_in % 8 == 0 && d_out % 8 == 0 && d_in <= kTcMaxAccum && d_out <= kTcMaxAccum &&
+         tma_encode_available();
 }
 
 int tc_ghost_parts(int T) {

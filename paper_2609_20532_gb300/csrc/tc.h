@@ -51,7 +51,7 @@ cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int 
 
 // Clipped sum for short examples (T < 32): c_i folded into a bf16 hi+lo
 // split of A in scratch (tc_prescaled_scratch_bytes), then one plain GEMM.
-bool tc_prescaled_supported(int T, int64_t d_in, int64_t d_out);
+bool tc_prescaled_supported(int B, int T, int64_t d_in, int64_t d_out);
 int64_t tc_prescaled_scratch_bytes(int B, int T, int64_t d_in);
 cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const float* c, int B,
                                         int T, int d_in, int d_out, float* out,

@@ -140,6 +140,61 @@ def test_llm_workload_sampled():
     _llm_sample_check(w, layers, res)
 
 
+def test_widest_layers_sampled():
+    """Layers at the widest size the library accepts (2^20 on one side): two
+    thin layers at T = 1 (per-example gradients stored) and a tensor-core
+    layer at T = 64 whose output has 2^26 parameters.  Every norm and clip
+    factor against the oracle, and sampled rows of every noisy output."""
+    M = 1 << 20
+    shapes = [(M, 8, 1), (8, M, 1), (64, M, 64)]
+    w = W.custom("widest", shapes, 2, 64, "bf16", C=0.5, sigma=0.7, d_std=0.05, wid=640)
+    layers = W.make_inputs(w, seed=0)
+    res = run_gpu_step(w, layers, seed=6, step=2)
+    # the cost model prefers the Gram form for the last layer, but its 2^20-long
+    # feature reductions exceed the tensor cores' accumulation bound: the
+    # materialised form on tensor cores (reductions of length T) serves it
+    assert [p[0] for p in res["paths"]] == [2, 2, 1], res["paths"]
+    assert res["modes"][2] == dp.DP_NORM_MATERIALISED
+    n_ref = np.stack([O.layer_sqnorms_ghost(W.to_f64(A), W.to_f64(D)) for A, D in layers])
+    s_ref, c_ref = O.clip_factors(n_ref, f32(w.C))
+    assert rel_err_elementwise(res["n"], n_ref) <= TOL["bf16"]
+    assert rel_err_elementwise(res["c"], c_ref) <= TOL["bf16"]
+    rng = np.random.default_rng(7)
+    off = 0
+    for l, (A, D) in enumerate(layers):
+        d_in, d_out = w.layers[l]
+        rows = np.sort(rng.choice(d_in, size=min(6, d_in), replace=False))
+        S_rows = O.clipped_sum(W.to_f64(A[:, :, rows]), W.to_f64(D), c_ref)
+        z = np.stack([O.gaussian_noise(6, 2, off + int(j) * d_out, d_out) for j in rows])
+        ref = S_rows + f32(w.sigma) * f32(w.C) * z
+        assert rel_err_normwise(res["out"][l][rows], ref) <= TOL["bf16"], l
+        off += d_in * d_out
+    # the Gram form forced on the wide layer runs on CUDA cores, also in bound
+    w1 = W.custom("widest_g", [(64, M)], 2, 64, "bf16", C=0.5, sigma=0.7, d_std=0.05, wid=641)
+    l1 = W.make_inputs(w1, seed=0)
+    g = run_gpu_step(w1, l1, norm_mode=dp.DP_NORM_GHOST, flags=dp.DP_NO_NOISE)
+    assert g["paths"][0][0] == 0 and g["modes"][0] == dp.DP_NORM_GHOST
+    n1 = O.layer_sqnorms_ghost(W.to_f64(l1[0][0]), W.to_f64(l1[0][1]))
+    assert rel_err_elementwise(g["n"][0], n1) <= TOL["bf16"]
+
+
+def test_long_reductions_leave_the_tensor_cores():
+    """Paths whose tensor-core reduction would exceed 2^16 terms run on CUDA
+    cores: T = 2^17 positions (an example's product), a 2^17-wide Gram side,
+    and a pre-scaled T < 32 batch of more than 2^15 rows."""
+    cases = [([(64, 64)], 1, 1 << 17, dp.DP_NORM_MATERIALISED, (0, 0)),
+             ([(64, 1 << 17)], 2, 64, dp.DP_NORM_GHOST, (0, 1)),
+             ([(64, 64)], 1 << 12, 16, dp.DP_NORM_MATERIALISED, (0, 0)),
+             ([(64, 64)], 1 << 10, 16, dp.DP_NORM_MATERIALISED, (0, 1))]
+    for shapes, B, T, mode, want in cases:
+        cfg = dp.make_config(shapes, B, T, "bf16", 1.0, 1.0, norm_mode=mode)
+        ctx = dp.dp_step_init(cfg)
+        try:
+            assert dp.dp_layer_path(ctx, 0) == want, (shapes, B, T)
+        finally:
+            dp.dp_step_destroy(ctx)
+
+
 # ---------------------------------------------------------------------------
 # norm modes, edge shapes and flags
 # ---------------------------------------------------------------------------
