@@ -865,8 +865,8 @@ bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out) {
 
 // (the whole batch, 2 B T rows of hi + lo, accumulates in one TMEM tile)
 bool tc_prescaled_supported(int B, int T, int64_t d_in, int64_t d_out) {
-  return T < 32 && 2 * prescale_rows(B, T) <= kTcMaxAccum && d_in % 8 == 0 && d_out % 8 == 0 &&
-         tma_encode_available();
+  return T <= kPrescaleMaxT && 2 * prescale_rows(B, T) <= kTcMaxAccum && d_in % 8 == 0 &&
+         d_out % 8 == 0 && tma_encode_available();
 }
 
 int64_t tc_prescaled_scratch_bytes(int B, int T, int64_t d_in) {

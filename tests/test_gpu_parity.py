@@ -498,8 +498,9 @@ TC_CASES = [
 ]
 
 SMALL_T_CASES = [
-    # T < 32: the clipped sum runs on the pre-scaled hi+lo operand
+    # T <= 64: the clipped sum runs on the pre-scaled hi+lo operand
     ([(264, 136)], 7, 3),
+    ([(3320, 264)], 5, 64),
     ([(4096, 1024)], 16, 1),
     ([(136, 72), (72, 8)], 33, 31),
 ]
@@ -780,7 +781,7 @@ def test_split_batch_tensor_core_layers(case, mode):
 ODD_BASE_CASES = [
     # (layers, B, T): a tensor-core layer whose first global parameter index
     # is not a multiple of 4, so its noise groups straddle two Philox quads
-    ([(1, 3), (264, 136)], 6, 64),      # direct tiles, p_base = 3
+    ([(1, 3), (264, 136)], 6, 128),     # direct tiles, p_base = 3
     ([(1, 5), (256, 64)], 64, 256),     # split ranges + reduce, p_base = 5
     ([(1, 3), (256, 256)], 16, 8),      # pre-scaled operand (T < 32), p_base = 3
 ]
