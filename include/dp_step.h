@@ -305,9 +305,9 @@ dp_status dp_set_noise_key(dp_ctx* ctx, uint64_t seed, uint64_t step);
  * does.  For bf16 layers the Gram norm does when d_in, d_out <= 65536; the
  * clipped sum and the materialised norm do when T is a multiple of 64 or
  * T >= 32 (each example padded to 64 positions) and T <= 65536, and for
- * T <= 64 the clipped sum of a dense layer runs on a pre-scaled copy of A
- * (c_i folded into a bf16 hi + lo pair held in context scratch, no
- * per-example fold) when 2 B T <= 65536 (rounded up to 64).  The bounds are accuracy bounds: a tensor-core fp32
+ * T < 32 the clipped sum runs on a pre-scaled copy of A (c_i folded into a
+ * bf16 hi + lo pair held in context scratch, no per-example fold) when
+ * 2 B T <= 65536 (rounded up to 64).  The bounds are accuracy bounds: a tensor-core fp32
  * accumulator drifts low by about 1.6 * 2^-24 per 16-long step of its
  * reduction, so longer reductions run on CUDA cores.  fp32 layers never use
  * tensor cores.  Thin layers whose

@@ -280,14 +280,7 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
                            : dpk::mat_simt_parts(static_cast<int>(p.d_in), static_cast<int>(p.d_out));
     }
     p.gemm_tc = 0;
-    // dense layers with short examples take the pre-scaled operand even where
-    // the direct kernel could run (tc.h: kPrescaleMaxT), unless the layer has
-    // so few tiles that the direct kernel splits its examples over the GPU
-    // (the pre-scaled GEMM is one long example and cannot split)
-    const bool pre_short =
-        bf16 && !p.conv && dpk::tc_prescaled_supported(cfg->B, T, p.d_in, p.d_out) &&
-        (T < 32 || dpk::tc_gemm_split(cfg->B, T, p.d_in, p.d_out) == 1);
-    if (!pre_short && bf16 && dpk::tc_gemm_supported(T, p.d_in, p.d_out)) {
+    if (bf16 && dpk::tc_gemm_supported(T, p.d_in, p.d_out)) {
       p.gemm_tc = 1;
       p.split = dpk::tc_gemm_split(cfg->B, T, p.d_in, p.d_out);
       if (p.split > 1) {

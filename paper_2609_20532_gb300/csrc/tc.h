@@ -52,14 +52,12 @@ cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int 
 // Clipped sum for short examples (T < 32): c_i folded into a bf16 hi+lo
 // split of A in scratch (tc_prescaled_scratch_bytes), then one plain GEMM.
 // Pre-scaled operand (c_i a as a bf16 hi + lo pair, one plain GEMM with no
-// per-example fold): every dense layer with T < 32, and with T <= 64 where
-// the layer has enough tiles to fill the GPU without splitting its examples:
-// there the fold after every K block costs more than the doubled MMA work
-// (same-box sweep of a 4096 x 4096 layer at T = 64: 0.21 -> 0.16 ms at
-// B = 32, 0.64 -> 0.55 ms at B = 128).  At T = 128 it lost (the 768-3072
-// wide block layers: 0.115 -> 0.295 ms), as it does for few-tile layers,
-// which the direct kernel splits and the one-example pre-scaled GEMM cannot.
-constexpr int kPrescaleMaxT = 64;
+// per-example fold) for T < 32, where the direct kernel's 3-D padding would
+// waste more than half of every K block.  At T = 64 and 128 the direct
+// kernel with its per-example fold is faster (same box, 4096 x 4096 layer at
+// T = 64: 0.41 against 0.54 ms at B = 128; the 768-3072 wide block layers at
+// T = 128: 0.115 against 0.295 ms).
+constexpr int kPrescaleMaxT = 31;
 bool tc_prescaled_supported(int B, int T, int64_t d_in, int64_t d_out);
 int64_t tc_prescaled_scratch_bytes(int B, int T, int64_t d_in);
 cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const float* c, int B,

@@ -498,9 +498,9 @@ TC_CASES = [
 ]
 
 SMALL_T_CASES = [
-    # T <= 64: the clipped sum runs on the pre-scaled hi+lo operand
+    # T < 32: the clipped sum runs on the pre-scaled hi+lo operand
     ([(264, 136)], 7, 3),
-    ([(3320, 264)], 5, 64),
+    ([(3320, 264)], 5, 31),
     ([(4096, 1024)], 16, 1),
     ([(136, 72), (72, 8)], 33, 31),
 ]
