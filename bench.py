@@ -163,8 +163,16 @@ def _stage_ms(fn, stream, args, use_graph):
         run = g_.replay
     else:
         run = fn
-    for _ in range(args.warmup):
+    # warm up for at least W calls and 0.1 s, so that a GPU whose clocks
+    # dropped while it idled is back at speed even for very short kernels
+    t_end = time.perf_counter() + 0.1
+    n = 0
+    while n < args.warmup or time.perf_counter() < t_end:
         run()
+        n += 1
+        if n % 64 == 0:
+            torch.cuda.synchronize()
+    torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     a.record(stream)
     for _ in range(args.steps):
