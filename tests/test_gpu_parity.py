@@ -1178,3 +1178,45 @@ def test_roberta_adapters_with_head_reduced():
     assert [n for n, _ in res["paths"][:8]] == [2] * 8
     ref = oracle_step(w, layers, seed=2, step=9, out_scale=1.0 / w.B)
     assert_step_matches(res, ref, "bf16")
+
+
+def test_data_parallel_step_on_one_rank():
+    """data_parallel_step through the library on a one-rank NCCL group: the
+    commitment, the (trivial) all-reduce and the noise added after it give
+    the same bits as an eager step of the same context."""
+    import socket
+    import torch.distributed as dist
+    from paper_2609_20532_gb300.data_parallel import data_parallel_step
+    w = W.custom("dp1", [(136, 72), (64, 200)], 5, 64, "bf16", C=0.05, sigma=0.7, d_std=0.1,
+                 wid=612)
+    layers = W.make_inputs(w)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    with socket.socket() as s_:
+        s_.bind(("127.0.0.1", 0))
+        port = s_.getsockname()[1]
+    dist.init_process_group("nccl", init_method=f"tcp://127.0.0.1:{port}", rank=0, world_size=1)
+    try:
+        stream = torch.cuda.current_stream()
+        cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
+                             seed=21, step=3)
+        outs = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+        ref = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+        ctx = dp.dp_step_init(cfg, stream)
+        try:
+            data_parallel_step(ctx, range(len(layers)), Ad, Dd, outs)
+            dp.dp_step_init(cfg, stream, ctx)
+            dp.run_step(ctx, Ad, Dd, ref, flags=dp.DP_NO_NOISE)
+            dp.dp_clipped_sum_noise_batch(ctx, list(range(len(layers))), None, None, ref,
+                                          dp.DP_NOISE_ONLY)
+        finally:
+            dp.dp_step_destroy(ctx)
+        torch.cuda.synchronize()
+    finally:
+        dist.destroy_process_group()
+    for a, b in zip(outs, ref):
+        assert torch.equal(a, b)
+    r = oracle_step(w, layers, seed=21, step=3, out_scale=1.0 / w.B)
+    for o, rr in zip(outs, r["out"]):
+        assert rel_err_normwise(o.cpu().numpy(), rr) <= TOL["bf16"]
