@@ -332,9 +332,9 @@ void dp_step_destroy(dp_ctx* ctx);
  * d_sqnorm_out: device fp32 [B]; cuda_stream: cudaStream_t (NULL = default).
  * Asynchronous.  Scratch is a library-owned static device array of 2^20 fp32
  * partial sums (4 MiB, held by every GPU that loads the library until exit):
- * B * ceil(T/128) * (ceil(T/128) + 1) * 2 (bf16) or
- * B * ceil(T/64) * (ceil(T/64) + 1) / 2 (fp32) must not exceed 2^20, else
- * DP_ERR_SHAPE.  The first call on a device looks up the array's address
+ * B * ceil(T/128) * (ceil(T/128) + 1) * 2 (bf16 with d_in, d_out <= 65536:
+ * tensor cores) or B * ceil(T/64) * (ceil(T/64) + 1) / 2 (fp32, or a side
+ * wider than 65536: CUDA cores) must not exceed 2^20, else DP_ERR_SHAPE.  The first call on a device looks up the array's address
  * and should come before any stream capture.  Calls share the array: calls
  * that overlap on the GPU race and must be ordered by the caller.  If a
  * tensor-core pipeline wait gives up, the outputs are NaN.
