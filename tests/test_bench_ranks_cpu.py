@@ -79,3 +79,26 @@ def test_traffic_lookup(tmp_path):
     assert bench._traffic("k", 250.0, str(p)) == 12500.0
     for key in ("stale", "old", "partial", "missing"):
         assert bench._traffic(key, 1.0, str(p)) is None
+
+
+def test_reference_arm_line_on_cpu():
+    """`bench.py --impl reference` times the oracle on the host cores and
+    prints the contract's JSON line: impl, the metric and unit of our arm,
+    a cpu_baseline describing the run and an e2e with no host copies."""
+    import json
+    import subprocess
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--workload", "single_fp32", "--steps", "3", "--warmup", "3"],
+                       capture_output=True, text=True, timeout=300, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    sys.path.insert(0, ROOT)
+    import bench
+    assert line["impl"] == "reference" and line["metric"] == bench.METRIC
+    assert line["unit"] == bench.UNIT and line["higher_is_better"] is True
+    assert line["steps"] == 3 and line["warmup"] == 3 and line["value"] > 0
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == line["value"]
+    assert "example 0 of single_fp32" in cb["sample"]
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"],
+                           "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
