@@ -152,3 +152,27 @@ def test_conv_layer_config_checked_on_host(L):
     nogeom = dp.make_config([(144, 32)], 2, 1, "bf16", 1.0, 1.0)
     nogeom.layers[0].kind = dp.DP_LAYER_CONV2D
     assert _init_status(L, nogeom)[0] == 1
+
+
+def test_header_is_plain_c_and_cpp():
+    """include/dp_step.h is a C ABI: it compiles as C99 and as C++17 with
+    warnings as errors, and a C translation unit can take the address of
+    every declared entry point."""
+    import shutil
+    import subprocess
+    import tempfile
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("gcc not available")
+    inc = os.path.join(ROOT, "include")
+    with tempfile.TemporaryDirectory() as td:
+        src = os.path.join(td, "use.c")
+        with open(src, "w") as f:
+            f.write('#include "dp_step.h"\n')
+            f.write("void* const entry_points[] = {\n")
+            f.write("".join(f"  (void*)&{n},\n" for n in header_functions()))
+            f.write("};\n")
+        for lang, std in (("c", "-std=c99"), ("c++", "-std=c++17")):
+            r = subprocess.run([gcc, "-fsyntax-only", std, "-Wall", "-Wextra", "-Werror",
+                                "-x", lang, "-I", inc, src], capture_output=True, text=True)
+            assert r.returncode == 0, (lang, r.stderr)
