@@ -153,6 +153,10 @@ typedef struct {
     int32_t audit_capacity;    /* max records per dp_audit_emit call, 0 .. B */
     const dp_conv2d* convs;    /* host array of L geometries, read for DP_LAYER_CONV2D
                                   layers only (NULL when there are none); copied */
+    uint64_t param_base;       /* global parameter index of layer 0's element (0, 0):
+                                  0 for a whole model; when the layers are split over
+                                  ranks, the parameters of the layers before this
+                                  context's (the noise keys are global indices) */
 } dp_config;
 
 /* Flags of dp_clipped_sum_noise. */
@@ -207,6 +211,23 @@ dp_status dp_layer_norms(dp_ctx* ctx, int32_t layer, const void* A, const void* 
 dp_status dp_layer_norms_batch(dp_ctx* ctx, int32_t n, const int32_t* layers,
                                const void* const* A, const void* const* D);
 
+/* Layers split over ranks (each rank's context holds a contiguous range of
+ * the model's layers, dp_config.param_base placing them in the global
+ * parameter vector).  Sec. 2.2's ||g_i|| runs over every trainable
+ * parameter, so the squared norms of all ranks' layers are summed before
+ * clipping:
+ *   dp_partial_sqnorms: d_sqnorm_local[i] = sum over this context's layers
+ *     of n_{l,i} (device fp32 [B]); needs every layer's norms, forms no clip
+ *     factor and leaves the call-order state unchanged;
+ *   dp_clip_factors_from: as dp_clip_factors, but with s_i =
+ *     d_sqnorm_total[i] (device fp32 [B], e.g. the sum over ranks of their
+ *     dp_partial_sqnorms) in place of this context's own sum.  Audit records
+ *     then hold this total and this context's layer norms.
+ * Errors: as dp_clip_factors (DP_ERR_ARG for a NULL array). */
+dp_status dp_partial_sqnorms(dp_ctx* ctx, float* d_sqnorm_local);
+dp_status dp_clip_factors_from(dp_ctx* ctx, const float* d_sqnorm_total, float* d_sqnorm_out,
+                               float* d_clip_out);
+
 /* Sum the per-layer norms and form the clip factors (Sec. 2.2; Algorithm 2):
  *   s_i = sum_l n_{l,i},   c_i = 1 if s_i <= C^2 else C / sqrt(s_i).
  * d_sqnorm_out [B] and d_clip_out [B] are optional device fp32 arrays that
@@ -237,6 +258,18 @@ dp_status dp_clip_factors(dp_ctx* ctx, float* d_sqnorm_out, float* d_clip_out);
  *   DP_NOISE_ONLY), DP_ERR_CUDA. */
 dp_status dp_clipped_sum_noise(dp_ctx* ctx, int32_t layer, const void* A, const void* D,
                                float* d_out, uint32_t flags);
+
+/* Released noise on a range of the global parameter vector (Algorithm 2:
+ * the noise added after the commitment), independent of layers:
+ *   d_out[e] += out_scale * sigma * C * z_{p_first + e},  0 <= e < n,
+ * with z as in dp_clipped_sum_noise.  It lets ranks that hold disjoint
+ * slices of the summed commitment (after a reduce-scatter) each add the
+ * noise of their own slice.  d_out: device fp32 [n], 16-byte aligned (the
+ * kernel reads and writes whole quads when p_first is a multiple of 4).
+ * Needs only an initialised context (the key of dp_step_init /
+ * dp_set_noise_key).  n = 0 launches nothing.
+ * Errors: DP_ERR_ARG (NULL or misaligned d_out, n < 0), DP_ERR_CUDA. */
+dp_status dp_noise_add_range(dp_ctx* ctx, uint64_t p_first, int64_t n, float* d_out);
 
 /* Clipped sum and noise of n listed layers (host arrays of n entries:
  * layer indices, each at most once, and their A, D and d_out pointers; A
@@ -331,13 +364,18 @@ void dp_step_destroy(dp_ctx* ctx);
  * A: [B][T][d_in], D: [B][T][d_out] device arrays of dtype, 16-byte aligned;
  * d_sqnorm_out: device fp32 [B]; cuda_stream: cudaStream_t (NULL = default).
  * Asynchronous.  Scratch is a library-owned static device array of 2^20 fp32
- * partial sums (4 MiB, held by every GPU that loads the library until exit):
- * B * ceil(T/128) * (ceil(T/128) + 1) * 2 (bf16 with d_in, d_out <= 65536:
- * tensor cores) or B * ceil(T/64) * (ceil(T/64) + 1) / 2 (fp32, or a side
- * wider than 65536: CUDA cores) must not exceed 2^20, else DP_ERR_SHAPE.  The first call on a device looks up the array's address
- * and should come before any stream capture.  Calls share the array: calls
- * that overlap on the GPU race and must be ordered by the caller.  If a
- * tensor-core pipeline wait gives up, the outputs are NaN.
+ * partial sums (4 MiB, held by every GPU that loads the library until exit).
+ * B times the partial sums per example must not exceed 2^20, else
+ * DP_ERR_SHAPE.  Per example that is, with m = ceil(ceil(T / 128) / 2):
+ *   tensor cores (bf16, d_in and d_out <= 65536, T <= 65536):
+ *     8 m (m + 1) when ceil(T / 128) is even, 8 m^2 when it is odd;
+ *   CUDA cores (fp32, or a side or T above 65536):
+ *     n (n + 1) / 2 with n = ceil(T / 64).
+ * The first call on a device looks up the array's address and does the
+ * kernels' per-device set-up; it should come before any stream capture.
+ * Calls share the array: calls that overlap on the GPU race and must be
+ * ordered by the caller.  If a tensor-core pipeline wait gives up, the
+ * outputs are NaN.
  * Errors: DP_ERR_ARG, DP_ERR_DTYPE, DP_ERR_SHAPE, DP_ERR_CUDA. */
 dp_status dp_layer_sqnorms_noalloc(const void* A, const void* D, int32_t B, int32_t T,
                                    int64_t d_in, int64_t d_out, dp_dtype dtype,
@@ -379,6 +417,19 @@ dp_status dp_kernel_launches(int64_t* count_out);
  * They expose the generator the noise uses so tests can compare it with the
  * oracle: raw Philox4x32-10 blocks and the Gaussian numbers z_p.
  * d_out is a device array; stream is a cudaStream_t (NULL = default).    */
+
+/* Make one bounded device wait run out, to exercise the failure path of the
+ * tensor-core pipelines (their waits give up after 2 s, record
+ * DP_ERR_TIMEOUT in the context's sticky error word and return, so the
+ * context stays usable; Algorithm 1's checker then rejects the step).  A
+ * one-warp kernel on the context's stream waits, with the same bounded-wait
+ * helper, on an mbarrier that nothing arrives on, gives up after limit_ns
+ * nanoseconds (1 .. 10^9) and sets the context's timeout bit; it issues no
+ * TMA copy and no MMA.  Synchronises the stream.  Returns DP_ERR_TIMEOUT when
+ * the wait gave up (dp_audit_emit of the same step then reports it too; the
+ * next dp_step_init clears it).  Errors: DP_ERR_ARG (NULL context, limit out
+ * of range), DP_ERR_CUDA. */
+dp_status dp_debug_bounded_wait(dp_ctx* ctx, int64_t limit_ns);
 
 /* d_out[4 r + w] = word w of the block for quad first_quad + r, r < n_quads. */
 dp_status dp_debug_philox(uint64_t seed, uint64_t step, uint64_t first_quad, int64_t n_quads,

@@ -53,8 +53,9 @@ EXPORTED_SYMBOLS = ["dp_step_init", "dp_layer_norms", "dp_layer_norms_batch", "d
                     "dp_layer_path", "dp_set_noise_key", "dp_step_destroy", "dp_last_error",
                     "dp_status_string", "dp_kernel_launches", "dp_conv2d_dims",
                     "dp_conv2d_unfold",
-                    "dp_debug_philox", "dp_debug_gaussian", "dp_layer_sqnorms_noalloc",
-                    "dp_noise_adamw"]
+                    "dp_debug_philox", "dp_debug_gaussian", "dp_debug_bounded_wait",
+                    "dp_layer_sqnorms_noalloc", "dp_noise_adamw", "dp_partial_sqnorms",
+                    "dp_clip_factors_from", "dp_noise_add_range"]
 
 
 class DPError(RuntimeError):
@@ -90,7 +91,8 @@ class dp_config(ctypes.Structure):
                 ("clip_C", ctypes.c_float), ("sigma", ctypes.c_float),
                 ("out_scale", ctypes.c_float), ("seed", ctypes.c_uint64),
                 ("step", ctypes.c_uint64), ("norm_mode", ctypes.c_int32),
-                ("audit_capacity", ctypes.c_int32), ("convs", ctypes.POINTER(dp_conv2d))]
+                ("audit_capacity", ctypes.c_int32), ("convs", ctypes.POINTER(dp_conv2d)),
+                ("param_base", ctypes.c_uint64)]
 
 
 _LIB = None
@@ -128,6 +130,10 @@ def lib() -> ctypes.CDLL:
         "dp_conv2d_unfold": ([ctypes.POINTER(dp_conv2d), i32, i32, vp, vp, vp], i32),
         "dp_debug_philox": ([u64, u64, u64, i64, vp, vp], i32),
         "dp_debug_gaussian": ([u64, u64, u64, i64, vp, vp], i32),
+        "dp_debug_bounded_wait": ([vp, i64], i32),
+        "dp_partial_sqnorms": ([vp, vp], i32),
+        "dp_clip_factors_from": ([vp, vp, vp, vp], i32),
+        "dp_noise_add_range": ([vp, u64, i64, vp], i32),
         "dp_layer_sqnorms_noalloc": ([vp, vp, i32, i32, i64, i64, i32, vp, vp], i32),
         "dp_noise_adamw": ([vp, i32, vp, vp, vp, vp, ctypes.POINTER(dp_adamw), u32], i32),
     }
@@ -169,11 +175,13 @@ def _stream(stream) -> Optional[int]:
 def make_config(layers: Sequence[Sequence[int]], B: int, T: int, dtype: str, C: float,
                 sigma: float, out_scale: float = 1.0, seed: int = 0, step: int = 0,
                 norm_mode: int = DP_NORM_AUTO, audit_capacity: int = 0,
-                convs: Optional[Sequence[Optional[dp_conv2d]]] = None) -> dp_config:
+                convs: Optional[Sequence[Optional[dp_conv2d]]] = None,
+                param_base: int = 0) -> dp_config:
     """A layer is (d_in, d_out) or (d_in, d_out, T); T = 0 takes the config's
     T.  convs, when given, has one entry per layer: a dp_conv2d makes that
     layer a DP_LAYER_CONV2D layer (its A is then the NHWC input), None keeps
-    it dense."""
+    it dense.  param_base: global parameter index of the first layer's first
+    element (layers split over ranks)."""
     kinds = [DP_LAYER_CONV2D if convs is not None and convs[i] is not None else DP_LAYER_DENSE
              for i in range(len(layers))]
     arr = (dp_layer * len(layers))(*[dp_layer(int(ly[0]), int(ly[1]),
@@ -186,7 +194,8 @@ def make_config(layers: Sequence[Sequence[int]], B: int, T: int, dtype: str, C: 
                     dtype=DP_BF16 if dtype == "bf16" else DP_F32, clip_C=C, sigma=sigma,
                     out_scale=out_scale, seed=seed & (2 ** 64 - 1), step=step & (2 ** 64 - 1),
                     norm_mode=norm_mode, audit_capacity=audit_capacity,
-                    convs=ctypes.cast(carr, ctypes.POINTER(dp_conv2d)) if carr is not None else None)
+                    convs=ctypes.cast(carr, ctypes.POINTER(dp_conv2d)) if carr is not None else None,
+                    param_base=param_base & (2 ** 64 - 1))
     cfg._keep = (arr, carr)  # keep the arrays alive with the struct
     return cfg
 
@@ -291,6 +300,28 @@ def dp_debug_philox(seed: int, step: int, first_quad: int, n_quads: int, out, st
 def dp_debug_gaussian(seed: int, step: int, first_index: int, n: int, out, stream=None):
     _check(lib().dp_debug_gaussian(seed & (2 ** 64 - 1), step & (2 ** 64 - 1),
                                    first_index & (2 ** 64 - 1), n, _ptr(out), _stream(stream)))
+
+
+def dp_partial_sqnorms(ctx: int, s_local) -> None:
+    """This context's layers' share of every example's squared norm into
+    ``s_local`` [B] (layers split over ranks; no clip factors yet)."""
+    _check(lib().dp_partial_sqnorms(ctx, _ptr(s_local)))
+
+
+def dp_clip_factors_from(ctx: int, s_total, sqnorm_out=None, clip_out=None) -> None:
+    """Clip factors from squared norms summed over every rank's layers."""
+    _check(lib().dp_clip_factors_from(ctx, _ptr(s_total), _ptr(sqnorm_out), _ptr(clip_out)))
+
+
+def dp_noise_add_range(ctx: int, p_first: int, n: int, out) -> None:
+    """out[e] += out_scale * sigma * C * z_{p_first + e} for e < n."""
+    _check(lib().dp_noise_add_range(ctx, p_first & (2 ** 64 - 1), n, _ptr(out)))
+
+
+def dp_debug_bounded_wait(ctx: int, limit_ns: int) -> int:
+    """Run one bounded device wait that nothing satisfies; returns the status
+    (DP_ERR_TIMEOUT when it gave up, as it should).  Test export."""
+    return lib().dp_debug_bounded_wait(ctx, limit_ns)
 
 
 def make_conv(H: int, W: int, C_in: int, kh: int, kw: int, stride=(1, 1), pad=(0, 0)) -> dp_conv2d:

@@ -131,6 +131,11 @@ struct dp_ctx {
 
 namespace {
 
+// Partial sums one example of one layer may need.  The partial buffer holds
+// L * B * NP floats; a forced Gram form on very long examples (about T^2 /
+// 8192 partials) or a materialised norm of an enormous layer would exceed it.
+constexpr int64_t kMaxPartsPerExample = int64_t(1) << 24;
+
 dp_status check_config(const dp_config* cfg) {
   if (!cfg) return fail(DP_ERR_ARG, "cfg is NULL");
   if (cfg->B < 1 || cfg->T < 1) return fail(DP_ERR_SHAPE, "B and T must be >= 1");
@@ -163,6 +168,14 @@ dp_status check_config(const dp_config* cfg) {
       return fail(DP_ERR_SHAPE, "layer %d: B*T exceeds 2^31-1", l);
     if (cfg->norm_mode == DP_NORM_RANK1 && T != 1)
       return fail(DP_ERR_SHAPE, "DP_NORM_RANK1 needs T == 1 for every layer");
+    // a forced Gram form beyond the tensor cores' T bound runs on CUDA cores
+    // with ceil(T/64) (ceil(T/64) + 1) / 2 partial sums per example
+    if (cfg->norm_mode == DP_NORM_GHOST && T > dpk::kTcGhostMaxT &&
+        dpk::ghost_simt_parts(T) > kMaxPartsPerExample)
+      return fail(DP_ERR_SHAPE,
+                  "layer %d: the Gram form at T = %d needs more than %lld partial sums per "
+                  "example; use DP_NORM_MATERIALISED for examples this long",
+                  l, T, static_cast<long long>(kMaxPartsPerExample));
   }
   if (!(cfg->clip_C > 0.f) || !std::isfinite(cfg->clip_C))
     return fail(DP_ERR_ARG, "clip_C must be finite and > 0");
@@ -211,11 +224,11 @@ bool use_pergrad(const dp_config* cfg, int T, int64_t d_in, int64_t d_out) {
   return 8.0 * double(d_in) * double(d_out) < double(T) * double(d_in + d_out) * elem;
 }
 
-void build_plan(dp_ctx* c, const dp_config* cfg) {
+dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
   c->plan.resize(cfg->n_layers);
-  uint64_t off = 0;
+  uint64_t off = cfg->param_base;
   int64_t grads = 0, splits = 0, unf = 0;
-  int NP = 1;
+  int64_t NP = 1;
   for (int l = 0; l < cfg->n_layers; ++l) {
     LayerPlan& p = c->plan[l];
     p.d_in = cfg->layers[l].d_in;
@@ -252,8 +265,8 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
       p.mode = DP_NORM_MATERIALISED;
       p.norm_tc = 0;
       p.gemm_tc = 0;
-      p.nparts = dpk::pergrad_parts(cfg->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, p.d_in,
-                                    p.d_out, T);
+      p.nparts = static_cast<int>(dpk::pergrad_parts(
+          cfg->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, p.d_in, p.d_out, T));
       p.g_off = grads;
       grads += static_cast<int64_t>(cfg->B) * p.d_in * p.d_out;
       if (p.nparts > NP) NP = p.nparts;
@@ -262,6 +275,13 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
     }
     p.mode = resolve_mode(cfg->norm_mode, T, p.d_in, p.d_out);
     const bool bf16 = cfg->dtype == DP_BF16;
+    // the cost model picked the Gram form for examples so long that its
+    // partial sums would not fit: the materialised form needs T-independent
+    // partials
+    if (cfg->norm_mode == DP_NORM_AUTO && p.mode == DP_NORM_GHOST &&
+        !(bf16 && dpk::tc_ghost_supported(T, p.d_in, p.d_out)) &&
+        dpk::ghost_simt_parts(T) > kMaxPartsPerExample)
+      p.mode = DP_NORM_MATERIALISED;
     // the cost model picked the Gram form, but a side wider than the tensor
     // cores' accumulation bound keeps it off them: the materialised form on
     // tensor cores (reductions of length T) beats the Gram form on CUDA cores
@@ -269,16 +289,24 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
         !dpk::tc_ghost_supported(T, p.d_in, p.d_out) && dpk::tc_gemm_supported(T, p.d_in, p.d_out))
       p.mode = DP_NORM_MATERIALISED;
     p.norm_tc = 0;
+    int64_t parts = 1;
     if (p.mode == DP_NORM_RANK1) {
-      p.nparts = dpk::rank1_parts();
+      parts = dpk::rank1_parts();
     } else if (p.mode == DP_NORM_GHOST) {
       p.norm_tc = bf16 && dpk::tc_ghost_supported(T, p.d_in, p.d_out);
-      p.nparts = p.norm_tc ? dpk::tc_ghost_parts(T) : dpk::ghost_simt_parts(T);
+      parts = p.norm_tc ? dpk::tc_ghost_parts(T) : dpk::ghost_simt_parts(T);
     } else {
       p.norm_tc = bf16 && dpk::tc_gemm_supported(T, p.d_in, p.d_out);
-      p.nparts = p.norm_tc ? dpk::tc_mat_parts(p.d_in, p.d_out)
-                           : dpk::mat_simt_parts(static_cast<int>(p.d_in), static_cast<int>(p.d_out));
+      parts = p.norm_tc ? dpk::tc_mat_parts(p.d_in, p.d_out)
+                        : dpk::mat_simt_parts(p.d_in, p.d_out);
     }
+    if (parts < 1 || parts > kMaxPartsPerExample)
+      return fail(DP_ERR_SHAPE,
+                  "layer %d: its norm form needs %lld partial sums per example (limit %lld)%s", l,
+                  static_cast<long long>(parts), static_cast<long long>(kMaxPartsPerExample),
+                  p.mode == DP_NORM_GHOST ? "; use DP_NORM_MATERIALISED for examples this long"
+                                          : "");
+    p.nparts = static_cast<int>(parts);
     p.gemm_tc = 0;
     if (bf16 && dpk::tc_gemm_supported(T, p.d_in, p.d_out)) {
       p.gemm_tc = 1;
@@ -293,7 +321,7 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
         p.implicit = 1;
         p.mode = DP_NORM_MATERIALISED;
         p.norm_tc = 1;
-        p.nparts = dpk::tc_mat_parts(p.d_in, p.d_out);
+        p.nparts = static_cast<int>(dpk::tc_mat_parts(p.d_in, p.d_out));
       }
     } else if (bf16 && dpk::tc_prescaled_supported(cfg->B, T, p.d_in, p.d_out)) {
       p.gemm_tc = 2;
@@ -303,10 +331,15 @@ void build_plan(dp_ctx* c, const dp_config* cfg) {
     if (p.conv && !p.implicit) need_unfold();
     if (p.nparts > NP) NP = p.nparts;
   }
-  c->NP = NP;
+  // the partial buffer [L][B][NP] and the row index layer * B + example
+  if (static_cast<double>(cfg->n_layers) * cfg->B > 0x7fffffff ||
+      static_cast<double>(cfg->n_layers) * cfg->B * NP * 4.0 > 0x1p50)
+    return fail(DP_ERR_SHAPE, "L * B * partial sums per example too large for the norm scratch");
+  c->NP = static_cast<int>(NP);
   c->grads_floats = grads;
   c->split_floats = splits;
   c->unf_bytes = unf;
+  return DP_OK;
 }
 
 void free_scratch(dp_ctx* c) {
@@ -625,7 +658,16 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
     const int64_t old_grads = c->grads_floats;
     const int64_t old_splits = c->split_floats;
     const int64_t old_unf = c->unf_bytes;
-    build_plan(c, cfg);
+    st = build_plan(c, cfg);
+    if (st != DP_OK) {
+      c->plan = old;
+      c->NP = oldNP;
+      c->prescaled_bytes = old_pre;
+      c->grads_floats = old_grads;
+      c->split_floats = old_splits;
+      c->unf_bytes = old_unf;
+      return st;
+    }
     c->prescaled_bytes = old_pre;  // shapes are unchanged, so is the pre-scale need
     if (c->NP > oldNP || c->grads_floats > old_grads || c->split_floats > old_splits ||
         c->unf_bytes > old_unf) {
@@ -660,7 +702,11 @@ dp_status dp_step_init(dp_ctx** ctx, const dp_config* cfg, void* cuda_stream) {
   c->dtype = cfg->dtype;
   cudaGetDevice(&c->device);
   set_scalars(c, cfg, cuda_stream);
-  build_plan(c, cfg);
+  st = build_plan(c, cfg);
+  if (st != DP_OK) {
+    delete c;
+    return st;
+  }
   st = alloc_scratch(c);
   if (st != DP_OK) {
     delete c;
@@ -785,6 +831,52 @@ dp_status dp_clip_factors(dp_ctx* c, float* d_sqnorm_out, float* d_clip_out) {
                                    c->d_flag, c->stream);
   if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clip kernel launch: %s", cudaGetErrorString(e));
   c->clip_done = true;
+  return DP_OK;
+}
+
+dp_status dp_partial_sqnorms(dp_ctx* c, float* d_sqnorm_local) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (!d_sqnorm_local) return fail(DP_ERR_ARG, "d_sqnorm_local is NULL");
+  for (int l = 0; l < c->L; ++l)
+    if (!c->norm_done[l]) return fail(DP_ERR_ORDER, "norms of layer %d not computed", l);
+  if (c->clip_done) return fail(DP_ERR_ORDER, "dp_partial_sqnorms after dp_clip_factors");
+  cudaError_t e = dpk::launch_clip(c->d_part, c->L, c->B, c->NP, c->d_nparts, c->C,
+                                   c->d_layer_sq, c->d_s, c->d_c, d_sqnorm_local, nullptr,
+                                   c->d_flag, c->stream, dpk::kClipLocal, nullptr);
+  if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clip kernel launch: %s", cudaGetErrorString(e));
+  return DP_OK;
+}
+
+dp_status dp_clip_factors_from(dp_ctx* c, const float* d_sqnorm_total, float* d_sqnorm_out,
+                               float* d_clip_out) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (!d_sqnorm_total) return fail(DP_ERR_ARG, "d_sqnorm_total is NULL");
+  for (int l = 0; l < c->L; ++l)
+    if (!c->norm_done[l]) return fail(DP_ERR_ORDER, "norms of layer %d not computed", l);
+  if (c->clip_done) return fail(DP_ERR_ORDER, "dp_clip_factors already called this step");
+  cudaError_t e = dpk::launch_clip(c->d_part, c->L, c->B, c->NP, c->d_nparts, c->C,
+                                   c->d_layer_sq, c->d_s, c->d_c, d_sqnorm_out, d_clip_out,
+                                   c->d_flag, c->stream, dpk::kClipGiven, d_sqnorm_total);
+  if (e != cudaSuccess) return fail(DP_ERR_CUDA, "clip kernel launch: %s", cudaGetErrorString(e));
+  c->clip_done = true;
+  return DP_OK;
+}
+
+dp_status dp_noise_add_range(dp_ctx* c, uint64_t p_first, int64_t n, float* d_out) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (n < 0) return fail(DP_ERR_ARG, "n < 0");
+  if (n == 0) return DP_OK;
+  if (!d_out) return fail(DP_ERR_ARG, "d_out is NULL");
+  if (!aligned16(d_out)) return fail(DP_ERR_ARG, "d_out must be 16-byte aligned");
+  dpk::NoiseAddBatch nb{};
+  nb.key = c->d_key;
+  nb.scale = c->out_scale * (c->sigma * c->C);
+  nb.out[0] = d_out;
+  nb.n[0] = n;
+  nb.p_base[0] = p_first;
+  nb.L = 1;
+  cudaError_t e = dpk::launch_noise_add(nb, c->stream);
+  if (e != cudaSuccess) return fail(DP_ERR_CUDA, "noise kernel: %s", cudaGetErrorString(e));
   return DP_OK;
 }
 
@@ -1040,6 +1132,19 @@ dp_status dp_conv2d_unfold(const dp_conv2d* conv, int32_t B, dp_dtype dtype, con
 dp_status dp_kernel_launches(int64_t* count_out) {
   if (!count_out) return fail(DP_ERR_ARG, "count_out is NULL");
   *count_out = dpk::launch_count();
+  return DP_OK;
+}
+
+dp_status dp_debug_bounded_wait(dp_ctx* c, int64_t limit_ns) {
+  if (!c) return fail(DP_ERR_ARG, "ctx is NULL");
+  if (limit_ns < 1 || limit_ns > 1000000000)
+    return fail(DP_ERR_ARG, "limit_ns must be in 1 .. 10^9");
+  DP_CUDA(dpk::launch_debug_wait(static_cast<uint64_t>(limit_ns), c->d_flag, c->stream));
+  DP_CUDA(cudaStreamSynchronize(c->stream));
+  int flag = 0;
+  DP_CUDA(cudaMemcpy(&flag, c->d_flag, sizeof(int), cudaMemcpyDeviceToHost));
+  if (flag & 2) return fail(DP_ERR_TIMEOUT, "the bounded wait gave up after %lld ns",
+                            static_cast<long long>(limit_ns));
   return DP_OK;
 }
 

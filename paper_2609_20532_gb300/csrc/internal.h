@@ -3,6 +3,8 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
+#include <functional>
+
 namespace dpk {
 
 enum InType { IN_F32 = 0, IN_BF16 = 1 };
@@ -28,9 +30,11 @@ struct Epilogue {
 
 // ---- per-example squared norms: partial sums into part[(row) * NP + p] ----
 // row = layer * B + example; every kernel writes exactly nparts(...) entries.
-int rank1_parts();
-int ghost_simt_parts(int T);
-int mat_simt_parts(int d_in, int d_out);
+// The counts are int64: a long example has ~T^2 / 8192 Gram tiles, more
+// than an int holds for T of a few million; callers bound them before launch.
+int64_t rank1_parts();
+int64_t ghost_simt_parts(int T);
+int64_t mat_simt_parts(int64_t d_in, int64_t d_out);
 
 cudaError_t launch_norm_rank1(InType t, const void* A, const void* D, int B, int d_in, int d_out,
                               float* part, int NP, int row0, cudaStream_t s);
@@ -40,9 +44,15 @@ cudaError_t launch_norm_mat_simt(InType t, const void* A, const void* D, int B, 
                                  int d_out, float* part, int NP, int row0, cudaStream_t s);
 
 // ---- cross-layer sum and clip factors ----
+// mode kClipFull: s_i = sum of this context's layer norms, then c_i.
+// mode kClipLocal: that sum into user_s only (a rank's share of s_i when the
+//   layers are split over ranks); no clip factor.
+// mode kClipGiven: s_i = s_given[i] (summed over every rank), then c_i.
+constexpr int kClipFull = 0, kClipLocal = 1, kClipGiven = 2;
 cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_nparts, float C,
                         float* layer_sq, float* s_out, float* c_out, float* user_s, float* user_c,
-                        int* flag, cudaStream_t s);
+                        int* flag, cudaStream_t s, int mode = kClipFull,
+                        const float* s_given = nullptr);
 
 // ---- clipped sum + noise (CUDA-core FFMA path) ----
 cudaError_t launch_gemm_simt(InType t, const void* A, const void* D, const float* c, int B, int T,
@@ -103,7 +113,7 @@ struct PerGradSumBatch {
   int L, B;
 };
 int pergrad_bucket(int r);                       // 1, 2, 4, ..., 32, or 0 if too wide
-int pergrad_parts(InType t, int64_t d_in, int64_t d_out, int T);  // partials per example
+int64_t pergrad_parts(InType t, int64_t d_in, int64_t d_out, int T);  // partials per example
 cudaError_t launch_pergrad_norm(InType t, PerGradBatch& g, cudaStream_t s);
 cudaError_t launch_pergrad_sum(PerGradSumBatch& g, cudaStream_t s);
 
@@ -136,6 +146,17 @@ struct ConvGeom {
 cudaError_t launch_conv_unfold(InType t, const void* x, void* a, const ConvGeom& g, int B,
                                cudaStream_t s);
 
+// ---- per-device kernel set-up ----
+// Kernel attributes (the dynamic shared-memory limit) and occupancy figures
+// belong to one device.  setup_once_per_device runs setup() the first time it
+// is asked for `key` (a kernel's address) on the current device, under a
+// process-wide lock, and returns its status; a failed set-up runs again on
+// the next call.  cached_per_device does the same for an integer (e.g. the
+// CTA pairs that fit on the device at once), computed by fn() once per
+// (key, device).
+cudaError_t setup_once_per_device(const void* key, const std::function<cudaError_t()>& setup);
+int cached_per_device(const void* key, const std::function<int()>& fn);
+
 // ---- launch count: every launcher calls note_launch() once per kernel it
 // issues (process-wide, thread-safe), read back by dp_kernel_launches() ----
 void note_launch();
@@ -147,6 +168,9 @@ void set_last_error(const char* msg);
 // ---- generator exports for tests ----
 cudaError_t launch_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
                                 uint32_t* out, cudaStream_t s);
+// one-warp kernel whose bounded mbarrier wait gives up after limit_ns and
+// sets the timeout bit (2) of *err
+cudaError_t launch_debug_wait(uint64_t limit_ns, int* err, cudaStream_t s);
 cudaError_t launch_debug_gauss(uint64_t seed, uint64_t step, uint64_t p0, int64_t n, float* out,
                                cudaStream_t s);
 

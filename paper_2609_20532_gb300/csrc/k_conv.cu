@@ -132,14 +132,13 @@ cudaError_t launch_unfold_t(const void* x, void* a, const ConvGeom& g, int B, in
   if (U <= kConvTab) {
     const int smem = 3 * U * static_cast<int>(sizeof(int));
     if (smem > 48 * 1024) {
-      static bool attr_set = false;
-      if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(k_conv_unfold_rows<Unit>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             3 * kConvTab * static_cast<int>(sizeof(int)));
-        if (e != cudaSuccess) return e;
-        attr_set = true;
-      }
+      cudaError_t e = setup_once_per_device(
+          reinterpret_cast<const void*>(&k_conv_unfold_rows<Unit>), [] {
+            return cudaFuncSetAttribute(k_conv_unfold_rows<Unit>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        3 * kConvTab * static_cast<int>(sizeof(int)));
+          });
+      if (e != cudaSuccess) return e;
     }
     const int64_t warps_needed = rows;  // at least one row per warp
     const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;

@@ -29,7 +29,8 @@ __global__ void __launch_bounds__(256) k_noise_adamw(float* __restrict__ grad, f
                                                      const uint64_t* __restrict__ key,
                                                      float noise_scale, int add_noise, int write_grad,
                                                      AdamWArgs h) {
-  const uint64_t seed = key[0], step = key[1];
+  const PhiloxKeys keys = philox_keys(key[0]);  // round keys formed once per thread
+  const uint64_t step = key[1];
   const uint64_t q_first = p_base >> 2;
   const int64_t nq = static_cast<int64_t>(((p_base + n - 1) >> 2) - q_first + 1);
   const bool vec = ((p_base & 3) == 0) &&
@@ -39,7 +40,7 @@ __global__ void __launch_bounds__(256) k_noise_adamw(float* __restrict__ grad, f
        gq += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const uint64_t q = q_first + gq;
     float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (add_noise) z = gauss_quad(seed, step, q);
+    if (add_noise) z = gauss_quad(keys, step, q);
     const int64_t e0 = static_cast<int64_t>(4 * q) - static_cast<int64_t>(p_base);
     if (vec && e0 + 3 < n) {
       float4 g = *reinterpret_cast<const float4*>(grad + e0);

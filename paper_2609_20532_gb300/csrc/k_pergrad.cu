@@ -672,13 +672,11 @@ __global__ void __launch_bounds__(kThreads) k_pergrad_sum(const __grid_constant_
 
 template <typename TIn, int R>
 cudaError_t launch_norm_t(const PerGradBatch& g, int blocks, cudaStream_t s) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_pergrad_norm<TIn, R>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kPerGradSmem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  cudaError_t e = setup_once_per_device(reinterpret_cast<const void*>(&k_pergrad_norm<TIn, R>), [] {
+    return cudaFuncSetAttribute(k_pergrad_norm<TIn, R>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, kPerGradSmem);
+  });
+  if (e != cudaSuccess) return e;
   note_launch();
   k_pergrad_norm<TIn, R><<<blocks, kThreads, kPerGradSmem, s>>>(g);
   return cudaGetLastError();
@@ -713,26 +711,23 @@ bool pergrad_mma(InType t, int64_t n, int r, int T) {
   return t == IN_BF16 && n % 8 == 0 && r > 0 && T <= kTcMaxAccum;
 }
 
-int pergrad_parts(InType t, int64_t d_in, int64_t d_out, int T) {
+int64_t pergrad_parts(InType t, int64_t d_in, int64_t d_out, int T) {
   const int r = static_cast<int>(d_in < d_out ? d_in : d_out);
   const int64_t n = d_in < d_out ? d_out : d_in;
   const int R = pergrad_bucket(r);
   if (R == 0) return 0;
-  if (pergrad_mma(t, n, r, T)) return static_cast<int>((n + kMmaCols - 1) / kMmaCols);
+  if (pergrad_mma(t, n, r, T)) return (n + kMmaCols - 1) / kMmaCols;
   const int vj = R <= 8 ? 4 : (R <= 16 ? 2 : 1);
-  return static_cast<int>((n + kThreads * vj - 1) / (kThreads * vj));
+  return (n + kThreads * vj - 1) / (kThreads * vj);
 }
 
 template <int NT>
 cudaError_t launch_mma_t(const PerGradBatch& g, int blocks, cudaStream_t s) {
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_pergrad_norm_mma<NT>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         MmaCfg<NT>::SMEM);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+  cudaError_t e = setup_once_per_device(reinterpret_cast<const void*>(&k_pergrad_norm_mma<NT>), [] {
+    return cudaFuncSetAttribute(k_pergrad_norm_mma<NT>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, MmaCfg<NT>::SMEM);
+  });
+  if (e != cudaSuccess) return e;
   note_launch();
   k_pergrad_norm_mma<NT><<<blocks, kMmaThreads, MmaCfg<NT>::SMEM, s>>>(g);
   return cudaGetLastError();

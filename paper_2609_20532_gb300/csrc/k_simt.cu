@@ -11,6 +11,7 @@
 
 #include "internal.h"
 #include "philox.cuh"
+#include "tc_util.cuh"
 
 namespace dpk {
 
@@ -246,10 +247,14 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
 // layers j, j + 32, ... (each layer's partials in slot order), then a fixed
 // butterfly adds the 32 lane sums, so the order never depends on timing.
 // ---------------------------------------------------------------------------
+// mode kClipLocal: only the layers' norms and their sum (into user_s); no
+// clip factor, no flag.  mode kClipGiven: s_i = s_given[i] (the squared norm
+// summed over every rank's layers) instead of this context's sum.
 __global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
                        const int* __restrict__ nparts, float C, float* __restrict__ layer_sq,
                        float* __restrict__ s_out, float* __restrict__ c_out,
-                       float* __restrict__ user_s, float* __restrict__ user_c, int* flag) {
+                       float* __restrict__ user_s, float* __restrict__ user_c, int* flag,
+                       int mode, const float* __restrict__ s_given) {
   const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = static_cast<int>(threadIdx.x) & 31;
   if (w >= B) return;  // the whole warp leaves together
@@ -266,6 +271,11 @@ __global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
   if (lane != 0) return;
+  if (mode == kClipLocal) {
+    user_s[i] = s;
+    return;
+  }
+  if (mode == kClipGiven) s = s_given[i];
   float c;
   if (!isfinite(s)) {
     atomicOr(flag, 1);
@@ -312,7 +322,8 @@ __device__ __forceinline__ void noise_store(float* __restrict__ out, int64_t e0,
 __global__ void __launch_bounds__(256) k_noise_add(const __grid_constant__ NoiseAddBatch b) {
   int l = 0;
   while (l + 1 < b.L && static_cast<int64_t>(blockIdx.x) >= b.block0[l + 1]) ++l;
-  const uint64_t seed = b.key[0], step = b.key[1];
+  const PhiloxKeys keys = philox_keys(b.key[0]);  // round keys formed once per thread
+  const uint64_t step = b.key[1];
   float* __restrict__ out = b.out[l];
   const int64_t n = b.n[l];
   const uint64_t p_base = b.p_base[l];
@@ -327,8 +338,8 @@ __global__ void __launch_bounds__(256) k_noise_add(const __grid_constant__ Noise
   for (int j = threadIdx.x; j < cnt; j += 512) {
     const bool has_b = j + 256 < cnt;
     const int jb = has_b ? j + 256 : j;
-    const float4 za = gauss_quad(seed, step, q0 + j);
-    const float4 zb = gauss_quad(seed, step, q0 + jb);
+    const float4 za = gauss_quad(keys, step, q0 + j);
+    const float4 zb = gauss_quad(keys, step, q0 + jb);
     noise_store(out, e_base + 4 * j, n, vec, b.scale, za);
     if (has_b) noise_store(out, e_base + 4 * jb, n, vec, b.scale, zb);
   }
@@ -378,15 +389,29 @@ __global__ void k_set_key(uint64_t seed, uint64_t step, uint64_t* __restrict__ k
   *flag = 0;
 }
 
+// A wait that runs out: one thread waits, with the pipelines' bounded-wait
+// helper, for phase 0 of an mbarrier that nothing ever arrives on; after
+// limit_ns it records the timeout in *err and the kernel returns.  No TMA
+// copy, no MMA and no TMEM are involved, so nothing is left in flight.
+__global__ void k_debug_wait(uint64_t limit_ns, int* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(&bar, 1);
+    abort_flag = 0;
+    tc::fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) tc::mbar_wait_for(&bar, 0, &abort_flag, err, limit_ns);
+}
+
 __global__ void k_debug_philox(uint64_t seed, uint64_t step, uint64_t q0, int64_t nq,
                                uint32_t* __restrict__ out) {
   for (int64_t r = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; r < nq;
        r += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const uint64_t q = q0 + r;
-    const uint4 w = philox4x32_10(
-        make_uint4(static_cast<uint32_t>(q), static_cast<uint32_t>(q >> 32),
-                   static_cast<uint32_t>(step), static_cast<uint32_t>(step >> 32)),
-        static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32));
+    const uint4 w = philox4x32_10(philox_counter(q, step), static_cast<uint32_t>(seed),
+                                  static_cast<uint32_t>(seed >> 32));
     out[4 * r + 0] = w.x;
     out[4 * r + 1] = w.y;
     out[4 * r + 2] = w.z;
@@ -413,13 +438,33 @@ int grid_for(int64_t work, int threads) {
 
 }  // namespace
 
-int rank1_parts() { return 1; }
-int ghost_simt_parts(int T) {
-  const int nb = (T + GT - 1) / GT;
+int64_t rank1_parts() { return 1; }
+int64_t ghost_simt_parts(int T) {
+  const int64_t nb = (static_cast<int64_t>(T) + GT - 1) / GT;
   return nb * (nb + 1) / 2;
 }
-int mat_simt_parts(int d_in, int d_out) {
+int64_t mat_simt_parts(int64_t d_in, int64_t d_out) {
   return ((d_in + SB - 1) / SB) * ((d_out + SB - 1) / SB);
+}
+
+// The per-example norm kernels below index examples with blockIdx.y / .z,
+// which stop at 65535: larger batches launch once per 65535 examples, each
+// launch on its slice of A, D and the partial-sum rows.
+constexpr int kMaxGridYZ = 65535;
+
+template <typename F>
+cudaError_t per_example_slices(InType t, const void* A, const void* D, int B, int T, int d_in,
+                               int d_out, int row0, F&& launch) {
+  const int64_t es = t == IN_F32 ? 4 : 2;
+  for (int b0 = 0; b0 < B; b0 += kMaxGridYZ) {
+    const int nb = B - b0 < kMaxGridYZ ? B - b0 : kMaxGridYZ;
+    const char* a = static_cast<const char*>(A) + static_cast<int64_t>(b0) * T * d_in * es;
+    const char* d = static_cast<const char*>(D) + static_cast<int64_t>(b0) * T * d_out * es;
+    launch(static_cast<const void*>(a), static_cast<const void*>(d), nb, row0 + b0);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_norm_rank1(InType t, const void* A, const void* D, int B, int d_in, int d_out,
@@ -438,41 +483,50 @@ cudaError_t launch_norm_rank1(InType t, const void* A, const void* D, int B, int
 
 cudaError_t launch_norm_ghost_simt(InType t, const void* A, const void* D, int B, int T, int d_in,
                                    int d_out, float* part, int NP, int row0, cudaStream_t s) {
-  const dim3 grid(ghost_simt_parts(T), B);
-  note_launch();
-  if (t == IN_F32)
-    k_norm_ghost_simt<float><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
-                                                   static_cast<const float*>(D), T, d_in, d_out,
-                                                   part, NP, row0);
-  else
-    k_norm_ghost_simt<__nv_bfloat16><<<grid, 256, 0, s>>>(
-        static_cast<const __nv_bfloat16*>(A), static_cast<const __nv_bfloat16*>(D), T, d_in,
-        d_out, part, NP, row0);
-  return cudaGetLastError();
+  const int64_t parts = ghost_simt_parts(T);
+  if (parts > NP || parts > 0x7fffffff) return cudaErrorInvalidValue;
+  return per_example_slices(t, A, D, B, T, d_in, d_out, row0,
+                            [&](const void* a, const void* d, int nb, int r0) {
+    const dim3 grid(static_cast<unsigned>(parts), nb);
+    note_launch();
+    if (t == IN_F32)
+      k_norm_ghost_simt<float><<<grid, 256, 0, s>>>(static_cast<const float*>(a),
+                                                     static_cast<const float*>(d), T, d_in, d_out,
+                                                     part, NP, r0);
+    else
+      k_norm_ghost_simt<__nv_bfloat16><<<grid, 256, 0, s>>>(
+          static_cast<const __nv_bfloat16*>(a), static_cast<const __nv_bfloat16*>(d), T, d_in,
+          d_out, part, NP, r0);
+  });
 }
 
 cudaError_t launch_norm_mat_simt(InType t, const void* A, const void* D, int B, int T, int d_in,
                                  int d_out, float* part, int NP, int row0, cudaStream_t s) {
-  const dim3 grid((d_out + SB - 1) / SB, (d_in + SB - 1) / SB, B);
-  Epilogue ep{};
-  note_launch();
-  if (t == IN_F32)
-    k_gemm_simt<float, true, SB><<<grid, 256, 0, s>>>(static_cast<const float*>(A),
-                                                       static_cast<const float*>(D), nullptr, T,
-                                                       B, d_in, d_out, nullptr, ep, part, NP, row0);
-  else
-    k_gemm_simt<__nv_bfloat16, true, SB><<<grid, 256, 0, s>>>(
-        static_cast<const __nv_bfloat16*>(A), static_cast<const __nv_bfloat16*>(D), nullptr, T,
-        B, d_in, d_out, nullptr, ep, part, NP, row0);
-  return cudaGetLastError();
+  if (mat_simt_parts(d_in, d_out) > NP || (d_in + SB - 1) / SB > kMaxGridYZ)
+    return cudaErrorInvalidValue;
+  return per_example_slices(t, A, D, B, T, d_in, d_out, row0,
+                            [&](const void* a, const void* d, int nb, int r0) {
+    const dim3 grid((d_out + SB - 1) / SB, (d_in + SB - 1) / SB, nb);
+    Epilogue ep{};
+    note_launch();
+    if (t == IN_F32)
+      k_gemm_simt<float, true, SB><<<grid, 256, 0, s>>>(static_cast<const float*>(a),
+                                                         static_cast<const float*>(d), nullptr, T,
+                                                         nb, d_in, d_out, nullptr, ep, part, NP,
+                                                         r0);
+    else
+      k_gemm_simt<__nv_bfloat16, true, SB><<<grid, 256, 0, s>>>(
+          static_cast<const __nv_bfloat16*>(a), static_cast<const __nv_bfloat16*>(d), nullptr, T,
+          nb, d_in, d_out, nullptr, ep, part, NP, r0);
+  });
 }
 
 cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_nparts, float C,
                         float* layer_sq, float* s_out, float* c_out, float* user_s, float* user_c,
-                        int* flag, cudaStream_t s) {
+                        int* flag, cudaStream_t s, int mode, const float* s_given) {
   note_launch();
   k_clip<<<(B + 7) / 8, 256, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out,
-                                      user_s, user_c, flag);
+                                      user_s, user_c, flag, mode, s_given);
   return cudaGetLastError();
 }
 
@@ -539,6 +593,12 @@ cudaError_t launch_load_key(const uint64_t* host_key_dev, uint64_t* key, int* fl
                             cudaStream_t s) {
   note_launch();
   k_load_key<<<1, 1, 0, s>>>(host_key_dev, key, flag);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_debug_wait(uint64_t limit_ns, int* err, cudaStream_t s) {
+  note_launch();
+  k_debug_wait<<<1, 32, 0, s>>>(limit_ns, err);
   return cudaGetLastError();
 }
 

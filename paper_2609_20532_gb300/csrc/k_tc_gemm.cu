@@ -473,7 +473,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
               // when p_base is a multiple of 4, else they straddle two (a
               // layer after one whose size is not a multiple of 4)
               if (k0 + 4 * q >= d_out) break;
-              const float4 z = gauss4_at(seed, step, prow + k0 + 4 * q);
+              const float4 z = gauss4_at<Root::kSqrt>(seed, step, prow + k0 + 4 * q);
               add_noise_slot<0, QPT, C::HALF>(S, q, z, g.sigmaC);
             }
           }
@@ -601,24 +601,25 @@ int gemm_nb(int64_t d_out) { return d_out <= 128 ? 128 : BN; }
 template <bool NORM, bool PAIR, int NB, bool CONV>
 cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
   using C = Cfg<PAIR, NB>;
-  static bool attr_set = false;
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<NORM, PAIR, NB, CONV>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         C::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    if constexpr (NB == 256) {
-      // setmaxnreg moves registers within what the block was launched with:
-      // the split must fit the compiled count, else the raise never returns
-      cudaFuncAttributes fa{};
-      e = cudaFuncGetAttributes(&fa, k_gemm_tc<NORM, PAIR, NB, CONV>);
-      if (e != cudaSuccess) return e;
-      if (fa.numRegs * GEMM_THREADS < 4 * 32 * REGS_CTRL + NUM_EPI_WARPS * 32 * REGS_EPI ||
-          fa.numRegs > REGS_EPI)
-        return cudaErrorInvalidConfiguration;
-    }
-    attr_set = true;
-  }
+  cudaError_t e = setup_once_per_device(
+      reinterpret_cast<const void*>(&k_gemm_tc<NORM, PAIR, NB, CONV>), []() -> cudaError_t {
+        cudaError_t r = cudaFuncSetAttribute(k_gemm_tc<NORM, PAIR, NB, CONV>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             C::SMEM_BYTES);
+        if (r != cudaSuccess) return r;
+        if constexpr (NB == 256) {
+          // setmaxnreg moves registers within what the block was launched with:
+          // the split must fit the compiled count, else the raise never returns
+          cudaFuncAttributes fa{};
+          r = cudaFuncGetAttributes(&fa, k_gemm_tc<NORM, PAIR, NB, CONV>);
+          if (r != cudaSuccess) return r;
+          if (fa.numRegs * GEMM_THREADS < 4 * 32 * REGS_CTRL + NUM_EPI_WARPS * 32 * REGS_EPI ||
+              fa.numRegs > REGS_EPI)
+            return cudaErrorInvalidConfiguration;
+        }
+        return cudaSuccess;
+      });
+  if (e != cudaSuccess) return e;
   g.tile_start[0] = 0;
   for (int l = 0; l < g.L; ++l) {
     g.n_m[l] = (g.d_in[l] + C::TILE_M - 1) / C::TILE_M;
@@ -630,7 +631,6 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
   const int sms = device_sm_count();
   if constexpr (PAIR) {
     // persistent grid: as many pairs as can be resident at once
-    static int max_pairs = 0;
     cudaLaunchConfig_t cfg = {};
     cfg.blockDim = dim3(GEMM_THREADS);
     cfg.dynamicSmemBytes = C::SMEM_BYTES;
@@ -642,16 +642,19 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (max_pairs == 0) {
-      cfg.gridDim = dim3(sms);
-      int n = 0;
-      if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<NORM, PAIR, NB, CONV>, &cfg) != cudaSuccess ||
-          n < 1) {
-        cudaGetLastError();
-        n = sms / 2;
-      }
-      max_pairs = n < sms / 2 ? n : sms / 2;
-    }
+    const int max_pairs =
+        cached_per_device(reinterpret_cast<const void*>(&k_gemm_tc<NORM, PAIR, NB, CONV>), [&] {
+          cudaLaunchConfig_t q = cfg;
+          q.gridDim = dim3(sms);
+          int n = 0;
+          if (cudaOccupancyMaxActiveClusters(&n, k_gemm_tc<NORM, PAIR, NB, CONV>, &q) !=
+                  cudaSuccess ||
+              n < 1) {
+            cudaGetLastError();
+            n = sms / 2;
+          }
+          return n < sms / 2 ? n : sms / 2;
+        });
     const int pairs = tiles < max_pairs ? tiles : max_pairs;
     cfg.gridDim = dim3(2 * pairs);
     note_launch();
@@ -908,12 +911,12 @@ cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const floa
   return launch_any<false>(g, s);
 }
 
-int tc_mat_parts(int64_t d_in, int64_t d_out) {
+int64_t tc_mat_parts(int64_t d_in, int64_t d_out) {
   const int64_t tile_m = use_pair(d_in) ? 2 * BM : BM;
   const int64_t ctas_per_tile = use_pair(d_in) ? 2 : 1;
   const int64_t nb = gemm_nb(d_out);
-  return static_cast<int>(((d_in + tile_m - 1) / tile_m) * ((d_out + nb - 1) / nb) *
-                          ctas_per_tile * NUM_EPI_WARPS);
+  return ((d_in + tile_m - 1) / tile_m) * ((d_out + nb - 1) / nb) * ctas_per_tile *
+         NUM_EPI_WARPS;
 }
 
 cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d_in, int d_out,

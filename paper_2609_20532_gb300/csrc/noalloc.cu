@@ -78,11 +78,13 @@ extern "C" dp_status dp_layer_sqnorms_noalloc(const void* A, const void* D, int3
     return noalloc_fail(DP_ERR_SHAPE, "bf16 rows must be a multiple of 16 bytes");
 
   const bool tc = dtype == DP_BF16 && dpk::tc_ghost_supported(T, d_in, d_out);
-  const int NP = tc ? dpk::tc_ghost_parts(T) : dpk::ghost_simt_parts(T);
-  if (int64_t(B) * NP > kNoallocMaxPartials)
+  // partials per example, counted in 64 bits (about T^2 / 8192 of them)
+  const int64_t parts = tc ? dpk::tc_ghost_parts(T) : dpk::ghost_simt_parts(T);
+  if (parts < 1 || parts > kNoallocMaxPartials || int64_t(B) * parts > kNoallocMaxPartials)
     return noalloc_fail(DP_ERR_SHAPE,
                         "B x partials-per-example exceeds the 2^20-float scratch of "
                         "dp_layer_sqnorms_noalloc; use dp_layer_norms instead");
+  const int NP = static_cast<int>(parts);
 
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
@@ -96,6 +98,15 @@ extern "C" dp_status dp_layer_sqnorms_noalloc(const void* A, const void* D, int3
       if (e != cudaSuccess || !p) {
         cudaGetLastError();
         return noalloc_fail(DP_ERR_CUDA, "cudaGetSymbolAddress of the scratch array failed");
+      }
+      // the tensor-core kernels' per-device set-up happens here too, so that
+      // calls after the first one make no set-up call of any kind
+      if (dpk::tma_encode_available()) {
+        e = dpk::tc_ghost_prepare();
+        if (e != cudaSuccess) {
+          cudaGetLastError();
+          return noalloc_fail(DP_ERR_CUDA, "set-up of the Gram kernels failed");
+        }
       }
       g_dev_ptr[dev] = static_cast<float*>(p);
     }

@@ -11,9 +11,17 @@ namespace dpk {
 
 // Gram-form per-example norms on tensor cores; one launch can serve up to
 // kGhostMaxLayers layers of a step.
+// T up to kTcGhostMaxT (a Gram of T^2 / 2 products per example; longer
+// examples take the materialised form).  tc_ghost_parts(T) partial sums per
+// example: CTA-pair items when ceil(T / 128) is even, single-CTA strips when
+// it is odd.
 constexpr int kGhostMaxLayers = 8;
+constexpr int kTcGhostMaxT = 1 << 16;
 bool tc_ghost_supported(int T, int64_t d_in, int64_t d_out);
-int tc_ghost_parts(int T);
+int64_t tc_ghost_parts(int T);
+// The once-per-device set-up of both Gram kernels (shared-memory limits, the
+// resident-pair count), so that later launches make no set-up calls.
+cudaError_t tc_ghost_prepare();
 cudaError_t tc_launch_ghost(const void* A, const void* D, int B, int T, int d_in, int d_out,
                             float* part, int NP, int row0, int* err, cudaStream_t s);
 cudaError_t tc_launch_ghost_batch(int L, const void* const* A, const void* const* D,
@@ -41,7 +49,7 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
                                     const ConvGeom* const* conv = nullptr);
 bool tc_conv_implicit_ok(const ConvGeom& g, int T);
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out);
-int tc_mat_parts(int64_t d_in, int64_t d_out);
+int64_t tc_mat_parts(int64_t d_in, int64_t d_out);
 cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d_in, int d_out,
                                float* part, int NP, int row0, int* err, cudaStream_t s,
                                const ConvGeom* conv = nullptr);

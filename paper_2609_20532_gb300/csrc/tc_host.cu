@@ -6,7 +6,9 @@
 #include <cudaTypedefs.h>
 
 #include <atomic>
+#include <map>
 #include <mutex>
+#include <utility>
 
 #include "tc.h"
 
@@ -77,6 +79,36 @@ bool make_tma_f32_split(CUtensorMap* m, void* base, int split, uint64_t rows, ui
   return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, d, st, b, es,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+namespace {
+std::mutex g_setup_mu;
+std::map<std::pair<const void*, int>, int> g_setup_done;   // (key, device) -> 1
+std::map<std::pair<const void*, int>, int> g_cached;       // (key, device) -> value
+}  // namespace
+
+cudaError_t setup_once_per_device(const void* key, const std::function<cudaError_t()>& setup) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lk(g_setup_mu);
+  const auto k = std::make_pair(key, dev);
+  if (g_setup_done.count(k)) return cudaSuccess;
+  e = setup();
+  if (e == cudaSuccess) g_setup_done[k] = 1;
+  return e;
+}
+
+int cached_per_device(const void* key, const std::function<int()>& fn) {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  std::lock_guard<std::mutex> lk(g_setup_mu);
+  const auto k = std::make_pair(key, dev);
+  auto it = g_cached.find(k);
+  if (it != g_cached.end()) return it->second;
+  const int v = fn();
+  g_cached[k] = v;
+  return v;
 }
 
 int device_sm_count() {

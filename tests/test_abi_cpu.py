@@ -176,3 +176,35 @@ def test_header_is_plain_c_and_cpp():
             r = subprocess.run([gcc, "-fsyntax-only", std, "-Wall", "-Wextra", "-Werror",
                                 "-x", lang, "-I", inc, src], capture_output=True, text=True)
             assert r.returncode == 0, (lang, r.stderr)
+
+
+@pytest.mark.parametrize("dtype,B,T,d", [
+    (dp.DP_BF16, 1, 1 << 22, 8),     # ~T^2/8192 partial sums would overflow 32-bit counts
+    (dp.DP_F32, 1, 1 << 22, 8),
+    (dp.DP_BF16, 1, 4_194_304, 4096),
+    (dp.DP_BF16, 4096, 1 << 17, 8),  # fits 32 bits, exceeds the 2^20-float scratch
+])
+def test_noalloc_rejects_long_examples_on_host(L, dtype, B, T, d):
+    """dp_layer_sqnorms_noalloc counts the Gram form's partial sums in 64 bits
+    and refuses requests beyond its static scratch on the host.  The pointers
+    are never dereferenced: the check comes before any CUDA call, so this
+    runs without a GPU and launches nothing."""
+    n0 = dp.dp_kernel_launches()
+    fake = ctypes.c_void_p(1 << 20)   # 16-byte aligned, never touched
+    st = L.dp_layer_sqnorms_noalloc(fake, fake, B, T, d, d, dtype, fake, None)
+    assert st == 2, (st, dp.dp_last_error())
+    assert "scratch" in dp.dp_last_error()
+    assert dp.dp_kernel_launches() == n0
+
+
+@pytest.mark.parametrize("mode,T,d", [
+    (dp.DP_NORM_GHOST, 1 << 22, 8),  # forced Gram form on very long examples
+])
+def test_init_rejects_gram_form_beyond_its_partials(L, mode, T, d):
+    """A forced Gram form whose partial sums per example exceed the norm
+    scratch's bound is refused on the host with DP_ERR_SHAPE (the count is
+    formed in 64 bits, so it cannot wrap into a small or negative number)."""
+    cfg = _cfg(layers=[(d, d)], B=1, T=T, dtype="bf16", norm_mode=mode)
+    st, h = _init_status(L, cfg)
+    assert st == 2 and not h, (st, dp.dp_last_error())
+    assert "partial sums" in dp.dp_last_error()

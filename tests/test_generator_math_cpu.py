@@ -52,18 +52,24 @@ def _ln_u0(u):
     return _fma(e.astype(np.float64), ln2, p)
 
 
-def _sincospi_0_2(x):
+def _sincospi_0_2(X):
+    """The kernel's steps on X = RN(x_odd), the float of the word; they give
+    sin / cos(pi x) for x = X 2^-31."""
     body = _body("void sincospi_0_2")
     ps_body = body[body.index("const float ps"):body.index("const float pc")]
     pc_body = body[body.index("const float pc"):body.index("const bool odd")]
     cs = [float(v) for v in re.findall(FLOAT, ps_body)]
     cc = [float(v) for v in re.findall(FLOAT, pc_body)]
     assert len(cs) == 5 and len(cc) == 5
-    x = _f32(x)
-    sh = _f32(2.0 * x + 12582912.0)              # fmaf(2, x, 1.5 * 2^23)
-    k = _f32(sh - 12582912.0)
+    X = _f32(X)
+    sh = _fma(X, 2.0 ** -30, 12582912.0)         # 2x + 1.5 * 2^23, rounded once
+    mk = _fma(sh, -0.5, 6291456.0)               # -k / 2, exact
     q = sh.astype(np.float32).view(np.int32)
-    y = _fma(-0.5, k, x)
+    y = _fma(X, 2.0 ** -31, mk)                  # x - k / 2
+    # the folded steps equal the plain ones: k = sh - 1.5 * 2^23, y = x - k / 2
+    k = _f32(sh - 12582912.0)
+    assert np.array_equal(mk, -0.5 * k)
+    assert np.array_equal(y, _fma(-0.5, k, _f32(X) * 2.0 ** -31))
     t = _f32(y * y)
     ps = np.full_like(t, cs[0])
     for c in cs[1:]:
@@ -112,8 +118,9 @@ def test_sincospi_error_bound_and_exact_zeros(seed):
     edges = np.array([0, 1, 1 << 30, 1 << 31, 3 << 30, (1 << 32) - 1, (1 << 29), (5 << 29)],
                      dtype=np.uint64)
     words = np.concatenate([words, edges])
-    two_u1 = _f32(words.astype(np.float64)) * 2.0 ** -31   # 2 u1 = RN(x_odd) 2^-31
-    s, c = _sincospi_0_2(two_u1)
+    X = _f32(words.astype(np.float64))                     # RN(x_odd)
+    two_u1 = X * 2.0 ** -31                                  # 2 u1 = RN(x_odd) 2^-31
+    s, c = _sincospi_0_2(X)
     s_ref, c_ref = O.sincospi(two_u1)
     for got, ref in ((s, s_ref), (c, c_ref)):
         zero = ref == 0

@@ -7,6 +7,7 @@ within the same bounds normwise per layer.
 """
 
 import math
+import time
 
 import numpy as np
 import pytest
@@ -305,6 +306,46 @@ def test_call_order_errors():
         dp.dp_step_destroy(ctx)
 
 
+def test_bounded_wait_that_runs_out_is_reported_and_context_stays_usable():
+    """The failure path of every pipeline wait: a device wait that nothing
+    satisfies gives up after its limit (1 ms here), the call and the step's
+    dp_audit_emit report DP_ERR_TIMEOUT, and after a re-key the same context
+    runs a correct step (Algorithm 1's checker would reject the failed one)."""
+    w = W.custom("timeout", [(136, 72), (64, 200)], 3, 80, "bf16", C=0.05, sigma=0.7,
+                 d_std=0.1, wid=611)
+    layers = W.make_inputs(w, seed=2)
+    dev = torch.device(DEV)
+    Ad = [A.to(dev) for A, _ in layers]
+    Dd = [D.to(dev) for _, D in layers]
+    out = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, seed=3, step=5,
+                         audit_capacity=w.B)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.run_step(ctx, Ad, Dd, out)
+        t0 = time.perf_counter()
+        assert dp.dp_debug_bounded_wait(ctx, 1_000_000) == 7          # DP_ERR_TIMEOUT
+        assert time.perf_counter() - t0 < 5.0
+        with pytest.raises(dp.DPError) as ei:
+            dp.dp_audit_emit(ctx, range(w.B), len(w.layers))
+        assert ei.value.status == 7
+        assert "gave up" in str(ei.value)
+        # a wait that is satisfied in time reports nothing: out of range is an argument error
+        assert dp.lib().dp_debug_bounded_wait(ctx, 0) == 1
+        # re-key: the flag is cleared and the next step is correct
+        dp.dp_step_init(cfg, None, ctx)
+        dp.run_step(ctx, Ad, Dd, out)
+        recs = dp.dp_audit_emit(ctx, range(w.B), len(w.layers))
+        torch.cuda.synchronize()
+    finally:
+        dp.dp_step_destroy(ctx)
+    ref = O.dp_step([(W.to_f64(A), W.to_f64(D)) for A, D in layers], f32(w.C), f32(w.sigma),
+                    3, 5)
+    assert rel_err_elementwise(recs["layer_sqnorm"].astype(np.float64).T, ref["n"]) <= TOL["bf16"]
+    for o, r in zip(out, ref["out"]):
+        assert rel_err_normwise(o.double().cpu().numpy(), r) <= TOL["bf16"]
+
+
 def test_commit_then_noise_equals_one_shot():
     """Commit (DP_NO_NOISE), re-key with the released seed, DP_NOISE_ONLY:
     equals the one-shot noisy output (Algorithm 2 commit-then-release)."""
@@ -600,6 +641,74 @@ def test_sweep_point_full_size(name):
     for i in range(w.B):                     # the oracle's sum, one example at a time
         S += O.clipped_sum(W.to_f64(A[i:i + 1, :, rows]), W.to_f64(D[i:i + 1]), ones)
     assert rel_err_normwise(resu["out"][0][rows], S) <= TOL["bf16"]
+    # the clipped, noisy output of the first run on the same rows, with the
+    # clip factors the GPU formed (checked above on the sampled examples)
+    c_gpu = res["c"].astype(np.float64)
+    Sc = np.zeros((rows.size, 4096))
+    for i in range(w.B):
+        Sc += O.clipped_sum(W.to_f64(A[i:i + 1, :, rows]), W.to_f64(D[i:i + 1]), c_gpu[i:i + 1])
+    z = np.stack([O.gaussian_noise(4, 9, int(j) * 4096, 4096) for j in rows])
+    ref = Sc + f32(w.sigma) * f32(w.C) * z
+    assert rel_err_normwise(res["out"][0][rows], ref) <= TOL["bf16"]
+
+
+def test_fused_noise_of_the_tensor_core_sum_elementwise():
+    """The noise the tensor-core clipped sum adds inside its main loop, alone:
+    with D = 0 every S_l is exactly 0, so out = out_scale * sigma * C * z and
+    each element must be within 1e-6 of the oracle's z (llm_bf16 shapes and
+    batch, sampled rows of every layer).  Then, on the real inputs, the noisy
+    output minus the noiseless commitment is that noise to 1e-6 plus the
+    fp32 rounding of the sums (a few ulp of each output)."""
+    w = W.get("llm_bf16")
+    dev = torch.device(DEV)
+    g = torch.Generator(device=dev)
+    g.manual_seed(5)
+    Ad = [torch.randn(w.B, w.T, i, generator=g, device=dev).to(torch.bfloat16)
+          for i, _ in w.layers]
+    Z = [torch.zeros(w.B, w.T, o, device=dev, dtype=torch.bfloat16) for _, o in w.layers]
+    outs = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+    scale, seed, step = 1.0 / w.B, 17, 4
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=scale, seed=seed,
+                         step=step)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        assert all(dp.dp_layer_path(ctx, l)[1] == 1 for l in range(len(w.layers)))
+        dp.run_step(ctx, Ad, Z, outs)
+        torch.cuda.synchronize()
+        rng = np.random.default_rng(8)
+        k = scale * f32(w.sigma) * f32(w.C)
+        off = 0
+        for l, (d_in, d_out) in enumerate(w.layers):
+            rows = np.sort(rng.choice(d_in, size=6, replace=False))
+            z = np.stack([O.gaussian_noise(seed, step, off + int(j) * d_out, d_out) for j in rows])
+            got = outs[l][torch.as_tensor(rows, device=dev)].double().cpu().numpy()
+            assert rel_err_elementwise(got, k * z) <= 1e-6, l
+            off += d_in * d_out
+        # real inputs: noisy minus noiseless
+        Dd = [(torch.randn(w.B, w.T, o, generator=g, device=dev) * w.d_std).to(torch.bfloat16)
+              for _, o in w.layers]
+        noisy = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+        clean = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+        dp.dp_step_init(cfg, None, ctx)
+        dp.run_step(ctx, Ad, Dd, noisy)
+        dp.dp_step_init(cfg, None, ctx)
+        dp.run_step(ctx, Ad, Dd, clean, flags=dp.DP_NO_NOISE)
+        torch.cuda.synchronize()
+        off = 0
+        for l, (d_in, d_out) in enumerate(w.layers):
+            rows = torch.as_tensor(np.sort(rng.choice(d_in, size=4, replace=False)), device=dev)
+            a = noisy[l][rows].double().cpu().numpy()
+            b = clean[l][rows].double().cpu().numpy()
+            z = np.stack([O.gaussian_noise(seed, step, off + int(j) * d_out, d_out)
+                          for j in rows.cpu().numpy()])
+            want = k * z
+            # each of the B folds into the fp32 accumulator rounds once, and the
+            # noisy run adds the noise before the folds, the clean one does not
+            bound = 1e-6 * np.abs(want) + w.B * 2.0 ** -24 * (np.abs(a) + np.abs(b))
+            assert np.all(np.abs((a - b) - want) <= bound), l
+            off += d_in * d_out
+    finally:
+        dp.dp_step_destroy(ctx)
 
 
 def test_batched_norms_equal_per_layer_calls():
@@ -1182,11 +1291,12 @@ def test_roberta_adapters_with_head_reduced():
 
 def test_data_parallel_step_on_one_rank():
     """data_parallel_step through the library on a one-rank NCCL group: the
-    commitment, the (trivial) all-reduce and the noise added after it give
-    the same bits as an eager step of the same context."""
+    commitment, the (trivial) reduce-scatter, the noise of the rank's slice
+    (all of it) and the all-gather give the same bits as an eager step of the
+    same context."""
     import socket
     import torch.distributed as dist
-    from paper_2609_20532_gb300.data_parallel import data_parallel_step
+    from paper_2609_20532_gb300.data_parallel import FlatOutputs, data_parallel_step
     w = W.custom("dp1", [(136, 72), (64, 200)], 5, 64, "bf16", C=0.05, sigma=0.7, d_std=0.1,
                  wid=612)
     layers = W.make_inputs(w)
@@ -1201,11 +1311,11 @@ def test_data_parallel_step_on_one_rank():
         stream = torch.cuda.current_stream()
         cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
                              seed=21, step=3)
-        outs = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+        fo = FlatOutputs(w.layers, 1, dev)
         ref = [torch.zeros(i, o, device=dev) for i, o in w.layers]
         ctx = dp.dp_step_init(cfg, stream)
         try:
-            data_parallel_step(ctx, range(len(layers)), Ad, Dd, outs)
+            data_parallel_step(ctx, Ad, Dd, fo)
             dp.dp_step_init(cfg, stream, ctx)
             dp.run_step(ctx, Ad, Dd, ref, flags=dp.DP_NO_NOISE)
             dp.dp_clipped_sum_noise_batch(ctx, list(range(len(layers))), None, None, ref,
@@ -1215,8 +1325,108 @@ def test_data_parallel_step_on_one_rank():
         torch.cuda.synchronize()
     finally:
         dist.destroy_process_group()
-    for a, b in zip(outs, ref):
+    for a, b in zip(fo.views, ref):
         assert torch.equal(a, b)
     r = oracle_step(w, layers, seed=21, step=3, out_scale=1.0 / w.B)
-    for o, rr in zip(outs, r["out"]):
+    for o, rr in zip(fo.views, r["out"]):
         assert rel_err_normwise(o.cpu().numpy(), rr) <= TOL["bf16"]
+
+
+DP2_SHAPES = [(136, 72), (64, 200), (96, 48)]
+DP2_B, DP2_T = 6, 64
+
+
+def _dp2_worker(rank, world, port, kind, out):
+    """One rank of a two-process step on cuda:0 through the real library;
+    the collectives run over gloo on host copies.  The ranks' kernels never
+    wait on each other: only the host-side collectives join them."""
+    import os
+    import sys
+    sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+    import torch
+    import torch.distributed as dist
+    import paper_2609_20532_gb300 as dp
+    import workloads as W
+    from paper_2609_20532_gb300 import data_parallel as P
+    torch.cuda.set_device(0)
+    dist.init_process_group("gloo", init_method=f"tcp://127.0.0.1:{port}", rank=rank,
+                            world_size=world)
+    try:
+        w = W.custom("dp2", DP2_SHAPES, DP2_B, DP2_T, "bf16", C=0.05, sigma=0.7, d_std=0.1,
+                     wid=613)
+        layers = W.make_inputs(w)
+        dev = torch.device("cuda:0")
+        stream = torch.cuda.current_stream()
+        if kind == "example":
+            start, count = P.shard_examples(w.B, world, rank)
+            Ad = [A[start:start + count].to(dev) for A, _ in layers]
+            Dd = [D[start:start + count].to(dev) for _, D in layers]
+            cfg = dp.make_config(w.layers, count, w.T, w.dtype, w.C, w.sigma,
+                                 out_scale=1.0 / w.B, seed=21, step=3)
+            fo = P.FlatOutputs(w.layers, world, dev)
+            ctx = dp.dp_step_init(cfg, stream)
+            try:
+                P.data_parallel_step(ctx, Ad, Dd, fo, host_staging=True)
+                torch.cuda.synchronize()
+            finally:
+                dp.dp_step_destroy(ctx)
+            out[rank] = [v.cpu().numpy() for v in fo.views]
+        else:
+            first, count, pbase = P.shard_layers(w.layers, world, rank)
+            mine = w.layers[first:first + count]
+            Ad = [layers[l][0].to(dev) for l in range(first, first + count)]
+            Dd = [layers[l][1].to(dev) for l in range(first, first + count)]
+            cfg = dp.make_config(mine, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
+                                 seed=21, step=3, param_base=pbase)
+            outs = [torch.zeros(i, o, device=dev) for i, o in mine]
+            s = torch.zeros(w.B, device=dev)
+            ctx = dp.dp_step_init(cfg, stream)
+            try:
+                P.layer_parallel_step(ctx, Ad, Dd, outs, w.B, host_staging=True, s_total=s)
+                torch.cuda.synchronize()
+            finally:
+                dp.dp_step_destroy(ctx)
+            out[rank] = (first, [o.cpu().numpy() for o in outs], s.cpu().numpy())
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("kind", ["example", "layer"])
+def test_two_rank_partitions_through_the_library(kind):
+    """Both multi-GPU partitions at world size 2 with the real library (two
+    processes sharing cuda:0, gloo collectives on host copies): by example,
+    every rank ends with the whole-batch oracle step; by layer, every rank's
+    outputs are the whole-model oracle step's for its layers and its summed
+    squared norms those of the whole model."""
+    import socket
+    import torch.multiprocessing as mp
+    with socket.socket() as s_:
+        s_.bind(("127.0.0.1", 0))
+        port = s_.getsockname()[1]
+    ctx = mp.get_context("spawn")
+    mgr = ctx.Manager()
+    out = mgr.dict()
+    procs = [ctx.Process(target=_dp2_worker, args=(r, 2, port, kind, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(timeout=300)
+        assert p.exitcode == 0
+    w = W.custom("dp2", DP2_SHAPES, DP2_B, DP2_T, "bf16", C=0.05, sigma=0.7, d_std=0.1, wid=613)
+    layers = W.make_inputs(w)
+    r = oracle_step(w, layers, seed=21, step=3, out_scale=1.0 / w.B)
+    if kind == "example":
+        for rank in range(2):
+            for o, rr in zip(out[rank], r["out"]):
+                assert rel_err_normwise(o, rr) <= TOL["bf16"]
+        for a, b in zip(out[0], out[1]):
+            assert np.array_equal(a, b)
+    else:
+        seen = []
+        for rank in range(2):
+            first, outs, s = out[rank]
+            assert rel_err_elementwise(s, r["n"].sum(axis=0)) <= TOL["bf16"]
+            for k, o in enumerate(outs):
+                assert rel_err_normwise(o, r["out"][first + k]) <= TOL["bf16"]
+                seen.append(first + k)
+        assert sorted(seen) == list(range(len(DP2_SHAPES)))
