@@ -10,6 +10,12 @@ bf16, B=16, T=512.  Prints ONE JSON line on rank 0.
 
 --impl reference times the fp64 CPU oracle (the plain implementation the
 kernels are checked against) on a bounded sample of the same workload.
+Under torchrun (N > 1) the step is sharded by example over the ranks (each
+rank B examples, the job's batch N * B): local norms, clip factors and
+clipped sums, a reduce-scatter of the commitment, each rank's slice of the
+noise, an all-gather (--replicas: N independent one-GPU steps instead).
+--table prints one record per configured workload (stages, rooflines, the
+oracle's time and the errors against it); --sweep the 4096x4096 sweep.
 """
 
 from __future__ import annotations
@@ -646,7 +652,7 @@ def run_ours(args, rank, world, local_rank):
                    "T": w.T, "C": w.C, "sigma": w.sigma, "out_scale": "1/B",
                    "audit_examples": len(idx),
                    "l2": f"inputs {in_bytes / 1e6:.0f} MB > 129 MB L2 (no flush needed)",
-                   "parallelism": "replicas" if world > 1 else "single",
+                   "parallelism": "replicas (no collective)" if world > 1 else "single",
                    "execution": execution},
         "roofline": roofline,
         "kernels": kernels,
@@ -656,6 +662,124 @@ def run_ours(args, rank, world, local_rank):
         # reset, norms, clip, clipped sums, audit gather of every step)
         "gpu_launches": timed_launches,
         "launches_per_stage": dict(stage_launches),
+        "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_data_parallel(args, rank, world, local_rank):
+    """The step on ``world`` GPUs sharded by example (data_parallel_step):
+    every rank holds B examples of the workload (weak scaling: the job's
+    batch is world * B), computes their norms, clip factors and clipped
+    sums, the ranks reduce-scatter the flat commitment, each adds the noise
+    of its own slice of the parameters and all-gathers the released
+    gradient; then each rank emits its audit records.  Timed from a barrier
+    to a barrier; the job's time is the slowest rank's.  The collectives'
+    own time is measured alone on the same buffer after the timed region."""
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_20532_gb300 as dp
+    import workloads as W
+    from paper_2609_20532_gb300.data_parallel import FlatOutputs, data_parallel_step
+
+    dev = torch.device(f"cuda:{0 if args.same_device else local_rank}")
+    torch.cuda.set_device(dev)
+    host = args.dist_backend == "gloo"
+    w = W.get(args.workload)
+    L = len(w.layers)
+    B_job = w.B * world
+    layers = W.make_inputs(w, seed=rank)        # this rank's B examples
+    A_d = [A.to(dev) for A, _ in layers]
+    D_d = [D.to(dev) for _, D in layers]
+    fo = FlatOutputs(w.layers, world, dev)
+    idx = W.audit_indices(w, seed=rank)
+    stream = torch.cuda.current_stream()
+    cfg = dp.make_config(w.specs, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / B_job,
+                         seed=1234, step=0, audit_capacity=len(idx))
+    ctx = dp.dp_step_init(cfg, stream)
+    in_bytes = sum(A.numel() * A.element_size() + D.numel() * D.element_size()
+                   for A, D in layers)
+
+    def step(t, A_, D_):
+        cfg.step = t
+        dp.dp_step_init(cfg, stream, ctx)
+        data_parallel_step(ctx, A_, D_, fo, host_staging=host)
+        return dp.dp_audit_emit(ctx, idx, L)
+
+    for t in range(args.warmup):
+        step(t, A_d, D_d)
+    torch.cuda.synchronize()
+    dist.barrier()
+    torch.cuda.synchronize()
+    n0 = dp.dp_kernel_launches()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(0 if args.same_device else local_rank) as clk:
+        e0.record(stream)
+        for t in range(args.steps):
+            step(args.warmup + t, A_d, D_d)
+        e1.record(stream)
+        torch.cuda.synchronize()
+    launches = dp.dp_kernel_launches() - n0
+    dist.barrier()
+    ms = max_over_ranks(e0.elapsed_time(e1), world, None if host else dev) / args.steps
+    # the two collectives alone on the same buffer
+    from paper_2609_20532_gb300.data_parallel import _Comm
+    comm = _Comm(None, host)
+    mine = fo.slice_buffer()
+    torch.cuda.synchronize()
+    dist.barrier()
+    c0, c1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    c0.record(stream)
+    for _ in range(args.steps):
+        comm.reduce_scatter(mine, fo.flat)
+        comm.all_gather(fo.flat, mine)
+    c1.record(stream)
+    torch.cuda.synchronize()
+    coll_ms = max_over_ranks(c0.elapsed_time(c1), world, None if host else dev) / args.steps
+    # end to end: each step copies this rank's inputs in from pinned host
+    # memory and the released gradient out (one copy of the flat vector)
+    e2e = None
+    if not args.no_e2e:
+        A_h = [A.pin_memory() for A, _ in layers]
+        D_h = [D.pin_memory() for _, D in layers]
+        O_h = torch.empty(fo.flat.numel(), dtype=torch.float32).pin_memory()
+        A_b = [torch.empty_like(a) for a in A_d]
+        D_b = [torch.empty_like(d) for d in D_d]
+        dist.barrier()
+        t0 = time.perf_counter()
+        for t in range(args.steps):
+            for l in range(L):
+                A_b[l].copy_(A_h[l], non_blocking=True)
+                D_b[l].copy_(D_h[l], non_blocking=True)
+            step(10_000 + t, A_b, D_b)
+            O_h.copy_(fo.flat, non_blocking=True)
+            torch.cuda.synchronize()
+        wall = max_over_ranks((time.perf_counter() - t0) / args.steps, world,
+                              None if host else dev)
+        e2e = {"value": B_job / wall, "unit": UNIT, "ms_per_step": 1e3 * wall,
+               "h2d_bytes_per_step": in_bytes * world,
+               "d2h_bytes_per_step": (4 * fo.flat.numel() + len(idx) * dp.dp_audit_record_bytes(L))
+               * world, "overlap": "none (copies, step and read-back in sequence)"}
+    dp.dp_step_destroy(ctx)
+    if rank != 0:
+        return
+    line = {
+        "metric": METRIC, "value": B_job / (ms * 1e-3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": _data_desc(w),
+        "config": {"workload": w.describe(), "global_batch": B_job, "B_per_rank": w.B,
+                   "T": w.T, "parallelism": "data-parallel by example",
+                   "collectives": f"{args.dist_backend}: reduce-scatter + all-gather of the "
+                                  f"flat commitment ({4 * fo.flat.numel()} bytes), "
+                                  "noise of each rank's slice in between",
+                   "l2": f"inputs {in_bytes / 1e6:.0f} MB per rank > 129 MB L2",
+                   "execution": "eager launches"},
+        "collective_ms_per_step": coll_ms,
+        "collective_bytes_per_rank": 2 * 4 * fo.flat.numel(),
+        "e2e": e2e,
+        "gpu_launches": launches,
         "clocks": clk.summary(),
     }
     print(json.dumps(line), flush=True)
@@ -829,6 +953,223 @@ def run_verifier(args):
 
 FAMILY_P = 0.1  # audit rate of every family in the paper's verifier table
 
+TABLE_CONFIGS = ["single_fp32", "mlp_fp32", "block_bf16", "llm_bf16"]
+
+
+def _oracle_one_thread(name: str) -> dict:
+    """The oracle's bounded sample of a workload on one host thread: a child
+    process whose BLAS pools are limited to one thread before numpy loads."""
+    env = dict(os.environ)
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS",
+              "BLIS_NUM_THREADS", "VECLIB_MAXIMUM_THREADS", "NUMEXPR_NUM_THREADS"):
+        env[k] = "1"
+    code = ("import json, sys; sys.path.insert(0, %r); import bench, workloads as W; "
+            "v, dt, d = bench.cpu_baseline_sample(W.get(%r)); "
+            "print(json.dumps({'value': v, 'seconds': dt}))") % (ROOT, name)
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                       timeout=900)
+    if r.returncode != 0:
+        return {"error": r.stderr.strip().splitlines()[-1] if r.stderr.strip() else "failed"}
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def _errors(got, ref):
+    """Elementwise relative error max over entries, and for outputs also the
+    normwise error and the max of |d| / max(|ref|, 1e-3 rms(ref))."""
+    import numpy as np
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    d = np.abs(got - ref)
+    rms = float(np.sqrt(np.mean(ref * ref))) if ref.size else 0.0
+    return {"elementwise": float(np.max(d / np.maximum(np.abs(ref), 1e-30))),
+            "normwise": float(np.linalg.norm(got - ref) / max(np.linalg.norm(ref), 1e-300)),
+            "max_scaled": float(np.max(d / np.maximum(np.abs(ref), 1e-3 * rms + 1e-300)))}
+
+
+def run_table(args):
+    """One JSON line with a record per configured workload (single_fp32,
+    mlp_fp32, block_bf16, llm_bf16 and the 12 points of the 4096x4096
+    sweep): the step through the C ABI (CUDA-graph replay, inputs resident,
+    no audit emit), its stages, their roofline fractions, the oracle on the
+    host cores (all cores; one thread for the three small workloads) and the
+    largest error of every output against the oracle -- in full for the
+    three small workloads, on sampled examples and rows (with the GPU's
+    clip factors for the sampled rows of the sums) for the large ones."""
+    import numpy as np
+    import torch
+
+    import paper_2609_20532_gb300 as dp
+    import workloads as W
+    from oracle import dp_oracle as O
+
+    dev = torch.device("cuda:0")
+    torch.cuda.set_device(dev)
+    peaks = _peaks()
+    ffma_peak = 152 * 128 * 2 * 2.07e9 / 1e12   # fp32 FFMA TFLOP/s at the maximum SM clock
+    cores = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+    stream = torch.cuda.Stream()
+    torch.cuda.set_stream(stream)
+    f32 = lambda x: float(np.float32(x))  # noqa: E731
+    names = (args.table_configs.split(",") if args.table_configs
+             else TABLE_CONFIGS + [w.name for w in W.SWEEP])
+    recs = []
+    for name in names:
+        w = W.get(name)
+        L = len(w.layers)
+        full = name in ("single_fp32", "mlp_fp32", "block_bf16")
+        if name.startswith("sweep_"):
+            g = torch.Generator(device=dev)
+            g.manual_seed(w.wid)
+            A_d = [torch.randn(w.B, w.T, 4096, generator=g, device=dev).to(torch.bfloat16)]
+            D_d = [torch.randn(w.B, w.T, 4096, generator=g, device=dev).to(torch.bfloat16)]
+            layers = None
+        else:
+            layers = W.make_inputs(w, seed=0)
+            A_d = [A.to(dev) for A, _ in layers]
+            D_d = [D.to(dev) for _, D in layers]
+        outs = [torch.zeros(i, o, device=dev) for i, o in w.layers]
+        s_dev = torch.empty(w.B, device=dev)
+        c_dev = torch.empty(w.B, device=dev)
+        seed, step = 5, 2
+        cfg = dp.make_config(w.specs, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=1.0 / w.B,
+                             seed=seed, step=step, audit_capacity=w.B)
+        ctx = dp.dp_step_init(cfg, stream)
+        ids = list(range(L))
+
+        def graph(fn):
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=stream):
+                fn()
+            torch.cuda.synchronize()
+            return gr
+
+        def timed(gr, reps):
+            # at least W replays and 0.1 s, so the SM clock is back up after an idle
+            t_end = time.perf_counter() + 0.1
+            k = 0
+            while k < max(3, args.warmup) or time.perf_counter() < t_end:
+                gr.replay()
+                k += 1
+                if k % 32 == 0:
+                    torch.cuda.synchronize()
+            torch.cuda.synchronize()
+            ts = []
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            for _ in range(reps):
+                e0.record(stream)
+                gr.replay()
+                e1.record(stream)
+                torch.cuda.synchronize()
+                ts.append(e0.elapsed_time(e1))
+            return statistics.median(ts)
+
+        def whole():
+            dp.dp_step_init(cfg, stream, ctx)
+            dp.dp_layer_norms_batch(ctx, ids, A_d, D_d)
+            dp.dp_clip_factors(ctx, s_dev, c_dev)
+            dp.dp_clipped_sum_noise_batch(ctx, ids, A_d, D_d, outs, 0)
+
+        g_step = graph(whole)
+        g_init = graph(lambda: dp.dp_step_init(cfg, stream, ctx))
+        g_norm = graph(lambda: dp.dp_layer_norms_batch(ctx, ids, A_d, D_d))
+        g_clip = graph(lambda: dp.dp_clip_factors(ctx, s_dev, c_dev))
+        g_sum = graph(lambda: dp.dp_clipped_sum_noise_batch(ctx, ids, A_d, D_d, outs, 0))
+        g_noise = graph(lambda: dp.dp_clipped_sum_noise_batch(ctx, ids, None, None, outs,
+                                                              dp.DP_NOISE_ONLY))
+        reps = args.steps
+        time.sleep(0.5)
+        t_step = timed(g_step, reps)
+        # stages one at a time, each after the step's earlier stages
+        g_init.replay()
+        t_norm = timed(g_norm, reps)
+        t_clip = timed(g_clip, reps)
+        t_sum = timed(g_sum, reps)
+        time.sleep(0.5)
+        t_noise = timed(g_noise, reps)
+        # the results of one step, with the audit records of every example
+        g_step.replay()
+        recs_a = dp.dp_audit_emit(ctx, range(w.B), L)
+        torch.cuda.synchronize()
+        modes = [dp.dp_layer_norm_mode(ctx, l) for l in range(L)]
+        paths = [dp.dp_layer_path(ctx, l) for l in range(L)]
+        dp.dp_step_destroy(ctx)
+        n_gpu = recs_a["layer_sqnorm"].astype(np.float64).T
+        s_gpu = recs_a["total_sqnorm"].astype(np.float64)
+        c_gpu = recs_a["clip_factor"].astype(np.float64)
+        out_gpu = [o.double().cpu().numpy() for o in outs]
+        in_bytes = sum(a.numel() * a.element_size() + d.numel() * d.element_size()
+                       for a, d in zip(A_d, D_d))
+        flops = sum(2.0 * w.B * T_ * i * o for i, o, T_ in w.specs)
+        rec = {"workload": w.describe(), "B": w.B, "T": w.T, "params": w.n_params,
+               "norm_modes": [{1: "rank1", 2: "gram", 3: "materialised"}[m] for m in modes],
+               "tensor_core": [list(p_) for p_ in paths],
+               "step_ms": t_step, "examples_per_s": w.B / (t_step * 1e-3),
+               "norm_ms": t_norm, "clip_ms": t_clip, "sum_ms": t_sum, "noise_ms": t_noise,
+               "k1_frac_hbm": in_bytes / (t_norm * 1e-3) / 1e9 / peaks["hbm_gbs"],
+               "k4_frac_hbm": 8.0 * w.n_params / (t_noise * 1e-3) / 1e9 / peaks["hbm_gbs"]}
+        tf = flops / (t_sum * 1e-3) / 1e12
+        if w.dtype == "bf16":
+            rec["k3_tflops"], rec["k3_frac_bf16"] = tf, tf / peaks["bf16_tflops"]
+        else:
+            rec["k3_tflops"], rec["k3_frac_fp32_ffma"] = tf, tf / ffma_peak
+        # ---- errors against the oracle ----
+        Cf, sf = f32(w.C), f32(w.sigma)
+        if full:
+            ref = O.dp_step([(W.to_f64(A), W.to_f64(D)) for A, D in layers], Cf, sf, seed, step,
+                            out_scale=f32(1.0 / w.B))
+            err = {"n": _errors(n_gpu, ref["n"])["elementwise"],
+                   "s": _errors(s_gpu, ref["s"])["elementwise"],
+                   "c": _errors(c_gpu, ref["c"])["elementwise"],
+                   "out": [_errors(o, r) for o, r in zip(out_gpu, ref["out"])],
+                   "compared": "every output in full"}
+        else:
+            rng = np.random.default_rng(w.wid)
+            ex = np.sort(rng.choice(w.B, size=min(2, w.B), replace=False))
+            if layers is None:   # sweep: the device inputs' bits
+                lay = [(A_d[0][ex].cpu(), D_d[0][ex].cpu())]
+            else:
+                lay = [(A[ex], D[ex]) for A, D in layers]
+            n_ref = np.stack([O.layer_sqnorms_ghost(W.to_f64(A), W.to_f64(D)) for A, D in lay])
+            s_ref, c_ref = O.clip_factors(n_ref, Cf)
+            out_err, off = [], 0
+            for l, (d_in, d_out) in enumerate(w.layers):
+                rows = np.sort(rng.choice(d_in, size=4, replace=False))
+                S = np.zeros((rows.size, d_out))
+                A_l, D_l = A_d[l], D_d[l]
+                for i in range(w.B):
+                    a = A_l[i, :, torch.as_tensor(rows, device=dev)].cpu()
+                    d_ = D_l[i].cpu()
+                    S += c_gpu[i] * (W.to_f64(a).T @ W.to_f64(d_))
+                z = np.stack([O.gaussian_noise(seed, step, off + int(j) * d_out, d_out)
+                              for j in rows])
+                ref_rows = f32(1.0 / w.B) * (S + sf * Cf * z)
+                out_err.append(_errors(out_gpu[l][rows], ref_rows))
+                off += d_in * d_out
+            err = {"n": _errors(n_gpu[:, ex], n_ref)["elementwise"],
+                   "s": _errors(s_gpu[ex], s_ref)["elementwise"],
+                   "c": _errors(c_gpu[ex], c_ref)["elementwise"],
+                   "out": out_err,
+                   "compared": f"norms, s, c of examples {ex.tolist()}; 4 sampled rows of "
+                               "every output (sums with the GPU's clip factors)"}
+        rec["max_rel_err"] = err
+        # ---- the oracle on the host cores ----
+        if not name.startswith("sweep_"):
+            v, dt, desc = cpu_baseline_sample(w)
+            rec["oracle"] = {"examples_per_s": v, "cores": cores, "sample": desc}
+            if full:
+                one = _oracle_one_thread(name)
+                rec["oracle"]["examples_per_s_1_thread"] = one.get("value")
+        recs.append(rec)
+        print(json.dumps({"partial": name, "step_ms": t_step}), file=sys.stderr, flush=True)
+        del A_d, D_d, outs, layers
+        torch.cuda.empty_cache()
+    line = {"impl": "table", "metric": METRIC, "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "peaks": peaks, "ffma_peak_tflops": ffma_peak,
+            "data": "synthetic (workloads recipe; the sweep's inputs from torch's seeded CUDA "
+                    "generator, N(0,1) rounded to bf16)",
+            "configs": recs}
+    print(json.dumps(line), flush=True)
+
 
 def main():
     ap = argparse.ArgumentParser()
@@ -846,6 +1187,17 @@ def main():
                     help="time the trusted-side checker of Algorithm 1 on the host cores")
     ap.add_argument("--sweep", action="store_true",
                     help="time every point of the 4096x4096 sweep instead of one workload")
+    ap.add_argument("--dist-backend", default="nccl", choices=["nccl", "gloo"],
+                    help="collective backend of a multi-rank run (gloo: host-staged copies)")
+    ap.add_argument("--same-device", action="store_true",
+                    help="every rank on cuda:0 (a gloo run of the multi-rank path on one GPU)")
+    ap.add_argument("--replicas", action="store_true",
+                    help="multi-rank: independent replicas of the one-GPU step, no collective")
+    ap.add_argument("--table", action="store_true",
+                    help="one record per configured workload: step, stages, rooflines, "
+                         "oracle timing and errors against the oracle")
+    ap.add_argument("--table-configs", default="",
+                    help="comma-separated workload names for --table (default: all)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3) if args.impl == "ours" else args.warmup
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -857,6 +1209,10 @@ def main():
     if args.sweep:
         run_sweep(args)
         return
+    if args.table:
+        if rank == 0:
+            run_table(args)
+        return
     if args.verifier:
         if rank == 0:
             run_verifier(args)
@@ -864,10 +1220,13 @@ def main():
     if world > 1:
         import torch
         import torch.distributed as dist
-        torch.cuda.set_device(local_rank)
-        dist.init_process_group("nccl")
+        torch.cuda.set_device(0 if args.same_device else local_rank)
+        dist.init_process_group(args.dist_backend)
     try:
-        run_ours(args, rank, world, local_rank)
+        if world > 1 and not args.replicas:
+            run_data_parallel(args, rank, world, local_rank)
+        else:
+            run_ours(args, rank, world, local_rank)
     finally:
         if world > 1:
             import torch.distributed as dist

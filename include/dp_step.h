@@ -80,9 +80,14 @@ typedef enum { DP_F32 = 0, DP_BF16 = 1 } dp_dtype;
  *   squared and summed; it is never written to memory.
  * AUTO: RANK1 when T == 1, else whichever of GHOST / MATERIALISED has the
  *   smaller arithmetic cost (T <= 2 d_in d_out / (d_in + d_out) picks GHOST),
- *   except that a bf16 layer wider than 65536 on either side takes
- *   MATERIALISED on tensor cores instead of GHOST on CUDA cores (see
- *   dp_layer_path). */
+ *   except that
+ *   - a bf16 layer wider than 65536 on either side takes MATERIALISED on
+ *     tensor cores instead of GHOST on CUDA cores (see dp_layer_path);
+ *   - a bf16 layer with T <= 128 whose Gram form has few work items (B times
+ *     the Gram layers of that T below half the SMs) takes MATERIALISED when
+ *     that is faster than one Gram item, whose (d_in + d_out) / 64 feature
+ *     steps run one after another on one SM (0.42 us each, measured),
+ *     against 2 B T d_in d_out flops at 0.9 PFLOP/s (measured). */
 typedef enum {
     DP_NORM_AUTO = 0,
     DP_NORM_RANK1 = 1,

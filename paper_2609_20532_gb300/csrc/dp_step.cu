@@ -199,6 +199,28 @@ dp_norm_mode resolve_mode(dp_norm_mode m, int T, int64_t d_in, int64_t d_out) {
   return ghost <= mat ? DP_NORM_GHOST : DP_NORM_MATERIALISED;
 }
 
+// Latency term of the norm-form choice.  When the Gram form has few work
+// items (B times the Gram layers that share T: fewer than half the SMs), its
+// time is one item's, whose K steps of 64 features run one after another on
+// one SM: about 0.42 us each on the GB300 (measured: 4096 x 4096 at T = 64,
+// 128 steps in 54 us), while the materialised form spreads over the whole
+// GPU at about 0.9 PFLOP/s for examples of one 64-position K block (measured
+// at T = 64).  Only examples of one 128-position block (T <= 128) are
+// concerned: longer ones give the Gram form CTA-pair items that fill the GPU
+// and it wins by its arithmetic.
+constexpr double kGramStepSeconds = 0.42e-6;
+constexpr double kMatShortRate = 0.9e15;
+
+bool gram_latency_prefers_materialised(int B, int T, int64_t d_in, int64_t d_out,
+                                       int64_t gram_items, int sms) {
+  if (T > 128 || gram_items * 2 >= sms) return false;
+  const double steps = static_cast<double>((d_in + 63) / 64 + (d_out + 63) / 64);
+  const double t_gram = steps * kGramStepSeconds;
+  const double t_mat = 2.0 * B * T * static_cast<double>(d_in) * static_cast<double>(d_out) /
+                       kMatShortRate;
+  return t_mat < t_gram;
+}
+
 // A thin layer (narrow side <= kThinMax) stores its per-example gradients
 // when writing and reading them back moves fewer bytes than reading A and D
 // a second time, 8 d_in d_out < T (d_in + d_out) elem, which also makes the
@@ -229,6 +251,50 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
   uint64_t off = cfg->param_base;
   int64_t grads = 0, splits = 0, unf = 0;
   int64_t NP = 1;
+  const bool bf16_cfg = cfg->dtype == DP_BF16;
+  // Gram-form tensor-core layers per T (they share norm launches), for the
+  // latency term of the AUTO choice
+  std::map<int, int64_t> gram_layers;
+  if (cfg->norm_mode == DP_NORM_AUTO && bf16_cfg) {
+    for (int l = 0; l < cfg->n_layers; ++l) {
+      const int T = layer_T(cfg, l);
+      const int64_t di = cfg->layers[l].d_in, dd = cfg->layers[l].d_out;
+      if (use_pergrad(cfg, T, di, dd)) continue;
+      if (resolve_mode(DP_NORM_AUTO, T, di, dd) == DP_NORM_GHOST &&
+          dpk::tc_ghost_supported(T, di, dd))
+        ++gram_layers[T];
+    }
+  }
+  const int sms = gram_layers.empty() ? 0 : dpk::device_sm_count();
+  // Tiles of the tensor-core clipped-sum launch each layer shares when every
+  // layer is summed in one batched call in layer order (consecutive layers of
+  // one tile shape and T, up to kGemmMaxLayers per launch): a layer's example
+  // split is chosen for that launch, then fixed.
+  std::vector<int64_t> group_tiles(cfg->n_layers, 0);
+  {
+    std::vector<int> cur;
+    auto close = [&]() {
+      int64_t t = 0;
+      for (int l : cur) t += dpk::tc_gemm_tiles(cfg->layers[l].d_in, cfg->layers[l].d_out);
+      for (int l : cur) group_tiles[l] = t;
+      cur.clear();
+    };
+    for (int l = 0; l < cfg->n_layers; ++l) {
+      const int T = layer_T(cfg, l);
+      const int64_t di = cfg->layers[l].d_in, dd = cfg->layers[l].d_out;
+      if (!bf16_cfg || use_pergrad(cfg, T, di, dd) || !dpk::tc_gemm_supported(T, di, dd))
+        continue;
+      if (!cur.empty()) {
+        const int f = cur[0];
+        if (!dpk::tc_clipsum_same_launch(cfg->layers[f].d_in, cfg->layers[f].d_out, di, dd) ||
+            layer_T(cfg, f) != T)
+          close();
+      }
+      cur.push_back(l);
+      if (static_cast<int>(cur.size()) == dpk::kGemmMaxLayers) close();
+    }
+    close();
+  }
   for (int l = 0; l < cfg->n_layers; ++l) {
     LayerPlan& p = c->plan[l];
     p.d_in = cfg->layers[l].d_in;
@@ -288,6 +354,13 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
     if (cfg->norm_mode == DP_NORM_AUTO && p.mode == DP_NORM_GHOST && bf16 &&
         !dpk::tc_ghost_supported(T, p.d_in, p.d_out) && dpk::tc_gemm_supported(T, p.d_in, p.d_out))
       p.mode = DP_NORM_MATERIALISED;
+    // few Gram items on short examples: the latency of one item decides
+    if (cfg->norm_mode == DP_NORM_AUTO && p.mode == DP_NORM_GHOST && bf16 &&
+        dpk::tc_ghost_supported(T, p.d_in, p.d_out) &&
+        dpk::tc_gemm_supported(T, p.d_in, p.d_out) &&
+        gram_latency_prefers_materialised(cfg->B, T, p.d_in, p.d_out,
+                                          static_cast<int64_t>(cfg->B) * gram_layers[T], sms))
+      p.mode = DP_NORM_MATERIALISED;
     p.norm_tc = 0;
     int64_t parts = 1;
     if (p.mode == DP_NORM_RANK1) {
@@ -310,7 +383,8 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
     p.gemm_tc = 0;
     if (bf16 && dpk::tc_gemm_supported(T, p.d_in, p.d_out)) {
       p.gemm_tc = 1;
-      p.split = dpk::tc_gemm_split(cfg->B, T, p.d_in, p.d_out);
+      p.split = dpk::tc_gemm_split(cfg->B, T, p.d_in, p.d_out,
+                                   group_tiles[l] - dpk::tc_gemm_tiles(p.d_in, p.d_out));
       if (p.split > 1) {
         p.s_off = splits;
         splits += static_cast<int64_t>(p.split) * p.d_in * p.d_out;
@@ -619,7 +693,7 @@ cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const vo
   A = dense_A(c, layer, A);
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
   if (p.gemm_tc == 1)
-    return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, p.T, din, dout, d_out,
+    return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, p.T, din, dout, p.split, d_out,
                                   p.split > 1 ? c->d_split + p.s_off : nullptr, ep, c->d_flag,
                                   c->stream, p.implicit ? &p.cg : nullptr);
   if (p.gemm_tc == 2)
@@ -948,9 +1022,11 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
     const dpk::ConvGeom* cg[dpk::kGemmMaxLayers];
     int din[dpk::kGemmMaxLayers], dout[dpk::kGemmMaxLayers];
     uint64_t pb[dpk::kGemmMaxLayers];
+    int sp[dpk::kGemmMaxLayers];
     for (size_t q = 0; q < grp.size(); ++q) {
       const int r = grp[q];
       const LayerPlan& p = c->plan[layers[r]];
+      sp[q] = p.split;
       a[q] = dense_A(c, layers[r], A[r]);
       d[q] = D[r];
       o[q] = d_out[r];
@@ -961,8 +1037,9 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
       pb[q] = p.p_base;
     }
     cudaError_t e = dpk::tc_launch_clipsum_batch(static_cast<int>(grp.size()), a, d, o, part, din,
-                                                 dout, pb, c->d_c, c->B, c->plan[layers[grp[0]]].T,
-                                                 ep, c->d_flag, c->stream, cg);
+                                                 dout, pb, sp, c->d_c, c->B,
+                                                 c->plan[layers[grp[0]]].T, ep, c->d_flag,
+                                                 c->stream, cg);
     grp.clear();
     return e;
   };

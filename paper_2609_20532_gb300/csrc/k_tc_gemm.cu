@@ -163,8 +163,10 @@ __device__ __forceinline__ ConvTaps conv_taps(const ConvGeom& v, int m0) {
   return t;
 }
 
-// TMA loads of one stage: A rows m0.. (two 64-column chunks) and the D
-// columns this CTA stages, for K block kb of example ex.  For a convolution
+// TMA loads of one K block of a stage: A rows m0.. (two 64-column chunks)
+// and the D columns this CTA stages, for K block kb of example ex.  The
+// leader (a single CTA: itself) announces tx_bytes, the bytes the whole stage
+// brings to its full barrier, with the stage's first block (0 for the rest).  For a convolution
 // an A chunk is 64 channels of one kernel tap at 64 output positions
 // starting at output row ho0, column wo0: one 4-D box [1 image][rows]
 // [columns][64 channels] of the NHWC input at the tap's offset, whose
@@ -172,9 +174,9 @@ __device__ __forceinline__ ConvTaps conv_taps(const ConvGeom& v, int m0) {
 // issues every stage, so nothing here divides.
 template <bool PAIR, int NB, bool CONV>
 __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, uint64_t* full,
-                                                  bool leader, uint8_t* sa, uint8_t* sb, int m0,
-                                                  int n0, int ex, int kb, const ConvTaps& ct,
-                                                  int ho0, int wo0) {
+                                                  bool leader, uint32_t tx_bytes, uint8_t* sa,
+                                                  uint8_t* sb, int m0, int n0, int ex, int kb,
+                                                  const ConvTaps& ct, int ho0, int wo0) {
   using C = Cfg<PAIR, NB>;
   const CUtensorMap* mapA = &g.mapA[layer];
   const CUtensorMap* mapD = &g.mapD[layer];
@@ -184,7 +186,7 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
   if constexpr (PAIR) {
     // both CTAs' loads complete on the leader's full barrier
     const uint32_t fb = mapa_shared(smem_u32(full), 0);
-    if (leader) mbar_arrive_expect_tx(full, 2 * C::STAGE_BYTES);
+    if (leader && tx_bytes) mbar_arrive_expect_tx(full, tx_bytes);
     if (CONV && g.conv[layer]) {
       tma_load_4d_pair(mapA, fb, sa, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
       tma_load_4d_pair(mapA, fb, sa + CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
@@ -205,7 +207,7 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
         tma_load_2d_pair(mapD, fb, sb + q * CHUNK, n0 + 64 * q, drow);
     }
   } else {
-    mbar_arrive_expect_tx(full, C::STAGE_BYTES);
+    if (tx_bytes) mbar_arrive_expect_tx(full, tx_bytes);
     if (CONV && g.conv[layer]) {
       tma_load_4d(mapA, full, sa, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
       tma_load_4d(mapA, full, sa + CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
@@ -282,6 +284,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   const int unit = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
   const int n_units = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
   const int kpe = (g.T + BK - 1) / BK;  // K-blocks per example
+  // CTA pairs take two K blocks per stage when an example has an even number
+  // of them (a stage never straddles two examples' folds): half the barrier
+  // round trips per MMA, measured faster; the stage memory is the same.
+  const int bps = (PAIR && (kpe % 2) == 0) ? 2 : 1;
+  const int nst = bps == 2 ? STAGES / 2 : STAGES;
   const int n_tiles = g.tile_start[g.L];
   volatile int* abrt = &abort_flag;
 
@@ -344,22 +351,28 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
         for (int ex = w.e0; ex < w.e1; ++ex) {
           int ho0 = 0, wo0 = 0;
-          for (int kb = 0; kb < kpe; ++kb) {
+          for (int kb = 0; kb < kpe; kb += bps) {
             if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
-            uint8_t* sa = smem + stage * C::STAGE_BYTES;
-            uint8_t* sb = sa + C::A_STAGE;
-            issue_stage_loads<PAIR, NB, CONV>(g, l, &full_bar[stage], leader, sa, sb, m0, n0, ex,
-                                              kb, s_taps, ho0, wo0);
-            if constexpr (CONV) {
-              if (rows_per_kb) {
-                ho0 += rows_per_kb;
-              } else if (wout > 1 && (wo0 += BK) == wout) {
-                wo0 = 0;
-                ++ho0;
+            for (int j = 0; j < bps; ++j) {
+              uint8_t* sa = smem + (stage * bps + j) * C::STAGE_BYTES;
+              uint8_t* sb = sa + C::A_STAGE;
+              issue_stage_loads<PAIR, NB, CONV>(g, l, &full_bar[stage], leader,
+                                                j == 0 ? static_cast<uint32_t>(
+                                                             bps * (PAIR ? 2 : 1) * C::STAGE_BYTES)
+                                                       : 0u,
+                                                sa, sb, m0, n0, ex,
+                                                kb + j, s_taps, ho0, wo0);
+              if constexpr (CONV) {
+                if (rows_per_kb) {
+                  ho0 += rows_per_kb;
+                } else if (wout > 1 && (wo0 += BK) == wout) {
+                  wo0 = 0;
+                  ++ho0;
+                }
               }
             }
             ++uses[stage];
-            if (++stage == STAGES) {
+            if (++stage == nst) {
               stage = 0;
               phase ^= 1;
             }
@@ -390,25 +403,27 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           if (!mbar_wait(&tempty_bar[buf], tph ^ 1, abrt, g.err)) goto mma_done;
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + buf * NB;
-          for (int kb = 0; kb < kpe; ++kb) {
+          for (int kb = 0; kb < kpe; kb += bps) {
             if (!mbar_wait(&full_bar[stage], phase, abrt, g.err)) goto mma_done;
             tc_fence_after();
-            const uint32_t sa = smem_u32(smem + stage * C::STAGE_BYTES);
-            const uint32_t sb = sa + C::A_STAGE;
+            for (int j = 0; j < bps; ++j) {
+              const uint32_t sa = smem_u32(smem + (stage * bps + j) * C::STAGE_BYTES);
+              const uint32_t sb = sa + C::A_STAGE;
 #pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk) {
-              const uint64_t ad = smem_desc_sw128(sa + kk * 16 * 128, LBO, SBO);
-              const uint64_t bd = smem_desc_sw128(sb + kk * 16 * 128, LBO, SBO);
-              if constexpr (PAIR)
-                mma_bf16_pair(d_tmem, ad, bd, C::IDESC, (kb | kk) != 0);
-              else
-                mma_bf16(d_tmem, ad, bd, C::IDESC, (kb | kk) != 0);
+              for (int kk = 0; kk < BK / 16; ++kk) {
+                const uint64_t ad = smem_desc_sw128(sa + kk * 16 * 128, LBO, SBO);
+                const uint64_t bd = smem_desc_sw128(sb + kk * 16 * 128, LBO, SBO);
+                if constexpr (PAIR)
+                  mma_bf16_pair(d_tmem, ad, bd, C::IDESC, ((kb + j) | kk) != 0);
+                else
+                  mma_bf16(d_tmem, ad, bd, C::IDESC, ((kb + j) | kk) != 0);
+              }
             }
             if constexpr (PAIR)
               mma_commit_pair(&empty_bar[stage]);
             else
               mma_commit(&empty_bar[stage]);
-            if (++stage == STAGES) {
+            if (++stage == nst) {
               stage = 0;
               phase ^= 1;
             }
@@ -823,13 +838,23 @@ __global__ void __launch_bounds__(256) k_split_reduce(const __grid_constant__ Sp
 // at least 8 K-blocks of work.  S depends only on the layer's own shape (and
 // the device's SM count), so a layer rounds the same in a batched launch and
 // in a launch of its own.
-int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out) {
-  const bool pair = use_pair(d_in);
-  const int64_t tile_m = pair ? 2 * BM : BM;
+int64_t tc_gemm_tiles(int64_t d_in, int64_t d_out) {
+  const int64_t tile_m = use_pair(d_in) ? 2 * BM : BM;
   const int64_t nb = gemm_nb(d_out);
-  const int64_t tiles = ((d_in + tile_m - 1) / tile_m) * ((d_out + nb - 1) / nb);
+  return ((d_in + tile_m - 1) / tile_m) * ((d_out + nb - 1) / nb);
+}
+
+// Example ranges per tile.  A launch whose tiles (this layer's and the
+// other_tiles of the layers sharing it) already give every unit a tile runs
+// unsplit: a split writes and re-reads S partial tiles, which costs more
+// than the partly empty last round it saves.  Otherwise S fills whole
+// rounds: the count with the largest items / (rounds x units), the smallest
+// on a tie, at least 8 K-blocks per range, at most 256.
+int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out, int64_t other_tiles) {
+  const bool pair = use_pair(d_in);
+  const int64_t tiles = tc_gemm_tiles(d_in, d_out);
   const int64_t units = pair ? device_sm_count() / 2 : device_sm_count();
-  if (tiles >= units || B < 2) return 1;
+  if (tiles + other_tiles >= units || B < 2) return 1;
   const int64_t kpe = (T + BK - 1) / BK;
   int64_t smax = static_cast<int64_t>(B) * kpe / 8;
   if (smax > B) smax = B;
@@ -837,7 +862,7 @@ int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out) {
   int64_t best = 1;
   double best_eff = 0.0;
   for (int64_t S = 1; S <= smax; ++S) {
-    const int64_t items = tiles * S;
+    const int64_t items = tiles * S + other_tiles;
     const int64_t rounds = (items + units - 1) / units;
     const double eff = static_cast<double>(items) / static_cast<double>(rounds * units);
     if (eff > best_eff + 1e-9) {
@@ -939,9 +964,9 @@ cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d
 
 cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
                                     float* const* out, float* const* part, const int* d_in,
-                                    const int* d_out, const uint64_t* p_base, const float* c,
-                                    int B, int T, const Epilogue& ep, int* err, cudaStream_t s,
-                                    const ConvGeom* const* conv) {
+                                    const int* d_out, const uint64_t* p_base, const int* split,
+                                    const float* c, int B, int T, const Epilogue& ep, int* err,
+                                    cudaStream_t s, const ConvGeom* const* conv) {
   if (L < 1 || L > kGemmMaxLayers) return cudaErrorInvalidValue;
   const bool pair = use_pair(d_in[0]);
   const int nb = gemm_nb(d_out[0]);
@@ -961,7 +986,8 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
     g.d_out[l] = d_out[l];
     g.out[l] = out[l];
     g.p_base[l] = p_base[l];
-    g.split[l] = tc_gemm_split(B, T, d_in[l], d_out[l]);
+    g.split[l] = split ? split[l] : tc_gemm_split(B, T, d_in[l], d_out[l]);
+    if (g.split[l] < 1 || g.split[l] > kGemmMaxSplit) return cudaErrorInvalidValue;
     if (!make_input_maps(A[l], D[l], g, l, conv ? conv[l] : nullptr)) return cudaErrorInvalidValue;
     if (g.split[l] > 1) {
       if (!part || !part[l] || (reinterpret_cast<uintptr_t>(part[l]) & 15) != 0 ||
@@ -992,10 +1018,10 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
 }
 
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
-                              int d_in, int d_out, float* out, float* part, const Epilogue& ep,
-                              int* err, cudaStream_t s, const ConvGeom* conv) {
-  return tc_launch_clipsum_batch(1, &A, &D, &out, &part, &d_in, &d_out, &ep.p_base, c, B, T, ep,
-                                 err, s, &conv);
+                              int d_in, int d_out, int split, float* out, float* part,
+                              const Epilogue& ep, int* err, cudaStream_t s, const ConvGeom* conv) {
+  return tc_launch_clipsum_batch(1, &A, &D, &out, &part, &d_in, &d_out, &ep.p_base, &split, c, B,
+                                 T, ep, err, s, &conv);
 }
 
 bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_out_a, int64_t d_in_b, int64_t d_out_b) {

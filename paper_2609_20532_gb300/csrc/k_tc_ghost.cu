@@ -61,11 +61,15 @@ constexpr uint32_t TMEM_COLS = 512;      // A-Gram 256 + D-Gram 256
 // K-major, 128-byte swizzle: rows 128 B apart, 8-row groups 1024 B apart.
 constexpr uint32_t LBO = 16, SBO = 1024;
 
-// single-CTA strips: a t-tile and two s-tiles per stage
-constexpr int STAGES = 4;
-constexpr int A_OFF = 0;                 // t-tile (off-diagonal strips only)
-constexpr int B_OFF = TILE_BYTES;        // two s-tiles, 256 rows
-constexpr int STAGE_BYTES = 3 * TILE_BYTES;
+// single-CTA strips.  A stage holds SLOTS boxes of 128 rows x 64 features.
+// A strip stages `nt` tiles per K step (its t-tile unless diagonal, then its
+// one or two s-tiles) and fits nbox = SLOTS / nt boxes of each per stage (a
+// K step of nbox * 64 features), laid out box by box: the slots of box b are
+// [t-tile, s-tile 0, s-tile 1] (t-tile absent on the diagonal), so the two
+// s-tiles of a 256-row B operand sit next to each other.
+constexpr int STAGES = 3;
+constexpr int SLOTS = 4;
+constexpr int STAGE_BYTES = SLOTS * TILE_BYTES;
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;
 constexpr uint32_t IDESC_N256 = idesc_bf16_f32(GT, 2 * GT, 0, 0);
 constexpr uint32_t IDESC_N128 = idesc_bf16_f32(GT, GT, 0, 0);
@@ -209,19 +213,29 @@ __global__ void __launch_bounds__(GHOST_THREADS, 1)
         const bool diag = st.tb == st.sb;
         const CUtensorMap* mA = &g.mapA[st.layer];
         const CUtensorMap* mD = &g.mapD[st.layer];
-        const int ka = (g.d_in[st.layer] + FK - 1) / FK, kd = (g.d_out[st.layer] + FK - 1) / FK;
-        const uint32_t bytes = (diag ? 0 : TILE_BYTES) + st.ns * TILE_BYTES;
+        const int nt = (diag ? 0 : 1) + st.ns;  // tiles per box
+        const int nbox = SLOTS / nt;
+        const int fks = nbox * FK;
+        const int ka = (g.d_in[st.layer] + fks - 1) / fks;
+        const int kd = (g.d_out[st.layer] + fks - 1) / fks;
+        const uint32_t bytes = static_cast<uint32_t>(nbox * nt) * TILE_BYTES;
         for (int k = 0; k < ka + kd; ++k) {
           const CUtensorMap* map = k < ka ? mA : mD;
-          const int f0 = (k < ka ? k : k - ka) * FK;
+          const int f0 = (k < ka ? k : k - ka) * fks;
           if (!mbar_wait(&empty_bar[stage], phase ^ 1, abrt, g.err)) goto producer_done;
           uint8_t* sp = smem + stage * STAGE_BYTES;
           mbar_arrive_expect_tx(&full_bar[stage], bytes);
-          if (!diag) tma_load_3d(map, &full_bar[stage], sp + A_OFF, f0, st.tb * GT, st.ex);
-          tma_load_3d(map, &full_bar[stage], sp + B_OFF, f0, st.sb * GT, st.ex);
-          if (st.ns == 2)
-            tma_load_3d(map, &full_bar[stage], sp + B_OFF + TILE_BYTES, f0, (st.sb + 1) * GT,
-                        st.ex);
+          for (int b = 0; b < nbox; ++b) {
+            uint8_t* bp = sp + b * nt * TILE_BYTES;
+            const int f = f0 + b * FK;
+            if (!diag) {
+              tma_load_3d(map, &full_bar[stage], bp, f, st.tb * GT, st.ex);
+              bp += TILE_BYTES;
+            }
+            tma_load_3d(map, &full_bar[stage], bp, f, st.sb * GT, st.ex);
+            if (st.ns == 2)
+              tma_load_3d(map, &full_bar[stage], bp + TILE_BYTES, f, (st.sb + 1) * GT, st.ex);
+          }
           ++uses[stage];
           if (++stage == STAGES) {
             stage = 0;
@@ -243,7 +257,11 @@ __global__ void __launch_bounds__(GHOST_THREADS, 1)
         const Strip st = decode(item, g);
         const bool diag = st.tb == st.sb;
         const uint32_t idesc = st.ns == 2 ? IDESC_N256 : IDESC_N128;
-        const int ka = (g.d_in[st.layer] + FK - 1) / FK, kd = (g.d_out[st.layer] + FK - 1) / FK;
+        const int nt = (diag ? 0 : 1) + st.ns;
+        const int nbox = SLOTS / nt;
+        const int fks = nbox * FK;
+        const int ka = (g.d_in[st.layer] + fks - 1) / fks;
+        const int kd = (g.d_out[st.layer] + fks - 1) / fks;
         if (!mbar_wait(&tempty_bar, (it & 1) ^ 1, abrt, g.err)) goto mma_done;
         tc_fence_after();
         for (int k = 0; k < ka + kd; ++k) {
@@ -253,13 +271,15 @@ __global__ void __launch_bounds__(GHOST_THREADS, 1)
           if (!mbar_wait(&full_bar[stage], phase, abrt, g.err)) goto mma_done;
           tc_fence_after();
           const uint32_t sp = smem_u32(smem + stage * STAGE_BYTES);
-          const uint32_t sb = sp + B_OFF;
-          const uint32_t sa = diag ? sb : sp + A_OFF;
+          for (int b = 0; b < nbox; ++b) {
+            const uint32_t sa = sp + b * nt * TILE_BYTES;
+            const uint32_t sb = diag ? sa : sa + TILE_BYTES;
 #pragma unroll
-          for (int kk = 0; kk < FK / 16; ++kk) {
-            const uint64_t ad = smem_desc_sw128(sa + kk * 32, LBO, SBO);
-            const uint64_t bd = smem_desc_sw128(sb + kk * 32, LBO, SBO);
-            mma_bf16(d_tmem, ad, bd, idesc, (kl | kk) != 0);
+            for (int kk = 0; kk < FK / 16; ++kk) {
+              const uint64_t ad = smem_desc_sw128(sa + kk * 32, LBO, SBO);
+              const uint64_t bd = smem_desc_sw128(sb + kk * 32, LBO, SBO);
+              mma_bf16(d_tmem, ad, bd, idesc, (kl | b | kk) != 0);
+            }
           }
           mma_commit(&empty_bar[stage]);
           if (++stage == STAGES) {

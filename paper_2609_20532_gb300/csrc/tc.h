@@ -36,17 +36,22 @@ cudaError_t tc_launch_ghost_batch(int L, const void* const* A, const void* const
 // clipped sum then writes one partial per range into the caller's scratch
 // (split * d_in * d_out fp32, 16-byte aligned) and a reduce pass adds them in
 // order with the noise; the materialised norm needs no scratch.
+// The split is fixed per layer when the step is planned (dp_step_init), from
+// the layer's shape and the tiles of the other layers that share its launch,
+// so a layer's sum rounds the same in a batched and a per-layer call.
 constexpr int kGemmMaxLayers = 8;
 constexpr int kGemmMaxSplit = 256;
-int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out);
+int64_t tc_gemm_tiles(int64_t d_in, int64_t d_out);
+int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out, int64_t other_tiles = 0);
 bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_out_a, int64_t d_in_b, int64_t d_out_b);
 // conv (per layer, NULL for a dense layer): A is then the NHWC input and the
 // kernels read its patch rows directly (tc_conv_implicit_ok must hold).
+// split: example ranges of each layer (as planned; NULL: tc_gemm_split alone).
 cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
                                     float* const* out, float* const* part, const int* d_in,
-                                    const int* d_out, const uint64_t* p_base, const float* c,
-                                    int B, int T, const Epilogue& ep, int* err, cudaStream_t s,
-                                    const ConvGeom* const* conv = nullptr);
+                                    const int* d_out, const uint64_t* p_base, const int* split,
+                                    const float* c, int B, int T, const Epilogue& ep, int* err,
+                                    cudaStream_t s, const ConvGeom* const* conv = nullptr);
 bool tc_conv_implicit_ok(const ConvGeom& g, int T);
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out);
 int64_t tc_mat_parts(int64_t d_in, int64_t d_out);
@@ -54,8 +59,9 @@ cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d
                                float* part, int NP, int row0, int* err, cudaStream_t s,
                                const ConvGeom* conv = nullptr);
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
-                              int d_in, int d_out, float* out, float* part, const Epilogue& ep,
-                              int* err, cudaStream_t s, const ConvGeom* conv = nullptr);
+                              int d_in, int d_out, int split, float* out, float* part,
+                              const Epilogue& ep, int* err, cudaStream_t s,
+                              const ConvGeom* conv = nullptr);
 
 // Clipped sum for short examples (T < 32): c_i folded into a bf16 hi+lo
 // split of A in scratch (tc_prescaled_scratch_bytes), then one plain GEMM.

@@ -607,6 +607,27 @@ def test_gram_strips_cover_every_block_pair(T):
         assert rel_err_elementwise(res["n"][l], ref) <= TOL["bf16"]
 
 
+@pytest.mark.parametrize("B,T,layers,want", [
+    (8, 64, [(4096, 4096)], dp.DP_NORM_MATERIALISED),   # 8 Gram items: one item's latency decides
+    (32, 64, [(4096, 4096)], dp.DP_NORM_GHOST),         # materialised work grows with B
+    (128, 64, [(4096, 4096)], dp.DP_NORM_GHOST),        # enough items to fill the GPU
+    (8, 512, [(4096, 4096)], dp.DP_NORM_GHOST),         # CTA-pair items, arithmetic decides
+    (32, 128, [(768, 2304), (768, 768), (768, 3072), (3072, 768)], dp.DP_NORM_GHOST),
+])
+def test_auto_norm_form_latency_term(B, T, layers, want):
+    """DP_NORM_AUTO's choice where the Gram form's few work items leave the
+    GPU mostly idle: at B = 8, T = 64 on the 4096 x 4096 layer the
+    materialised form is faster (measured 0.038 against 0.056 ms) and AUTO
+    takes it; at larger B, longer examples or several layers sharing the
+    Gram launch (block_bf16) it keeps the Gram form."""
+    cfg = dp.make_config(layers, B, T, "bf16", 1.0, 1.0)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        assert all(dp.dp_layer_norm_mode(ctx, l) == want for l in range(len(layers)))
+    finally:
+        dp.dp_step_destroy(ctx)
+
+
 def test_ghost_and_materialised_agree_on_block_workload():
     w = W.get("block_bf16")
     layers = W.make_inputs(w)
@@ -1430,3 +1451,33 @@ def test_two_rank_partitions_through_the_library(kind):
                 assert rel_err_normwise(o, r["out"][first + k]) <= TOL["bf16"]
                 seen.append(first + k)
         assert sorted(seen) == list(range(len(DP2_SHAPES)))
+
+
+def test_bench_data_parallel_path_two_ranks_one_gpu():
+    """bench.py's multi-rank path (data_parallel_step under torchrun) at two
+    ranks sharing cuda:0 with gloo collectives on host copies: it runs to
+    completion and rank 0 prints one JSON line that counts both ranks'
+    examples and names the partition."""
+    import json
+    import os
+    import socket
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    with socket.socket() as s_:
+        s_.bind(("127.0.0.1", 0))
+        port = s_.getsockname()[1]
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node=2",
+           "--master-addr", "127.0.0.1", "--master-port", str(port), "bench.py", "--gpus", "2",
+           "--steps", "2", "--warmup", "3", "--workload", "block_bf16", "--dist-backend", "gloo",
+           "--same-device", "--no-e2e"]
+    r = subprocess.run(cmd, cwd=root, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-3000:]
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1, r.stdout[-2000:]
+    line = json.loads(lines[0])
+    w = W.get("block_bf16")
+    assert line["n_gpus"] == 2 and line["config"]["global_batch"] == 2 * w.B
+    assert line["config"]["parallelism"] == "data-parallel by example"
+    assert line["value"] == pytest.approx(2 * w.B / (line["ms_per_step"] * 1e-3))
+    assert line["gpu_launches"] > 0 and line["collective_bytes_per_rank"] > 0
