@@ -614,9 +614,36 @@ def run_ours(args, rank, world, local_rank):
         run(k, 1000)
         torch.cuda.synchronize()                   # last outputs are in host memory
         wall = max_over_ranks((time.perf_counter() - t0) / k, world, dev)
+
+        # the host link alone: each direction by itself, then both at once, on
+        # the same pinned buffers; the e2e floor is the slower of the link's
+        # per-step time and the device step
+        def copies(h2d, d2h):
+            torch.cuda.synchronize()
+            t1 = time.perf_counter()
+            if h2d:
+                with torch.cuda.stream(s_in):
+                    for l in range(L):
+                        A_b[1][l].copy_(A_h[l], non_blocking=True)
+                        D_b[1][l].copy_(D_h[l], non_blocking=True)
+            if d2h:
+                with torch.cuda.stream(s_out):
+                    for l in range(L):
+                        O_h[1][l].copy_(O_b[1][l], non_blocking=True)
+            torch.cuda.synchronize()
+            return time.perf_counter() - t1
+        link = {}
+        for key, a_, b_ in (("h2d", True, False), ("d2h", False, True), ("both", True, True)):
+            link[key] = min(copies(a_, b_) for _ in range(3))
+        floor = max(link["both"], ms_step * 1e-3)
         e2e = {"value": replica_throughput(w.B, world, wall), "unit": UNIT, "ms_per_step": 1e3 * wall,
                "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out_bytes + rec_bytes,
-               "steps": k, "overlap": "double-buffered copies on separate streams"}
+               "steps": k, "overlap": "double-buffered copies on separate streams",
+               "link": {"h2d_gbs": in_bytes / link["h2d"] / 1e9,
+                        "d2h_gbs": out_bytes / link["d2h"] / 1e9,
+                        "both_gbs": (in_bytes + out_bytes) / link["both"] / 1e9,
+                        "floor_ms": 1e3 * floor,
+                        "overlap_efficiency": floor / wall}}
 
     dp.dp_step_destroy(ctx)
     if rank != 0:
@@ -788,7 +815,8 @@ def run_data_parallel(args, rank, world, local_rank):
 def run_sweep(args):
     """One JSON line with a record per point of the 4096x4096 sweep: step
     time, per-kernel times, the norm kernel the cost model picked, both norm
-    kernels timed (the measured crossover) and roofline fractions.  Inputs are
+    forms timed up to the clip factors (the measured crossover) and roofline
+    fractions.  Inputs are
     drawn on the device (torch's seeded CUDA generator, N(0,1) rounded to
     bf16) so the whole sweep stays under a minute."""
     import torch
@@ -833,6 +861,13 @@ def run_sweep(args):
                 dp.dp_step_init(cfg, stream, ctx)
                 dp.dp_layer_norms(ctx, 0, A, D)
 
+            def norms_and_factors():
+                # the two forms leave different partial sums for the clip
+                # kernel to add (a few per example against one per tile), so
+                # the norm stage is compared up to the clip factors
+                norms()
+                dp.dp_clip_factors(ctx)
+
             def gemm():
                 dp.dp_clipped_sum_noise(ctx, 0, A, D, out, 0)
 
@@ -844,7 +879,7 @@ def run_sweep(args):
             for _ in range(args.warmup):
                 step()
             torch.cuda.synchronize()
-            rec[f"norm_{mode_name}_ms"] = timed(norms, args.steps)
+            rec[f"norm_{mode_name}_ms"] = timed(norms_and_factors, args.steps)
             if mode_name == "auto":
                 rec["auto_picked"] = {1: "rank1", 2: "ghost", 3: "materialised"}[
                     dp.dp_layer_norm_mode(ctx, 0)]

@@ -243,9 +243,11 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
 }
 
 // ---------------------------------------------------------------------------
-// Cross-layer sum and clip factors.  One warp per example: lane j adds the
-// layers j, j + 32, ... (each layer's partials in slot order), then a fixed
-// butterfly adds the 32 lane sums, so the order never depends on timing.
+// Cross-layer sum and clip factors.  One warp per example.  For each layer
+// in turn, lane j adds the partials j, j + 32, ... (coalesced: a layer can
+// hold thousands of partials per example, one per tile and epilogue warp of
+// the materialised form), then a fixed butterfly adds the 32 lane sums; lane
+// 0 adds the layer sums in layer order.  The order never depends on timing.
 // ---------------------------------------------------------------------------
 // mode kClipLocal: only the layers' norms and their sum (into user_s); no
 // clip factor, no flag.  mode kClipGiven: s_i = s_given[i] (the squared norm
@@ -260,16 +262,16 @@ __global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
   if (w >= B) return;  // the whole warp leaves together
   const int i = static_cast<int>(w);
   float s = 0.f;
-  for (int l = lane; l < L; l += 32) {
+  for (int l = 0; l < L; ++l) {
     const float* p = part + (static_cast<int64_t>(l) * B + i) * NP;
-    float n = 0.f;
     const int np = nparts[l];
-    for (int q = 0; q < np; ++q) n += p[q];
-    layer_sq[static_cast<int64_t>(l) * B + i] = n;
+    float n = 0.f;
+    for (int q = lane; q < np; q += 32) n += p[q];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) n += __shfl_xor_sync(0xffffffffu, n, o);
+    if (lane == 0) layer_sq[static_cast<int64_t>(l) * B + i] = n;
     s += n;
   }
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
   if (lane != 0) return;
   if (mode == kClipLocal) {
     user_s[i] = s;

@@ -62,11 +62,15 @@ constexpr uint32_t LBO = CHUNK, SBO = 1024;
 // with d_out <= 128 (no MMA work on columns past the layer).
 template <bool PAIR, int NB>
 struct Cfg {
-  static constexpr int STAGES = PAIR ? 6 : 4;
   static constexpr int B_COLS = PAIR ? NB / 2 : NB;         // D columns staged per CTA
   static constexpr int A_STAGE = BM * BK * 2;               // 16 KB
-  static constexpr int B_STAGE = B_COLS * BK * 2;           // 16 / 32 KB
-  static constexpr int STAGE_BYTES = A_STAGE + B_STAGE;     // 32 / 48 KB
+  static constexpr int B_STAGE = B_COLS * BK * 2;           // 8 / 16 / 32 KB
+  static constexpr int STAGE_BYTES = A_STAGE + B_STAGE;     // 24 / 32 / 48 KB
+  // 192 KB of stages whatever the tile: the operand bytes in flight set the
+  // rate at which L2 delivers them (a stage's round trip is about the same
+  // for every tile), so the narrow tiles get more stages: 8, 6 or 4
+  static constexpr int STAGES = (192 * 1024) / STAGE_BYTES;
+  static_assert(STAGES % 2 == 0 && STAGES * STAGE_BYTES == 192 * 1024, "stage split");
   static constexpr int TILE_M = PAIR ? 2 * BM : BM;
   // pipeline stages, then one 4 KB store-staging block per epilogue warp
   static constexpr int STAGING = STAGES * STAGE_BYTES;

@@ -465,6 +465,38 @@ def test_deterministic_and_step_keyed():
     assert np.array_equal(r1["n"], r2["n"]) and np.array_equal(r1["c"], r2["c"])
 
 
+@pytest.mark.parametrize("p_first,n", [(0, 4096), (3, 1001), (140_000_001, 77), (1 << 40, 4099)])
+def test_noise_add_range_matches_oracle(p_first, n):
+    """dp_noise_add_range adds out_scale * sigma * C * z_{p_first + e} to any
+    range of global parameter indices (a rank's slice of the commitment):
+    elementwise against the oracle to 1e-6, with unaligned starts and ragged
+    ends; n = 0 launches nothing."""
+    w = W.custom("range", [(8, 8)], 2, 1, "f32", C=0.7, sigma=1.3, wid=612)
+    dev = torch.device(DEV)
+    scale = 0.25
+    cfg = dp.make_config(w.layers, w.B, w.T, w.dtype, w.C, w.sigma, out_scale=scale,
+                         seed=(1 << 62) + 9, step=17)
+    ctx = dp.dp_step_init(cfg)
+    g = torch.Generator().manual_seed(n)
+    init = torch.randn(n + 8, generator=g)
+    buf = init.clone().to(dev)
+    try:
+        n0 = dp.dp_kernel_launches()
+        dp.dp_noise_add_range(ctx, p_first, 0, buf)
+        assert dp.dp_kernel_launches() == n0
+        dp.dp_noise_add_range(ctx, p_first, n, buf)
+        torch.cuda.synchronize()
+    finally:
+        dp.dp_step_destroy(ctx)
+    got = buf.double().cpu().numpy()
+    z = O.gaussian_noise((1 << 62) + 9, 17, p_first, n)
+    want = scale * f32(w.sigma) * f32(w.C) * z
+    added = got[:n] - init.double().numpy()[:n]
+    bound = 1e-6 * np.abs(want) + 2 * 2.0 ** -24 * np.abs(got[:n])
+    assert np.all(np.abs(added - want) <= bound)
+    assert np.array_equal(got[n:], init.double().numpy()[n:])   # nothing past the range
+
+
 def test_noise_statistics_on_device():
     """Noise-only output over a large layer: mean ~ 0, variance ~ (out_scale sigma C)^2."""
     w = W.custom("stat", [(4096, 4096)], 2, 1, "bf16", C=0.5, sigma=1.3, wid=604)
