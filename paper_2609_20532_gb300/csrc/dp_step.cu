@@ -201,15 +201,16 @@ dp_norm_mode resolve_mode(dp_norm_mode m, int T, int64_t d_in, int64_t d_out) {
 
 // Latency term of the norm-form choice.  When the Gram form has few work
 // items (B times the Gram layers that share T: fewer than half the SMs), its
-// time is one item's, whose K steps of 64 features run one after another on
-// one SM: about 0.42 us each on the GB300 (measured: 4096 x 4096 at T = 64,
-// 128 steps in 54 us), while the materialised form spreads over the whole
-// GPU at about 0.9 PFLOP/s for examples of one 64-position K block (measured
-// at T = 64).  Only examples of one 128-position block (T <= 128) are
-// concerned: longer ones give the Gram form CTA-pair items that fill the GPU
-// and it wins by its arithmetic.
-constexpr double kGramStepSeconds = 0.42e-6;
-constexpr double kMatShortRate = 0.9e15;
+// time is one item's, whose K steps run one after another on one SM: about
+// 0.25 us per 64 features on the GB300 (measured: 4096 x 4096 at T = 64,
+// 128 x 64 features in 32 us), while the materialised form spreads over the
+// whole GPU at about 0.64 PFLOP/s for examples of one 64-position K block
+// (measured at T = 64: 17.2 GFLOP in 27 us).  Both forms then reduce their
+// partial sums in the clip kernel at about the same cost.  Only examples of
+// one 128-position block (T <= 128) are concerned: longer ones give the Gram
+// form CTA-pair items that fill the GPU and it wins by its arithmetic.
+constexpr double kGramStepSeconds = 0.25e-6;
+constexpr double kMatShortRate = 0.64e15;
 
 bool gram_latency_prefers_materialised(int B, int T, int64_t d_in, int64_t d_out,
                                        int64_t gram_items, int sms) {

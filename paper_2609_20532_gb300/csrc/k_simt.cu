@@ -243,36 +243,51 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
 }
 
 // ---------------------------------------------------------------------------
-// Cross-layer sum and clip factors.  One warp per example.  For each layer
-// in turn, lane j adds the partials j, j + 32, ... (coalesced: a layer can
-// hold thousands of partials per example, one per tile and epilogue warp of
-// the materialised form), then a fixed butterfly adds the 32 lane sums; lane
-// 0 adds the layer sums in layer order.  The order never depends on timing.
+// Cross-layer sum and clip factors.  A group of WARPS warps per example (one
+// warp, or a block of eight where a layer holds thousands of partials per
+// example: one per tile and epilogue warp of the materialised form).  For
+// each layer in turn, thread j of the group adds the partials j, j + G, ...
+// (G = 32 WARPS threads; coalesced), a fixed butterfly adds each warp's 32 sums, and the
+// warps' sums are added in warp order; thread 0 adds the layer sums in layer
+// order.  The order never depends on timing.
 // ---------------------------------------------------------------------------
 // mode kClipLocal: only the layers' norms and their sum (into user_s); no
 // clip factor, no flag.  mode kClipGiven: s_i = s_given[i] (the squared norm
 // summed over every rank's layers) instead of this context's sum.
+template <int WARPS>
 __global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
                        const int* __restrict__ nparts, float C, float* __restrict__ layer_sq,
                        float* __restrict__ s_out, float* __restrict__ c_out,
                        float* __restrict__ user_s, float* __restrict__ user_c, int* flag,
                        int mode, const float* __restrict__ s_given) {
-  const int64_t w = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const int lane = static_cast<int>(threadIdx.x) & 31;
-  if (w >= B) return;  // the whole warp leaves together
+  constexpr int G = 32 * WARPS;  // threads per example
+  __shared__ float red[WARPS];
+  const int64_t gid = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const int64_t w = gid / G;
+  const int t = static_cast<int>(gid - w * G);
+  const int lane = t & 31;
+  if (w >= B) return;  // a whole group leaves together (WARPS > 1: one group per block)
   const int i = static_cast<int>(w);
   float s = 0.f;
   for (int l = 0; l < L; ++l) {
     const float* p = part + (static_cast<int64_t>(l) * B + i) * NP;
     const int np = nparts[l];
     float n = 0.f;
-    for (int q = lane; q < np; q += 32) n += p[q];
+    for (int q = t; q < np; q += G) n += p[q];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) n += __shfl_xor_sync(0xffffffffu, n, o);
-    if (lane == 0) layer_sq[static_cast<int64_t>(l) * B + i] = n;
+    if constexpr (WARPS > 1) {
+      if (lane == 0) red[t >> 5] = n;
+      __syncthreads();
+      n = 0.f;
+#pragma unroll
+      for (int k = 0; k < WARPS; ++k) n += red[k];
+      __syncthreads();
+    }
+    if (t == 0) layer_sq[static_cast<int64_t>(l) * B + i] = n;
     s += n;
   }
-  if (lane != 0) return;
+  if (t != 0) return;
   if (mode == kClipLocal) {
     user_s[i] = s;
     return;
@@ -527,8 +542,12 @@ cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_np
                         float* layer_sq, float* s_out, float* c_out, float* user_s, float* user_c,
                         int* flag, cudaStream_t s, int mode, const float* s_given) {
   note_launch();
-  k_clip<<<(B + 7) / 8, 256, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out,
-                                      user_s, user_c, flag, mode, s_given);
+  if (NP >= 512)  // thousands of partials per example: a block of eight warps each
+    k_clip<8><<<B, 256, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out, user_s,
+                                user_c, flag, mode, s_given);
+  else
+    k_clip<1><<<(B + 7) / 8, 256, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out,
+                                          user_s, user_c, flag, mode, s_given);
   return cudaGetLastError();
 }
 
