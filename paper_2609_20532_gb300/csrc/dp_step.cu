@@ -76,6 +76,10 @@ struct LayerPlan {
   int64_t g_off;       // offset (floats) of its [B][d_in][d_out] gradients in d_grads
   int split;           // tensor-core clipped sum: example ranges per tile (tc_gemm_split)
   int64_t s_off;       // offset (floats) of its [split][d_in][d_out] partials in d_split
+  // tensor-core clipped sum: its tiles from tail_from on run as tail_split
+  // pieces of the batch (the last round of its launch group, tc_plan_tail);
+  // fixed at planning so any grouping of the calls gives the same bits
+  int tail_from, tail_split;
   // convolutions (kind DP_LAYER_CONV2D; A is the NHWC input)
   int kind;            // dp_layer.kind as given
   int conv;            // 1: a convolution whose patch rows differ from its input
@@ -121,6 +125,8 @@ struct dp_ctx {
   int64_t grads_floats = 0;
   float* d_split = nullptr;     // partial sums of tensor-core layers whose batch is split
   int64_t split_floats = 0;
+  float* d_tail = nullptr;      // partial tiles of a clipped-sum launch's tail pieces
+  int64_t tail_bytes = 0;
   uint8_t* d_unf = nullptr;     // patch rows of convolutions formed in scratch
   int64_t unf_bytes = 0;
   size_t part_bytes = 0;
@@ -272,12 +278,14 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
   // one tile shape and T, up to kGemmMaxLayers per launch): a layer's example
   // split is chosen for that launch, then fixed.
   std::vector<int64_t> group_tiles(cfg->n_layers, 0);
+  std::vector<std::vector<int>> groups;
   {
     std::vector<int> cur;
     auto close = [&]() {
       int64_t t = 0;
       for (int l : cur) t += dpk::tc_gemm_tiles(cfg->layers[l].d_in, cfg->layers[l].d_out);
       for (int l : cur) group_tiles[l] = t;
+      if (!cur.empty()) groups.push_back(cur);
       cur.clear();
     };
     for (int l = 0; l < cfg->n_layers; ++l) {
@@ -308,6 +316,8 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
     p.g_off = 0;
     p.split = 1;
     p.s_off = 0;
+    p.tail_from = 0;
+    p.tail_split = 1;
     p.kind = cfg->layers[l].kind;
     p.conv = p.kind == DP_LAYER_CONV2D ? 1 : 0;
     p.cg = dpk::ConvGeom{};
@@ -406,6 +416,23 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
     if (p.conv && !p.implicit) need_unfold();
     if (p.nparts > NP) NP = p.nparts;
   }
+  // the last round of each launch group of tensor-core clipped sums
+  for (const std::vector<int>& grp : groups) {
+    bool ok = grp.size() <= static_cast<size_t>(dpk::kGemmMaxLayers);
+    for (int l : grp) ok = ok && c->plan[l].gemm_tc == 1 && c->plan[l].split == 1;
+    if (!ok) continue;
+    int64_t di[dpk::kGemmMaxLayers], dd[dpk::kGemmMaxLayers];
+    int tf[dpk::kGemmMaxLayers], ts[dpk::kGemmMaxLayers];
+    for (size_t q = 0; q < grp.size(); ++q) {
+      di[q] = c->plan[grp[q]].d_in;
+      dd[q] = c->plan[grp[q]].d_out;
+    }
+    dpk::tc_plan_tail(static_cast<int>(grp.size()), di, dd, cfg->B, tf, ts);
+    for (size_t q = 0; q < grp.size(); ++q) {
+      c->plan[grp[q]].tail_from = tf[q];
+      c->plan[grp[q]].tail_split = ts[q];
+    }
+  }
   // the partial buffer [L][B][NP] and the row index layer * B + example
   if (static_cast<double>(cfg->n_layers) * cfg->B > 0x7fffffff ||
       static_cast<double>(cfg->n_layers) * cfg->B * NP * 4.0 > 0x1p50)
@@ -413,6 +440,9 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
   c->NP = static_cast<int>(NP);
   c->grads_floats = grads;
   c->split_floats = splits;
+  c->tail_bytes = 0;
+  for (const LayerPlan& p : c->plan)
+    if (p.gemm_tc == 1) c->tail_bytes = dpk::tc_tail_scratch_bytes();
   c->unf_bytes = unf;
   return DP_OK;
 }
@@ -430,10 +460,12 @@ void free_scratch(dp_ctx* c) {
   cudaFree(c->d_prescaled);
   cudaFree(c->d_grads);
   cudaFree(c->d_split);
+  cudaFree(c->d_tail);
   cudaFree(c->d_unf);
   c->d_prescaled = nullptr;
   c->d_grads = nullptr;
   c->d_split = nullptr;
+  c->d_tail = nullptr;
   c->d_unf = nullptr;
   cudaFree(c->d_key);
   cudaFreeHost(c->h_key);
@@ -470,6 +502,7 @@ dp_status alloc_scratch(dp_ctx* c) {
   if (c->prescaled_bytes > 0) DP_ALLOC(c->d_prescaled, static_cast<size_t>(c->prescaled_bytes));
   if (c->grads_floats > 0) DP_ALLOC(c->d_grads, sizeof(float) * static_cast<size_t>(c->grads_floats));
   if (c->split_floats > 0) DP_ALLOC(c->d_split, sizeof(float) * static_cast<size_t>(c->split_floats));
+  if (c->tail_bytes > 0) DP_ALLOC(c->d_tail, static_cast<size_t>(c->tail_bytes));
   if (c->unf_bytes > 0) DP_ALLOC(c->d_unf, static_cast<size_t>(c->unf_bytes));
   DP_ALLOC(c->d_key, 2 * sizeof(uint64_t));
 #undef DP_ALLOC
@@ -696,7 +729,8 @@ cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const vo
   if (p.gemm_tc == 1)
     return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, p.T, din, dout, p.split, d_out,
                                   p.split > 1 ? c->d_split + p.s_off : nullptr, ep, c->d_flag,
-                                  c->stream, p.implicit ? &p.cg : nullptr);
+                                  c->stream, p.implicit ? &p.cg : nullptr, p.tail_from,
+                                  p.tail_split, c->d_tail, c->tail_bytes);
   if (p.gemm_tc == 2)
     return dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, p.T, din, dout, d_out, ep,
                                             c->d_flag, c->d_prescaled, c->stream);
@@ -1023,7 +1057,7 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
     const dpk::ConvGeom* cg[dpk::kGemmMaxLayers];
     int din[dpk::kGemmMaxLayers], dout[dpk::kGemmMaxLayers];
     uint64_t pb[dpk::kGemmMaxLayers];
-    int sp[dpk::kGemmMaxLayers];
+    int sp[dpk::kGemmMaxLayers], tf[dpk::kGemmMaxLayers], ts[dpk::kGemmMaxLayers];
     for (size_t q = 0; q < grp.size(); ++q) {
       const int r = grp[q];
       const LayerPlan& p = c->plan[layers[r]];
@@ -1036,11 +1070,14 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
       din[q] = static_cast<int>(p.d_in);
       dout[q] = static_cast<int>(p.d_out);
       pb[q] = p.p_base;
+      tf[q] = p.tail_from;
+      ts[q] = p.tail_split;
     }
     cudaError_t e = dpk::tc_launch_clipsum_batch(static_cast<int>(grp.size()), a, d, o, part, din,
                                                  dout, pb, sp, c->d_c, c->B,
                                                  c->plan[layers[grp[0]]].T, ep, c->d_flag,
-                                                 c->stream, cg);
+                                                 c->stream, cg, tf, ts, c->d_tail,
+                                                 c->tail_bytes);
     grp.clear();
     return e;
   };

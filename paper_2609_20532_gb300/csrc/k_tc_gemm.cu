@@ -87,6 +87,7 @@ struct GemmArgs {
   CUtensorMap mapA[kGemmMaxLayers];
   CUtensorMap mapD[kGemmMaxLayers];
   CUtensorMap mapO[kGemmMaxLayers];  // fp32 outputs, 32 x 32 boxes ([split][d_in][d_out] when split)
+  CUtensorMap mapT;                   // tail pieces' partial tiles [piece][TILE_M][NB] (fp32)
   float* out[kGemmMaxLayers];
   uint64_t p_base[kGemmMaxLayers];  // global parameter index of element (0, 0)
   int d_in[kGemmMaxLayers], d_out[kGemmMaxLayers];
@@ -94,7 +95,18 @@ struct GemmArgs {
   int split[kGemmMaxLayers];  // example ranges per tile (1: the whole batch)
   int conv[kGemmMaxLayers];   // 1: mapA is the NHWC input of a convolution (patch rows on the fly)
   ConvGeom cg[kGemmMaxLayers];
-  int tile_start[kGemmMaxLayers + 1];  // first work item of each layer
+  int tile_start[kGemmMaxLayers + 1];  // first work item of each layer (whole tiles)
+  // Tail split: a layer's tiles from tail_from on (the tiles that would
+  // leave most units idle in the launch's last round) run as pieces, each
+  // over about B / tail_split examples, after every whole tile of the
+  // launch.  Pieces of layer l are items tile_start[L] + piece_start[l] ..;
+  // piece q of the layer covers its tail tile q % n and example range
+  // q / n (n tail tiles).  A clipped-sum piece stores its partial tile into
+  // mapT at its piece index for the tail reduce; a norm piece writes its
+  // examples' partials like a whole tile.
+  int tail_from[kGemmMaxLayers], tail_split[kGemmMaxLayers];
+  int piece_start[kGemmMaxLayers + 1];
+  int n_items;
   int L;
   const float* c;  // clip factors [B]; nullptr: all ones (pre-scaled operand)
   float* part;     // materialised-norm partials (L == 1)
@@ -113,20 +125,37 @@ struct GemmArgs {
 // different tiles of the same examples and share their operand rows in L2.
 struct GemmItem {
   int l, lt, s, e0, e1;
+  int z;  // tail piece index, -1 for a tile of its own
 };
 
 __device__ __forceinline__ GemmItem gemm_item(const GemmArgs& g, int item) {
   GemmItem w;
   int l = 0;
+  if (item >= g.tile_start[g.L]) {
+    // a tail piece (tail tiles are unsplit layers' last tiles)
+    const int p = item - g.tile_start[g.L];
+    while (p >= g.piece_start[l + 1]) ++l;
+    const int q = p - g.piece_start[l];
+    const int n = g.n_m[l] * g.n_n[l] - g.tail_from[l];
+    const int r = q / n;
+    w.l = l;
+    w.s = 0;
+    w.lt = g.tail_from[l] + (q - r * n);
+    w.e0 = static_cast<int>(static_cast<int64_t>(g.B) * r / g.tail_split[l]);
+    w.e1 = static_cast<int>(static_cast<int64_t>(g.B) * (r + 1) / g.tail_split[l]);
+    w.z = p;
+    return w;
+  }
   while (item >= g.tile_start[l + 1]) ++l;
   const int li = item - g.tile_start[l];
-  const int tiles = g.n_m[l] * g.n_n[l];
   const int S = g.split[l];
+  const int tiles = S > 1 ? g.n_m[l] * g.n_n[l] : g.tail_from[l];  // whole tiles per range
   w.l = l;
   w.s = li / tiles;
   w.lt = li - w.s * tiles;
   w.e0 = static_cast<int>(static_cast<int64_t>(g.B) * w.s / S);
   w.e1 = static_cast<int>(static_cast<int64_t>(g.B) * (w.s + 1) / S);
+  w.z = -1;
   return w;
 }
 
@@ -257,7 +286,9 @@ __device__ __forceinline__ void add_noise_slot(float (&S)[SZ], int q, float4 z, 
 // with m fastest, so the tiles in flight at one time share an A panel of
 // kRasterM tiles that stays in L2 while the D panels stream past it.
 constexpr int kRasterM = 8;
-__device__ __forceinline__ void tile_mn(int t, int n_m, int n_n, int& mt, int& nt) {
+// most tail tiles one launch may split (the units of a GPU of 152 SMs)
+constexpr int kTailMaxTiles = 152;
+__host__ __device__ __forceinline__ void tile_mn(int t, int n_m, int n_n, int& mt, int& nt) {
   const int per_group = kRasterM * n_n;
   const int grp = t / per_group;
   const int r = t - grp * per_group;
@@ -293,7 +324,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   // round trips per MMA, measured faster; the stage memory is the same.
   const int bps = (PAIR && (kpe % 2) == 0) ? 2 : 1;
   const int nst = bps == 2 ? STAGES / 2 : STAGES;
-  const int n_tiles = g.tile_start[g.L];
+  const int n_tiles = g.n_items;
   volatile int* abrt = &abort_flag;
 
   if (threadIdx.x == 0) {
@@ -465,9 +496,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       const GemmItem w = gemm_item(g, tile);
       const int l = w.l, lt = w.lt;
       const int d_in = g.d_in[l], d_out = g.d_out[l];
-      // a split tile stores its partial sum unscaled and without noise; the
-      // reduce pass adds the ranges in order, then the noise
-      const bool part_out = g.split[l] > 1;
+      // a split tile or a tail piece stores its partial sum unscaled and
+      // without noise; the reduce pass adds the ranges in order, then the noise
+      const bool part_out = g.split[l] > 1 || w.z >= 0;
       int mt, nt;
       tile_mn(lt, g.n_m[l], g.n_n[l], mt, nt);
       const int m0 = mt * C::TILE_M + static_cast<int>(rank) * BM;
@@ -558,7 +589,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) {
-            if (part_out)
+            if (w.z >= 0)
+              tma_store_3d(&g.mapT, stg, k0 - n0 + 32 * c4, y - mt * C::TILE_M, w.z);
+            else if (part_out)
               tma_store_3d(&g.mapO[l], stg, k0 + 32 * c4, y, w.s);
             else if (g.accumulate)
               tma_reduce_add_2d(&g.mapO[l], stg, k0 + 32 * c4, y);
@@ -618,7 +651,8 @@ bool use_pair(int64_t d_in) { return d_in > BM; }
 int gemm_nb(int64_t d_out) { return d_out <= 128 ? 128 : BN; }
 
 template <bool NORM, bool PAIR, int NB, bool CONV>
-cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
+cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s, float* tail = nullptr,
+                        int64_t tail_cap = 0) {
   using C = Cfg<PAIR, NB>;
   cudaError_t e = setup_once_per_device(
       reinterpret_cast<const void*>(&k_gemm_tc<NORM, PAIR, NB, CONV>), []() -> cudaError_t {
@@ -639,15 +673,57 @@ cudaError_t launch_gemm(GemmArgs& g, cudaStream_t s) {
         return cudaSuccess;
       });
   if (e != cudaSuccess) return e;
-  g.tile_start[0] = 0;
-  for (int l = 0; l < g.L; ++l) {
-    g.n_m[l] = (g.d_in[l] + C::TILE_M - 1) / C::TILE_M;
-    g.n_n[l] = (g.d_out[l] + NB - 1) / NB;
-    if (g.split[l] < 1) g.split[l] = 1;
-    g.tile_start[l + 1] = g.tile_start[l] + g.n_m[l] * g.n_n[l] * g.split[l];
-  }
-  const int tiles = g.tile_start[g.L];
   const int sms = device_sm_count();
+  // whole tiles and tail pieces of every layer (a tail needs tail_split >= 2
+  // on an unsplit layer; the norm kernel plans its own below)
+  auto count_items = [&]() -> bool {
+    g.tile_start[0] = 0;
+    g.piece_start[0] = 0;
+    for (int l = 0; l < g.L; ++l) {
+      g.n_m[l] = (g.d_in[l] + C::TILE_M - 1) / C::TILE_M;
+      g.n_n[l] = (g.d_out[l] + NB - 1) / NB;
+      if (g.split[l] < 1) g.split[l] = 1;
+      const int tl = g.n_m[l] * g.n_n[l];
+      int whole = tl * g.split[l], pieces = 0;
+      if (g.tail_split[l] >= 2) {
+        if (g.split[l] != 1 || g.tail_from[l] < 0 || g.tail_from[l] >= tl ||
+            g.tail_split[l] > g.B || g.d_rows > 0)
+          return false;
+        whole = g.tail_from[l];
+        pieces = (tl - g.tail_from[l]) * g.tail_split[l];
+      } else {
+        g.tail_from[l] = tl;
+        g.tail_split[l] = 1;
+      }
+      g.tile_start[l + 1] = g.tile_start[l] + whole;
+      g.piece_start[l + 1] = g.piece_start[l] + pieces;
+    }
+    g.n_items = g.tile_start[g.L] + g.piece_start[g.L];
+    return true;
+  };
+  if (!count_items()) return cudaErrorInvalidValue;
+  if constexpr (NORM) {
+    // a norm launch (one layer) splits its own last round: a piece's
+    // examples keep their partial slots, so the result does not change
+    auto plan_norm_tail = [&](int units) {
+      const int tiles = g.tile_start[1];
+      const int r = tiles % units;
+      if (g.L != 1 || g.split[0] != 1 || tiles <= units || r == 0 || g.d_rows > 0) return;
+      int S = units / r;
+      if (S > g.B) S = g.B;
+      if (S < 2) return;
+      g.tail_from[0] = tiles - r;
+      g.tail_split[0] = S;
+      count_items();
+    };
+    plan_norm_tail(PAIR ? sms / 2 : sms);
+  } else if (g.piece_start[g.L] > 0) {
+    const int64_t bytes = static_cast<int64_t>(g.piece_start[g.L]) * C::TILE_M * NB * 4;
+    if (!tail || (reinterpret_cast<uintptr_t>(tail) & 15) != 0 || bytes > tail_cap ||
+        !make_tma_f32_split(&g.mapT, tail, g.piece_start[g.L], C::TILE_M, NB))
+      return cudaErrorInvalidValue;
+  }
+  const int tiles = g.n_items;
   if constexpr (PAIR) {
     // persistent grid: as many pairs as can be resident at once
     cudaLaunchConfig_t cfg = {};
@@ -720,7 +796,7 @@ bool make_input_maps(const void* A, const void* D, GemmArgs& g, int l,
 }
 
 template <bool NORM>
-cudaError_t launch_any(GemmArgs& g, cudaStream_t s) {
+cudaError_t launch_any(GemmArgs& g, cudaStream_t s, float* tail = nullptr, int64_t tail_cap = 0) {
   // every layer of a launch shares the tile shape (use_pair, gemm_nb); a
   // convolution read in place always has pairs (tc_conv_implicit_ok)
   bool conv = false;
@@ -728,12 +804,13 @@ cudaError_t launch_any(GemmArgs& g, cudaStream_t s) {
   const bool pair = use_pair(g.d_in[0]);
   if (conv && !pair) return cudaErrorInvalidValue;
   if (gemm_nb(g.d_out[0]) == 128) {
-    if (conv) return launch_gemm<NORM, true, 128, true>(g, s);
-    return pair ? launch_gemm<NORM, true, 128, false>(g, s)
-                : launch_gemm<NORM, false, 128, false>(g, s);
+    if (conv) return launch_gemm<NORM, true, 128, true>(g, s, tail, tail_cap);
+    return pair ? launch_gemm<NORM, true, 128, false>(g, s, tail, tail_cap)
+                : launch_gemm<NORM, false, 128, false>(g, s, tail, tail_cap);
   }
-  if (conv) return launch_gemm<NORM, true, BN, true>(g, s);
-  return pair ? launch_gemm<NORM, true, BN, false>(g, s) : launch_gemm<NORM, false, BN, false>(g, s);
+  if (conv) return launch_gemm<NORM, true, BN, true>(g, s, tail, tail_cap);
+  return pair ? launch_gemm<NORM, true, BN, false>(g, s, tail, tail_cap)
+              : launch_gemm<NORM, false, BN, false>(g, s, tail, tail_cap);
 }
 
 void set_epilogue(GemmArgs& g, const Epilogue& ep) {
@@ -823,6 +900,66 @@ __global__ void __launch_bounds__(256) k_split_reduce(const __grid_constant__ Sp
   v.z = g.out_scale * fmaf(g.sigmaC, z.z, s.z);
   v.w = g.out_scale * fmaf(g.sigmaC, z.w, s.w);
   float4* o = reinterpret_cast<float4*>(P.out + e);
+  if (g.accumulate) {
+    const float4 a = *o;
+    v.x += a.x;
+    v.y += a.y;
+    v.z += a.z;
+    v.w += a.w;
+  }
+  *o = v;
+}
+
+// The tail pieces of one clipped-sum launch: for each tail tile its partial
+// tiles added in example order, then the noise, the output scale and the
+// store (or add) into the layer's output, as for a split layer.
+struct TailReduceArgs {
+  const float* tail;  // [pieces][tile_m][nb]
+  float* out[kGemmMaxLayers];
+  uint64_t p_base[kGemmMaxLayers];
+  int d_in[kGemmMaxLayers], d_out[kGemmMaxLayers];
+  // per tail tile: its layer and origin, and its pieces first, first +
+  // stride, ... (count of them, in example order)
+  int layer[kTailMaxTiles], row0[kTailMaxTiles], col0[kTailMaxTiles];
+  int first[kTailMaxTiles], stride[kTailMaxTiles], count[kTailMaxTiles];
+  int n, tile_m, nb;
+  const uint64_t* key;
+  float out_scale, sigmaC;
+  int add_noise, accumulate;
+};
+
+__global__ void __launch_bounds__(256) k_tail_reduce(const __grid_constant__ TailReduceArgs g) {
+  const int per_row = g.nb / 4;
+  const int per_tile = g.tile_m * per_row;
+  const int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (q >= static_cast<int64_t>(g.n) * per_tile) return;
+  const int t = static_cast<int>(q / per_tile);
+  const int r = static_cast<int>(q - static_cast<int64_t>(t) * per_tile);
+  const int row = r / per_row, col = (r - row * per_row) * 4;
+  const int l = g.layer[t];
+  const int j = g.row0[t] + row, k = g.col0[t] + col;
+  if (j >= g.d_in[l] || k >= g.d_out[l]) return;  // d_out is a multiple of 8
+  const int64_t tile_elems = static_cast<int64_t>(g.tile_m) * g.nb;
+  const float* src =
+      g.tail + g.first[t] * tile_elems + static_cast<int64_t>(row) * g.nb + col;
+  const int64_t step = g.stride[t] * tile_elems;
+  float4 s = __ldcs(reinterpret_cast<const float4*>(src));
+  for (int p = 1; p < g.count[t]; ++p) {
+    const float4 v = __ldcs(reinterpret_cast<const float4*>(src + p * step));
+    s.x += v.x;
+    s.y += v.y;
+    s.z += v.z;
+    s.w += v.w;
+  }
+  const uint64_t e = static_cast<uint64_t>(j) * g.d_out[l] + k;
+  float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (g.add_noise) z = gauss4_at<Root::kSqrt>(g.key[0], g.key[1], g.p_base[l] + e);
+  float4 v;
+  v.x = g.out_scale * fmaf(g.sigmaC, z.x, s.x);
+  v.y = g.out_scale * fmaf(g.sigmaC, z.y, s.y);
+  v.z = g.out_scale * fmaf(g.sigmaC, z.z, s.z);
+  v.w = g.out_scale * fmaf(g.sigmaC, z.w, s.w);
+  float4* o = reinterpret_cast<float4*>(g.out[l] + e);
   if (g.accumulate) {
     const float4 a = *o;
     v.x += a.x;
@@ -970,10 +1107,31 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
                                     float* const* out, float* const* part, const int* d_in,
                                     const int* d_out, const uint64_t* p_base, const int* split,
                                     const float* c, int B, int T, const Epilogue& ep, int* err,
-                                    cudaStream_t s, const ConvGeom* const* conv) {
+                                    cudaStream_t s, const ConvGeom* const* conv,
+                                    const int* tail_from, const int* tail_split, float* tail,
+                                    int64_t tail_bytes) {
   if (L < 1 || L > kGemmMaxLayers) return cudaErrorInvalidValue;
   const bool pair = use_pair(d_in[0]);
   const int nb = gemm_nb(d_out[0]);
+  const int tile_m = pair ? 2 * BM : BM;
+  // the planned tails' pieces must fit the scratch: else one launch per layer
+  // (a layer's pieces always fit; the bits do not depend on the grouping)
+  if (tail_split && L > 1) {
+    int64_t pieces = 0;
+    for (int l = 0; l < L; ++l)
+      if (tail_split[l] >= 2)
+        pieces += (tc_gemm_tiles(d_in[l], d_out[l]) - tail_from[l]) * tail_split[l];
+    if (pieces * tile_m * nb * 4 > tail_bytes) {
+      for (int l = 0; l < L; ++l) {
+        cudaError_t e = tc_launch_clipsum_batch(
+            1, A + l, D + l, out + l, part ? part + l : nullptr, d_in + l, d_out + l, p_base + l,
+            split ? split + l : nullptr, c, B, T, ep, err, s, conv ? conv + l : nullptr,
+            tail_from + l, tail_split + l, tail, tail_bytes);
+        if (e != cudaSuccess) return e;
+      }
+      return cudaSuccess;
+    }
+  }
   GemmArgs g{};
   g.L = L;
   g.c = c;
@@ -992,6 +1150,10 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
     g.p_base[l] = p_base[l];
     g.split[l] = split ? split[l] : tc_gemm_split(B, T, d_in[l], d_out[l]);
     if (g.split[l] < 1 || g.split[l] > kGemmMaxSplit) return cudaErrorInvalidValue;
+    if (tail_split && tail_split[l] >= 2) {
+      g.tail_from[l] = tail_from[l];
+      g.tail_split[l] = tail_split[l];
+    }
     if (!make_input_maps(A[l], D[l], g, l, conv ? conv[l] : nullptr)) return cudaErrorInvalidValue;
     if (g.split[l] > 1) {
       if (!part || !part[l] || (reinterpret_cast<uintptr_t>(part[l]) & 15) != 0 ||
@@ -1009,8 +1171,45 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
       return cudaErrorInvalidValue;
     }
   }
-  cudaError_t e = launch_any<false>(g, s);
-  if (e != cudaSuccess || r.L == 0) return e;
+  cudaError_t e = launch_any<false>(g, s, tail, tail_bytes);
+  if (e != cudaSuccess) return e;
+  if (g.piece_start[L] > 0) {
+    TailReduceArgs t{};
+    t.tail = tail;
+    t.tile_m = tile_m;
+    t.nb = nb;
+    for (int l = 0; l < L; ++l) {
+      t.out[l] = out[l];
+      t.p_base[l] = p_base[l];
+      t.d_in[l] = d_in[l];
+      t.d_out[l] = d_out[l];
+      const int tl = g.n_m[l] * g.n_n[l];
+      const int n = tl - g.tail_from[l];
+      for (int q = 0; q < n && g.tail_split[l] >= 2; ++q) {
+        if (t.n == kTailMaxTiles) return cudaErrorInvalidValue;
+        int mt, nt;
+        tile_mn(g.tail_from[l] + q, g.n_m[l], g.n_n[l], mt, nt);
+        t.layer[t.n] = l;
+        t.row0[t.n] = mt * tile_m;
+        t.col0[t.n] = nt * nb;
+        t.first[t.n] = g.piece_start[l] + q;
+        t.stride[t.n] = n;
+        t.count[t.n] = g.tail_split[l];
+        ++t.n;
+      }
+    }
+    t.key = ep.key;
+    t.out_scale = ep.out_scale;
+    t.sigmaC = ep.sigmaC;
+    t.add_noise = ep.add_noise;
+    t.accumulate = ep.accumulate;
+    const int64_t nthreads = static_cast<int64_t>(t.n) * tile_m * nb / 4;
+    note_launch();
+    k_tail_reduce<<<static_cast<int>((nthreads + 255) / 256), 256, 0, s>>>(t);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  if (r.L == 0) return cudaSuccess;
   r.key = ep.key;
   r.out_scale = ep.out_scale;
   r.sigmaC = ep.sigmaC;
@@ -1023,9 +1222,45 @@ cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* con
 
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
                               int d_in, int d_out, int split, float* out, float* part,
-                              const Epilogue& ep, int* err, cudaStream_t s, const ConvGeom* conv) {
+                              const Epilogue& ep, int* err, cudaStream_t s, const ConvGeom* conv,
+                              int tail_from, int tail_split, float* tail, int64_t tail_bytes) {
   return tc_launch_clipsum_batch(1, &A, &D, &out, &part, &d_in, &d_out, &ep.p_base, &split, c, B,
-                                 T, ep, err, s, &conv);
+                                 T, ep, err, s, &conv, &tail_from, &tail_split, tail, tail_bytes);
+}
+
+// Tail of a launch group of clipped sums (the layers that share one batched
+// launch, in order, unsplit): with tiles > units and r = tiles mod units,
+// the last r tiles become r * S pieces, S = min(units / r, B) >= 2, so the
+// last round fills the units.  Returns, per layer, the first tail tile
+// (tiles: none) and S (1: none).
+void tc_plan_tail(int L, const int64_t* d_in, const int64_t* d_out, int B, int* tail_from,
+                  int* tail_split) {
+  int64_t tiles = 0;
+  for (int l = 0; l < L; ++l) {
+    tail_from[l] = static_cast<int>(tc_gemm_tiles(d_in[l], d_out[l]));
+    tail_split[l] = 1;
+    tiles += tail_from[l];
+  }
+  if (L < 1) return;
+  const int64_t units = use_pair(d_in[0]) ? device_sm_count() / 2 : device_sm_count();
+  const int64_t r = tiles % units;
+  if (tiles <= units || r == 0 || r > kTailMaxTiles) return;
+  int64_t S = units / r;
+  if (S > B) S = B;
+  if (S < 2) return;
+  int64_t left = r;
+  for (int l = L - 1; l >= 0 && left > 0; --l) {
+    const int64_t n = left < tail_from[l] ? left : tail_from[l];
+    tail_from[l] -= static_cast<int>(n);
+    tail_split[l] = static_cast<int>(S);
+    left -= n;
+  }
+}
+
+// Scratch for the tail pieces of one clipped-sum launch: at most one partial
+// tile per unit of the GPU (256 x 256 per CTA pair, 128 x 256 per CTA).
+int64_t tc_tail_scratch_bytes() {
+  return static_cast<int64_t>(device_sm_count()) * BM * BN * 4;
 }
 
 bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_out_a, int64_t d_in_b, int64_t d_out_b) {

@@ -47,11 +47,21 @@ bool tc_clipsum_same_launch(int64_t d_in_a, int64_t d_out_a, int64_t d_in_b, int
 // conv (per layer, NULL for a dense layer): A is then the NHWC input and the
 // kernels read its patch rows directly (tc_conv_implicit_ok must hold).
 // split: example ranges of each layer (as planned; NULL: tc_gemm_split alone).
+// tail_from / tail_split (per layer, as planned by tc_plan_tail; NULL: no
+// tail): the layer's tiles from tail_from on run as tail_split pieces of the
+// batch each, into `tail` (tail_bytes, 16-byte aligned;
+// tc_tail_scratch_bytes is always enough), added up by a reduce launch.
 cudaError_t tc_launch_clipsum_batch(int L, const void* const* A, const void* const* D,
                                     float* const* out, float* const* part, const int* d_in,
                                     const int* d_out, const uint64_t* p_base, const int* split,
                                     const float* c, int B, int T, const Epilogue& ep, int* err,
-                                    cudaStream_t s, const ConvGeom* const* conv = nullptr);
+                                    cudaStream_t s, const ConvGeom* const* conv = nullptr,
+                                    const int* tail_from = nullptr,
+                                    const int* tail_split = nullptr, float* tail = nullptr,
+                                    int64_t tail_bytes = 0);
+int64_t tc_tail_scratch_bytes();
+void tc_plan_tail(int L, const int64_t* d_in, const int64_t* d_out, int B, int* tail_from,
+                  int* tail_split);
 bool tc_conv_implicit_ok(const ConvGeom& g, int T);
 bool tc_gemm_supported(int T, int64_t d_in, int64_t d_out);
 int64_t tc_mat_parts(int64_t d_in, int64_t d_out);
@@ -61,7 +71,8 @@ cudaError_t tc_launch_mat_norm(const void* A, const void* D, int B, int T, int d
 cudaError_t tc_launch_clipsum(const void* A, const void* D, const float* c, int B, int T,
                               int d_in, int d_out, int split, float* out, float* part,
                               const Epilogue& ep, int* err, cudaStream_t s,
-                              const ConvGeom* conv = nullptr);
+                              const ConvGeom* conv = nullptr, int tail_from = 0,
+                              int tail_split = 1, float* tail = nullptr, int64_t tail_bytes = 0);
 
 // Clipped sum for short examples (T < 32): c_i folded into a bf16 hi+lo
 // split of A in scratch (tc_prescaled_scratch_bytes), then one plain GEMM.

@@ -594,6 +594,46 @@ def test_tensor_core_paths(case, mode):
     assert_step_matches(res, ref, "bf16")
 
 
+def test_tail_split_of_the_last_round():
+    """A 2304 x 2304 layer is 81 CTA-pair tiles of 256 x 256.  On a GPU of
+    76 resident pairs the last round holds 5 tiles; they run as 5 x 15
+    pieces of 1-2 examples on every pair, the clipped sums' pieces are added
+    by one more launch (the tail reduce, which also adds the noise), the
+    materialised norm's pieces write their examples' partials directly.
+    Full output, norms and factors against the oracle for both norm forms;
+    DP_ACCUMULATE adds the same bits again."""
+    units = torch.cuda.get_device_properties(0).multi_processor_count // 2
+    tiles = 81
+    r = tiles % units
+    tail = tiles > units and r > 0 and units // r >= 2
+    w = W.custom("tail81", [(2304, 2304)], 16, 128, "bf16", C=0.2, sigma=0.5, d_std=0.05,
+                 wid=771)
+    layers = W.make_inputs(w, seed=4)
+    ref = oracle_step(w, layers, seed=6, step=3, norm="ghost")
+    for mode in (dp.DP_NORM_GHOST, dp.DP_NORM_MATERIALISED):
+        res = run_gpu_step(w, layers, seed=6, step=3, norm_mode=mode)
+        assert res["paths"] == [(1, 1)]
+        assert_step_matches(res, ref, "bf16")
+    dev = torch.device(DEV)
+    A, D = [t.to(dev) for t in layers[0]]
+    cfg = dp.make_config(w.layers, w.B, w.T, "bf16", w.C, w.sigma, seed=6, step=3)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.dp_layer_norms(ctx, 0, A, D)
+        dp.dp_clip_factors(ctx)
+        out = torch.zeros(2304, 2304, device=dev)
+        n0 = dp.dp_kernel_launches()
+        dp.dp_clipped_sum_noise(ctx, 0, A, D, out, 0)
+        assert dp.dp_kernel_launches() - n0 == (2 if tail else 1)
+        twice = out.clone()
+        dp.dp_clipped_sum_noise(ctx, 0, A, D, twice, dp.DP_ACCUMULATE)
+        torch.cuda.synchronize()
+    finally:
+        dp.dp_step_destroy(ctx)
+    assert torch.equal(twice, 2 * out)
+    assert rel_err_normwise(out.cpu().numpy(), ref["out"][0]) <= TOL["bf16"]
+
+
 @pytest.mark.parametrize("case", range(len(SMALL_T_CASES)))
 def test_small_T_prescaled_clipped_sum(case):
     shapes, B, T = SMALL_T_CASES[case]
