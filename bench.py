@@ -465,6 +465,28 @@ def run_ours(args, rank, world, local_rank):
                         "launches_per_step": stage_launches["norm"]},
         "clip": {"ms_per_step": per_step_ms("clip")},
     }
+    # The Gram form on tensor cores does T^2 (d_in + d_out) work per example
+    # and layer, so at long T it is bound by the tensor pipe, not by reading
+    # its inputs: report what the tensor pipe executes (issued: 128 x 128
+    # position blocks, CTA-pair items of 2 x 2 blocks when the block count is
+    # even, whose mirrored lower block is computed and not used) and the
+    # upper triangle of blocks the sum needs.
+    modes = [dp.dp_layer_norm_mode(ctx, l) for l in range(L)]
+    if all(m == dp.DP_NORM_GHOST for m in modes) and all(
+            dp.dp_layer_path(ctx, l)[0] == 1 for l in range(L)):
+        issued = needed = 0.0
+        for i, o, T_ in w.specs:
+            nb = -(-T_ // 128)
+            unit = 2.0 * 128 * 128 * (i + o) * w.B
+            m = nb // 2
+            issued += unit * (2 * m * (m + 1) if nb % 2 == 0 else nb * (nb + 1) // 2)
+            needed += unit * nb * (nb + 1) // 2
+        tf = issued / (norm_ms * 1e-3) / 1e12
+        kernels["layer_norms"]["tensor"] = {
+            "gflop_issued": issued / 1e9, "gflop_block_triangle": needed / 1e9,
+            "tflops_issued": tf, "frac_bf16_burst": tf / peaks["bf16_tflops"],
+            "frac_bf16_sustained": (tf / peaks["bf16_tflops_sustained"]
+                                    if peaks.get("bf16_tflops_sustained") else None)}
     # thin layers (norm path 2): the norm pass reads the inputs and writes
     # the per-example gradients (4 B x B x params), the clipped sum reads
     # them back and writes the output; both are HBM-bound CUDA-core kernels
