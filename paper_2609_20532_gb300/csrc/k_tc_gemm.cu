@@ -88,6 +88,8 @@ struct GemmArgs {
   CUtensorMap mapD[kGemmMaxLayers];
   CUtensorMap mapO[kGemmMaxLayers];  // fp32 outputs, 32 x 32 boxes ([split][d_in][d_out] when split)
   CUtensorMap mapT;                   // tail pieces' partial tiles [piece][TILE_M][NB] (fp32)
+  // a strided convolution's parity maps 1-3 (map 0 is mapA; conv_taps)
+  CUtensorMap mapS[kGemmMaxLayers][3];
   float* out[kGemmMaxLayers];
   uint64_t p_base[kGemmMaxLayers];  // global parameter index of element (0, 0)
   int d_in[kGemmMaxLayers], d_out[kGemmMaxLayers];
@@ -172,10 +174,14 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity, int* 
 
 // A convolution's two A chunks of a tile: 64 channels of one kernel tap
 // each, fixed for the whole work item.  cc: first channel (C_in for a chunk
-// past K: a box wholly out of range, read as zeros); dx, dy: the tap's
-// offset from the output position, padding included.
+// past K: a box wholly out of range, read as zeros).  The input pixel of
+// output position (ho, wo) under tap offset (dy, dx) (padding included) is
+// (s ho + dy, s wo + dx) for stride s.  With dy = s qy + ry (0 <= ry < s) that
+// is pixel (ho + qy, wo + qx) of the parity map (ry, rx), the input's pixels
+// whose row and column are ry and rx modulo s: map = ry s + rx (0 for a unit
+// stride, whose one map is the input), dy, dx hold qy, qx.
 struct ConvTaps {
-  int cc[2], dx[2], dy[2];
+  int cc[2], dx[2], dy[2], map[2];
 };
 
 __device__ __forceinline__ ConvTaps conv_taps(const ConvGeom& v, int m0) {
@@ -189,9 +195,13 @@ __device__ __forceinline__ ConvTaps conv_taps(const ConvGeom& v, int m0) {
       cc = v.C_in;
     }
     const int ki = tap / v.kw;
+    const int dx = (tap - ki * v.kw) - v.pad_w, dy = ki - v.pad_h;
+    const int rx = ((dx % v.stride_w) + v.stride_w) % v.stride_w;
+    const int ry = ((dy % v.stride_h) + v.stride_h) % v.stride_h;
     t.cc[q] = cc;
-    t.dx[q] = (tap - ki * v.kw) - v.pad_w;
-    t.dy[q] = ki - v.pad_h;
+    t.dx[q] = (dx - rx) / v.stride_w;
+    t.dy[q] = (dy - ry) / v.stride_h;
+    t.map[q] = ry * v.stride_w + rx;
   }
   return t;
 }
@@ -221,8 +231,10 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
     const uint32_t fb = mapa_shared(smem_u32(full), 0);
     if (leader && tx_bytes) mbar_arrive_expect_tx(full, tx_bytes);
     if (CONV && g.conv[layer]) {
-      tma_load_4d_pair(mapA, fb, sa, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
-      tma_load_4d_pair(mapA, fb, sa + CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
+      const CUtensorMap* map0 = ct.map[0] ? &g.mapS[layer][ct.map[0] - 1] : mapA;
+      const CUtensorMap* map1 = ct.map[1] ? &g.mapS[layer][ct.map[1] - 1] : mapA;
+      tma_load_4d_pair(map0, fb, sa, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
+      tma_load_4d_pair(map1, fb, sa + CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
 #pragma unroll
       for (int q = 0; q < C::B_COLS / 64; ++q)
         tma_load_2d_pair(mapD, fb, sb + q * CHUNK, n0 + 64 * q, drow);
@@ -242,8 +254,10 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
   } else {
     if (tx_bytes) mbar_arrive_expect_tx(full, tx_bytes);
     if (CONV && g.conv[layer]) {
-      tma_load_4d(mapA, full, sa, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
-      tma_load_4d(mapA, full, sa + CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
+      const CUtensorMap* map0 = ct.map[0] ? &g.mapS[layer][ct.map[0] - 1] : mapA;
+      const CUtensorMap* map1 = ct.map[1] ? &g.mapS[layer][ct.map[1] - 1] : mapA;
+      tma_load_4d(map0, full, sa, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
+      tma_load_4d(map1, full, sa + CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
 #pragma unroll
       for (int q = 0; q < C::B_COLS / 64; ++q)
         tma_load_2d(mapD, full, sb + q * CHUNK, n0 + 64 * q, drow);
@@ -777,15 +791,27 @@ bool make_input_maps(const void* A, const void* D, GemmArgs& g, int l,
     g.conv[l] = 1;
     g.cg[l] = v;
     const uint64_t c = static_cast<uint64_t>(v.C_in);
-    const uint64_t dims[4] = {c, static_cast<uint64_t>(v.W), static_cast<uint64_t>(v.H),
-                              static_cast<uint64_t>(g.B)};
-    const uint64_t strides[3] = {c * 2, c * v.W * 2, c * v.W * v.H * 2};
     const uint32_t rows = v.W_out <= BK ? static_cast<uint32_t>(BK / v.W_out) : 1u;
     const uint32_t cols = v.W_out <= BK ? static_cast<uint32_t>(v.W_out) : static_cast<uint32_t>(BK);
     const uint32_t box[4] = {64, cols, rows, 1};
+    // one map per parity (ry, rx) of the stride s: the pixels (s i + ry,
+    // s j + rx), i.e. the input from pixel (ry, rx) on with s times its
+    // row and pixel strides (s = 1: the input itself)
+    const int s = v.stride_h;
+    for (int ry = 0; ry < s; ++ry)
+      for (int rx = 0; rx < s; ++rx) {
+        const uint64_t dims[4] = {c, static_cast<uint64_t>((v.W - rx + s - 1) / s),
+                                  static_cast<uint64_t>((v.H - ry + s - 1) / s),
+                                  static_cast<uint64_t>(g.B)};
+        const uint64_t strides[3] = {c * 2 * s, c * v.W * 2 * s, c * v.W * v.H * 2};
+        const void* base =
+            static_cast<const __nv_bfloat16*>(A) + (static_cast<uint64_t>(ry) * v.W + rx) * c;
+        const int k = ry * s + rx;
+        if (!make_tma_bf16(k == 0 ? &g.mapA[l] : &g.mapS[l][k - 1], base, 4, dims, strides, box))
+          return false;
+      }
     const uint64_t rows_all = static_cast<uint64_t>(g.B) * g.T;
-    return make_tma_bf16(&g.mapA[l], A, 4, dims, strides, box) &&
-           make_map_2d(&g.mapD[l], D, g.d_out[l], rows_all, BK);
+    return make_map_2d(&g.mapD[l], D, g.d_out[l], rows_all, BK);
   }
   if (g.pad3d)
     return make_map_3d(&g.mapA[l], A, g.d_in[l], g.T, g.B, BK) &&
@@ -1016,11 +1042,14 @@ int tc_gemm_split(int B, int T, int64_t d_in, int64_t d_out, int64_t other_tiles
 
 // Patch rows on the fly: 64-channel chunks never straddle a tap (C_in a
 // multiple of 64), K blocks are whole boxes of output positions (T a
-// multiple of 64, W_out dividing 64 or 64 dividing W_out), unit strides.
+// multiple of 64, W_out dividing 64 or 64 dividing W_out), stride 1 or 2 in
+// both directions (a stride-2 tap reads one of four parity maps).
 bool tc_conv_implicit_ok(const ConvGeom& g, int T) {
   if (g.C_in % 64 != 0 || T % BK != 0 || T != g.H_out * g.W_out) return false;
   if (!use_pair(static_cast<int64_t>(g.kh) * g.kw * g.C_in)) return false;
-  if (g.stride_h != 1 || g.stride_w != 1) return false;
+  // unit stride, or stride 2 in both directions (four parity maps)
+  if (g.stride_h != g.stride_w || g.stride_h < 1 || g.stride_h > 2) return false;
+  if (g.H < g.stride_h || g.W < g.stride_w) return false;
   if (g.W_out <= BK) return BK % g.W_out == 0;
   return g.W_out % BK == 0;
 }

@@ -92,14 +92,22 @@ CONV_NETS = [
      [(64, 10, 1), (1, 10, 1)], 8, "bf16"),
     ([(6, 6, 4, 8, 3, 3, 1, 1), (6, 6, 8, 8, 3, 3, 2, 1)], [(8, 3, 1)], 5, "f32"),
     # channels in multiples of 64: patch rows read in place by the tensor-core
-    # kernels (W_out = 16, 8 and 128), a 1x1 identity, a strided convolution
-    # (patch rows in scratch)
+    # kernels (W_out = 16, 8 and 128), a 1x1 identity, strided convolutions
+    # (four parity maps of the input)
     ([(16, 16, 64, 64, 3, 3, 1, 1),       # T = 256, W_out = 16
       (8, 8, 128, 128, 3, 3, 1, 1),       # T = 64, W_out = 8
       (4, 128, 64, 64, 3, 3, 1, 1),       # W_out = 128: boxes are half rows
       (16, 16, 64, 128, 1, 1, 1, 0),      # 1x1 stride 1: the input is the patch rows
       (16, 16, 64, 128, 3, 3, 2, 1)],     # stride 2
      [], 6, "bf16"),
+    # stride 2 read in place: odd input sizes (parity maps of unequal size),
+    # no padding, a 5x5 kernel (tap offsets -2 .. 2), a 4x4 kernel (offsets
+    # -1 .. 2: parities 1, 0, 1, 0), all with 8 x 8 outputs
+    ([(15, 15, 64, 64, 3, 3, 2, 1),
+      (17, 17, 64, 128, 3, 3, 2, 0),
+      (16, 16, 128, 64, 5, 5, 2, 2),
+      (16, 16, 64, 64, 4, 4, 2, 1)],
+     [], 5, "bf16"),
 ]
 
 
@@ -121,7 +129,9 @@ def test_conv_net_step_matches_oracle(case, conv_mode):
 
 @pytest.mark.parametrize("conv,launches", [
     ((16, 16, 64, 64, 3, 3, 1, 1), 1),    # read in place: the norm kernel alone
-    ((16, 16, 64, 128, 3, 3, 2, 1), 2),   # strided: unfold into scratch, then the norm
+    ((16, 16, 64, 128, 3, 3, 2, 1), 1),   # stride 2, read in place through parity maps
+    ((15, 15, 64, 64, 3, 3, 2, 1), 1),    # the same with odd input sizes
+    ((16, 16, 64, 128, 3, 3, 3, 1), 2),   # stride 3: unfold into scratch, then the norm
     ((16, 16, 64, 128, 1, 1, 1, 0), 1),   # 1x1 identity: the input is the patch rows
 ])
 def test_library_conv_paths_and_launches(conv, launches):
