@@ -80,6 +80,11 @@ struct LayerPlan {
   // pieces of the batch (the last round of its launch group, tc_plan_tail);
   // fixed at planning so any grouping of the calls gives the same bits
   int tail_from, tail_split;
+  // tensor-core clipped sum (direct or pre-scaled) of a short batch
+  // (B T <= kNoiseAfterMaxK): the noise is added by the noise-add kernel
+  // after the GEMM instead of inside its epilogue, where generating it would
+  // take longer than the products
+  int noise_after;
   // convolutions (kind DP_LAYER_CONV2D; A is the NHWC input)
   int kind;            // dp_layer.kind as given
   int conv;            // 1: a convolution whose patch rows differ from its input
@@ -141,6 +146,15 @@ namespace {
 // L * B * NP floats; a forced Gram form on very long examples (about T^2 /
 // 8192 partials) or a materialised norm of an enormous layer would exceed it.
 constexpr int64_t kMaxPartsPerExample = int64_t(1) << 24;
+// The tensor-core clipped sum generates its noise in the epilogue while the
+// tensor core works on the examples: about 0.2 G Gaussians per second per
+// launch, hidden behind the products when a tile runs over a few thousand
+// rows of K = B T.  With K <= 1024 the products are the shorter part, so the
+// GEMM writes the noiseless sum and the noise-add kernel (about 0.6 G
+// Gaussians per second) adds the noise after it (4096 x 4096 layer: 0.080 ->
+// 0.055 ms at B = 8, T = 1; 0.086 -> 0.073 ms at B = 8, T = 64; at K = 2048,
+// B = 32, T = 64, the noise inside the GEMM is faster, 0.125 against 0.130).
+constexpr int64_t kNoiseAfterMaxK = 1024;
 
 dp_status check_config(const dp_config* cfg) {
   if (!cfg) return fail(DP_ERR_ARG, "cfg is NULL");
@@ -318,6 +332,7 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
     p.s_off = 0;
     p.tail_from = 0;
     p.tail_split = 1;
+    p.noise_after = 0;
     p.kind = cfg->layers[l].kind;
     p.conv = p.kind == DP_LAYER_CONV2D ? 1 : 0;
     p.cg = dpk::ConvGeom{};
@@ -394,6 +409,7 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
     p.gemm_tc = 0;
     if (bf16 && dpk::tc_gemm_supported(T, p.d_in, p.d_out)) {
       p.gemm_tc = 1;
+      p.noise_after = static_cast<int64_t>(cfg->B) * T <= kNoiseAfterMaxK ? 1 : 0;
       p.split = dpk::tc_gemm_split(cfg->B, T, p.d_in, p.d_out,
                                    group_tiles[l] - dpk::tc_gemm_tiles(p.d_in, p.d_out));
       if (p.split > 1) {
@@ -410,6 +426,7 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
       }
     } else if (bf16 && dpk::tc_prescaled_supported(cfg->B, T, p.d_in, p.d_out)) {
       p.gemm_tc = 2;
+      p.noise_after = static_cast<int64_t>(cfg->B) * T <= kNoiseAfterMaxK ? 1 : 0;
       const int64_t need = dpk::tc_prescaled_scratch_bytes(cfg->B, T, p.d_in);
       if (need > c->prescaled_bytes) c->prescaled_bytes = need;
     }
@@ -704,20 +721,31 @@ dpk::Epilogue make_epilogue(const dp_ctx* c, uint32_t flags, uint64_t p_base) {
   return ep;
 }
 
+// out_l += out_scale sigma C z over every parameter of layers[0 .. n), in
+// launches of up to kNoiseMaxLayers layers (the DP_NOISE_ONLY arithmetic).
+cudaError_t launch_noise_layers(dp_ctx* c, int n, const int32_t* layers, float* const* d_out) {
+  dpk::NoiseAddBatch nb{};
+  nb.key = c->d_key;
+  nb.scale = c->out_scale * (c->sigma * c->C);
+  for (int r = 0; r < n; ++r) {
+    const LayerPlan& p = c->plan[layers[r]];
+    nb.out[nb.L] = d_out[r];
+    nb.n[nb.L] = p.d_in * p.d_out;
+    nb.p_base[nb.L] = p.p_base;
+    if (++nb.L == dpk::kNoiseMaxLayers || r == n - 1) {
+      cudaError_t e = dpk::launch_noise_add(nb, c->stream);
+      if (e != cudaSuccess) return e;
+      nb.L = 0;
+    }
+  }
+  return cudaSuccess;
+}
+
 cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const void* D,
                                float* d_out, uint32_t flags) {
   const LayerPlan& p = c->plan[layer];
   const dpk::Epilogue ep = make_epilogue(c, flags, p.p_base);
-  if (flags & DP_NOISE_ONLY) {
-    dpk::NoiseAddBatch nb{};
-    nb.key = c->d_key;
-    nb.scale = c->out_scale * ep.sigmaC;
-    nb.out[0] = d_out;
-    nb.n[0] = p.d_in * p.d_out;
-    nb.p_base[0] = p.p_base;
-    nb.L = 1;
-    return dpk::launch_noise_add(nb, c->stream);
-  }
+  if (flags & DP_NOISE_ONLY) return launch_noise_layers(c, 1, &layer, &d_out);
   if (p.pergrad) {
     dpk::PerGradSumBatch g = pergrad_sum_batch(c, flags);
     fill_pergrad_sum(c, layer, d_out, g.l[0]);
@@ -726,14 +754,26 @@ cudaError_t launch_clipped_sum(dp_ctx* c, int32_t layer, const void* A, const vo
   }
   A = dense_A(c, layer, A);
   const int din = static_cast<int>(p.d_in), dout = static_cast<int>(p.d_out);
-  if (p.gemm_tc == 1)
-    return dpk::tc_launch_clipsum(A, D, c->d_c, c->B, p.T, din, dout, p.split, d_out,
-                                  p.split > 1 ? c->d_split + p.s_off : nullptr, ep, c->d_flag,
-                                  c->stream, p.implicit ? &p.cg : nullptr, p.tail_from,
-                                  p.tail_split, c->d_tail, c->tail_bytes);
-  if (p.gemm_tc == 2)
-    return dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, p.T, din, dout, d_out, ep,
-                                            c->d_flag, c->d_prescaled, c->stream);
+  if (p.gemm_tc == 1) {
+    const bool after = p.noise_after && ep.add_noise;
+    dpk::Epilogue eg = ep;
+    if (after) eg.add_noise = 0;
+    cudaError_t e = dpk::tc_launch_clipsum(
+        A, D, c->d_c, c->B, p.T, din, dout, p.split, d_out,
+        p.split > 1 ? c->d_split + p.s_off : nullptr, eg, c->d_flag, c->stream,
+        p.implicit ? &p.cg : nullptr, p.tail_from, p.tail_split, c->d_tail, c->tail_bytes);
+    if (e != cudaSuccess || !after) return e;
+    return launch_noise_layers(c, 1, &layer, &d_out);
+  }
+  if (p.gemm_tc == 2) {
+    const bool after = p.noise_after && ep.add_noise;
+    dpk::Epilogue eg = ep;
+    if (after) eg.add_noise = 0;
+    cudaError_t e = dpk::tc_launch_clipsum_prescaled(A, D, c->d_c, c->B, p.T, din, dout, d_out,
+                                                     eg, c->d_flag, c->d_prescaled, c->stream);
+    if (e != cudaSuccess || !after) return e;
+    return launch_noise_layers(c, 1, &layer, &d_out);
+  }
   return dpk::launch_gemm_simt(c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, A, D, c->d_c,
                                c->B, p.T, din, dout, d_out, ep, c->stream);
 }
@@ -1021,20 +1061,8 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
   dpk::Epilogue ep = make_epilogue(c, flags, 0);
   // noise only: every listed layer in one launch (up to kNoiseMaxLayers each)
   if (flags & DP_NOISE_ONLY) {
-    dpk::NoiseAddBatch nb{};
-    nb.key = c->d_key;
-    nb.scale = c->out_scale * (c->sigma * c->C);
-    for (int r = 0; r < n; ++r) {
-      const LayerPlan& p = c->plan[layers[r]];
-      nb.out[nb.L] = d_out[r];
-      nb.n[nb.L] = p.d_in * p.d_out;
-      nb.p_base[nb.L] = p.p_base;
-      if (++nb.L == dpk::kNoiseMaxLayers || r == n - 1) {
-        cudaError_t e = dpk::launch_noise_add(nb, c->stream);
-        if (e != cudaSuccess) return fail(DP_ERR_CUDA, "noise kernel: %s", cudaGetErrorString(e));
-        nb.L = 0;
-      }
-    }
+    cudaError_t e = launch_noise_layers(c, n, layers, d_out);
+    if (e != cudaSuccess) return fail(DP_ERR_CUDA, "noise kernel: %s", cudaGetErrorString(e));
     return DP_OK;
   }
   // thin layers: one summing launch over their stored per-example gradients
@@ -1073,11 +1101,20 @@ dp_status dp_clipped_sum_noise_batch(dp_ctx* c, int32_t n, const int32_t* layers
       tf[q] = p.tail_from;
       ts[q] = p.tail_split;
     }
+    // the group shares B and T, hence noise_after
+    const bool after = c->plan[layers[grp[0]]].noise_after && ep.add_noise;
+    dpk::Epilogue eg = ep;
+    if (after) eg.add_noise = 0;
     cudaError_t e = dpk::tc_launch_clipsum_batch(static_cast<int>(grp.size()), a, d, o, part, din,
                                                  dout, pb, sp, c->d_c, c->B,
-                                                 c->plan[layers[grp[0]]].T, ep, c->d_flag,
+                                                 c->plan[layers[grp[0]]].T, eg, c->d_flag,
                                                  c->stream, cg, tf, ts, c->d_tail,
                                                  c->tail_bytes);
+    if (e == cudaSuccess && after) {
+      int32_t ls[dpk::kGemmMaxLayers];
+      for (size_t q = 0; q < grp.size(); ++q) ls[q] = layers[grp[q]];
+      e = launch_noise_layers(c, static_cast<int>(grp.size()), ls, o);
+    }
     grp.clear();
     return e;
   };

@@ -597,7 +597,7 @@ def test_tensor_core_paths(case, mode):
 def test_tail_split_of_the_last_round():
     """A 2304 x 2304 layer is 81 CTA-pair tiles of 256 x 256.  On a GPU of
     76 resident pairs the last round holds 5 tiles; they run as 5 x 15
-    pieces of 1-2 examples on every pair, the clipped sums' pieces are added
+    pieces of 1-2 examples on 75 pairs, the clipped sums' pieces are added
     by one more launch (the tail reduce, which also adds the noise), the
     materialised norm's pieces write their examples' partials directly.
     Full output, norms and factors against the oracle for both norm forms;
@@ -606,7 +606,8 @@ def test_tail_split_of_the_last_round():
     tiles = 81
     r = tiles % units
     tail = tiles > units and r > 0 and units // r >= 2
-    w = W.custom("tail81", [(2304, 2304)], 16, 128, "bf16", C=0.2, sigma=0.5, d_std=0.05,
+    # B T = 4096: the GEMM adds the noise itself (the tail reduce for its pieces)
+    w = W.custom("tail81", [(2304, 2304)], 16, 256, "bf16", C=0.2, sigma=0.5, d_std=0.05,
                  wid=771)
     layers = W.make_inputs(w, seed=4)
     ref = oracle_step(w, layers, seed=6, step=3, norm="ghost")
@@ -632,6 +633,39 @@ def test_tail_split_of_the_last_round():
         dp.dp_step_destroy(ctx)
     assert torch.equal(twice, 2 * out)
     assert rel_err_normwise(out.cpu().numpy(), ref["out"][0]) <= TOL["bf16"]
+
+
+@pytest.mark.parametrize("B,T", [(8, 64), (16, 64), (128, 1)])
+def test_noise_added_after_a_short_gemm(B, T):
+    """With B T <= 1024 the tensor-core clipped sum writes the noiseless sum
+    and the noise-add kernel adds the noise (one more launch): the output
+    against the oracle, and two DP_ACCUMULATE calls against twice the
+    oracle's step."""
+    w = W.custom(f"nafter{B}_{T}", [(1024, 1536)], B, T, "bf16", C=0.3, sigma=0.7, d_std=0.05,
+                 wid=780 + B + T)
+    layers = W.make_inputs(w, seed=6)
+    res = run_gpu_step(w, layers, seed=2, step=5)
+    assert res["paths"][0][1] == 1   # tensor cores (direct, or pre-scaled at T < 32)
+    ref = oracle_step(w, layers, seed=2, step=5, norm="ghost")
+    assert_step_matches(res, ref, "bf16")
+    dev = torch.device(DEV)
+    A, D = [t.to(dev) for t in layers[0]]
+    cfg = dp.make_config(w.layers, w.B, w.T, "bf16", w.C, w.sigma, seed=2, step=5)
+    ctx = dp.dp_step_init(cfg)
+    try:
+        dp.dp_layer_norms(ctx, 0, A, D)
+        dp.dp_clip_factors(ctx)
+        out = torch.zeros(1024, 1536, device=dev)
+        n0 = dp.dp_kernel_launches()
+        dp.dp_clipped_sum_noise(ctx, 0, A, D, out, dp.DP_ACCUMULATE)
+        gemm_launches = dp.dp_kernel_launches() - n0
+        dp.dp_clipped_sum_noise(ctx, 0, A, D, out, dp.DP_ACCUMULATE)
+        torch.cuda.synchronize()
+    finally:
+        dp.dp_step_destroy(ctx)
+    # the GEMM (with its pre-scale pass or split reduce), then the noise
+    assert gemm_launches in (2, 3)
+    assert rel_err_normwise(out.cpu().numpy(), 2 * ref["out"][0]) <= TOL["bf16"]
 
 
 @pytest.mark.parametrize("case", range(len(SMALL_T_CASES)))
