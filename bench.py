@@ -1193,10 +1193,14 @@ def run_table(args):
         if full:
             ref = O.dp_step([(W.to_f64(A), W.to_f64(D)) for A, D in layers], Cf, sf, seed, step,
                             out_scale=f32(1.0 / w.B))
+            # the checker's own measure (Alg. 1): z = ||g_GPU - g_64||_2 / C over
+            # every parameter, g the averaged gradient (out_scale = 1/B)
+            dz = sum(float(np.sum((o - r) ** 2)) for o, r in zip(out_gpu, ref["out"]))
             err = {"n": _errors(n_gpu, ref["n"])["elementwise"],
                    "s": _errors(s_gpu, ref["s"])["elementwise"],
                    "c": _errors(c_gpu, ref["c"])["elementwise"],
                    "out": [_errors(o, r) for o, r in zip(out_gpu, ref["out"])],
+                   "z_over_C": float(np.sqrt(dz)) / float(Cf),
                    "compared": "every output in full"}
         else:
             rng = np.random.default_rng(w.wid)
