@@ -243,13 +243,19 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
 }
 
 // ---------------------------------------------------------------------------
-// Cross-layer sum and clip factors.  A group of WARPS warps per example (one
-// warp, or a block of eight where a layer holds thousands of partials per
-// example: one per tile and epilogue warp of the materialised form).  For
-// each layer in turn, thread j of the group adds the partials j, j + G, ...
-// (G = 32 WARPS threads; coalesced), a fixed butterfly adds each warp's 32 sums, and the
-// warps' sums are added in warp order; thread 0 adds the layer sums in layer
-// order.  The order never depends on timing.
+// Cross-layer sum and clip factors, in one of three arrangements chosen by
+// the partials per example of a layer (NP); the order of the additions
+// never depends on timing.
+//   WARPS = 0 (NP < 64: few partials, maybe many layers, e.g. LoRA factors):
+//     one warp per example, lane j adds the layers j, j + 32, ... (each
+//     layer's partials in slot order), then a fixed butterfly adds the 32
+//     lane sums;
+//   WARPS = 1 or 8 (thousands of partials per layer: one per tile and
+//     epilogue warp of the materialised form): a group of WARPS warps per
+//     example; for each layer in turn, thread j of the group adds the
+//     partials j, j + G, ... (G = 32 WARPS threads; coalesced), a fixed
+//     butterfly adds each warp's 32 sums and the warps' sums are added in
+//     warp order; thread 0 adds the layer sums in layer order.
 // ---------------------------------------------------------------------------
 // mode kClipLocal: only the layers' norms and their sum (into user_s); no
 // clip factor, no flag.  mode kClipGiven: s_i = s_given[i] (the squared norm
@@ -260,8 +266,8 @@ __global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
                        float* __restrict__ s_out, float* __restrict__ c_out,
                        float* __restrict__ user_s, float* __restrict__ user_c, int* flag,
                        int mode, const float* __restrict__ s_given) {
-  constexpr int G = 32 * WARPS;  // threads per example
-  __shared__ float red[WARPS];
+  constexpr int G = WARPS > 0 ? 32 * WARPS : 32;  // threads per example
+  __shared__ float red[WARPS > 0 ? WARPS : 1];
   const int64_t gid = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   const int64_t w = gid / G;
   const int t = static_cast<int>(gid - w * G);
@@ -269,7 +275,19 @@ __global__ void k_clip(const float* __restrict__ part, int L, int B, int NP,
   if (w >= B) return;  // a whole group leaves together (WARPS > 1: one group per block)
   const int i = static_cast<int>(w);
   float s = 0.f;
-  for (int l = 0; l < L; ++l) {
+  if constexpr (WARPS == 0) {
+    for (int l = lane; l < L; l += 32) {
+      const float* p = part + (static_cast<int64_t>(l) * B + i) * NP;
+      const int np = nparts[l];
+      float n = 0.f;
+      for (int q = 0; q < np; ++q) n += p[q];
+      layer_sq[static_cast<int64_t>(l) * B + i] = n;
+      s += n;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  }
+  for (int l = 0; l < (WARPS > 0 ? L : 0); ++l) {
     const float* p = part + (static_cast<int64_t>(l) * B + i) * NP;
     const int np = nparts[l];
     float n = 0.f;
@@ -545,8 +563,11 @@ cudaError_t launch_clip(const float* part, int L, int B, int NP, const int* d_np
   if (NP >= 512)  // thousands of partials per example: a block of eight warps each
     k_clip<8><<<B, 256, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out, user_s,
                                 user_c, flag, mode, s_given);
-  else
+  else if (NP >= 64)
     k_clip<1><<<(B + 7) / 8, 256, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out,
+                                          user_s, user_c, flag, mode, s_given);
+  else  // few partials per layer: the layers in parallel over the lanes
+    k_clip<0><<<(B + 7) / 8, 256, 0, s>>>(part, L, B, NP, d_nparts, C, layer_sq, s_out, c_out,
                                           user_s, user_c, flag, mode, s_given);
   return cudaGetLastError();
 }
