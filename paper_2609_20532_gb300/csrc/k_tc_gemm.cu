@@ -21,10 +21,11 @@
 //   single CTA (PAIR = false): tile 128 x 256, 4 stages of 48 KB;
 //   CTA pair (PAIR = true, cluster of 2, tcgen05 cta_group::2): tile
 //     256 x 256; each CTA stages its 128 rows of A and its 128 columns of D
-//     (6 stages of 32 KB), the leader CTA issues the pair MMA and its
-//     commits arrive on the barriers of both CTAs; each CTA's TMEM holds its
-//     128 rows.  Half the shared-memory bytes per MMA, so the same stage
-//     memory covers 1.5x more load latency.
+//     (6 stages of 32 KB, taken two at a time when an example has an even
+//     number of K blocks, then as 128-row boxes), the leader CTA issues the
+//     pair MMA and its commits arrive on the barriers of both CTAs; each
+//     CTA's TMEM holds its 128 rows.  Half the shared-memory bytes per MMA,
+//     so the same stage memory covers 1.5x more load latency.
 //
 // Warp roles (3 warpgroups = 384 threads, one CTA per SM, persistent):
 //   warpgroup 0: warp 0 TMA producer (one lane), warp 1 TMEM allocator +
@@ -215,6 +216,20 @@ __device__ __forceinline__ ConvTaps conv_taps(const ConvGeom& v, int m0) {
 // [columns][64 channels] of the NHWC input at the tap's offset, whose
 // out-of-range pixels (the zero padding) read as zeros.  The producer thread
 // issues every stage, so nothing here divides.
+// A CTA pair's stage of two K blocks reads its rows of the 2-D maps as
+// 128-row boxes: one TMA copy per 64-column chunk and stage instead of one
+// per chunk and K block (an in-place convolution's patch rows stay one box
+// per tap and K block, placed in the same layout).  The producer's rate is set by the
+// copies it issues more than by their bytes (same bytes, the launch 4%
+// shorter on the LLM layers).  Such a stage holds each chunk's 128 rows
+// together, the A chunks and then the D chunks 16 KB apart (the MMA's
+// leading-dimension offset), and K block j of the stage starts 64 j rows in.
+// Two K blocks per stage means an even number per example (T % 128 == 0);
+// the pre-scaled operand (d_rows > 0) keeps 64-row boxes.
+__host__ __device__ __forceinline__ bool tall_boxes(int T, int d_rows) {
+  return T % (2 * BK) == 0 && d_rows == 0;
+}
+
 template <bool PAIR, int NB, bool CONV>
 __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, uint64_t* full,
                                                   bool leader, uint32_t tx_bytes, uint8_t* sa,
@@ -231,19 +246,40 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
     const uint32_t fb = mapa_shared(smem_u32(full), 0);
     if (leader && tx_bytes) mbar_arrive_expect_tx(full, tx_bytes);
     if (CONV && g.conv[layer]) {
+      // patch rows: one box per tap and K block; D rows as 128-row boxes
+      // when the stage holds two K blocks (j: this block's place in it)
+      const bool tall = tall_boxes(g.T, 0);
+      const int j = tall ? (kb & 1) : 0;
+      uint8_t* s0 = sa - j * C::STAGE_BYTES;
       const CUtensorMap* map0 = ct.map[0] ? &g.mapS[layer][ct.map[0] - 1] : mapA;
       const CUtensorMap* map1 = ct.map[1] ? &g.mapS[layer][ct.map[1] - 1] : mapA;
-      tma_load_4d_pair(map0, fb, sa, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
-      tma_load_4d_pair(map1, fb, sa + CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
+      tma_load_4d_pair(map0, fb, tall ? s0 + j * CHUNK : sa, ct.cc[0], wo0 + ct.dx[0],
+                       ho0 + ct.dy[0], ex);
+      tma_load_4d_pair(map1, fb, tall ? s0 + (2 + j) * CHUNK : sa + CHUNK, ct.cc[1],
+                       wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
+      if (!tall) {
 #pragma unroll
-      for (int q = 0; q < C::B_COLS / 64; ++q)
-        tma_load_2d_pair(mapD, fb, sb + q * CHUNK, n0 + 64 * q, drow);
+        for (int q = 0; q < C::B_COLS / 64; ++q)
+          tma_load_2d_pair(mapD, fb, sb + q * CHUNK, n0 + 64 * q, drow);
+      } else if (j == 0) {
+#pragma unroll
+        for (int q = 0; q < C::B_COLS / 64; ++q)
+          tma_load_2d_pair(mapD, fb, s0 + 2 * C::A_STAGE + q * 2 * CHUNK, n0 + 64 * q, drow);
+      }
     } else if (g.pad3d) {
       tma_load_3d_pair(mapA, fb, sa, m0, trow, ex);
       tma_load_3d_pair(mapA, fb, sa + CHUNK, m0 + 64, trow, ex);
 #pragma unroll
       for (int q = 0; q < C::B_COLS / 64; ++q)
         tma_load_3d_pair(mapD, fb, sb + q * CHUNK, n0 + 64 * q, trow, ex);
+    } else if (tall_boxes(g.T, g.d_rows)) {
+      if ((kb & 1) == 0) {  // the stage's first K block loads both
+        tma_load_2d_pair(mapA, fb, sa, m0, arow);
+        tma_load_2d_pair(mapA, fb, sa + 2 * CHUNK, m0 + 64, arow);
+#pragma unroll
+        for (int q = 0; q < C::B_COLS / 64; ++q)
+          tma_load_2d_pair(mapD, fb, sa + 2 * C::A_STAGE + q * 2 * CHUNK, n0 + 64 * q, drow);
+      }
     } else {
       tma_load_2d_pair(mapA, fb, sa, m0, arow);
       tma_load_2d_pair(mapA, fb, sa + CHUNK, m0 + 64, arow);
@@ -452,16 +488,20 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           if (!mbar_wait(&tempty_bar[buf], tph ^ 1, abrt, g.err)) goto mma_done;
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + buf * NB;
+          const bool tall = PAIR && tall_boxes(g.T, g.d_rows);
+          const uint32_t lbo = tall ? 2 * CHUNK : LBO;
           for (int kb = 0; kb < kpe; kb += bps) {
             if (!mbar_wait(&full_bar[stage], phase, abrt, g.err)) goto mma_done;
             tc_fence_after();
             for (int j = 0; j < bps; ++j) {
-              const uint32_t sa = smem_u32(smem + (stage * bps + j) * C::STAGE_BYTES);
-              const uint32_t sb = sa + C::A_STAGE;
+              const uint32_t s0 = smem_u32(smem + stage * bps * C::STAGE_BYTES);
+              const uint32_t sa =
+                  tall ? s0 + j * BK * 128 : smem_u32(smem + (stage * bps + j) * C::STAGE_BYTES);
+              const uint32_t sb = tall ? s0 + 2 * C::A_STAGE + j * BK * 128 : sa + C::A_STAGE;
 #pragma unroll
               for (int kk = 0; kk < BK / 16; ++kk) {
-                const uint64_t ad = smem_desc_sw128(sa + kk * 16 * 128, LBO, SBO);
-                const uint64_t bd = smem_desc_sw128(sb + kk * 16 * 128, LBO, SBO);
+                const uint64_t ad = smem_desc_sw128(sa + kk * 16 * 128, lbo, SBO);
+                const uint64_t bd = smem_desc_sw128(sb + kk * 16 * 128, lbo, SBO);
                 if constexpr (PAIR)
                   mma_bf16_pair(d_tmem, ad, bd, C::IDESC, ((kb + j) | kk) != 0);
                 else
@@ -811,14 +851,15 @@ bool make_input_maps(const void* A, const void* D, GemmArgs& g, int l,
           return false;
       }
     const uint64_t rows_all = static_cast<uint64_t>(g.B) * g.T;
-    return make_map_2d(&g.mapD[l], D, g.d_out[l], rows_all, BK);
+    return make_map_2d(&g.mapD[l], D, g.d_out[l], rows_all, tall_boxes(g.T, 0) ? 2 * BK : BK);
   }
   if (g.pad3d)
     return make_map_3d(&g.mapA[l], A, g.d_in[l], g.T, g.B, BK) &&
            make_map_3d(&g.mapD[l], D, g.d_out[l], g.T, g.B, BK);
   const uint64_t rows = static_cast<uint64_t>(g.B) * g.T;
-  return make_map_2d(&g.mapA[l], A, g.d_in[l], rows, BK) &&
-         make_map_2d(&g.mapD[l], D, g.d_out[l], rows, BK);
+  const uint32_t br = (use_pair(g.d_in[l]) && tall_boxes(g.T, 0)) ? 2 * BK : BK;  // tall_boxes
+  return make_map_2d(&g.mapA[l], A, g.d_in[l], rows, br) &&
+         make_map_2d(&g.mapD[l], D, g.d_out[l], rows, br);
 }
 
 template <bool NORM>
