@@ -568,6 +568,10 @@ TC_CASES = [
     ([(264, 136), (64, 8)], 4, 97),      # padded, ragged
     ([(3320, 3320)], 2, 64),             # 13 x 13 pair tiles, ragged in M and N
     ([(3320, 4096)], 2, 96),             # 13 x 16 pair tiles, 3-D maps
+    # stages of two K blocks loaded as 128-row boxes (pairs, T % 128 == 0),
+    # beside a single-CTA layer of the same step that keeps 64-row boxes
+    ([(264, 520), (120, 296)], 3, 256),
+    ([(704, 136)], 2, 384),              # six K blocks per example, ragged M and N
 ]
 
 SMALL_T_CASES = [
