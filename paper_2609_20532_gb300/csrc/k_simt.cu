@@ -136,10 +136,15 @@ __global__ void __launch_bounds__(256) k_norm_ghost_simt(const TIn* __restrict__
 }
 
 // ---------------------------------------------------------------------------
-// FFMA GEMM over positions: tile TB (d_in) x TB (d_out), K-chunks of 16,
-// 256 threads with (TB/16) x (TB/16) outputs each.
+// FFMA GEMM over positions: tile TB (d_in) x TB (d_out), K-chunks of SK rows,
+// 256 threads with 8 x 8 outputs each.
 // CLIPSUM: S = sum_k c[k / T] A[k, :]^T D[k, :] over all B*T rows, + epilogue.
 // NORM:    per example (blockIdx.z), G tile = A_i^T D_i, writes sum of squares.
+// TB = 128: one group of 256 threads walks all chunks.  TB = 64 (grids too
+// small to fill the GPU twice with 128-wide tiles): four groups of 64
+// threads each walk every fourth chunk, so a block keeps four chains of
+// loads and multiply-adds in flight, and the groups' tiles are added in
+// shared memory in a fixed order, ((g0 + g2) + (g1 + g3)).
 // ---------------------------------------------------------------------------
 constexpr int SB = 128, SK = 16;
 
@@ -150,12 +155,17 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
                                                    int d_in, int d_out, float* __restrict__ out,
                                                    Epilogue ep, float* __restrict__ part, int NP,
                                                    int row0) {
-  constexpr int MT = TB / 16;  // outputs per thread along each axis
-  constexpr int NH = MT / 4;   // 4-wide groups per thread along each axis
-  __shared__ __align__(16) float As[SK][TB];
-  __shared__ __align__(16) float Ds[SK][TB];
+  constexpr int KG = TB == 128 ? 1 : 4;  // K groups
+  constexpr int GTH = 256 / KG;          // threads per group
+  constexpr int TD = TB / 8;             // a group's threads per tile row
+  constexpr int HALF = TB / 2;
+  constexpr int LPT = (SK * TB) / GTH;   // A (and D) elements per thread and chunk
+  static_assert(TD * TD == GTH && TB % 64 == 0, "8 x 8 outputs per thread");
+  static_assert(KG == 1 || KG * SK * TB == TB * TB, "a group's tile fits one operand buffer");
+  __shared__ __align__(16) float As[KG][SK][TB];
+  __shared__ __align__(16) float Ds[KG][SK][TB];
   __shared__ float red[32];
-  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const int tid = threadIdx.x, grp = tid / GTH, gt = tid % GTH, tx = gt % TD, ty = gt / TD;
   const int j0 = blockIdx.y * TB, k0 = blockIdx.x * TB;
   int64_t K;
   if (NORM) {
@@ -166,63 +176,146 @@ __global__ void __launch_bounds__(256) k_gemm_simt(const TIn* __restrict__ A,
   } else {
     K = static_cast<int64_t>(B) * T;
   }
-  float acc[MT][MT] = {};
-  for (int64_t kk = 0; kk < K; kk += SK) {
+  const int64_t nch = (K + SK - 1) / SK;
+  float acc[8][8] = {};
+  // The group's next chunk is loaded into registers while the current one is
+  // multiplied out of shared memory; the loads only load (the clip factor is
+  // applied when the chunk is stored to shared memory), so all of a chunk's
+  // loads are in flight together.  Rows stay below B T <= 2^31 - 1, so a
+  // row's example index is a 32-bit division.
+  float ra[LPT], rc[LPT], rd[LPT];
+  auto load = [&](int64_t ch) {
+    const int64_t kk = ch * SK;
 #pragma unroll
-    for (int r = 0; r < (SK * TB) / 256; ++r) {
-      const int e = tid + 256 * r;
+    for (int r = 0; r < LPT; ++r) {
+      const int e = gt + GTH * r;
       const int row = e / TB, col = e % TB;
       const int64_t kr = kk + row;
       const int j = j0 + col, k = k0 + col;
-      float va = 0.f, vd = 0.f;
-      if (kr < K) {
-        if (j < d_in) {
-          va = to_f(A[kr * d_in + j]);
-          if (!NORM) va *= cvec[kr / T];
-        }
-        if (k < d_out) vd = to_f(D[kr * d_out + k]);
+      const bool in_k = kr < K;
+      ra[r] = in_k && j < d_in ? to_f(A[kr * d_in + j]) : 0.f;
+      rc[r] = !NORM && in_k ? cvec[static_cast<uint32_t>(kr) / static_cast<uint32_t>(T)] : 1.f;
+      rd[r] = in_k && k < d_out ? to_f(D[kr * d_out + k]) : 0.f;
+    }
+  };
+  if (grp < nch) load(grp);
+  const int64_t rounds = (nch + KG - 1) / KG;
+  for (int64_t rnd = 0; rnd < rounds; ++rnd) {
+    const int64_t ch = rnd * KG + grp;
+    const bool have = ch < nch;
+    if (have) {
+#pragma unroll
+      for (int r = 0; r < LPT; ++r) {
+        const int e = gt + GTH * r;
+        As[grp][e / TB][e % TB] = NORM ? ra[r] : ra[r] * rc[r];
+        Ds[grp][e / TB][e % TB] = rd[r];
       }
-      As[row][col] = va;
-      Ds[row][col] = vd;
     }
     __syncthreads();
+    if (ch + KG < nch) load(ch + KG);
+    if (have) {
 #pragma unroll
-    for (int q = 0; q < SK; ++q) {
-      float av[MT], bv[MT];
+      for (int q = 0; q < SK; ++q) {
+        float av[8], bv[8];
 #pragma unroll
-      for (int h = 0; h < NH; ++h) {
-        const float4 a = *reinterpret_cast<const float4*>(&As[q][h * 64 + ty * 4]);
-        const float4 b = *reinterpret_cast<const float4*>(&Ds[q][h * 64 + tx * 4]);
-        av[4 * h + 0] = a.x; av[4 * h + 1] = a.y; av[4 * h + 2] = a.z; av[4 * h + 3] = a.w;
-        bv[4 * h + 0] = b.x; bv[4 * h + 1] = b.y; bv[4 * h + 2] = b.z; bv[4 * h + 3] = b.w;
+        for (int h = 0; h < 2; ++h) {
+          const float4 a = *reinterpret_cast<const float4*>(&As[grp][q][h * HALF + ty * 4]);
+          const float4 b = *reinterpret_cast<const float4*>(&Ds[grp][q][h * HALF + tx * 4]);
+          av[4 * h + 0] = a.x; av[4 * h + 1] = a.y; av[4 * h + 2] = a.z; av[4 * h + 3] = a.w;
+          bv[4 * h + 0] = b.x; bv[4 * h + 1] = b.y; bv[4 * h + 2] = b.z; bv[4 * h + 3] = b.w;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+#pragma unroll
+          for (int v = 0; v < 8; ++v) acc[u][v] = fmaf(av[u], bv[v], acc[u][v]);
       }
-#pragma unroll
-      for (int u = 0; u < MT; ++u)
-#pragma unroll
-        for (int v = 0; v < MT; ++v) acc[u][v] = fmaf(av[u], bv[v], acc[u][v]);
     }
     __syncthreads();
   }
+  // tile row and column of this thread's output (u, v)
+  auto trow = [&](int u) { return (u / 4) * HALF + ty * 4 + (u % 4); };
+  auto tcol = [&](int v) { return (v / 4) * HALF + tx * 4 + (v % 4); };
 
-  if constexpr (NORM) {
+  if constexpr (KG > 1) {
+    // ((g0 + g2) + (g1 + g3)) through the two operand buffers, one tile each
+    auto slot = [&](int i) { return i ? &Ds[0][0][0] : &As[0][0][0]; };
+    auto put = [&](float* t) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+#pragma unroll
+        for (int v = 0; v < 8; ++v) t[trow(u) * TB + tcol(v)] = acc[u][v];
+    };
+    auto add = [&](const float* t) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+#pragma unroll
+        for (int v = 0; v < 8; ++v) acc[u][v] += t[trow(u) * TB + tcol(v)];
+    };
+    if (grp >= 2) put(slot(grp - 2));
+    __syncthreads();
+    if (grp < 2) add(slot(grp));
+    __syncthreads();
+    if (grp == 1) put(slot(0));
+    __syncthreads();
+    if (grp == 0) {
+      add(slot(0));
+      put(slot(0));
+    }
+    __syncthreads();
+    // the block's tile is in slot 0; every thread takes 4 quads of it
+    const float* tile = slot(0);
+    if constexpr (NORM) {
+      float sq = 0.f;
+#pragma unroll
+      for (int m = 0; m < (TB * TB) / 256; ++m) {
+        const float x = tile[tid + 256 * m];
+        sq = fmaf(x, x, sq);  // padding is zero
+      }
+      sq = block_sum(sq, red);
+      if (tid == 0) {
+        const int t_ = blockIdx.y * gridDim.x + blockIdx.x;
+        part[static_cast<int64_t>(row0 + blockIdx.z) * NP + t_] = sq;
+      }
+    } else {
+#pragma unroll
+      for (int m = 0; m < (TB * TB) / (4 * 256); ++m) {
+        const int qd = tid + 256 * m;
+        const int r = qd / (TB / 4), c4 = (qd % (TB / 4)) * 4;
+        const int j = j0 + r, kb = k0 + c4;
+        if (j >= d_in || kb >= d_out) continue;
+        float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (ep.add_noise) z = gauss4_at(ep.key[0], ep.key[1], ep.p_base + static_cast<uint64_t>(j) * d_out + kb);
+        const float zv[4] = {z.x, z.y, z.z, z.w};
+        float* o = out + static_cast<int64_t>(j) * d_out;
+#pragma unroll
+        for (int v = 0; v < 4; ++v) {
+          const int k = kb + v;
+          if (k < d_out) {
+            const float val = ep.out_scale * fmaf(ep.sigmaC, zv[v], tile[r * TB + c4 + v]);
+            o[k] = ep.accumulate ? o[k] + val : val;
+          }
+        }
+      }
+    }
+  } else if constexpr (NORM) {
     float sq = 0.f;
 #pragma unroll
-    for (int u = 0; u < MT; ++u)
+    for (int u = 0; u < 8; ++u)
 #pragma unroll
-      for (int v = 0; v < MT; ++v) sq = fmaf(acc[u][v], acc[u][v], sq);  // padding is zero
+      for (int v = 0; v < 8; ++v) sq = fmaf(acc[u][v], acc[u][v], sq);  // padding is zero
     sq = block_sum(sq, red);
     if (tid == 0) {
-      const int tile = blockIdx.y * gridDim.x + blockIdx.x;
-      part[static_cast<int64_t>(row0 + blockIdx.z) * NP + tile] = sq;
+      const int t_ = blockIdx.y * gridDim.x + blockIdx.x;
+      part[static_cast<int64_t>(row0 + blockIdx.z) * NP + t_] = sq;
     }
   } else {
 #pragma unroll
-    for (int u = 0; u < MT; ++u) {
-      const int j = j0 + (u / 4) * 64 + ty * 4 + (u % 4);
+    for (int u = 0; u < 8; ++u) {
+      const int j = j0 + trow(u);
       if (j >= d_in) continue;
 #pragma unroll
-      for (int h = 0; h < NH; ++h) {
-        const int kb = k0 + h * 64 + tx * 4;
+      for (int h = 0; h < 2; ++h) {
+        const int kb = k0 + h * HALF + tx * 4;
         if (kb >= d_out) continue;
         float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
         const uint64_t p0 = ep.p_base + static_cast<uint64_t>(j) * d_out + kb;

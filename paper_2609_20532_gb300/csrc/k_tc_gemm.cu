@@ -892,20 +892,24 @@ void set_epilogue(GemmArgs& g, const Epilogue& ep) {
 // hi = RN_bf16(c_i a) and rows [R, 2R) hold lo = RN_bf16(c_i a - hi) for the
 // B*T input rows (zeros in the padding rows), so hi + lo carries c_i a to
 // about 2^-16 relative and S = A2^T [D; D] needs no per-example fold.
+// IDX: the type of the vector index (32-bit when the 2 R d_in / 8 vectors
+// fit, so that the row and column come from a 32-bit division).
+template <typename IDX>
 __global__ void k_prescale_hilo(const __nv_bfloat16* __restrict__ A, const float* __restrict__ c,
                                 int T, int64_t BT, int64_t R, int d_in,
                                 __nv_bfloat16* __restrict__ A2) {
-  const int vpr = d_in / 8;  // 16-byte vectors per row
-  const int64_t nvec = 2 * R * vpr;
-  for (int64_t v = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; v < nvec;
-       v += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t row = v / vpr;
+  const IDX vpr = static_cast<IDX>(d_in / 8);  // 16-byte vectors per row
+  const IDX nvec = static_cast<IDX>(2 * R) * vpr;
+  for (IDX v = static_cast<IDX>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec;
+       v += static_cast<IDX>(gridDim.x) * blockDim.x) {
+    const int64_t row = static_cast<int64_t>(v / vpr);
     const int col = static_cast<int>(v % vpr) * 8;
     const bool lo = row >= R;
     const int64_t k = lo ? row - R : row;
     uint4 outv = make_uint4(0u, 0u, 0u, 0u);
     if (k < BT) {
-      const float ci = c[k / T];
+      // k < B T <= 2^31 - 1
+      const float ci = c[static_cast<uint32_t>(k) / static_cast<uint32_t>(T)];
       const uint4 in = *reinterpret_cast<const uint4*>(A + k * d_in + col);
       const __nv_bfloat16* x = reinterpret_cast<const __nv_bfloat16*>(&in);
       __nv_bfloat16 y[8];
@@ -1124,8 +1128,13 @@ cudaError_t tc_launch_clipsum_prescaled(const void* A, const void* D, const floa
   const int64_t cap = static_cast<int64_t>(device_sm_count()) * 8;
   note_launch();
   if (blocks > cap) blocks = cap;
-  k_prescale_hilo<<<static_cast<int>(blocks), 256, 0, s>>>(
-      static_cast<const __nv_bfloat16*>(A), c, T, BT, R, d_in, A2);
+  // 32-bit indices while v + the grid's stride stays below 2^32
+  if (nvec + blocks * 256 < (int64_t(1) << 32))
+    k_prescale_hilo<uint32_t><<<static_cast<int>(blocks), 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(A), c, T, BT, R, d_in, A2);
+  else
+    k_prescale_hilo<uint64_t><<<static_cast<int>(blocks), 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(A), c, T, BT, R, d_in, A2);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   GemmArgs g{};
