@@ -34,6 +34,17 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+L2_BYTES = 129 * 10**6          # GB300 L2
+L2_FLUSH_BYTES = 256 << 20      # the write that flushes it
+
+
+def _l2_flush_buffer(dev, in_bytes):
+    """A buffer whose write flushes L2 between timed replays when the inputs
+    (in_bytes) could stay resident in it, else None."""
+    import torch
+    return (torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+            if in_bytes < 2 * L2_BYTES else None)
+
 METRIC = "examples/sec per DP-SGD step (1 GB300) + % BF16 tensor peak / % HBM GB/s"
 UNIT = "examples/s"
 
@@ -370,14 +381,20 @@ def run_ours(args, rank, world, local_rank):
             graph.replay()
             dp.dp_audit_emit(ctx, idx, L)
         torch.cuda.synchronize()
+    # Inputs that L2 could keep between steps: a write larger than L2 before
+    # every timed step, outside that step's events.
+    flush = _l2_flush_buffer(dev, in_bytes)
     barrier()
     torch.cuda.synchronize()
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     marks = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     host_launches0 = dp.dp_kernel_launches()
     with ClockSampler(local_rank) as clk:
         start.record(stream)
         for t in range(args.steps):
+            if flush is not None:
+                flush.fill_(t & 0xFF)
             marks[t].record(stream)
             if graph is not None:
                 dp.dp_set_noise_key(ctx, cfg.seed, args.warmup + t)
@@ -385,6 +402,7 @@ def run_ours(args, rank, world, local_rank):
                 dp.dp_audit_emit(ctx, idx, L)
             else:
                 step(args.warmup + t, timed=True)
+            ends[t].record(stream)
         marks[args.steps].record(stream)
         stop.record(stream)
         torch.cuda.synchronize()
@@ -396,22 +414,36 @@ def run_ours(args, rank, world, local_rank):
                                            for k in ("init", "norm", "clip", "gemm"))
     barrier()
     torch.cuda.synchronize()
-    ms = max_over_ranks(start.elapsed_time(stop), world, dev)
+    per_step = [marks[t].elapsed_time(ends[t]) for t in range(args.steps)]
+    # flushed: the sum of the steps' own times; else the whole loop
+    ms = max_over_ranks(sum(per_step) if flush is not None else start.elapsed_time(stop),
+                        world, dev)
     ms_step = ms / args.steps
     value = replica_throughput(w.B, world, ms_step * 1e-3)
-    ms_median = statistics.median(marks[t].elapsed_time(marks[t + 1]) for t in range(args.steps))
+    ms_median = statistics.median(per_step)
 
-    # the step without the audit emit: replays back to back under one key
-    # (the emit's synchronisation is what lets each replay take a new key)
+    # the step without the audit emit: replays under one key (the emit's
+    # synchronisation is what lets each replay take a new key), back to back
+    # or, with the flush, each between its own events
     ms_no_audit = None
     if graph is not None:
-        e_a, e_b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e_a.record(stream)
+        ea = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+        ea[0].record(stream)
+        tot = 0.0
         for t in range(args.steps):
-            graph.replay()
-        e_b.record(stream)
+            if flush is not None:
+                e_f = torch.cuda.Event(enable_timing=True)
+                flush.fill_(t & 0xFF)
+                e_f.record(stream)
+                graph.replay()
+                ea[t + 1].record(stream)
+                torch.cuda.synchronize()
+                tot += e_f.elapsed_time(ea[t + 1])
+            else:
+                graph.replay()
+                ea[t + 1].record(stream)
         torch.cuda.synchronize()
-        ms_no_audit = e_a.elapsed_time(e_b) / args.steps
+        ms_no_audit = (tot if flush is not None else ea[0].elapsed_time(ea[-1])) / args.steps
 
     if graph is not None:
         # per-kernel split: the step's stages captured as separate graphs and
@@ -706,7 +738,12 @@ def run_ours(args, rank, world, local_rank):
         "config": {"workload": w.describe(), "layers": [list(x) for x in w.layers], "B": w.B,
                    "T": w.T, "C": w.C, "sigma": w.sigma, "out_scale": "1/B",
                    "audit_examples": len(idx),
-                   "l2": f"inputs {in_bytes / 1e6:.0f} MB > 129 MB L2 (no flush needed)",
+                   "l2": (f"inputs {in_bytes / 1e6:.0f} MB < 2 x the {L2_BYTES / 1e6:.0f} MB L2: "
+                          f"a {L2_FLUSH_BYTES >> 20} MB write before every timed step, outside "
+                          "its events (the per-kernel split replays back to back, inputs "
+                          "L2-resident)" if flush is not None else
+                          f"inputs {in_bytes / 1e6:.0f} MB > 2 x the {L2_BYTES / 1e6:.0f} MB L2 "
+                          "(no flush needed)"),
                    "parallelism": "replicas (no collective)" if world > 1 else "single",
                    "execution": execution},
         "roofline": roofline,
@@ -835,7 +872,11 @@ def run_data_parallel(args, rank, world, local_rank):
                    "collectives": f"{args.dist_backend}: reduce-scatter + all-gather of the "
                                   f"flat commitment ({4 * fo.flat.numel()} bytes), "
                                   "noise of each rank's slice in between",
-                   "l2": f"inputs {in_bytes / 1e6:.0f} MB per rank > 129 MB L2",
+                   "l2": (f"inputs {in_bytes / 1e6:.0f} MB per rank > 2 x the "
+                          f"{L2_BYTES / 1e6:.0f} MB L2 (no flush needed)"
+                          if in_bytes >= 2 * L2_BYTES else
+                          f"inputs {in_bytes / 1e6:.0f} MB per rank < 2 x the "
+                          f"{L2_BYTES / 1e6:.0f} MB L2, not flushed"),
                    "execution": "eager launches"},
         "collective_ms_per_step": coll_ms,
         "collective_bytes_per_rank": 2 * 4 * fo.flat.numel(),
@@ -880,13 +921,17 @@ def run_sweep(args):
             torch.cuda.synchronize()
             return gr
 
+        flush = _l2_flush_buffer(dev, A.numel() * 2 + D.numel() * 2)
+
         def timed(gr, reps):
             for _ in range(max(3, args.warmup)):
                 gr.replay()
             torch.cuda.synchronize()
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             ts = []
-            for _ in range(reps):
+            for r in range(reps):
+                if flush is not None:
+                    flush.fill_(r & 0xFF)
                 e0.record(stream)
                 gr.replay()
                 e1.record(stream)
@@ -1119,6 +1164,10 @@ def run_table(args):
             torch.cuda.synchronize()
             return gr
 
+        in_bytes = sum(a.numel() * a.element_size() + d.numel() * d.element_size()
+                       for a, d in zip(A_d, D_d))
+        flush = _l2_flush_buffer(dev, in_bytes)
+
         def timed(gr, reps):
             # at least W replays and 0.1 s, so the SM clock is back up after an idle
             t_end = time.perf_counter() + 0.1
@@ -1131,7 +1180,9 @@ def run_table(args):
             torch.cuda.synchronize()
             ts = []
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            for _ in range(reps):
+            for r in range(reps):
+                if flush is not None:
+                    flush.fill_(r & 0xFF)
                 e0.record(stream)
                 gr.replay()
                 e1.record(stream)
