@@ -229,6 +229,12 @@ __device__ __forceinline__ ConvTaps conv_taps(const ConvGeom& v, int m0) {
 __host__ __device__ __forceinline__ bool tall_boxes(int T, int d_rows) {
   return T % (2 * BK) == 0 && d_rows == 0;
 }
+// An in-place convolution whose K block is whole output rows (W_out divides
+// 64) reads a stage of two K blocks as one patch box of 128 positions per
+// tap: 128 / W_out output rows.
+__host__ __device__ __forceinline__ bool conv_tall_box(const ConvGeom& v, int T) {
+  return tall_boxes(T, 0) && v.W_out <= BK;
+}
 
 template <bool PAIR, int NB, bool CONV>
 __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, uint64_t* full,
@@ -246,17 +252,24 @@ __device__ __forceinline__ void issue_stage_loads(const GemmArgs& g, int layer, 
     const uint32_t fb = mapa_shared(smem_u32(full), 0);
     if (leader && tx_bytes) mbar_arrive_expect_tx(full, tx_bytes);
     if (CONV && g.conv[layer]) {
-      // patch rows: one box per tap and K block; D rows as 128-row boxes
-      // when the stage holds two K blocks (j: this block's place in it)
+      // patch rows: one box per tap and K block, or, when the stage holds two
+      // K blocks of whole output rows, one box of both (conv_tall_box); D
+      // rows as 128-row boxes when the stage holds two K blocks (j: this
+      // block's place in it)
       const bool tall = tall_boxes(g.T, 0);
       const int j = tall ? (kb & 1) : 0;
       uint8_t* s0 = sa - j * C::STAGE_BYTES;
       const CUtensorMap* map0 = ct.map[0] ? &g.mapS[layer][ct.map[0] - 1] : mapA;
       const CUtensorMap* map1 = ct.map[1] ? &g.mapS[layer][ct.map[1] - 1] : mapA;
-      tma_load_4d_pair(map0, fb, tall ? s0 + j * CHUNK : sa, ct.cc[0], wo0 + ct.dx[0],
-                       ho0 + ct.dy[0], ex);
-      tma_load_4d_pair(map1, fb, tall ? s0 + (2 + j) * CHUNK : sa + CHUNK, ct.cc[1],
-                       wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
+      if (!conv_tall_box(g.cg[layer], g.T)) {
+        tma_load_4d_pair(map0, fb, tall ? s0 + j * CHUNK : sa, ct.cc[0], wo0 + ct.dx[0],
+                         ho0 + ct.dy[0], ex);
+        tma_load_4d_pair(map1, fb, tall ? s0 + (2 + j) * CHUNK : sa + CHUNK, ct.cc[1],
+                         wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
+      } else if (j == 0) {
+        tma_load_4d_pair(map0, fb, s0, ct.cc[0], wo0 + ct.dx[0], ho0 + ct.dy[0], ex);
+        tma_load_4d_pair(map1, fb, s0 + 2 * CHUNK, ct.cc[1], wo0 + ct.dx[1], ho0 + ct.dy[1], ex);
+      }
       if (!tall) {
 #pragma unroll
         for (int q = 0; q < C::B_COLS / 64; ++q)
@@ -831,7 +844,9 @@ bool make_input_maps(const void* A, const void* D, GemmArgs& g, int l,
     g.conv[l] = 1;
     g.cg[l] = v;
     const uint64_t c = static_cast<uint64_t>(v.C_in);
-    const uint32_t rows = v.W_out <= BK ? static_cast<uint32_t>(BK / v.W_out) : 1u;
+    const uint32_t rows = v.W_out <= BK ? static_cast<uint32_t>(
+                                              (conv_tall_box(v, g.T) ? 2 * BK : BK) / v.W_out)
+                                        : 1u;
     const uint32_t cols = v.W_out <= BK ? static_cast<uint32_t>(v.W_out) : static_cast<uint32_t>(BK);
     const uint32_t box[4] = {64, cols, rows, 1};
     // one map per parity (ry, rx) of the stride s: the pixels (s i + ry,
