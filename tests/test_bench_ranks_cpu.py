@@ -1,8 +1,8 @@
-"""Multi-rank bookkeeping of bench.py on CPU (gloo, world size 2).
+"""Host logic of bench.py on CPU.
 
-The step has no data-path collective: every rank runs its own replica, the
-job's time is the slowest rank's and its throughput counts every rank's
-examples.  This checks that host logic with two gloo processes."""
+Multi-rank bookkeeping (gloo, world size 2): the job's time is the slowest
+rank's and its throughput counts every rank's examples.  Timing rules: the
+L2 flush between timed steps for inputs that L2 could keep."""
 
 import os
 import socket
@@ -102,3 +102,18 @@ def test_reference_arm_line_on_cpu():
     assert "example 0 of single_fp32" in cb["sample"]
     assert line["e2e"] == {"value": line["value"], "unit": line["unit"],
                            "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_l2_flush_applies_only_to_inputs_that_l2_could_keep(monkeypatch):
+    """Timed steps flush L2 (a write larger than it) when the inputs are
+    below twice its size; the LLM-scale inputs (763 MB) need no flush."""
+    import torch
+    sys.path.insert(0, ROOT)
+    import bench
+    assert bench.L2_FLUSH_BYTES > bench.L2_BYTES
+    monkeypatch.setattr(bench, "L2_FLUSH_BYTES", 4096)   # keep the test's buffer small
+    small = bench._l2_flush_buffer(torch.device("cpu"), 3 * 10**6)
+    assert small is not None and small.numel() == 4096 and small.dtype == torch.uint8
+    assert bench._l2_flush_buffer(torch.device("cpu"), 2 * bench.L2_BYTES - 1) is not None
+    assert bench._l2_flush_buffer(torch.device("cpu"), 2 * bench.L2_BYTES) is None
+    assert bench._l2_flush_buffer(torch.device("cpu"), 763 * 10**6) is None
