@@ -209,6 +209,11 @@ EDGE = [
     ([(1, 1)], 1, 1, "f32"),
     ([(5, 7)], 4, 65, "f32"),
     ([(256, 128)], 2, 256, "bf16"),
+    # FFMA clipped sum: 64-wide tiles walked by four K groups over 21 chunks
+    # (the last one partial), ragged in both directions; and the 128-wide
+    # tiles of a grid large enough for them (20 x 16 tiles)
+    ([(200, 136)], 9, 37, "f32"),
+    ([(2560, 2048)], 2, 3, "f32"),
 ]
 
 
