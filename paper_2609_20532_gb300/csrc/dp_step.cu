@@ -92,6 +92,10 @@ struct LayerPlan {
   int implicit;        // 1: the tensor-core kernels read its patch rows from A directly
   int unfold;          // 1: its patch rows are formed in d_unf when its norms are computed
   int64_t u_off;       // byte offset of those patch rows in d_unf
+  // a thin convolution whose input per example fits in shared memory: its
+  // per-example gradients come straight from the NHWC input
+  // (launch_conv_thin_norm), no patch rows, one norm partial per example
+  int fused;
 };
 
 struct dp_ctx {
@@ -327,6 +331,7 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
     p.p_base = off;
     off += static_cast<uint64_t>(p.d_in) * p.d_out;
     p.pergrad = use_pergrad(cfg, T, p.d_in, p.d_out) ? 1 : 0;
+    p.fused = 0;
     p.g_off = 0;
     p.split = 1;
     p.s_off = 0;
@@ -361,8 +366,13 @@ dp_status build_plan(dp_ctx* c, const dp_config* cfg) {
           cfg->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32, p.d_in, p.d_out, T));
       p.g_off = grads;
       grads += static_cast<int64_t>(cfg->B) * p.d_in * p.d_out;
+      if (p.conv && dpk::conv_thin_norm_ok(p.cg, p.d_out)) {
+        p.fused = 1;
+        p.nparts = 1;
+      } else if (p.conv) {
+        need_unfold();
+      }
       if (p.nparts > NP) NP = p.nparts;
-      if (p.conv) need_unfold();
       continue;
     }
     p.mode = resolve_mode(cfg->norm_mode, T, p.d_in, p.d_out);
@@ -668,6 +678,10 @@ dpk::PerGradSumBatch pergrad_sum_batch(const dp_ctx* c, uint32_t flags) {
 cudaError_t launch_layer_norms(dp_ctx* c, int32_t layer, const void* A, const void* D) {
   const LayerPlan& p = c->plan[layer];
   const dpk::InType it = c->dtype == DP_BF16 ? dpk::IN_BF16 : dpk::IN_F32;
+  if (p.fused)
+    return dpk::launch_conv_thin_norm(it, A, D, p.cg, static_cast<int>(p.d_out), c->B,
+                                      c->d_grads + p.g_off, c->d_part, c->NP, layer * c->B,
+                                      c->stream);
   if (p.pergrad) {
     dpk::PerGradBatch g{};
     fill_pergrad(c, layer, A, D, g.l[0]);
@@ -947,7 +961,9 @@ dp_status dp_layer_norms_batch(dp_ctx* c, int32_t n, const int32_t* layers, cons
   for (int r = 0; r < n; ++r) {
     const LayerPlan& p = c->plan[layers[r]];
     cudaError_t e = cudaSuccess;
-    if (p.pergrad) {
+    if (p.fused) {
+      e = launch_layer_norms(c, layers[r], Ad[r], D[r]);
+    } else if (p.pergrad) {
       const int nar = static_cast<int>(p.d_in < p.d_out ? p.d_in : p.d_out);
       std::vector<int>& v = thin[std::make_pair(dpk::pergrad_bucket(nar), p.T)];
       v.push_back(r);

@@ -159,7 +159,160 @@ cudaError_t launch_unfold_t(const void* x, void* a, const ConvGeom& g, int B, in
   return cudaGetLastError();
 }
 
+// ---------------------------------------------------------------------------
+// Thin convolution, per-example gradient from the input in shared memory:
+//   G_i[j][k] = sum_t a_i[t][j] d_i[t][k]
+// with a the patch rows above, for a layer whose per-example gradient the
+// step stores (few output channels) and whose input per example fits in
+// shared memory.  One block per example holds x_i [H][W][C_in] (fp32) and
+// walks the output positions in chunks of kThinChunk, the chunk's output
+// gradients [chunk][C_out] staged in shared memory.  Thread (j, q) owns
+// gradient row j (tap (ki, kj), channel c) for the positions q, q + Q, ... of
+// every chunk and all C_out columns; the Q partial rows are then added in q
+// order, the row is written to G_i, and the squares of the example's rows are
+// summed in a fixed order into its single norm partial.  No patch row is
+// formed in memory; the result differs from the unfolded path's only in the
+// order of the fp32 additions.
+// ---------------------------------------------------------------------------
+constexpr int kThinThreads = 256;
+constexpr int kThinChunk = 256;  // positions per staged chunk of d_i
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+// Sum over the block's threads: warp butterflies, then the warps' sums in
+// warp order (a fixed order).
+__device__ __forceinline__ float block_sum(float v, float* red) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) red[w] = v;
+  __syncthreads();
+  float t = lane < static_cast<int>(blockDim.x >> 5) ? red[lane] : 0.f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+  return t;
+}
+
+template <typename TIn, int CO>
+__global__ void __launch_bounds__(kThinThreads)
+    k_conv_thin_norm(const TIn* __restrict__ x, const TIn* __restrict__ d, ConvGeom g,
+                     int c_out, float* __restrict__ G, float* __restrict__ part, int NP,
+                     int row0) {
+  extern __shared__ __align__(16) float sm[];
+  __shared__ float red[32];
+  const int HWC = g.H * g.W * g.C_in;
+  float* img = sm;                         // [H][W][C_in]
+  float* buf = sm + ((HWC + 3) & ~3);      // chunk [kThinChunk][C_out], then [Q][K][C_out]
+  const int i = blockIdx.x;
+  const int K = g.kh * g.kw * g.C_in;      // <= kThinThreads (host check)
+  const int T = g.H_out * g.W_out;
+  const int Q = kThinThreads / K;
+  const int tid = threadIdx.x;
+  const TIn* xi = x + static_cast<int64_t>(i) * HWC;
+  const TIn* di = d + static_cast<int64_t>(i) * T * c_out;
+  for (int e = tid; e < HWC; e += kThinThreads) img[e] = to_f(xi[e]);
+  const int j = tid / Q, q = tid - j * Q;
+  const bool own = j < K;
+  int ki = 0, kj = 0, ch = 0;
+  if (own) {
+    const int tap = j / g.C_in;
+    ch = j - tap * g.C_in;
+    ki = tap / g.kw;
+    kj = tap - ki * g.kw;
+  }
+  float acc[CO];
+#pragma unroll
+  for (int k = 0; k < CO; ++k) acc[k] = 0.f;
+  for (int t0 = 0; t0 < T; t0 += kThinChunk) {
+    const int nt = T - t0 < kThinChunk ? T - t0 : kThinChunk;
+    __syncthreads();  // the image is in place; the previous chunk is used up
+    for (int e = tid; e < nt * c_out; e += kThinThreads)
+      buf[e] = to_f(di[static_cast<int64_t>(t0) * c_out + e]);
+    __syncthreads();
+    if (own) {
+      for (int tt = q; tt < nt; tt += Q) {
+        const int t = t0 + tt;
+        const int ho = t / g.W_out, wo = t - ho * g.W_out;
+        const int y = ho * g.stride_h + ki - g.pad_h, xx = wo * g.stride_w + kj - g.pad_w;
+        if (y < 0 || y >= g.H || xx < 0 || xx >= g.W) continue;  // zero padding
+        const float v = img[(y * g.W + xx) * g.C_in + ch];
+        const float* dr = buf + tt * c_out;
+#pragma unroll
+        for (int k = 0; k < CO; ++k)
+          if (k < c_out) acc[k] = fmaf(v, dr[k], acc[k]);
+      }
+    }
+  }
+  __syncthreads();
+  if (own) {
+#pragma unroll
+    for (int k = 0; k < CO; ++k)
+      if (k < c_out) buf[(q * K + j) * c_out + k] = acc[k];
+  }
+  __syncthreads();
+  float sq = 0.f;
+  if (tid < K) {
+    float* gi = G + (static_cast<int64_t>(i) * K + tid) * c_out;
+    for (int k = 0; k < c_out; ++k) {
+      float s = 0.f;
+      for (int r = 0; r < Q; ++r) s += buf[(r * K + tid) * c_out + k];
+      gi[k] = s;
+      sq = fmaf(s, s, sq);
+    }
+  }
+  sq = block_sum(sq, red);
+  if (tid == 0) part[static_cast<int64_t>(row0 + i) * NP] = sq;
+}
+
+int thin_smem_bytes(const ConvGeom& g, int c_out) {
+  const int64_t hwc = static_cast<int64_t>(g.H) * g.W * g.C_in;
+  return static_cast<int>((((hwc + 3) & ~int64_t(3)) + int64_t(kThinChunk) * c_out) * 4);
+}
+
+template <typename TIn, int CO>
+cudaError_t launch_thin_t(const void* x, const void* d, const ConvGeom& g, int c_out, int B,
+                          float* G, float* part, int NP, int row0, cudaStream_t s) {
+  const int smem = thin_smem_bytes(g, c_out);
+  if (smem > 48 * 1024) {
+    cudaError_t e = setup_once_per_device(
+        reinterpret_cast<const void*>(&k_conv_thin_norm<TIn, CO>), [] {
+          return cudaFuncSetAttribute(k_conv_thin_norm<TIn, CO>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      kConvThinMaxSmem);
+        });
+    if (e != cudaSuccess) return e;
+  }
+  note_launch();
+  k_conv_thin_norm<TIn, CO><<<B, kThinThreads, smem, s>>>(
+      static_cast<const TIn*>(x), static_cast<const TIn*>(d), g, c_out, G, part, NP, row0);
+  return cudaGetLastError();
+}
+
+template <typename TIn>
+cudaError_t launch_thin_co(const void* x, const void* d, const ConvGeom& g, int c_out, int B,
+                           float* G, float* part, int NP, int row0, cudaStream_t s) {
+  if (c_out <= 16) return launch_thin_t<TIn, 16>(x, d, g, c_out, B, G, part, NP, row0, s);
+  if (c_out <= 32) return launch_thin_t<TIn, 32>(x, d, g, c_out, B, G, part, NP, row0, s);
+  return launch_thin_t<TIn, 64>(x, d, g, c_out, B, G, part, NP, row0, s);
+}
+
 }  // namespace
+
+bool conv_thin_norm_ok(const ConvGeom& g, int64_t c_out) {
+  const int64_t K = static_cast<int64_t>(g.kh) * g.kw * g.C_in;
+  return K >= 1 && K <= kThinThreads && c_out >= 1 && c_out <= 64 &&
+         thin_smem_bytes(g, static_cast<int>(c_out)) <= kConvThinMaxSmem;
+}
+
+cudaError_t launch_conv_thin_norm(InType t, const void* x, const void* d, const ConvGeom& g,
+                                  int c_out, int B, float* G, float* part, int NP, int row0,
+                                  cudaStream_t s) {
+  if (B < 1) return cudaSuccess;
+  if (!conv_thin_norm_ok(g, c_out)) return cudaErrorInvalidValue;
+  if (t == IN_F32) return launch_thin_co<float>(x, d, g, c_out, B, G, part, NP, row0, s);
+  return launch_thin_co<__nv_bfloat16>(x, d, g, c_out, B, G, part, NP, row0, s);
+}
 
 cudaError_t launch_conv_unfold(InType t, const void* x, void* a, const ConvGeom& g, int B,
                                cudaStream_t s) {

@@ -133,6 +133,9 @@ def test_conv_net_step_matches_oracle(case, conv_mode):
     ((15, 15, 64, 64, 3, 3, 2, 1), 1),    # the same with odd input sizes
     ((16, 16, 64, 128, 3, 3, 3, 1), 2),   # stride 3: unfold into scratch, then the norm
     ((16, 16, 64, 128, 1, 1, 1, 0), 1),   # 1x1 identity: the input is the patch rows
+    ((16, 16, 3, 16, 3, 3, 1, 1), 1),     # thin, 3 channels: gradients straight from the input
+    ((20, 21, 5, 12, 3, 2, 1, 1), 1),     # thin, 3x2 kernel, odd sizes
+    ((16, 16, 3, 16, 3, 3, 2, 1), 1),     # thin, stride 2
 ])
 def test_library_conv_paths_and_launches(conv, launches):
     """A DP_LAYER_CONV2D layer: how many kernels its norm call issues shows
