@@ -12,6 +12,7 @@
 #include <vector>
 
 #include "../../include/dp_step.h"
+#include "conv_thin.h"
 #include "internal.h"
 #include "tc.h"
 

@@ -145,14 +145,6 @@ struct ConvGeom {
 };
 cudaError_t launch_conv_unfold(InType t, const void* x, void* a, const ConvGeom& g, int B,
                                cudaStream_t s);
-// A thin convolution (per-example gradient stored) whose input per example
-// fits in shared memory: G_i = a_i^T d_i straight from the NHWC input, one
-// norm partial per example (partial slot 0 of row row0 + i).
-constexpr int kConvThinMaxSmem = 200 * 1024;
-bool conv_thin_norm_ok(const ConvGeom& g, int64_t c_out);
-cudaError_t launch_conv_thin_norm(InType t, const void* x, const void* d, const ConvGeom& g,
-                                  int c_out, int B, float* G, float* part, int NP, int row0,
-                                  cudaStream_t s);
 
 // ---- per-device kernel set-up ----
 // Kernel attributes (the dynamic shared-memory limit) and occupancy figures

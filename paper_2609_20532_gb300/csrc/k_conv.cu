@@ -11,6 +11,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include "conv_thin.h"
 #include "internal.h"
 #include "tc.h"
 
