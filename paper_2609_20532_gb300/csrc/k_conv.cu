@@ -266,15 +266,15 @@ __global__ void __launch_bounds__(kThinThreads)
   if (tid == 0) part[static_cast<int64_t>(row0 + i) * NP] = sq;
 }
 
-int thin_smem_bytes(const ConvGeom& g, int c_out) {
+int64_t thin_smem_bytes(const ConvGeom& g, int64_t c_out) {
   const int64_t hwc = static_cast<int64_t>(g.H) * g.W * g.C_in;
-  return static_cast<int>((((hwc + 3) & ~int64_t(3)) + int64_t(kThinChunk) * c_out) * 4);
+  return (((hwc + 3) & ~int64_t(3)) + int64_t(kThinChunk) * c_out) * 4;
 }
 
 template <typename TIn, int CO>
 cudaError_t launch_thin_t(const void* x, const void* d, const ConvGeom& g, int c_out, int B,
                           float* G, float* part, int NP, int row0, cudaStream_t s) {
-  const int smem = thin_smem_bytes(g, c_out);
+  const int smem = static_cast<int>(thin_smem_bytes(g, c_out));  // <= kConvThinMaxSmem
   if (smem > 48 * 1024) {
     cudaError_t e = setup_once_per_device(
         reinterpret_cast<const void*>(&k_conv_thin_norm<TIn, CO>), [] {
@@ -302,8 +302,8 @@ cudaError_t launch_thin_co(const void* x, const void* d, const ConvGeom& g, int 
 
 bool conv_thin_norm_ok(const ConvGeom& g, int64_t c_out) {
   const int64_t K = static_cast<int64_t>(g.kh) * g.kw * g.C_in;
-  return K >= 1 && K <= kThinThreads && c_out >= 1 && c_out <= 64 &&
-         thin_smem_bytes(g, static_cast<int>(c_out)) <= kConvThinMaxSmem;
+  return K >= 1 && K <= kThinThreads && c_out >= 1 && c_out <= 64 && g.H >= 1 && g.W >= 1 &&
+         thin_smem_bytes(g, c_out) <= kConvThinMaxSmem;
 }
 
 cudaError_t launch_conv_thin_norm(InType t, const void* x, const void* d, const ConvGeom& g,
