@@ -169,11 +169,11 @@ cudaError_t launch_unfold_t(const void* x, void* a, const ConvGeom& g, int B, in
 // walks the output positions in chunks of kThinChunk, the chunk's output
 // gradients [chunk][C_out] staged in shared memory.  Thread (j, q) owns
 // gradient row j (tap (ki, kj), channel c) for the positions q, q + Q, ... of
-// every chunk and all C_out columns; the Q partial rows are then added in q
-// order, the row is written to G_i, and the squares of the example's rows are
-// summed in a fixed order into its single norm partial.  No patch row is
-// formed in memory; the result differs from the unfolded path's only in the
-// order of the fp32 additions.
+// every chunk and all C_out columns (thread q K + j); the Q partial rows are
+// then added in q order, the row is written to G_i, and the squares of the
+// example's rows are summed in a fixed order into its single norm partial.
+// No patch row is formed in memory; the result differs from the unfolded
+// path's only in the order of the fp32 additions.
 // ---------------------------------------------------------------------------
 constexpr int kThinThreads = 256;
 constexpr int kThinChunk = 256;  // positions per staged chunk of d_i
@@ -213,8 +213,10 @@ __global__ void __launch_bounds__(kThinThreads)
   const TIn* xi = x + static_cast<int64_t>(i) * HWC;
   const TIn* di = d + static_cast<int64_t>(i) * T * c_out;
   for (int e = tid; e < HWC; e += kThinThreads) img[e] = to_f(xi[e]);
-  const int j = tid / Q, q = tid - j * Q;
-  const bool own = j < K;
+  // consecutive threads take consecutive rows j at the same positions, so a
+  // warp's reads of a staged output-gradient row are one broadcast
+  const int q = tid / K, j = tid - q * K;
+  const bool own = q < Q;
   int ki = 0, kj = 0, ch = 0;
   if (own) {
     const int tap = j / g.C_in;
